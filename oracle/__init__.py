@@ -1,0 +1,144 @@
+"""CPU oracle for the naive W4A4 linear layer (test infrastructure only).
+
+Only ``tests/``, ``__graft_entry__.smoke()`` and the cpu-baseline/reference
+leg of ``bench.py`` may import this package.  The product library never does.
+
+The arithmetic lives in ``jq_oracle.c`` (plain C, compiled with gcc, no
+fast-math, no FMA contraction); this module only compiles it and marshals
+numpy arrays through ctypes.  Layout conventions used here:
+
+* activation codes / weight codes: ``int8 [rows, K]`` (one code per element);
+* packed codes: ``uint8 [rows, K/2]``, element 2j in the low nibble;
+* activation scales ``s_a``: ``float32 [M, K/G]``;
+* weight scales ``s_w``: ``float32 [N, K/G]`` (per output channel);
+* bf16 values travel as their ``uint16`` bit patterns.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import subprocess
+import threading
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_SRC = os.path.join(_HERE, "jq_oracle.c")
+_LIB = os.path.join(_HERE, "liboracle.so")
+_lock = threading.Lock()
+_lib = None
+
+_CFLAGS = ["-O2", "-ffp-contract=off", "-fno-fast-math", "-fopenmp", "-fPIC", "-shared", "-std=c11"]
+
+
+def build(force: bool = False) -> str:
+    """Compile the oracle into ``oracle/liboracle.so`` (gcc, seconds)."""
+    if force or not os.path.exists(_LIB) or os.path.getmtime(_LIB) < max(
+        os.path.getmtime(_SRC), os.path.getmtime(os.path.join(_HERE, "jq_oracle.h"))
+    ):
+        tmp = _LIB + f".tmp{os.getpid()}"
+        subprocess.check_call(["gcc", *_CFLAGS, "-o", tmp, _SRC, "-lm"])
+        os.replace(tmp, _LIB)
+    return _LIB
+
+
+def _load():
+    global _lib
+    with _lock:
+        if _lib is None:
+            lib = ctypes.CDLL(build())
+            i64, vp = ctypes.c_int64, ctypes.c_void_p
+            lib.oracle_bf16_rne.argtypes = [ctypes.c_double]
+            lib.oracle_bf16_rne.restype = ctypes.c_uint16
+            lib.oracle_quantize_bf16.argtypes = [vp, i64, i64, i64, i64, vp, vp]
+            lib.oracle_quantize_f32.argtypes = [vp, i64, i64, i64, vp, vp]
+            lib.oracle_pack.argtypes = [vp, i64, i64, vp]
+            lib.oracle_unpack.argtypes = [vp, i64, i64, vp]
+            lib.oracle_group_partials.argtypes = [vp, vp, i64, i64, i64, i64, vp]
+            lib.oracle_linear.argtypes = [vp, vp, vp, vp, vp, i64, i64, i64, i64, vp, vp]
+            for f in ("oracle_quantize_bf16", "oracle_quantize_f32", "oracle_pack", "oracle_unpack",
+                      "oracle_group_partials", "oracle_linear"):
+                getattr(lib, f).restype = None
+            _lib = lib
+    return _lib
+
+
+def _p(a):
+    return None if a is None else a.ctypes.data_as(ctypes.c_void_p)
+
+
+def _c(a, dtype):
+    return np.ascontiguousarray(a, dtype=dtype)
+
+
+def bf16_rne(v: float) -> int:
+    """fp64 -> bf16 bits, round to nearest even."""
+    return int(_load().oracle_bf16_rne(float(v)))
+
+
+def quantize_bf16(x_bits: np.ndarray, group: int):
+    """bf16 activations (uint16 bits, [M, K] or a strided view) -> (codes int8 [M,K], s_a f32 [M,K/G])."""
+    x_bits = np.asarray(x_bits)
+    assert x_bits.dtype == np.uint16 and x_bits.ndim == 2
+    M, K = x_bits.shape
+    assert K % group == 0
+    if x_bits.strides[1] != 2 or x_bits.strides[0] % 2:
+        x_bits = np.ascontiguousarray(x_bits)
+    ldx = x_bits.strides[0] // 2
+    codes = np.empty((M, K), np.int8)
+    scales = np.empty((M, K // group), np.float32)
+    _load().oracle_quantize_bf16(_p(x_bits), M, K, ldx, group, _p(codes), _p(scales))
+    return codes, scales
+
+
+def quantize_f32(w: np.ndarray, group: int):
+    """fp32 weights [N, K] -> (codes int8 [N,K], s_w f32 [N,K/G])."""
+    w = _c(w, np.float32)
+    N, K = w.shape
+    assert K % group == 0
+    codes = np.empty((N, K), np.int8)
+    scales = np.empty((N, K // group), np.float32)
+    _load().oracle_quantize_f32(_p(w), N, K, group, _p(codes), _p(scales))
+    return codes, scales
+
+
+def pack(codes: np.ndarray) -> np.ndarray:
+    codes = _c(codes, np.int8)
+    R, K = codes.shape
+    assert K % 2 == 0
+    out = np.empty((R, K // 2), np.uint8)
+    _load().oracle_pack(_p(codes), R, K, _p(out))
+    return out
+
+
+def unpack(packed: np.ndarray) -> np.ndarray:
+    packed = _c(packed, np.uint8)
+    R, H = packed.shape
+    out = np.empty((R, 2 * H), np.int8)
+    _load().oracle_unpack(_p(packed), R, 2 * H, _p(out))
+    return out
+
+
+def group_partials(qa: np.ndarray, qw: np.ndarray, group: int) -> np.ndarray:
+    """Exact per-group integer partials, int32 [M, N, K/G]."""
+    qa, qw = _c(qa, np.int8), _c(qw, np.int8)
+    M, K = qa.shape
+    N, K2 = qw.shape
+    assert K == K2 and K % group == 0
+    acc = np.empty((M, N, K // group), np.int32)
+    _load().oracle_group_partials(_p(qa), _p(qw), M, N, K, group, _p(acc))
+    return acc
+
+
+def linear(qa, s_a, qw, s_w, bias, group: int):
+    """(y64 float64 [M,N], y_bf16 uint16 [M,N]) of the dequantising linear layer."""
+    qa, qw = _c(qa, np.int8), _c(qw, np.int8)
+    s_a, s_w = _c(s_a, np.float32), _c(s_w, np.float32)
+    M, K = qa.shape
+    N = qw.shape[0]
+    assert s_a.shape == (M, K // group) and s_w.shape == (N, K // group)
+    b = None if bias is None else _c(bias, np.float32)
+    y64 = np.empty((M, N), np.float64)
+    yb = np.empty((M, N), np.uint16)
+    _load().oracle_linear(_p(qa), _p(s_a), _p(qw), _p(s_w), _p(b), M, N, K, group, _p(y64), _p(yb))
+    return y64, yb

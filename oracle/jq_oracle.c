@@ -1,0 +1,206 @@
+/*
+ * jq_oracle.c -- plain, slow, obviously-correct CPU oracle for the naive
+ * W4A4 linear layer of JustQuant (arxiv 2609.33601).
+ *
+ * TEST INFRASTRUCTURE ONLY.  Nothing in the product path may link, load or
+ * call this file: only tests/, __graft_entry__.smoke() and the cpu_baseline /
+ * reference leg of bench.py use it.  It shares no code, header, table or
+ * constant with the CUDA library (paper_2609_33601_gb300/csrc).
+ *
+ * What the paper fixes (and what this file computes):
+ *   - The deployed graph is a "plain low-bit operator graph": quantise, pack,
+ *     low-bit GEMM, with no smoothing, rotation, normalisation or SVD branch
+ *     (Sec. 1 contributions; Appendix FAQ Q7).
+ *   - Transformer-block linears run INT4 weights and INT4 activations with
+ *     group-wise scales: group128 for DiT-XL/2 and ELF-B (Appendix tables
+ *     "DiT-XL/2 experimental details", "ELF-B and LLaDA-8B experimental
+ *     details"), group64 for FLUX (Sec. 4.2 "FLUX"; Appendix table "FLUX
+ *     experimental details").
+ *   - The paper prints no quantiser formula.  The reading used here (and in
+ *     the GPU path) is the symmetric INT4 rule: for each row and each run of
+ *     G consecutive reduction-axis elements,
+ *         amax = max |x|,  s = fl32(amax / 7),
+ *         q = clamp(rint(fl32(x / s)), -8, 7)      (round half to even)
+ *     with s = 0 and q = 0 when amax == 0.  Codes are packed two per byte,
+ *     element 2j in the low nibble, 4-bit two's complement.
+ *   - The linear layer: acc[m,n,g] = sum_{k in g} qa[m,k]*qw[n,k] (exact
+ *     integers), y[m,n] = sum_g acc*s_a[m,g]*s_w[n,g] + bias[n], evaluated
+ *     here in fp64 and rounded once to bf16 (round to nearest even).
+ *
+ * Floating point: compile with -O2 -ffp-contract=off and without fast-math,
+ * so float division is the IEEE-754 single-precision correctly-rounded one
+ * and rintf rounds half to even (default rounding mode).  OpenMP only splits
+ * independent rows across threads; it never changes any arithmetic.
+ */
+#include <math.h>
+#include <stdint.h>
+#include <stdlib.h>
+#include <string.h>
+
+#include "jq_oracle.h"
+
+/* ---- bf16 helpers ------------------------------------------------------ */
+
+/* bf16 -> fp32 is exact: a bf16 is the top half of an fp32. */
+static float bf16_bits_to_float(uint16_t b) {
+  uint32_t u = ((uint32_t)b) << 16;
+  float f;
+  memcpy(&f, &u, sizeof f);
+  return f;
+}
+
+/*
+ * Round an fp64 value to the nearest bf16 (ties to even), by exact scaling:
+ * find the bf16 quantum (ulp) of |v|, round |v|/ulp to an integer with rint
+ * (fp64, ties to even), scale back.  bf16 has 8 significant bits, normal
+ * exponents down to 2^-126 and subnormals in steps of 2^-133.
+ */
+uint16_t oracle_bf16_rne(double v) {
+  if (isnan(v)) return 0x7FC0;
+  const int neg = signbit(v) ? 1 : 0;
+  double a = fabs(v);
+  double r;
+  if (a == 0.0) {
+    r = 0.0;
+  } else if (isinf(a)) {
+    r = INFINITY;
+  } else {
+    int e;
+    (void)frexp(a, &e);           /* a = f * 2^e, f in [0.5, 1) -> a in [2^(e-1), 2^e) */
+    int ulp_exp = (e - 1) - 7;    /* 8 significant bits */
+    if (ulp_exp < -133) ulp_exp = -133;  /* subnormal quantum */
+    double q = ldexp(a, -ulp_exp);       /* exact */
+    double n = rint(q);                  /* ties to even */
+    r = ldexp(n, ulp_exp);
+    /* largest finite bf16 is (2 - 2^-7) * 2^127; anything rounding above it is inf */
+    if (r > ldexp(255.0, 120)) r = INFINITY;
+  }
+  float f = (float)r; /* exact: r is representable in bf16, hence in fp32 */
+  uint32_t u;
+  memcpy(&u, &f, sizeof u);
+  uint16_t b = (uint16_t)(u >> 16);
+  if (neg) b |= 0x8000;
+  return b;
+}
+
+/* ---- quantiser (one group) --------------------------------------------- */
+
+/*
+ * Symmetric INT4 quantisation of one group of G consecutive values already
+ * widened to fp32 (the rule in the file header).  Writes G codes and returns
+ * the group scale.
+ */
+static float quantize_group(const float* xf, int64_t G, int8_t* q) {
+  float amax = 0.0f;
+  for (int64_t k = 0; k < G; ++k) {
+    float a = fabsf(xf[k]);
+    if (a > amax) amax = a;
+  }
+  if (amax == 0.0f) {
+    for (int64_t k = 0; k < G; ++k) q[k] = 0;
+    return 0.0f;
+  }
+  const float s = amax / 7.0f;            /* IEEE single division */
+  for (int64_t k = 0; k < G; ++k) {
+    float t = xf[k] / s;                  /* IEEE single division */
+    float r = rintf(t);                   /* half to even */
+    if (r > 7.0f) r = 7.0f;
+    if (r < -8.0f) r = -8.0f;
+    q[k] = (int8_t)r;
+  }
+  return s;
+}
+
+/* Activations: bf16 [M, K] with row stride ldx (elements) -> codes [M, K] and
+ * scales [M, K/G] (row-major, one scale per token and K-group). */
+void oracle_quantize_bf16(const uint16_t* x, int64_t M, int64_t K, int64_t ldx,
+                          int64_t G, int8_t* codes, float* scales) {
+  const int64_t ng = K / G;
+#pragma omp parallel for schedule(static)
+  for (int64_t m = 0; m < M; ++m) {
+    float* xf = (float*)malloc((size_t)K * sizeof(float));
+    for (int64_t k = 0; k < K; ++k) xf[k] = bf16_bits_to_float(x[m * ldx + k]);
+    for (int64_t g = 0; g < ng; ++g)
+      scales[m * ng + g] = quantize_group(xf + g * G, G, codes + m * K + g * G);
+    free(xf);
+  }
+}
+
+/* Weights: fp32 [N, K] row-major -> codes [N, K] and scales [N, K/G] (one
+ * scale per output channel and K-group). */
+void oracle_quantize_f32(const float* w, int64_t N, int64_t K, int64_t G,
+                         int8_t* codes, float* scales) {
+  const int64_t ng = K / G;
+#pragma omp parallel for schedule(static)
+  for (int64_t n = 0; n < N; ++n) {
+    for (int64_t g = 0; g < ng; ++g) {
+      scales[n * ng + g] = quantize_group(w + n * K + g * G, G, codes + n * K + g * G);
+    }
+  }
+}
+
+/* ---- packing ------------------------------------------------------------ */
+
+/* codes [rows, K] -> bytes [rows, K/2]: element 2j in the low nibble, 2j+1 in
+ * the high nibble, each as 4-bit two's complement. */
+void oracle_pack(const int8_t* codes, int64_t rows, int64_t K, uint8_t* packed) {
+  for (int64_t r = 0; r < rows; ++r)
+    for (int64_t j = 0; j < K / 2; ++j) {
+      uint8_t lo = (uint8_t)(codes[r * K + 2 * j] & 0x0F);
+      uint8_t hi = (uint8_t)(codes[r * K + 2 * j + 1] & 0x0F);
+      packed[r * (K / 2) + j] = (uint8_t)(lo | (hi << 4));
+    }
+}
+
+/* Inverse of oracle_pack: sign-extend each nibble. */
+void oracle_unpack(const uint8_t* packed, int64_t rows, int64_t K, int8_t* codes) {
+  for (int64_t r = 0; r < rows; ++r)
+    for (int64_t j = 0; j < K / 2; ++j) {
+      uint8_t b = packed[r * (K / 2) + j];
+      int lo = b & 0x0F, hi = (b >> 4) & 0x0F;
+      codes[r * K + 2 * j] = (int8_t)(lo >= 8 ? lo - 16 : lo);
+      codes[r * K + 2 * j + 1] = (int8_t)(hi >= 8 ? hi - 16 : hi);
+    }
+}
+
+/* ---- integer GEMM and the dequantising epilogue ------------------------- */
+
+/* acc[m, n, g] = sum over the G elements of group g of qa[m,k] * qw[n,k]. */
+void oracle_group_partials(const int8_t* qa, const int8_t* qw, int64_t M, int64_t N,
+                           int64_t K, int64_t G, int32_t* acc) {
+  const int64_t ng = K / G;
+#pragma omp parallel for schedule(static)
+  for (int64_t m = 0; m < M; ++m)
+    for (int64_t n = 0; n < N; ++n)
+      for (int64_t g = 0; g < ng; ++g) {
+        int32_t s = 0;
+        for (int64_t k = g * G; k < (g + 1) * G; ++k) s += (int32_t)qa[m * K + k] * (int32_t)qw[n * K + k];
+        acc[(m * N + n) * ng + g] = s;
+      }
+}
+
+/*
+ * y64[m, n] = sum_g acc[m,n,g] * s_a[m,g] * s_w[n,g] + bias[n]   (fp64)
+ * ybf16     = bf16_rne(y64)
+ * s_a is [M, K/G], s_w is [N, K/G] (per output channel), bias is [N] or NULL.
+ * The partial sums are recomputed here, one group at a time, from the codes.
+ * Either output pointer may be NULL.
+ */
+void oracle_linear(const int8_t* qa, const float* s_a, const int8_t* qw, const float* s_w,
+                   const float* bias, int64_t M, int64_t N, int64_t K, int64_t G,
+                   double* y64, uint16_t* ybf16) {
+  const int64_t ng = K / G;
+#pragma omp parallel for schedule(static)
+  for (int64_t m = 0; m < M; ++m)
+    for (int64_t n = 0; n < N; ++n) {
+      double y = 0.0;
+      for (int64_t g = 0; g < ng; ++g) {
+        int32_t s = 0;
+        for (int64_t k = g * G; k < (g + 1) * G; ++k) s += (int32_t)qa[m * K + k] * (int32_t)qw[n * K + k];
+        y += ((double)s * (double)s_a[m * ng + g]) * (double)s_w[n * ng + g];
+      }
+      if (bias) y += (double)bias[n];
+      if (y64) y64[m * N + n] = y;
+      if (ybf16) ybf16[m * N + n] = oracle_bf16_rne(y);
+    }
+}

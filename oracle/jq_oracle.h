@@ -1,0 +1,24 @@
+/* jq_oracle.h -- declarations of the CPU oracle (test infrastructure only;
+ * see jq_oracle.c for the definitions and the passages they follow). */
+#ifndef JQ_ORACLE_H
+#define JQ_ORACLE_H
+#include <stdint.h>
+#ifdef __cplusplus
+extern "C" {
+#endif
+uint16_t oracle_bf16_rne(double v);
+void oracle_quantize_bf16(const uint16_t* x, int64_t M, int64_t K, int64_t ldx, int64_t G,
+                          int8_t* codes, float* scales);
+void oracle_quantize_f32(const float* w, int64_t N, int64_t K, int64_t G, int8_t* codes,
+                         float* scales);
+void oracle_pack(const int8_t* codes, int64_t rows, int64_t K, uint8_t* packed);
+void oracle_unpack(const uint8_t* packed, int64_t rows, int64_t K, int8_t* codes);
+void oracle_group_partials(const int8_t* qa, const int8_t* qw, int64_t M, int64_t N, int64_t K,
+                           int64_t G, int32_t* acc);
+void oracle_linear(const int8_t* qa, const float* s_a, const int8_t* qw, const float* s_w,
+                   const float* bias, int64_t M, int64_t N, int64_t K, int64_t G, double* y64,
+                   uint16_t* ybf16);
+#ifdef __cplusplus
+}
+#endif
+#endif
