@@ -1,0 +1,144 @@
+/*
+ * jq.h -- C ABI of libjq: the naive W4A4 linear layer of JustQuant (arxiv 2609.33601)
+ * on one GB300 (sm_103a).
+ *
+ * The paper deploys a "plain low-bit operator graph": activations and weights are quantised
+ * to INT4 with per-group scales, packed, and multiplied by a low-bit GEMM, with no smoothing,
+ * rotation, normalisation or SVD branch (Sec. 1; Appendix FAQ Q7: low-bit execution "still
+ * requires suitable quantization, packing, and matrix-multiplication kernels").  Group sizes
+ * are fixed by the paper: group64 for FLUX transformer-block linears (Sec. 4.2 "FLUX";
+ * Appendix table "FLUX experimental details"), group128 for DiT-XL/2 and ELF-B (Appendix
+ * tables "DiT-XL/2 experimental details", "ELF-B and LLaDA-8B experimental details").
+ * Per-token / per-channel scaling is the special case group == K.
+ *
+ * Quantiser (the paper prints no formula; this is the symmetric INT4 reading):
+ *     per row and per run of `group` consecutive K elements:
+ *     amax = max|x|,  s = fl32(amax / 7),  q = clamp(rint(fl32(x / s)), -8, 7)
+ *     (IEEE fp32 division, round half to even; s = 0 and q = 0 when amax == 0).
+ * Linear layer:
+ *     acc[m,n,g] = sum_{k in group g} qa[m,k] * qw[n,k]            (exact integers)
+ *     y[m,n]     = bf16_rne( sum_g acc[m,n,g] * s_a[m,g] * s_w[g,n] + bias[n] )  (fp32 math)
+ *
+ * Conventions shared by every entry point
+ *   - Matrices are row-major with K contiguous.  Packed codes: 4-bit two's complement, two per
+ *     byte, element 2j in the low nibble of byte j; a row of K codes is K/2 bytes.
+ *   - Activation scales s_a: fp32 [M, K/group] (one per token and K-group).
+ *     Weight scales s_w:     fp32 [K/group, N] (group-major: one row of N channel scales per
+ *     K-group).  bias: fp32 [N] or NULL.  Outputs y: bf16 [M, N].
+ *   - All data pointers are DEVICE pointers owned by the caller.  The library allocates
+ *     nothing, never synchronises, and enqueues its kernels on `stream` (a cudaStream_t passed
+ *     as void*; NULL = legacy default stream).
+ *   - Supported shapes: group in {64, 128, K}; K % 128 == 0; K <= 262016 (so every exact
+ *     per-group sum, |acc| <= 64*K, stays below 2^24); N % 8 == 0; M >= 0 (M == 0 is a no-op).
+ *   - Pointers must be 16-byte aligned and ldx*2 a multiple of 16 bytes.
+ *   - Arguments are checked synchronously before any launch; a failed check returns an error
+ *     status and launches nothing.  A failed launch returns JQ_ERR_CUDA.  No exception
+ *     crosses the ABI.
+ *   - Every on-GPU wait is bounded (about a second).  A kernel that gives up records
+ *     JQ_ERR_TIMEOUT in a device status word read by jq_device_status().
+ */
+#ifndef JQ_H
+#define JQ_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#if defined(__GNUC__)
+#define JQ_API __attribute__((visibility("default")))
+#else
+#define JQ_API
+#endif
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  JQ_OK = 0,
+  JQ_ERR_INVALID_ARG = 1,  /* null pointer, bad size, unsupported group/K/N combination */
+  JQ_ERR_MISALIGNED = 2,   /* a pointer or a row pitch breaks the 16-byte rule */
+  JQ_ERR_UNSUPPORTED = 3,  /* no CUDA device of the required architecture (sm_103) */
+  JQ_ERR_CUDA = 4,         /* a CUDA runtime/driver call or kernel launch failed */
+  JQ_ERR_TIMEOUT = 5,      /* a kernel gave up a bounded wait (reported by jq_device_status) */
+  JQ_ERR_WORKSPACE = 6     /* workspace pointer NULL/misaligned or smaller than required */
+} jq_status;
+
+/* Human-readable name of a status code (static string, never NULL). */
+JQ_API const char* jq_status_string(jq_status s);
+
+/*
+ * Activation quantiser (per token and K-group; rule above).
+ *   x_bf16 : bf16 [M, ldx] (the first K columns are used), ldx >= K, ldx*2 % 16 == 0
+ *   q      : uint8 [M, K/2] packed codes (output)
+ *   s_a    : fp32 [M, K/group] scales (output)
+ * Errors: JQ_ERR_INVALID_ARG (null, K/group unsupported, ldx < K), JQ_ERR_MISALIGNED.
+ */
+JQ_API jq_status jq_quantize_act(const void* x_bf16, int64_t M, int64_t K, int64_t ldx, int32_t group,
+                          uint8_t* q, float* s_a, void* stream);
+
+/*
+ * Weight packer (offline; the same rule per output channel and K-group).
+ *   w   : fp32 [N, K] row-major
+ *   qw  : uint8 [N, K/2] packed codes (output)
+ *   s_w : fp32 [K/group, N] scales (output, group-major)
+ * Errors as jq_quantize_act.
+ */
+JQ_API jq_status jq_pack_weight(const float* w, int64_t N, int64_t K, int32_t group, uint8_t* qw, float* s_w,
+                         void* stream);
+
+/*
+ * Bytes of device scratch the two linear entry points need for this shape
+ * (fused != 0: jq_fused_quant_linear, else jq_w4a4_linear).  The caller owns it.
+ */
+JQ_API size_t jq_workspace_size(int64_t M, int64_t N, int64_t K, int32_t group, int32_t fused);
+
+/*
+ * W4A4 linear on pre-quantised activations:
+ *   y = bf16( sum_g acc[m,n,g] * s_a[m,g] * s_w[g,n] + bias[n] ).
+ *   q         : uint8 [M, K/2] packed activation codes (jq_quantize_act)
+ *   s_a       : fp32 [M, K/group]
+ *   qw, s_w   : packed weights and scales (jq_pack_weight, or any codes/finite scales in
+ *               these layouts, including the code -8)
+ *   bias      : fp32 [N] or NULL
+ *   y_bf16    : bf16 [M, N] (output)
+ *   workspace : >= jq_workspace_size(M, N, K, group, 0) bytes of device memory, 16-byte aligned
+ * Errors: JQ_ERR_INVALID_ARG, JQ_ERR_MISALIGNED, JQ_ERR_WORKSPACE, JQ_ERR_CUDA.
+ */
+JQ_API jq_status jq_w4a4_linear(const uint8_t* q, const float* s_a, const uint8_t* qw, const float* s_w,
+                         const float* bias, void* y_bf16, int64_t M, int64_t N, int64_t K, int32_t group,
+                         void* workspace, size_t workspace_bytes, void* stream);
+
+/*
+ * W4A4 linear straight from bf16 activations: quantises x (rule above, per token and
+ * K-group) directly into the GEMM's operand layout, then runs the same GEMM.  Results are
+ * bit-identical to jq_quantize_act followed by jq_w4a4_linear.
+ *   x_bf16    : bf16 [M, ldx]
+ *   workspace : >= jq_workspace_size(M, N, K, group, 1) bytes
+ * Other arguments and errors as jq_w4a4_linear.
+ */
+JQ_API jq_status jq_fused_quant_linear(const void* x_bf16, int64_t ldx, const uint8_t* qw, const float* s_w,
+                                const float* bias, void* y_bf16, int64_t M, int64_t N, int64_t K,
+                                int32_t group, void* workspace, size_t workspace_bytes, void* stream);
+
+/*
+ * Verification export of the exact per-group integer partials of the GEMM:
+ *   acc : int32 [M, N, K/group], acc[m,n,g] = sum_{k in g} qa[m,k] * qw[n,k].
+ * Runs the same mainloop as jq_w4a4_linear with the dequantising epilogue replaced by an
+ * integer store; meant for small shapes.  workspace as jq_w4a4_linear.
+ */
+JQ_API jq_status jq_w4a4_group_partials(const uint8_t* q, const uint8_t* qw, int32_t* acc, int64_t M, int64_t N,
+                                 int64_t K, int32_t group, void* workspace, size_t workspace_bytes,
+                                 void* stream);
+
+/*
+ * Synchronises `stream` and returns JQ_ERR_TIMEOUT if any kernel of this library on the
+ * current device gave up a bounded wait since the last reset (reset != 0 clears the flag),
+ * JQ_ERR_CUDA if the stream reports an error, JQ_OK otherwise.
+ */
+JQ_API jq_status jq_device_status(void* stream, int32_t reset);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* JQ_H */

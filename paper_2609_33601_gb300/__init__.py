@@ -1,0 +1,180 @@
+"""GB300-native naive W4A4 linear layer of JustQuant (arxiv 2609.33601).
+
+Python binding of ``libjq.so`` (the C ABI in ``include/jq.h``).  The functions carry the C
+names and only marshal arguments: torch tensors provide device memory and the current CUDA
+stream, and every step of the computation runs in the library's sm_103a kernels.  There is no
+CPU or PyTorch fallback: if ``libjq.so`` is missing or the device is not an sm_103 GPU, the
+calls raise.
+
+    q, s_a  = jq_quantize_act(x_bf16, group)              # INT4 codes, per (token, K-group) scales
+    qw, s_w = jq_pack_weight(w_fp32, group)               # offline
+    y       = jq_w4a4_linear(q, s_a, qw, s_w, bias, group)
+    y       = jq_fused_quant_linear(x_bf16, qw, s_w, bias, group)
+
+Layouts: x bf16 [M, K] (row stride may exceed K); q uint8 [M, K/2]; s_a fp32 [M, K/G];
+qw uint8 [N, K/2]; s_w fp32 [K/G, N]; bias fp32 [N] or None; y bf16 [M, N].
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import threading
+
+import torch
+
+__all__ = [
+    "JQError", "library_path", "jq_quantize_act", "jq_pack_weight", "jq_workspace_size", "jq_w4a4_linear",
+    "jq_fused_quant_linear", "jq_w4a4_group_partials", "jq_device_status", "jq_status_string",
+]
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+library_path = os.path.join(_HERE, "libjq.so")
+
+JQ_STATUS = {0: "JQ_OK", 1: "JQ_ERR_INVALID_ARG", 2: "JQ_ERR_MISALIGNED", 3: "JQ_ERR_UNSUPPORTED",
+             4: "JQ_ERR_CUDA", 5: "JQ_ERR_TIMEOUT", 6: "JQ_ERR_WORKSPACE"}
+
+_lock = threading.Lock()
+_lib = None
+
+
+class JQError(RuntimeError):
+    def __init__(self, fn: str, code: int):
+        super().__init__(f"{fn} failed: {JQ_STATUS.get(code, code)}")
+        self.code = code
+
+
+def _load() -> ctypes.CDLL:
+    global _lib
+    with _lock:
+        if _lib is None:
+            if not os.path.exists(library_path):
+                raise RuntimeError(
+                    f"{library_path} is not built; run `python -m paper_2609_33601_gb300.build` "
+                    "(needs nvcc for sm_103a). There is no fallback implementation.")
+            lib = ctypes.CDLL(library_path)
+            i64, i32, vp, sz = ctypes.c_int64, ctypes.c_int32, ctypes.c_void_p, ctypes.c_size_t
+            sig = {
+                "jq_quantize_act": [vp, i64, i64, i64, i32, vp, vp, vp],
+                "jq_pack_weight": [vp, i64, i64, i32, vp, vp, vp],
+                "jq_w4a4_linear": [vp, vp, vp, vp, vp, vp, i64, i64, i64, i32, vp, sz, vp],
+                "jq_fused_quant_linear": [vp, i64, vp, vp, vp, vp, i64, i64, i64, i32, vp, sz, vp],
+                "jq_w4a4_group_partials": [vp, vp, vp, i64, i64, i64, i32, vp, sz, vp],
+                "jq_device_status": [vp, i32],
+            }
+            for name, args in sig.items():
+                f = getattr(lib, name)
+                f.argtypes = args
+                f.restype = ctypes.c_int
+            lib.jq_workspace_size.argtypes = [i64, i64, i64, i32, i32]
+            lib.jq_workspace_size.restype = ctypes.c_size_t
+            lib.jq_status_string.argtypes = [ctypes.c_int]
+            lib.jq_status_string.restype = ctypes.c_char_p
+            _lib = lib
+    return _lib
+
+
+def _check(name: str, code: int) -> None:
+    if code != 0:
+        raise JQError(name, code)
+
+
+def _ptr(t):
+    return None if t is None else ctypes.c_void_p(t.data_ptr())
+
+
+def _stream(stream=None):
+    s = torch.cuda.current_stream() if stream is None else stream
+    return ctypes.c_void_p(s.cuda_stream)
+
+
+def _need_cuda(*ts):
+    for t in ts:
+        if t is not None and not t.is_cuda:
+            raise ValueError("libjq works on CUDA tensors only")
+
+
+def jq_status_string(code: int) -> str:
+    return _load().jq_status_string(code).decode()
+
+
+def jq_workspace_size(M: int, N: int, K: int, group: int, fused: bool = False) -> int:
+    return int(_load().jq_workspace_size(M, N, K, group, 1 if fused else 0))
+
+
+def _workspace(M, N, K, group, fused, device, workspace):
+    need = jq_workspace_size(M, N, K, group, fused)
+    if workspace is None:
+        workspace = torch.empty(max(need, 16), dtype=torch.uint8, device=device)
+    return workspace, workspace.numel() * workspace.element_size()
+
+
+def jq_quantize_act(x: torch.Tensor, group: int, q: torch.Tensor | None = None, s_a: torch.Tensor | None = None,
+                    stream=None):
+    """bf16 activations [M, K] (row stride >= K) -> (packed codes uint8 [M, K/2], scales fp32 [M, K/G])."""
+    assert x.dtype == torch.bfloat16 and x.dim() == 2 and x.stride(1) == 1
+    _need_cuda(x)
+    M, K = x.shape
+    if q is None:
+        q = torch.empty((M, K // 2), dtype=torch.uint8, device=x.device)
+    if s_a is None:
+        s_a = torch.empty((M, K // group if group else 0), dtype=torch.float32, device=x.device)
+    _check("jq_quantize_act", _load().jq_quantize_act(_ptr(x), M, K, x.stride(0), group, _ptr(q), _ptr(s_a),
+                                                      _stream(stream)))
+    return q, s_a
+
+
+def jq_pack_weight(w: torch.Tensor, group: int, stream=None):
+    """fp32 weights [N, K] -> (packed codes uint8 [N, K/2], scales fp32 [K/G, N])."""
+    assert w.dtype == torch.float32 and w.dim() == 2 and w.is_contiguous()
+    _need_cuda(w)
+    N, K = w.shape
+    qw = torch.empty((N, K // 2), dtype=torch.uint8, device=w.device)
+    s_w = torch.empty((K // group if group else 0, N), dtype=torch.float32, device=w.device)
+    _check("jq_pack_weight", _load().jq_pack_weight(_ptr(w), N, K, group, _ptr(qw), _ptr(s_w), _stream(stream)))
+    return qw, s_w
+
+
+def jq_w4a4_linear(q, s_a, qw, s_w, bias, group: int, y=None, workspace=None, stream=None):
+    """y = bf16(sum_g acc * s_a * s_w + bias) from packed activation and weight codes."""
+    _need_cuda(q, s_a, qw, s_w, bias)
+    M, K = q.shape[0], q.shape[1] * 2
+    N = qw.shape[0]
+    if y is None:
+        y = torch.empty((M, N), dtype=torch.bfloat16, device=q.device)
+    ws, ws_bytes = _workspace(M, N, K, group, False, q.device, workspace)
+    _check("jq_w4a4_linear", _load().jq_w4a4_linear(_ptr(q), _ptr(s_a), _ptr(qw), _ptr(s_w), _ptr(bias), _ptr(y),
+                                                    M, N, K, group, _ptr(ws), ws_bytes, _stream(stream)))
+    return y
+
+
+def jq_fused_quant_linear(x, qw, s_w, bias, group: int, y=None, workspace=None, stream=None):
+    """Same result as jq_w4a4_linear(*jq_quantize_act(x, group), ...), straight from bf16 x."""
+    assert x.dtype == torch.bfloat16 and x.dim() == 2 and x.stride(1) == 1
+    _need_cuda(x, qw, s_w, bias)
+    M, K = x.shape
+    N = qw.shape[0]
+    if y is None:
+        y = torch.empty((M, N), dtype=torch.bfloat16, device=x.device)
+    ws, ws_bytes = _workspace(M, N, K, group, True, x.device, workspace)
+    _check("jq_fused_quant_linear",
+           _load().jq_fused_quant_linear(_ptr(x), x.stride(0), _ptr(qw), _ptr(s_w), _ptr(bias), _ptr(y), M, N, K,
+                                         group, _ptr(ws), ws_bytes, _stream(stream)))
+    return y
+
+
+def jq_w4a4_group_partials(q, qw, group: int, workspace=None, stream=None):
+    """Exact per-group integer partials int32 [M, N, K/G] (verification export)."""
+    _need_cuda(q, qw)
+    M, K = q.shape[0], q.shape[1] * 2
+    N = qw.shape[0]
+    acc = torch.empty((M, N, K // group), dtype=torch.int32, device=q.device)
+    ws, ws_bytes = _workspace(M, N, K, group, False, q.device, workspace)
+    _check("jq_w4a4_group_partials",
+           _load().jq_w4a4_group_partials(_ptr(q), _ptr(qw), _ptr(acc), M, N, K, group, _ptr(ws), ws_bytes,
+                                          _stream(stream)))
+    return acc
+
+
+def jq_device_status(reset: bool = True, stream=None) -> int:
+    """Synchronises the stream; returns the library's status code (5 = a kernel timed out)."""
+    return int(_load().jq_device_status(_stream(stream), 1 if reset else 0))

@@ -1,0 +1,192 @@
+// api.cu -- the C ABI declared in include/jq.h: synchronous argument checks, then kernel
+// launches on the caller's stream.  No allocation, no synchronisation (except in
+// jq_device_status), no exceptions.
+#include <cstdint>
+#include <cuda_runtime.h>
+
+#include "jq.h"
+#include "kernels.cuh"
+
+namespace {
+
+constexpr int kMaxDevices = 64;
+constexpr int64_t kMaxK = 262016;  // 64 * K < 2^24 keeps every exact group sum representable
+
+// One status word per device, written by kernels that give up a bounded wait.
+__device__ uint32_t g_device_status = 0;
+
+struct DeviceInfo {
+  bool probed = false;
+  bool ok = false;
+  int sms = 0;
+  uint32_t* status = nullptr;
+};
+DeviceInfo g_devices[kMaxDevices];
+
+// Resolves the current device once: it must be an sm_103 part.
+const DeviceInfo* current_device() {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return nullptr;
+  DeviceInfo& d = g_devices[dev];
+  if (!d.probed) {
+    d.probed = true;
+    cudaDeviceProp prop;
+    if (cudaGetDeviceProperties(&prop, dev) != cudaSuccess) return nullptr;
+    d.sms = prop.multiProcessorCount;
+    void* p = nullptr;
+    d.ok = (prop.major == 10 && prop.minor == 3) && cudaGetSymbolAddress(&p, g_device_status) == cudaSuccess;
+    d.status = static_cast<uint32_t*>(p);
+  }
+  return d.ok ? &d : nullptr;
+}
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+bool group_ok(int64_t K, int32_t group) {
+  if (K <= 0 || K % 128 != 0 || K > kMaxK) return false;
+  return group == 64 || group == 128 || group == K;
+}
+
+size_t round_up(size_t v, size_t a) { return (v + a - 1) / a * a; }
+
+jq_status from_cuda(cudaError_t e) { return e == cudaSuccess ? JQ_OK : JQ_ERR_CUDA; }
+
+}  // namespace
+
+extern "C" {
+
+const char* jq_status_string(jq_status s) {
+  switch (s) {
+    case JQ_OK: return "JQ_OK";
+    case JQ_ERR_INVALID_ARG: return "JQ_ERR_INVALID_ARG";
+    case JQ_ERR_MISALIGNED: return "JQ_ERR_MISALIGNED";
+    case JQ_ERR_UNSUPPORTED: return "JQ_ERR_UNSUPPORTED";
+    case JQ_ERR_CUDA: return "JQ_ERR_CUDA";
+    case JQ_ERR_TIMEOUT: return "JQ_ERR_TIMEOUT";
+    case JQ_ERR_WORKSPACE: return "JQ_ERR_WORKSPACE";
+  }
+  return "JQ_ERR_UNKNOWN";
+}
+
+jq_status jq_quantize_act(const void* x_bf16, int64_t M, int64_t K, int64_t ldx, int32_t group, uint8_t* q,
+                          float* s_a, void* stream) {
+  if (M < 0 || !group_ok(K, group) || ldx < K) return JQ_ERR_INVALID_ARG;
+  if (M == 0) return JQ_OK;
+  if (x_bf16 == nullptr || q == nullptr || s_a == nullptr) return JQ_ERR_INVALID_ARG;
+  if (!aligned16(x_bf16) || !aligned16(q) || !aligned16(s_a) || (ldx * 2) % 16 != 0) return JQ_ERR_MISALIGNED;
+  const DeviceInfo* d = current_device();
+  if (d == nullptr) return JQ_ERR_UNSUPPORTED;
+  return from_cuda(jq::launch_quantize_act(x_bf16, M, K, ldx, group, q, s_a, static_cast<cudaStream_t>(stream),
+                                           d->sms));
+}
+
+jq_status jq_pack_weight(const float* w, int64_t N, int64_t K, int32_t group, uint8_t* qw, float* s_w,
+                         void* stream) {
+  if (N < 0 || !group_ok(K, group)) return JQ_ERR_INVALID_ARG;
+  if (N == 0) return JQ_OK;
+  if (w == nullptr || qw == nullptr || s_w == nullptr) return JQ_ERR_INVALID_ARG;
+  if (!aligned16(w) || !aligned16(qw) || !aligned16(s_w)) return JQ_ERR_MISALIGNED;
+  const DeviceInfo* d = current_device();
+  if (d == nullptr) return JQ_ERR_UNSUPPORTED;
+  return from_cuda(jq::launch_pack_weight(w, N, K, group, qw, s_w, static_cast<cudaStream_t>(stream), d->sms));
+}
+
+size_t jq_workspace_size(int64_t M, int64_t N, int64_t K, int32_t group, int32_t fused) {
+  (void)N;
+  if (M <= 0 || K <= 0 || group <= 0 || K % group != 0) return 0;
+  size_t bytes = round_up(static_cast<size_t>(M) * static_cast<size_t>(K), 256);  // A operand bytes
+  if (fused) bytes += round_up(static_cast<size_t>(M) * static_cast<size_t>(K / group) * sizeof(float), 256);
+  return bytes;
+}
+
+namespace {
+
+jq_status check_linear(int64_t M, int64_t N, int64_t K, int32_t group, const void* qw, const float* s_w,
+                       const float* bias, const void* y, size_t ws_need, const void* ws, size_t ws_bytes) {
+  if (M < 0 || N < 0 || N % 8 != 0 || N > INT32_MAX || M > INT32_MAX || !group_ok(K, group))
+    return JQ_ERR_INVALID_ARG;
+  if (qw == nullptr || s_w == nullptr || y == nullptr) return JQ_ERR_INVALID_ARG;
+  if (!aligned16(qw) || !aligned16(s_w) || !aligned16(y) || (bias != nullptr && !aligned16(bias)))
+    return JQ_ERR_MISALIGNED;
+  if (ws == nullptr || !aligned16(ws) || ws_bytes < ws_need) return JQ_ERR_WORKSPACE;
+  return JQ_OK;
+}
+
+}  // namespace
+
+jq_status jq_w4a4_linear(const uint8_t* q, const float* s_a, const uint8_t* qw, const float* s_w, const float* bias,
+                         void* y_bf16, int64_t M, int64_t N, int64_t K, int32_t group, void* workspace,
+                         size_t workspace_bytes, void* stream) {
+  if (M == 0 || N == 0) return (M < 0 || N < 0) ? JQ_ERR_INVALID_ARG : JQ_OK;
+  if (q == nullptr || s_a == nullptr) return JQ_ERR_INVALID_ARG;
+  jq_status st = check_linear(M, N, K, group, qw, s_w, bias, y_bf16, jq_workspace_size(M, N, K, group, 0),
+                              workspace, workspace_bytes);
+  if (st != JQ_OK) return st;
+  if (!aligned16(q) || !aligned16(s_a)) return JQ_ERR_MISALIGNED;
+  const DeviceInfo* d = current_device();
+  if (d == nullptr) return JQ_ERR_UNSUPPORTED;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  uint8_t* a_op = static_cast<uint8_t*>(workspace);
+  cudaError_t e = jq::launch_expand_operand(q, M, K, a_op, s, d->sms);
+  if (e != cudaSuccess) return JQ_ERR_CUDA;
+  jq::GemmProblem p{static_cast<int>(M), static_cast<int>(N), static_cast<int>(K), group, a_op, s_a, qw, s_w, bias,
+                    y_bf16, nullptr, d->status};
+  return from_cuda(jq::launch_w4a4_gemm(p, s, d->sms));
+}
+
+jq_status jq_fused_quant_linear(const void* x_bf16, int64_t ldx, const uint8_t* qw, const float* s_w,
+                                const float* bias, void* y_bf16, int64_t M, int64_t N, int64_t K, int32_t group,
+                                void* workspace, size_t workspace_bytes, void* stream) {
+  if (M == 0 || N == 0) return (M < 0 || N < 0) ? JQ_ERR_INVALID_ARG : JQ_OK;
+  if (x_bf16 == nullptr || ldx < K) return JQ_ERR_INVALID_ARG;
+  jq_status st = check_linear(M, N, K, group, qw, s_w, bias, y_bf16, jq_workspace_size(M, N, K, group, 1),
+                              workspace, workspace_bytes);
+  if (st != JQ_OK) return st;
+  if (!aligned16(x_bf16) || (ldx * 2) % 16 != 0) return JQ_ERR_MISALIGNED;
+  const DeviceInfo* d = current_device();
+  if (d == nullptr) return JQ_ERR_UNSUPPORTED;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  uint8_t* a_op = static_cast<uint8_t*>(workspace);
+  float* s_a = reinterpret_cast<float*>(a_op + round_up(static_cast<size_t>(M) * static_cast<size_t>(K), 256));
+  cudaError_t e = jq::launch_quantize_act_operand(x_bf16, M, K, ldx, group, a_op, s_a, s, d->sms);
+  if (e != cudaSuccess) return JQ_ERR_CUDA;
+  jq::GemmProblem p{static_cast<int>(M), static_cast<int>(N), static_cast<int>(K), group, a_op, s_a, qw, s_w, bias,
+                    y_bf16, nullptr, d->status};
+  return from_cuda(jq::launch_w4a4_gemm(p, s, d->sms));
+}
+
+jq_status jq_w4a4_group_partials(const uint8_t* q, const uint8_t* qw, int32_t* acc, int64_t M, int64_t N, int64_t K,
+                                 int32_t group, void* workspace, size_t workspace_bytes, void* stream) {
+  if (M == 0 || N == 0) return (M < 0 || N < 0) ? JQ_ERR_INVALID_ARG : JQ_OK;
+  if (q == nullptr || acc == nullptr) return JQ_ERR_INVALID_ARG;
+  if (M < 0 || N < 0 || N % 8 != 0 || !group_ok(K, group) || qw == nullptr) return JQ_ERR_INVALID_ARG;
+  if (!aligned16(q) || !aligned16(qw) || !aligned16(acc)) return JQ_ERR_MISALIGNED;
+  if (workspace == nullptr || !aligned16(workspace) || workspace_bytes < jq_workspace_size(M, N, K, group, 0))
+    return JQ_ERR_WORKSPACE;
+  const DeviceInfo* d = current_device();
+  if (d == nullptr) return JQ_ERR_UNSUPPORTED;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  uint8_t* a_op = static_cast<uint8_t*>(workspace);
+  cudaError_t e = jq::launch_expand_operand(q, M, K, a_op, s, d->sms);
+  if (e != cudaSuccess) return JQ_ERR_CUDA;
+  // The export path needs scale tensors only for their layout; it never reads their values,
+  // but the weight-scale tensor map must point at valid memory: reuse the packed weights.
+  jq::GemmProblem p{static_cast<int>(M), static_cast<int>(N), static_cast<int>(K), group, a_op, nullptr, qw,
+                    reinterpret_cast<const float*>(qw), nullptr, nullptr, acc, d->status};
+  return from_cuda(jq::launch_w4a4_gemm(p, s, d->sms));
+}
+
+jq_status jq_device_status(void* stream, int32_t reset) {
+  const DeviceInfo* d = current_device();
+  if (d == nullptr) return JQ_ERR_UNSUPPORTED;
+  if (cudaStreamSynchronize(static_cast<cudaStream_t>(stream)) != cudaSuccess) return JQ_ERR_CUDA;
+  uint32_t v = 0;
+  if (cudaMemcpy(&v, d->status, sizeof v, cudaMemcpyDeviceToHost) != cudaSuccess) return JQ_ERR_CUDA;
+  if (reset && v != 0) {
+    const uint32_t zero = 0;
+    if (cudaMemcpy(d->status, &zero, sizeof zero, cudaMemcpyHostToDevice) != cudaSuccess) return JQ_ERR_CUDA;
+  }
+  return v == 0 ? JQ_OK : JQ_ERR_TIMEOUT;
+}
+
+}  // extern "C"

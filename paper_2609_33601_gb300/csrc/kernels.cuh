@@ -1,0 +1,37 @@
+// kernels.cuh -- internal launchers behind the C ABI (no argument checking here; api.cu does it).
+#pragma once
+#include <cstdint>
+#include <cuda.h>
+#include <cuda_runtime.h>
+
+namespace jq {
+
+// bf16 activations [M, ldx] -> packed codes [M, K/2] + scales [M, K/G].
+cudaError_t launch_quantize_act(const void* x, int64_t M, int64_t K, int64_t ldx, int G, uint8_t* q, float* s_a,
+                                cudaStream_t stream, int sms);
+// bf16 activations -> GEMM operand bytes [M, K] + scales [M, K/G] (fused path).
+cudaError_t launch_quantize_act_operand(const void* x, int64_t M, int64_t K, int64_t ldx, int G, uint8_t* op,
+                                        float* s_a, cudaStream_t stream, int sms);
+// fp32 weights [N, K] -> packed codes [N, K/2] + scales [K/G, N].
+cudaError_t launch_pack_weight(const float* w, int64_t N, int64_t K, int G, uint8_t* qw, float* s_w,
+                               cudaStream_t stream, int sms);
+// packed codes [rows, K/2] -> operand bytes [rows, K].
+cudaError_t launch_expand_operand(const uint8_t* packed, int64_t rows, int64_t K, uint8_t* op, cudaStream_t stream,
+                                  int sms);
+
+struct GemmProblem {
+  int M, N, K, G;
+  const uint8_t* a_operand;  // [M, K] operand bytes (workspace)
+  const float* s_a;          // [M, K/G]
+  const uint8_t* qw;         // [N, K/2] packed
+  const float* s_w;          // [K/G, N]
+  const float* bias;         // [N] or nullptr
+  void* y;                   // bf16 [M, N] (or nullptr when exporting partials)
+  int32_t* partials;         // int32 [M, N, K/G] or nullptr
+  uint32_t* status;          // device status word
+};
+
+// Encodes the tensor maps and launches the persistent tcgen05 GEMM.
+cudaError_t launch_w4a4_gemm(const GemmProblem& p, cudaStream_t stream, int sms);
+
+}  // namespace jq

@@ -1,0 +1,247 @@
+// quantize.cu -- symmetric INT4 quantisers (activations and weights) and the conversion of
+// packed codes into the GEMM's E4M3 operand bytes.
+//
+// Rule (per row and per run of G consecutive K elements; group64 / group128 as the paper fixes
+// them in Sec. 4.2 "FLUX" and the Appendix experimental-detail tables, G = K for per-token):
+//     amax = max|x|,  s = fl32(amax / 7),  q = clamp(rint(fl32(x / s)), -8, 7),  s = q = 0 if amax = 0.
+//
+// Exact division without a division per element: with r = RN(1/s) (one correctly rounded
+// reciprocal per group) and y = RN(x * r), |y - x/s| < 2^-20 and |fl(x/s) - x/s| < 2^-21 for
+// |x/s| <= 7.5, so rint(y) == rint(fl(x/s)) unless y lies within 2^-19 of a half-integer.
+// Those rare elements (and groups whose scale is subnormal, where 1/s may overflow) take the
+// IEEE division __fdiv_rn.  rint(y) itself comes from one fp32 add of 1.5*2^23 + 8: the sum is
+// an integer 0x4B400008 + rint(y) whose low nibble is the offset code q + 8.
+#include <cstdint>
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+
+#include "kernels.cuh"
+#include "operand.cuh"
+
+namespace jq {
+
+namespace {
+
+constexpr float kRintMagic = 12582920.0f;  // 1.5 * 2^23 + 8
+constexpr float kHalfGuard = 0.5f - 0x1p-19f;
+
+// Loads 32 consecutive values of a row as fp32.
+__device__ __forceinline__ void load32(const __nv_bfloat16* p, float (&x)[32]) {
+  const uint4* v = reinterpret_cast<const uint4*>(p);
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const uint4 u = __ldg(v + i);
+    const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      x[8 * i + 2 * j] = __uint_as_float(w[j] << 16);
+      x[8 * i + 2 * j + 1] = __uint_as_float(w[j] & 0xFFFF0000u);
+    }
+  }
+}
+__device__ __forceinline__ void load32(const float* p, float (&x)[32]) {
+  const float4* v = reinterpret_cast<const float4*>(p);
+#pragma unroll
+  for (int i = 0; i < 8; ++i) {
+    const float4 u = __ldg(v + i);
+    x[4 * i] = u.x;
+    x[4 * i + 1] = u.y;
+    x[4 * i + 2] = u.z;
+    x[4 * i + 3] = u.w;
+  }
+}
+
+__device__ __forceinline__ float amax32(const float (&x)[32]) {
+  float m = 0.0f;
+#pragma unroll
+  for (int i = 0; i < 32; ++i) m = fmaxf(m, fabsf(x[i]));
+  return m;
+}
+
+// One code as its offset nibble u = q + 8 in [0, 15].
+__device__ __forceinline__ uint32_t code_offset(float x, float s, float r, bool exact_only) {
+  const float y = x * r;
+  const float t = y + kRintMagic;
+  const float d = y - (t - kRintMagic);
+  if (exact_only || fabsf(d) > kHalfGuard) {
+    float q = rintf(__fdiv_rn(x, s));
+    q = fminf(fmaxf(q, -8.0f), 7.0f);
+    return static_cast<uint32_t>(static_cast<int>(q) + 8);
+  }
+  return __float_as_uint(t) & 0xFu;
+}
+
+// 32 values of one group (scale s) -> 4 words of packed two's complement nibbles.
+__device__ __forceinline__ void quantize32(const float (&x)[32], float s, uint32_t (&pk)[4]) {
+  if (s == 0.0f) {
+#pragma unroll
+    for (int i = 0; i < 4; ++i) pk[i] = 0u;
+    return;
+  }
+  const bool exact_only = !(s >= 0x1p-126f);  // subnormal scale: 1/s may not be representable
+  const float r = __frcp_rn(s);
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    uint32_t w = 0;
+#pragma unroll
+    for (int j = 0; j < 8; ++j) w |= code_offset(x[8 * i + j], s, r, exact_only) << (4 * j);
+    pk[i] = w ^ 0x88888888u;  // offset (q + 8) -> two's complement nibble
+  }
+}
+
+template <bool kOperand>
+__device__ __forceinline__ void store32(uint8_t* out_row, int64_t col, const uint32_t (&pk)[4]) {
+  const uint4 p = make_uint4(pk[0], pk[1], pk[2], pk[3]);
+  if constexpr (kOperand) {
+    uint4 lo, hi;
+    nib32_to_operand(p, lo, hi);
+    uint4* dst = reinterpret_cast<uint4*>(out_row + col);
+    dst[0] = lo;
+    dst[1] = hi;
+  } else {
+    *reinterpret_cast<uint4*>(out_row + col / 2) = p;
+  }
+}
+
+// G = 32 * L (L = 2 or 4): each thread quantises 32 consecutive elements; the L threads of a
+// group are adjacent lanes and reduce amax with xor-shuffles.
+template <typename In, int L, bool kOperand, bool kScaleT>
+__global__ void __launch_bounds__(256) quantize_groups_kernel(const In* __restrict__ x, int64_t M, int64_t K,
+                                                              int64_t ldx, uint8_t* __restrict__ out,
+                                                              float* __restrict__ scales) {
+  const int64_t chunks_per_row = K / 32;
+  const int64_t total = M * chunks_per_row;
+  const int64_t ng = K / (32 * L);
+  const int64_t out_ld = kOperand ? K : K / 2;
+  for (int64_t c = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; c - (threadIdx.x & 31) < total;
+       c += (int64_t)gridDim.x * blockDim.x) {
+    const bool valid = c < total;
+    const int64_t row = valid ? c / chunks_per_row : 0;
+    const int64_t col = valid ? (c % chunks_per_row) * 32 : 0;
+    float v[32];
+    if (valid) {
+      load32(x + row * ldx + col, v);
+    } else {
+#pragma unroll
+      for (int i = 0; i < 32; ++i) v[i] = 0.0f;
+    }
+    float a = amax32(v);
+#pragma unroll
+    for (int o = 1; o < L; o <<= 1) a = fmaxf(a, __shfl_xor_sync(0xFFFFFFFFu, a, o));
+    const float s = __fdiv_rn(a, 7.0f);
+    if (valid) {
+      uint32_t pk[4];
+      quantize32(v, s, pk);
+      store32<kOperand>(out + row * out_ld, col, pk);
+      if ((threadIdx.x & (L - 1)) == 0) {
+        const int64_t g = col / (32 * L);
+        if constexpr (kScaleT) scales[g * M + row] = s;
+        else scales[row * ng + g] = s;
+      }
+    }
+  }
+}
+
+// G = K: one block per row; pass 1 reduces the row amax, pass 2 quantises (the second read
+// of the row hits L1/L2).
+template <typename In, bool kOperand, bool kScaleT>
+__global__ void __launch_bounds__(128) quantize_rows_kernel(const In* __restrict__ x, int64_t M, int64_t K,
+                                                            int64_t ldx, uint8_t* __restrict__ out,
+                                                            float* __restrict__ scales) {
+  __shared__ float red[4];
+  const int64_t out_ld = kOperand ? K : K / 2;
+  for (int64_t row = blockIdx.x; row < M; row += gridDim.x) {
+    const In* xr = x + row * ldx;
+    float a = 0.0f;
+    for (int64_t col = threadIdx.x * 32; col < K; col += 32 * blockDim.x) {
+      float v[32];
+      load32(xr + col, v);
+      a = fmaxf(a, amax32(v));
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) a = fmaxf(a, __shfl_xor_sync(0xFFFFFFFFu, a, o));
+    if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = a;
+    __syncthreads();
+    a = fmaxf(fmaxf(red[0], red[1]), fmaxf(red[2], red[3]));
+    __syncthreads();
+    const float s = __fdiv_rn(a, 7.0f);
+    for (int64_t col = threadIdx.x * 32; col < K; col += 32 * blockDim.x) {
+      float v[32];
+      load32(xr + col, v);
+      uint32_t pk[4];
+      quantize32(v, s, pk);
+      store32<kOperand>(out + row * out_ld, col, pk);
+    }
+    if (threadIdx.x == 0) {
+      if constexpr (kScaleT) scales[row] = s;  // [1, M]
+      else scales[row] = s;                    // [M, 1]
+    }
+  }
+}
+
+// Packed codes [rows, K/2] -> operand bytes [rows, K] (16 bytes in, 32 bytes out per thread).
+__global__ void __launch_bounds__(256) expand_operand_kernel(const uint8_t* __restrict__ packed,
+                                                             int64_t chunks, uint8_t* __restrict__ op) {
+  for (int64_t c = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; c < chunks; c += (int64_t)gridDim.x * blockDim.x) {
+    const uint4 p = __ldg(reinterpret_cast<const uint4*>(packed) + c);
+    uint4 lo, hi;
+    nib32_to_operand(p, lo, hi);
+    uint4* dst = reinterpret_cast<uint4*>(op) + 2 * c;
+    dst[0] = lo;
+    dst[1] = hi;
+  }
+}
+
+int grid_for(int64_t work_items, int threads, int sms) {
+  int64_t blocks = (work_items + threads - 1) / threads;
+  const int64_t cap = static_cast<int64_t>(sms) * 8;
+  if (blocks > cap) blocks = cap;
+  if (blocks < 1) blocks = 1;
+  return static_cast<int>(blocks);
+}
+
+template <typename In, bool kOperand, bool kScaleT>
+cudaError_t launch_quantize(const In* x, int64_t M, int64_t K, int64_t ldx, int G, uint8_t* out, float* scales,
+                            cudaStream_t stream, int sms) {
+  if (M == 0) return cudaSuccess;
+  if (G == K) {
+    int blocks = static_cast<int>(M < static_cast<int64_t>(sms) * 16 ? M : static_cast<int64_t>(sms) * 16);
+    quantize_rows_kernel<In, kOperand, kScaleT><<<blocks, 128, 0, stream>>>(x, M, K, ldx, out, scales);
+  } else if (G == 64) {
+    quantize_groups_kernel<In, 2, kOperand, kScaleT>
+        <<<grid_for(M * (K / 32), 256, sms), 256, 0, stream>>>(x, M, K, ldx, out, scales);
+  } else {
+    quantize_groups_kernel<In, 4, kOperand, kScaleT>
+        <<<grid_for(M * (K / 32), 256, sms), 256, 0, stream>>>(x, M, K, ldx, out, scales);
+  }
+  return cudaGetLastError();
+}
+
+}  // namespace
+
+cudaError_t launch_quantize_act(const void* x, int64_t M, int64_t K, int64_t ldx, int G, uint8_t* q, float* s_a,
+                                cudaStream_t stream, int sms) {
+  return launch_quantize<__nv_bfloat16, false, false>(static_cast<const __nv_bfloat16*>(x), M, K, ldx, G, q, s_a,
+                                                      stream, sms);
+}
+
+cudaError_t launch_quantize_act_operand(const void* x, int64_t M, int64_t K, int64_t ldx, int G, uint8_t* op,
+                                        float* s_a, cudaStream_t stream, int sms) {
+  return launch_quantize<__nv_bfloat16, true, false>(static_cast<const __nv_bfloat16*>(x), M, K, ldx, G, op, s_a,
+                                                     stream, sms);
+}
+
+cudaError_t launch_pack_weight(const float* w, int64_t N, int64_t K, int G, uint8_t* qw, float* s_w,
+                               cudaStream_t stream, int sms) {
+  return launch_quantize<float, false, true>(w, N, K, K, G, qw, s_w, stream, sms);
+}
+
+cudaError_t launch_expand_operand(const uint8_t* packed, int64_t rows, int64_t K, uint8_t* op, cudaStream_t stream,
+                                  int sms) {
+  const int64_t chunks = rows * (K / 32);
+  if (chunks == 0) return cudaSuccess;
+  expand_operand_kernel<<<grid_for(chunks, 256, sms), 256, 0, stream>>>(packed, chunks, op);
+  return cudaGetLastError();
+}
+
+}  // namespace jq

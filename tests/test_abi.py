@@ -1,0 +1,113 @@
+"""Host-side checks of the C ABI (no GPU needed): the library builds and loads, exports every
+entry point include/jq.h declares, and rejects bad arguments synchronously, before touching a
+device, with the documented status codes."""
+import ctypes
+import os
+import re
+
+import pytest
+import torch
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "jq.h")
+
+OK, INVALID, MISALIGNED, UNSUPPORTED, CUDA, TIMEOUT, WORKSPACE = range(7)
+
+
+@pytest.fixture(scope="module")
+def lib():
+    from paper_2609_33601_gb300 import build
+    path = build.build()
+    return ctypes.CDLL(path)
+
+
+def declared_functions():
+    text = open(HEADER).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(jq_[a-z0-9_]+)\s*\(", text)))
+
+
+def test_header_declares_the_boundary():
+    names = declared_functions()
+    for need in ("jq_quantize_act", "jq_pack_weight", "jq_w4a4_linear", "jq_fused_quant_linear",
+                 "jq_status_string", "jq_workspace_size", "jq_w4a4_group_partials", "jq_device_status"):
+        assert need in names
+
+
+def test_library_exports_every_declared_symbol(lib):
+    for name in declared_functions():
+        assert hasattr(lib, name), name
+
+
+def test_status_strings(lib):
+    lib.jq_status_string.restype = ctypes.c_char_p
+    lib.jq_status_string.argtypes = [ctypes.c_int]
+    names = [lib.jq_status_string(i).decode() for i in range(7)]
+    assert names == ["JQ_OK", "JQ_ERR_INVALID_ARG", "JQ_ERR_MISALIGNED", "JQ_ERR_UNSUPPORTED", "JQ_ERR_CUDA",
+                     "JQ_ERR_TIMEOUT", "JQ_ERR_WORKSPACE"]
+
+
+def test_workspace_size(lib):
+    f = lib.jq_workspace_size
+    f.argtypes = [ctypes.c_int64] * 3 + [ctypes.c_int32] * 2
+    f.restype = ctypes.c_size_t
+    assert f(1024, 12288, 4096, 128, 0) == 1024 * 4096
+    assert f(1024, 12288, 4096, 128, 1) == 1024 * 4096 + 1024 * 32 * 4
+    assert f(3, 8, 256, 64, 0) == 768  # rounded up to 256
+    assert f(0, 8, 256, 64, 0) == 0
+
+
+def _fake(addr):
+    return ctypes.c_void_p(addr)
+
+
+def test_argument_checks_reject_before_launch(lib):
+    i64, i32, vp, sz = ctypes.c_int64, ctypes.c_int32, ctypes.c_void_p, ctypes.c_size_t
+    lib.jq_quantize_act.argtypes = [vp, i64, i64, i64, i32, vp, vp, vp]
+    lib.jq_pack_weight.argtypes = [vp, i64, i64, i32, vp, vp, vp]
+    lib.jq_w4a4_linear.argtypes = [vp, vp, vp, vp, vp, vp, i64, i64, i64, i32, vp, sz, vp]
+    lib.jq_fused_quant_linear.argtypes = [vp, i64, vp, vp, vp, vp, i64, i64, i64, i32, vp, sz, vp]
+    A = _fake(0x10000)       # 16-byte aligned fake device addresses: never dereferenced here
+    odd = _fake(0x10008)
+    q = lib.jq_quantize_act
+    assert q(None, 4, 256, 256, 64, A, A, None) == INVALID
+    assert q(A, 4, 256, 256, 32, A, A, None) == INVALID          # unsupported group
+    assert q(A, 4, 192, 192, 64, A, A, None) == INVALID          # K % 128 != 0
+    assert q(A, 4, 256, 128, 64, A, A, None) == INVALID          # ldx < K
+    assert q(A, -1, 256, 256, 64, A, A, None) == INVALID
+    assert q(A, 0, 256, 256, 64, None, None, None) == OK         # M == 0 is a no-op
+    assert q(odd, 4, 256, 256, 64, A, A, None) == MISALIGNED
+    assert q(A, 4, 256, 260, 64, A, A, None) == MISALIGNED       # row pitch 520 B
+    assert q(A, 4, 262144, 262144, 262144, A, A, None) == INVALID  # K too large for exact sums
+    p = lib.jq_pack_weight
+    assert p(None, 8, 256, 64, A, A, None) == INVALID
+    assert p(A, 8, 256, 100, A, A, None) == INVALID
+    assert p(A, 8, 256, 64, odd, A, None) == MISALIGNED
+    L = lib.jq_w4a4_linear
+    big = 1 << 30
+    assert L(A, A, A, A, None, A, 4, 12, 256, 64, A, big, None) == INVALID     # N % 8
+    assert L(A, A, A, A, None, A, 4, 16, 256, 96, A, big, None) == INVALID     # group
+    assert L(None, A, A, A, None, A, 4, 16, 256, 64, A, big, None) == INVALID
+    assert L(A, A, A, A, odd, A, 4, 16, 256, 64, A, big, None) == MISALIGNED   # bias
+    assert L(A, A, A, A, None, A, 4, 16, 256, 64, None, big, None) == WORKSPACE
+    assert L(A, A, A, A, None, A, 4, 16, 256, 64, A, 16, None) == WORKSPACE
+    assert L(A, A, A, A, None, A, 0, 16, 256, 64, None, 0, None) == OK        # M == 0
+    F = lib.jq_fused_quant_linear
+    assert F(A, 200, A, A, None, A, 4, 16, 256, 64, A, big, None) == INVALID   # ldx < K
+    assert F(A, 260, A, A, None, A, 4, 16, 256, 64, A, big, None) == MISALIGNED
+    assert F(A, 256, A, A, None, A, 4, 16, 256, 64, A, 1024, None) == WORKSPACE
+
+
+@pytest.mark.skipif(torch.cuda.is_available(), reason="checks the no-device path; a GPU is present")
+def test_valid_arguments_without_a_device_report_unsupported(lib):
+    i64, i32, vp = ctypes.c_int64, ctypes.c_int32, ctypes.c_void_p
+    lib.jq_quantize_act.argtypes = [vp, i64, i64, i64, i32, vp, vp, vp]
+    A = _fake(0x10000)
+    assert lib.jq_quantize_act(A, 4, 256, 256, 64, A, A, None) == UNSUPPORTED
+
+
+def test_binding_fails_loudly_without_cuda_tensors():
+    import paper_2609_33601_gb300 as jq
+    x = torch.zeros((4, 256), dtype=torch.bfloat16)
+    with pytest.raises(ValueError):
+        jq.jq_quantize_act(x, 64)
