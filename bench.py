@@ -1,0 +1,348 @@
+"""Benchmark of the naive W4A4 linear layer (JustQuant, arxiv 2609.33601) on GB300.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--workload dllm] [--impl ours|reference]
+
+One step = one pass of the deployed hot path over one batch: the activation quantiser
+(jq_quantize_act) followed by the W4A4 GEMM with its dequantise + bias epilogue
+(jq_w4a4_linear), on the dLLM gate/up projection (M=1024 tokens x K=4096 -> N=12288,
+group128).  Weights are packed once, offline, as the paper's deployment does.  Six input/weight
+sets (about 200 MB, more than the 129 MB L2) rotate between steps, so every step streams its
+operands from HBM.  Metric: W4A4 linear TOPS (2*M*N*K per step), whole job over all ranks.
+
+Under torchrun each rank runs its own replica of the workload (the layer shards along tokens
+with no exchange), so scaling is weak and no collective sits on the data path; a barrier and a
+max-reduction of the timings bracket the timed region.
+
+--impl reference times the CPU oracle (oracle/, the plain C reference of the same layer) on
+the host cores, on a bounded row sample of the same workload.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+WORKLOADS = {
+    # name: (description, M, K, N, G, bias)
+    "dllm": ("dLLM 8B gate/up projection: M=1024 tokens x K=4096 -> N=12288, group128", 1024, 4096, 12288, 128),
+    "flux_qkv": ("FLUX 12B DiT fused QKV+MLP-in: M=4608 x K=3072 -> N=21504, group64", 4608, 3072, 21504, 64),
+    "flux_out": ("FLUX 12B DiT output projection: M=4608 x K=15360 -> N=3072, group64", 4608, 15360, 3072, 64),
+}
+PEAKS_PATH = os.path.join(ROOT, "MEASURED_PEAKS.json")
+FP8_PER_BF16 = 2.0  # nominal dense FP8 / BF16 tensor-core ratio on GB300 (4.5 / 2.25 PFLOP/s)
+
+# DRAM traffic of one GEMM launch (dram__bytes_read.sum + dram__bytes_write.sum) from the ncu
+# capture summarised in profiles/, keyed by the hash of the kernel source it was taken on; once
+# the kernel changes the figure no longer applies and the bench reports null.
+GEMM_TRAFFIC = {
+    ("dllm", "d598a837a9b8975a"): 31.25e6 + 0.15e6,  # profiles/w4a4_gemm_dllm_full.md
+}
+
+
+def kernel_hash() -> str:
+    h = hashlib.sha256()
+    for f in ("gemm.cu", "operand.cuh", "ptx.cuh"):
+        with open(os.path.join(ROOT, "paper_2609_33601_gb300", "csrc", f), "rb") as fh:
+            h.update(fh.read())
+    return h.hexdigest()[:16]
+
+
+def dist_env():
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return rank, world, local
+
+
+class ClockSampler:
+    """Samples SM clocks and throttle reasons with nvidia-smi while the timed region runs."""
+
+    QUERY = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+             "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+             "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.samples = []
+        self._stop = threading.Event()
+        self._thread = None
+
+    def _run(self):
+        while not self._stop.is_set():
+            try:
+                out = subprocess.run(["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.QUERY}",
+                                      "--format=csv,noheader,nounits"], capture_output=True, text=True, timeout=5)
+                if out.returncode == 0 and out.stdout.strip():
+                    self.samples.append([v.strip() for v in out.stdout.strip().split(",")])
+            except Exception:
+                return
+            self._stop.wait(0.2)
+
+    def __enter__(self):
+        self._thread = threading.Thread(target=self._run, daemon=True)
+        self._thread.start()
+        return self
+
+    def __exit__(self, *exc):
+        self._stop.set()
+        if self._thread:
+            self._thread.join(timeout=10)
+
+    def summary(self):
+        if not self.samples:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unsampled"]}
+        sm = [float(s[1]) for s in self.samples if s[1].replace(".", "").isdigit()]
+        mx = [float(s[2]) for s in self.samples if s[2].replace(".", "").isdigit()]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({n for s in self.samples for n, v in zip(names, s[5:9]) if v.lower() == "active"})
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(mx) if mx else None,
+                "reasons": reasons, "samples": len(self.samples)}
+
+
+def measured_peaks():
+    try:
+        with open(PEAKS_PATH) as f:
+            p = json.load(f)
+        return float(p["bf16_tflops"]), float(p["hbm_gbs"]), "measured"
+    except Exception:
+        return 1900.0, 6800.0, "fallback"
+
+
+# ----------------------------------------------------------------------------- reference arm
+
+class OracleSample:
+    """The CPU oracle, as it stands, on a bounded row sample of the workload: quantise the
+    sampled activation rows and evaluate the linear layer for them (the weights are packed
+    once, outside the timing, as on the GPU)."""
+
+    def __init__(self, name: str, seed: int = 7):
+        import oracle
+        from paper_2609_33601_gb300 import workloads as wl
+        self.oracle = oracle
+        self.name = name
+        self.desc, self.M, self.K, self.N, self.G = WORKLOADS[name]
+        w = wl.make(name, seed=seed)
+        self.x_bits, self.bias = w.x_bits, w.bias
+        self.qw, self.sw = oracle.quantize_f32(w.w, self.G)
+        self.rows = 8
+
+    def run(self, rows: int) -> float:
+        t0 = time.perf_counter()
+        qa, sa = self.oracle.quantize_bf16(self.x_bits[:rows], self.G)
+        self.oracle.linear(qa, sa, self.qw, self.sw, self.bias, self.G)
+        return time.perf_counter() - t0
+
+    def calibrate(self, target_s: float) -> int:
+        rows = 8
+        while True:
+            dt = self.run(rows)
+            if dt >= 0.8 * target_s or rows >= self.M:
+                break
+            rows = min(self.M, max(rows * 2, int(rows * target_s / max(dt, 1e-3))))
+        self.rows = rows
+        return rows
+
+    def ops(self) -> float:
+        return 2.0 * self.rows * self.N * self.K
+
+    def describe(self, dt: float) -> dict:
+        cores = int(os.environ.get("OMP_NUM_THREADS", os.cpu_count() or 1))
+        return {"value": self.ops() / dt / 1e12, "unit": "TOPS", "cores": min(cores, self.rows), "kind": "oracle",
+                "sample": f"{self.rows} of {self.M} token rows of the {self.name} workload (all N={self.N} "
+                          f"outputs), quantise + linear, {dt:.2f} s per sample"}
+
+
+def run_reference(args):
+    rank, world, _ = dist_env()
+    if rank != 0:
+        return 0
+    o = OracleSample(args.workload)
+    per_step = min(args.ref_seconds, 120.0 / (args.steps + args.warmup))
+    o.calibrate(per_step)
+    for _ in range(args.warmup):
+        o.run(o.rows)
+    times = [o.run(o.rows) for _ in range(args.steps)]
+    mean = sum(times) / len(times)
+    cb = o.describe(mean)
+    value = cb["value"]
+    line = {"impl": "reference", "metric": "W4A4 linear TOPS", "value": value, "unit": "TOPS", "n_gpus": args.gpus,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": mean * 1e3, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "int4", "data": "synthetic",
+            "config": {"workload": o.desc, "M": o.M, "K": o.K, "N": o.N, "group": o.G},
+            "cpu_baseline": cb, "e2e": {"value": value, "unit": "TOPS", "h2d_bytes_per_step": 0,
+                                        "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+# ----------------------------------------------------------------------------- our arm
+
+def run_ours(args):
+    import torch
+
+    rank, world, local = dist_env()
+    torch.cuda.set_device(local)
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    from paper_2609_33601_gb300 import build as jq_build
+    jq_build.build()
+    import paper_2609_33601_gb300 as jq
+    from paper_2609_33601_gb300 import workloads as wl
+
+    desc, M, K, N, G = WORKLOADS[args.workload]
+    dev = torch.device("cuda", local)
+    sets = []
+    n_sets = args.sets
+    for i in range(n_sets):
+        w = wl.make(args.workload, seed=100 + 17 * rank + i)
+        x = torch.from_numpy(w.x_bits.view(np.int16)).to(dev).view(torch.bfloat16)
+        qw, sw = jq.jq_pack_weight(torch.from_numpy(w.w).to(dev), G)
+        b = None if w.bias is None else torch.from_numpy(w.bias).to(dev)
+        sets.append((x, qw, sw, b))
+        del w
+    torch.cuda.synchronize()
+    q = torch.empty((M, K // 2), dtype=torch.uint8, device=dev)
+    s_a = torch.empty((M, K // G), dtype=torch.float32, device=dev)
+    y = torch.empty((M, N), dtype=torch.bfloat16, device=dev)
+    ws = torch.empty(jq.jq_workspace_size(M, N, K, G, False), dtype=torch.uint8, device=dev)
+    stream = torch.cuda.current_stream()
+
+    def step(i, ev=None):
+        x, qw, sw, b = sets[i % n_sets]
+        jq.jq_quantize_act(x, G, q, s_a, stream=stream)
+        if ev is not None:
+            ev[0].record(stream)
+        jq.jq_w4a4_linear(q, s_a, qw, sw, b, G, y=y, workspace=ws, stream=stream)
+        if ev is not None:
+            ev[1].record(stream)
+
+    def barrier():
+        if world > 1:
+            import torch.distributed as dist
+            dist.barrier()
+
+    for i in range(args.warmup):
+        step(i)
+    torch.cuda.synchronize()
+    assert jq.jq_device_status() == 0, "a kernel reported a bounded-wait timeout"
+
+    gemm_ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
+    t_start, t_end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    barrier()
+    torch.cuda.synchronize()
+    with ClockSampler(local) as clocks:
+        t_start.record(stream)
+        for i in range(args.steps):
+            step(i, gemm_ev[i])
+        t_end.record(stream)
+        torch.cuda.synchronize()
+    barrier()
+    total_ms = t_start.elapsed_time(t_end)
+    gemm_ms = sum(a.elapsed_time(b) for a, b in gemm_ev) / args.steps
+    if world > 1:
+        import torch.distributed as dist
+        t = torch.tensor([total_ms, gemm_ms], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        total_ms, gemm_ms = float(t[0]), float(t[1])
+    assert jq.jq_device_status() == 0, "a kernel reported a bounded-wait timeout"
+
+    # end to end through the public API: pinned host activations in, host result out
+    x_host = [sets[i][0].cpu().pin_memory() for i in range(min(2, n_sets))]
+    y_host = torch.empty((M, N), dtype=torch.bfloat16).pin_memory()
+    x_dev = torch.empty((M, K), dtype=torch.bfloat16, device=dev)
+
+    def e2e_step(i):
+        x_dev.copy_(x_host[i % len(x_host)], non_blocking=True)
+        _, qw, sw, b = sets[i % n_sets]
+        jq.jq_quantize_act(x_dev, G, q, s_a, stream=stream)
+        jq.jq_w4a4_linear(q, s_a, qw, sw, b, G, y=y, workspace=ws, stream=stream)
+        y_host.copy_(y, non_blocking=True)
+
+    for i in range(args.warmup):
+        e2e_step(i)
+    torch.cuda.synchronize()
+    barrier()
+    e0 = time.perf_counter()
+    for i in range(args.steps):
+        e2e_step(i)
+    torch.cuda.synchronize()
+    e2e_s = time.perf_counter() - e0
+    if world > 1:
+        import torch.distributed as dist
+        t = torch.tensor([e2e_s], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        e2e_s = float(t[0])
+
+    ops_step = 2.0 * M * N * K
+    value = world * ops_step * args.steps / (total_ms * 1e-3) / 1e12
+    e2e_value = world * ops_step * args.steps / e2e_s / 1e12
+    bf16_peak, _, peak_src = measured_peaks()
+    fp8_peak = bf16_peak * FP8_PER_BF16
+    achieved = ops_step / (gemm_ms * 1e-3) / 1e12
+    traffic = GEMM_TRAFFIC.get((args.workload, kernel_hash()))
+
+    if rank != 0:
+        if world > 1:
+            import torch.distributed as dist
+            dist.destroy_process_group()
+        return 0
+    cpu = None
+    if world == 1 and not args.no_cpu_baseline:
+        o = OracleSample(args.workload)
+        o.calibrate(args.ref_seconds)
+        cpu = o.describe(o.run(o.rows))
+    line = {
+        "metric": "W4A4 linear TOPS", "value": value, "unit": "TOPS", "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": total_ms / args.steps, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "int4", "data": "synthetic",
+        "config": {"workload": desc, "M": M, "K": K, "N": N, "group": G,
+                   "step": "jq_quantize_act + jq_w4a4_linear", "parallelism": f"replicas x{world}",
+                   "l2": f"{n_sets} rotating input/weight sets larger than L2"},
+        "roofline": {"bound": "tensor", "achieved": achieved, "peak": fp8_peak, "unit": "TFLOP/s",
+                     "frac": achieved / fp8_peak, "traffic": traffic,
+                     "kernel": "jq_w4a4_linear (operand expansion + tcgen05 GEMM), CUDA events per launch",
+                     "peak_source": f"{peak_src} bf16 {bf16_peak} TFLOP/s x nominal FP8/BF16 ratio {FP8_PER_BF16}"},
+        "cpu_baseline": cpu,
+        "e2e": {"value": e2e_value, "unit": "TOPS", "h2d_bytes_per_step": M * K * 2, "d2h_bytes_per_step": M * N * 2},
+        "gpu_launches": 3 * args.steps,
+        "clocks": clocks.summary(),
+    }
+    print(json.dumps(line), flush=True)
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+    return 0
+
+
+def main():
+    ap = argparse.ArgumentParser(description=__doc__.splitlines()[0])
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=50)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--workload", choices=sorted(WORKLOADS), default="dllm")
+    ap.add_argument("--sets", type=int, default=6, help="rotating input/weight sets (working set > L2)")
+    ap.add_argument("--ref-seconds", type=float, default=10.0, help="CPU seconds per oracle sample")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    if args.warmup < 3:
+        ap.error("--warmup must be at least 3")
+    if args.impl == "reference":
+        return run_reference(args)
+    return run_ours(args)
+
+
+if __name__ == "__main__":
+    sys.exit(main())
