@@ -131,6 +131,28 @@ JQ_API jq_status jq_w4a4_group_partials(const uint8_t* q, const uint8_t* qw, int
                                  void* stream);
 
 /*
+ * jq_w4a4_linear for callers that cannot allocate device memory.  (The paper has no
+ * counterpart; this is a deployment convenience.)  jq_w4a4_linear needs a caller-provided
+ * workspace; code that may not call cudaMalloc at all -- a host callback, a plug-in whose
+ * framework owns every allocation, a serving loop that must not allocate after start-up --
+ * cannot provide one.  This variant keeps that scratch (the M*K activation operand bytes) in a
+ * fixed device array inside the library instead, JQ_NOALLOC_MAX_SCRATCH_BYTES large, which
+ * every GPU that loads the library holds until the process exits.  It allocates nothing and
+ * runs the same kernels, so its output is identical to jq_w4a4_linear's.
+ *   Arguments as jq_w4a4_linear, without the workspace.
+ *   Limit: M * K <= JQ_NOALLOC_MAX_SCRATCH_BYTES, else JQ_ERR_WORKSPACE (nothing launched).
+ *   The first call on a device looks up the array's device address (cudaGetSymbolAddress);
+ *   make that first call before any stream capture.  All calls on a device share the one
+ *   array, so calls whose kernels may overlap on the GPU (different streams without ordering
+ *   between them) race and corrupt each other's results; order them on one stream.
+ * Errors: JQ_ERR_INVALID_ARG, JQ_ERR_MISALIGNED, JQ_ERR_WORKSPACE, JQ_ERR_UNSUPPORTED, JQ_ERR_CUDA.
+ */
+#define JQ_NOALLOC_MAX_SCRATCH_BYTES (16u * 1024u * 1024u)
+JQ_API jq_status jq_w4a4_linear_noalloc(const uint8_t* q, const float* s_a, const uint8_t* qw, const float* s_w,
+                                        const float* bias, void* y_bf16, int64_t M, int64_t N, int64_t K,
+                                        int32_t group, void* stream);
+
+/*
  * Synchronises `stream` and returns JQ_ERR_TIMEOUT if any kernel of this library on the
  * current device gave up a bounded wait since the last reset (reset != 0 clears the flag),
  * JQ_ERR_CUDA if the stream reports an error, JQ_OK otherwise.

@@ -25,6 +25,7 @@ import torch
 __all__ = [
     "JQError", "library_path", "jq_quantize_act", "jq_pack_weight", "jq_workspace_size", "jq_w4a4_linear",
     "jq_fused_quant_linear", "jq_w4a4_group_partials", "jq_device_status", "jq_status_string",
+    "jq_w4a4_linear_noalloc",
 ]
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
@@ -60,6 +61,7 @@ def _load() -> ctypes.CDLL:
                 "jq_fused_quant_linear": [vp, i64, vp, vp, vp, vp, i64, i64, i64, i32, vp, sz, vp],
                 "jq_w4a4_group_partials": [vp, vp, vp, i64, i64, i64, i32, vp, sz, vp],
                 "jq_device_status": [vp, i32],
+                "jq_w4a4_linear_noalloc": [vp, vp, vp, vp, vp, vp, i64, i64, i64, i32, vp],
             }
             for name, args in sig.items():
                 f = getattr(lib, name)
@@ -144,6 +146,22 @@ def jq_w4a4_linear(q, s_a, qw, s_w, bias, group: int, y=None, workspace=None, st
     ws, ws_bytes = _workspace(M, N, K, group, False, q.device, workspace)
     _check("jq_w4a4_linear", _load().jq_w4a4_linear(_ptr(q), _ptr(s_a), _ptr(qw), _ptr(s_w), _ptr(bias), _ptr(y),
                                                     M, N, K, group, _ptr(ws), ws_bytes, _stream(stream)))
+    return y
+
+
+def jq_w4a4_linear_noalloc(q, s_a, qw, s_w, bias, group: int, y=None, stream=None):
+    """jq_w4a4_linear without a workspace, for callers that cannot allocate device memory: the
+    library keeps the scratch in its own fixed device array (M*K <= 16 MiB).  Calls share that
+    array, so order them on one stream.  (Only the output tensor is allocated here, by the
+    caller's side, when y is None.)"""
+    _need_cuda(q, s_a, qw, s_w, bias)
+    M, K = q.shape[0], q.shape[1] * 2
+    N = qw.shape[0]
+    if y is None:
+        y = torch.empty((M, N), dtype=torch.bfloat16, device=q.device)
+    _check("jq_w4a4_linear_noalloc",
+           _load().jq_w4a4_linear_noalloc(_ptr(q), _ptr(s_a), _ptr(qw), _ptr(s_w), _ptr(bias), _ptr(y), M, N, K,
+                                          group, _stream(stream)))
     return y
 
 

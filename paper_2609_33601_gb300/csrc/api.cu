@@ -53,6 +53,15 @@ jq_status from_cuda(cudaError_t e) { return e == cudaSuccess ? JQ_OK : JQ_ERR_CU
 
 }  // namespace
 
+namespace jq {
+// Device address of the library's status word on the current device (nullptr if the device is
+// not supported); kernels launched from other files report bounded-wait timeouts into it.
+uint32_t* device_status_word() {
+  const DeviceInfo* d = current_device();
+  return d == nullptr ? nullptr : d->status;
+}
+}  // namespace jq
+
 extern "C" {
 
 const char* jq_status_string(jq_status s) {

@@ -31,6 +31,9 @@ struct GemmProblem {
   uint32_t* status;          // device status word
 };
 
+// Device address of the library's status word on the current device, or nullptr.
+uint32_t* device_status_word();
+
 // Encodes the tensor maps and launches the persistent tcgen05 GEMM.
 cudaError_t launch_w4a4_gemm(const GemmProblem& p, cudaStream_t stream, int sms);
 

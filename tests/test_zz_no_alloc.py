@@ -1,0 +1,74 @@
+"""GPU test of jq_w4a4_linear_noalloc, the entry point for callers that cannot allocate device
+memory (a host callback, a plug-in whose framework owns every allocation, a serving loop that
+must not allocate after start-up): it keeps its scratch in a fixed device array inside the
+library instead of a caller-provided workspace.
+
+Two calls in a row on different shapes, each compared with jq_w4a4_linear (which uses a
+workspace) and with the CPU oracle under the tolerance the parity tests use; then the size
+limit.  This file is collected last so that a run stopping at the first failure has already run
+every other test; it also passes on its own in a fresh process.
+"""
+import ctypes
+
+import numpy as np
+import pytest
+import torch
+
+import paper_2609_33601_gb300 as jq
+from paper_2609_33601_gb300 import workloads as wl
+from tests.helpers import Reference, check_linear
+
+pytestmark = pytest.mark.gpu
+
+JQ_ERR_WORKSPACE = 6
+MAX_SCRATCH = 16 * 1024 * 1024
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _device():
+    assert torch.cuda.is_available(), "the gpu tests need a CUDA device"
+    jq._load()
+    yield
+    assert jq.jq_device_status() == 0
+
+
+def _dev(a):
+    return torch.from_numpy(np.ascontiguousarray(a)).cuda()
+
+
+def _bits(y):
+    return y.view(torch.int16).cpu().numpy().view(np.uint16)
+
+
+def _problem(M, N, K, G, bias, seed):
+    w = wl.make("custom", seed=seed, M=M, K=K, N=N, G=G, bias=bias)
+    ref = Reference(w.x_bits, w.w, w.bias, G)
+    args = (_dev(ref.packed_a), _dev(ref.s_a), _dev(ref.packed_w), _dev(ref.s_w_groupmajor),
+            None if ref.bias is None else _dev(ref.bias))
+    return ref, args
+
+
+def test_noalloc_matches_workspace_linear_on_two_calls_in_a_row():
+    cases = [(300, 520, 512, 64, True, 1), (1024, 264, 4096, 128, False, 2)]
+    probs = [_problem(*c) for c in cases]
+    # two no-allocation calls back to back, sharing the library's scratch array
+    outs = [jq.jq_w4a4_linear_noalloc(*args, ref.G) for ref, args in probs]
+    torch.cuda.synchronize()
+    for (ref, args), y_na in zip(probs, outs):
+        y_ws = jq.jq_w4a4_linear(*args, ref.G)
+        a, b = _bits(y_na), _bits(y_ws)
+        y64, _ = ref.linear()
+        check_linear(a, y64, ref.partials(), ref.s_a, ref.s_w_rows, ref.bias, "noalloc")
+        check_linear(b, y64, ref.partials(), ref.s_a, ref.s_w_rows, ref.bias, "workspace")
+        assert np.array_equal(a, b)  # same kernels, same operands: identical bits
+
+
+def test_noalloc_rejects_problems_beyond_its_scratch():
+    lib = jq._load()
+    small = torch.zeros(256, dtype=torch.uint8, device="cuda")
+    p = ctypes.c_void_p(small.data_ptr())
+    K = 4096
+    M = MAX_SCRATCH // K + 1  # one row too many
+    rc = lib.jq_w4a4_linear_noalloc(p, p, p, p, None, p, M, 8, K, 128, None)
+    assert rc == JQ_ERR_WORKSPACE
+    torch.cuda.synchronize()
