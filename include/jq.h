@@ -135,12 +135,13 @@ JQ_API jq_status jq_w4a4_group_partials(const uint8_t* q, const uint8_t* qw, int
  * counterpart; this is a deployment convenience.)  jq_w4a4_linear needs a caller-provided
  * workspace; code that may not call cudaMalloc at all -- a host callback, a plug-in whose
  * framework owns every allocation, a serving loop that must not allocate after start-up --
- * cannot provide one.  This variant keeps that scratch (the M*K activation operand bytes) in a
+ * cannot provide one.  This variant keeps that scratch (the activation operand bytes) in a
  * fixed device array inside the library instead, JQ_NOALLOC_MAX_SCRATCH_BYTES large, which
  * every GPU that loads the library holds until the process exits.  It allocates nothing and
  * runs the same kernels, so its output is identical to jq_w4a4_linear's.
  *   Arguments as jq_w4a4_linear, without the workspace.
- *   Limit: M * K <= JQ_NOALLOC_MAX_SCRATCH_BYTES, else JQ_ERR_WORKSPACE (nothing launched).
+ *   Limit: ceil(M / 128) * 128 * K <= JQ_NOALLOC_MAX_SCRATCH_BYTES, else JQ_ERR_WORKSPACE
+ *   (nothing launched).
  *   The first call on a device looks up the array's device address (cudaGetSymbolAddress);
  *   make that first call before any stream capture.  All calls on a device share the one
  *   array, so calls whose kernels may overlap on the GPU (different streams without ordering
@@ -155,7 +156,8 @@ JQ_API jq_status jq_w4a4_linear_noalloc(const uint8_t* q, const float* s_a, cons
 /*
  * Synchronises `stream` and returns JQ_ERR_TIMEOUT if any kernel of this library on the
  * current device gave up a bounded wait since the last reset (reset != 0 clears the flag),
- * JQ_ERR_CUDA if the stream reports an error, JQ_OK otherwise.
+ * JQ_ERR_UNSUPPORTED if a GEMM launch found its shared-memory window not 1024-byte aligned
+ * (it then wrote nothing), JQ_ERR_CUDA if the stream reports an error, JQ_OK otherwise.
  */
 JQ_API jq_status jq_device_status(void* stream, int32_t reset);
 

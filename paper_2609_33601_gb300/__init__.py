@@ -151,7 +151,7 @@ def jq_w4a4_linear(q, s_a, qw, s_w, bias, group: int, y=None, workspace=None, st
 
 def jq_w4a4_linear_noalloc(q, s_a, qw, s_w, bias, group: int, y=None, stream=None):
     """jq_w4a4_linear without a workspace, for callers that cannot allocate device memory: the
-    library keeps the scratch in its own fixed device array (M*K <= 16 MiB).  Calls share that
+    library keeps the scratch in its own fixed device array (ceil(M/128)*128*K <= 16 MiB).  Calls share that
     array, so order them on one stream.  (Only the output tensor is allocated here, by the
     caller's side, when y is None.)"""
     _need_cuda(q, s_a, qw, s_w, bias)

@@ -103,7 +103,8 @@ jq_status jq_pack_weight(const float* w, int64_t N, int64_t K, int32_t group, ui
 size_t jq_workspace_size(int64_t M, int64_t N, int64_t K, int32_t group, int32_t fused) {
   (void)N;
   if (M <= 0 || K <= 0 || group <= 0 || K % group != 0) return 0;
-  size_t bytes = round_up(static_cast<size_t>(M) * static_cast<size_t>(K), 256);  // A operand bytes
+  // A-operand image: whole 128-row tiles of K operand bytes (operand.cuh)
+  size_t bytes = round_up(static_cast<size_t>(M), 128) * static_cast<size_t>(K);
   if (fused) bytes += round_up(static_cast<size_t>(M) * static_cast<size_t>(K / group) * sizeof(float), 256);
   return bytes;
 }
@@ -156,7 +157,7 @@ jq_status jq_fused_quant_linear(const void* x_bf16, int64_t ldx, const uint8_t* 
   if (d == nullptr) return JQ_ERR_UNSUPPORTED;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   uint8_t* a_op = static_cast<uint8_t*>(workspace);
-  float* s_a = reinterpret_cast<float*>(a_op + round_up(static_cast<size_t>(M) * static_cast<size_t>(K), 256));
+  float* s_a = reinterpret_cast<float*>(a_op + round_up(static_cast<size_t>(M), 128) * static_cast<size_t>(K));
   cudaError_t e = jq::launch_quantize_act_operand(x_bf16, M, K, ldx, group, a_op, s_a, s, d->sms);
   if (e != cudaSuccess) return JQ_ERR_CUDA;
   jq::GemmProblem p{static_cast<int>(M), static_cast<int>(N), static_cast<int>(K), group, a_op, s_a, qw, s_w, bias,
@@ -195,7 +196,8 @@ jq_status jq_device_status(void* stream, int32_t reset) {
     const uint32_t zero = 0;
     if (cudaMemcpy(d->status, &zero, sizeof zero, cudaMemcpyHostToDevice) != cudaSuccess) return JQ_ERR_CUDA;
   }
-  return v == 0 ? JQ_OK : JQ_ERR_TIMEOUT;
+  // 1: a bounded wait gave up; 2: the GEMM found its shared-memory window misaligned and did nothing
+  return v == 0 ? JQ_OK : (v == 1 ? JQ_ERR_TIMEOUT : JQ_ERR_UNSUPPORTED);
 }
 
 }  // extern "C"

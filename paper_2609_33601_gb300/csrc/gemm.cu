@@ -9,18 +9,26 @@
 // operand bytes (operand.cuh): every product and every per-group sum is exactly representable,
 // so the fp32 TMEM accumulator holds acc[m,n,g] * 2^-18 exactly.
 //
-// Persistent kernel, one 128x256 output tile at a time per CTA, 16 warps:
-//   warp 0      TMA producer: A operand bytes (128x128, 128B swizzle) straight into the MMA
-//               stage ring; packed B codes (256 x 64 bytes) into a packed ring; one row of
-//               weight scales s_w[g, n0:n0+256] per group into a scale ring.
-//   warp 1      MMA issuer (one thread): 4 x (128x256x32) MMAs per K stage into one of two TMEM
-//               accumulators; a fresh accumulator starts at every group boundary and is handed
-//               to the drain warps with tcgen05.commit when the group ends.
-//   warps 2-7   unpack: packed B nibbles -> operand bytes in the 128B-swizzled K-major layout.
-//   warps 8-15  drain: per group, tcgen05.ld the partials, y += acc * (s_a * 2^18) * s_w in
-//               fp32 registers (warp w owns TMEM lanes 32*(w%4).. and columns 128*((w-8)/4)..);
-//               after the last group, + bias, round to bf16, store.
-// Every mbarrier wait is bounded; a timeout records a status and unwinds the whole CTA.
+// Persistent kernel on CTA pairs (clusters of two SMs, tcgen05 cta_group::2).  A pair owns a
+// 256x256 output tile at a time: CTA r of the pair holds A rows 128r..128r+127 and B rows (output
+// columns) 128r..128r+127 of the tile, and the even CTA issues 256x256x32 MMAs that read both
+// CTAs' shared memory and write 128 rows x 256 columns into each CTA's TMEM.  Per SM this halves
+// the B bytes the tensor core reads and the B nibbles each SM unpacks, against a one-SM 128x256
+// tile.  K stages of 128; 16 warps per CTA:
+//   warp 0      A producer: one 2-D TMA per two K stages (256 rows x 128 bytes of the
+//               pre-swizzled A-operand image, 32 KB) -> A ring, completing on the even CTA's
+//               barrier
+//   warp 1      TMEM owner; in the even CTA also the MMA issuer (one thread): 4 MMAs per K stage
+//               into one of two TMEM accumulators; a new accumulator starts at every group
+//               boundary and is handed to both CTAs' drain warps when the group ends
+//   warps 4-7   unpack: packed nibbles straight from global memory (two stages in flight in
+//               registers) -> E4M3 operand bytes in the 128B-swizzled K-major layout -> B ring
+//   warps 8-15  drain: per group, tcgen05.ld the partials (the load of the next 16 columns in
+//               flight while the previous 16 are scaled), y += (acc * s_w) * (s_a * 2^18) in fp32
+//               registers (warp w owns TMEM lanes 32*(w%4).. and columns 128*((w-8)/4)..); after
+//               the last group, + bias, round to bf16, store
+// Every mbarrier wait is bounded; a timeout records a status and unwinds the CTA, and both CTAs
+// of a pair meet at a final cluster barrier before the pair's TMEM is released.
 #include <cfloat>
 #include <cstdint>
 #include <cuda.h>
@@ -36,44 +44,72 @@ namespace jq {
 
 namespace {
 
-constexpr int kBM = 128, kBN = 256, kBK = 128;
-constexpr int kStagesOp = 3;    // operand ring (A via TMA + B via unpack)
-constexpr int kStagesPk = 4;    // packed-B ring
-constexpr int kScaleSlots = 12;  // weight-scale ring (one slot per group; deep enough not to gate loads)
+constexpr int kBM = 128;            // A rows per CTA (a pair covers 256)
+constexpr int kPairM = 2 * kBM;
+constexpr int kBN = 256;            // output columns per pair tile
+constexpr int kBNHalf = kBN / 2;    // B rows per CTA
+constexpr int kBK = 128;
+constexpr int kStagesPerSlot = 2;   // K stages per ring slot (one A transfer, two unpacked B stages)
+constexpr int kSlots = 3;           // operand ring: each slot holds A and B for kStagesPerSlot stages
 constexpr int kThreads = 512;
-constexpr int kUnpackWarp0 = 2, kNumUnpackWarps = 6;
+constexpr int kWarpProdA = 0, kWarpMma = 1;
+constexpr int kUnpackWarp0 = 4, kUnpackThreads = 128;
+constexpr int kUnpackGroups = 2, kUnpackGroupThreads = kUnpackThreads / kUnpackGroups;  // alternate K stages
+constexpr int kUnpackGroupWarps = kUnpackGroupThreads / 32;
 constexpr int kDrainWarp0 = 8, kNumDrainWarps = 8;
-constexpr int kUnpackThreads = kNumUnpackWarps * 32;
 constexpr int kDrainThreads = kNumDrainWarps * 32;
-constexpr uint32_t kTmemCols = 512;  // two 256-column fp32 accumulators
+constexpr int kChunksPerThread = kBNHalf * (kBK / 2) / 16 / kUnpackGroupThreads;  // 8 packed 16-byte chunks
+constexpr uint32_t kTmemCols = 512;  // two 256-column accumulators
+constexpr int kRegsCtl = 40, kRegsUnpack = 120, kRegsDrain = 176;
+static_assert(4 * 32 * (kRegsCtl + kRegsUnpack + 2 * kRegsDrain) == 65536, "register split must use the launch budget");
+static_assert(kChunksPerThread == 8, "unpack assumes eight chunks per thread per stage");
 
-constexpr uint32_t kOpABytes = kBM * kBK;
-constexpr uint32_t kOpBBytes = kBN * kBK;
-constexpr uint32_t kPkBBytes = kBN * kBK / 2;
-constexpr uint32_t kScaleBytes = kBN * 4;
+constexpr uint32_t kOpABytes = kBM * kBK;                     // 16 KB per K stage per CTA
+constexpr uint32_t kSlotABytes = kStagesPerSlot * kOpABytes;  // 32 KB
+constexpr uint32_t kOpBBytes = kBNHalf * kBK;                 // 16 KB per K stage per CTA
+constexpr uint32_t kSlotBBytes = kStagesPerSlot * kOpBBytes;  // 32 KB
 
-constexpr uint32_t kOffOpA = 0;
-constexpr uint32_t kOffOpB = kOffOpA + kStagesOp * kOpABytes;
-constexpr uint32_t kOffPkB = kOffOpB + kStagesOp * kOpBBytes;
-constexpr uint32_t kOffSw = kOffPkB + kStagesPk * kPkBBytes;
-constexpr uint32_t kOffBar = kOffSw + kScaleSlots * kScaleBytes;
-constexpr uint32_t kNumBars = 3 * kStagesOp + 2 * kStagesPk + 2 * kScaleSlots + 4 + 1;
+constexpr uint32_t kOffA = 0;
+constexpr uint32_t kOffB = kOffA + kSlots * kSlotABytes;
+constexpr uint32_t kOffBar = kOffB + kSlots * kSlotBBytes;
+constexpr uint32_t kNumBars = 2 * kSlots + 4 + 1 + 4;
 constexpr uint32_t kOffMisc = kOffBar + kNumBars * 8;
-constexpr uint32_t kSmemBytes = kOffMisc + 16 + 1024;  // + slack to align the base to 1024
-
+constexpr uint32_t kOffSw = (kOffMisc + 16 + 127) & ~127u;  // two slots of kBN fp32 weight scales
+constexpr uint32_t kSmemBytes = kOffSw + 2 * kBN * 4;
+static_assert(kOffBar % 8 == 0 && kOffMisc % 8 == 0 && kOffSw % 16 == 0, "mbarriers need 8 bytes, v4 loads 16");
+static_assert(kOffA % 1024 == 0 && kOffB % 1024 == 0 && kOpABytes % 1024 == 0 && kOpBBytes % 1024 == 0,
+              "128B-swizzled operand slots need 1024-byte alignment");
+// The rings need a 1024-byte aligned base (128B swizzle atoms); the dynamic shared memory
+// window is declared with that alignment and the kernel checks it before touching anything.
 static_assert(kSmemBytes <= 232448, "shared memory budget");
 
 struct Args {
   int M, N, K, G;
-  int num_m_tiles, num_tiles;
+  int num_m2, num_tiles, k_stages, slots_per_tile;
+  const uint8_t* qw;
   const float* s_a;
+  const float* s_w;
   const float* bias;
   __nv_bfloat16* y;
   int32_t* partials;
   uint32_t* status;
 };
 
-__device__ __forceinline__ uint32_t ring_parity(uint32_t it, uint32_t stages) { return (it / stages) & 1u; }
+struct Bars {
+  uint64_t *full, *empty;  // operand ring: A and B of a slot arrive on full, leave on empty
+  uint64_t *acc_full, *acc_empty, *mma_done;
+  uint64_t *sw_full, *sw_empty;  // weight-scale slots of the drain (two groups)
+};
+
+struct Pair {
+  uint32_t rank;     // 0 = the CTA that issues the MMAs
+  int cluster;       // pair index
+  int num_clusters;  // pairs in the grid
+};
+
+__device__ __forceinline__ uint32_t ring_parity(uint32_t it, uint32_t slots) { return (it / slots) & 1u; }
+// Address of a barrier of this CTA's layout in the even CTA of the pair.
+__device__ __forceinline__ uint32_t leader_bar(uint64_t* bar) { return mapa_shared(smem_u32(bar), 0); }
 
 // A bounded wait that ignores the CTA abort flag (used while draining in-flight async work).
 __device__ __forceinline__ void drain_wait(uint64_t* bar, uint32_t parity, uint32_t* status) {
@@ -81,300 +117,470 @@ __device__ __forceinline__ void drain_wait(uint64_t* bar, uint32_t parity, uint3
   mbar_wait(bar, parity, &dummy, status);
 }
 
+// ------------------------------------------------------------------ drain + epilogue
 template <bool kExport>
-__device__ __forceinline__ void drain_role(const Args& args, uint32_t tmem_base, const float* sw, uint64_t* full_s,
-                                           uint64_t* empty_s, uint64_t* acc_full, uint64_t* acc_empty,
-                                           volatile int* abort_flag) {
+__device__ __forceinline__ void drain_role(const Args& args, const Pair& pr, uint32_t tmem_base, const Bars& b,
+                                           float* sw_smem, volatile int* abort_flag) {
   const uint32_t warp = warp_id(), lane = lane_id();
-  const int M = args.M, N = args.N, K = args.K, G = args.G;
-  const int groups = K / G;
-    // ------------------------------------------------------------------ drain + epilogue
-    const uint32_t quarter = warp & 3u, half = (warp - kDrainWarp0) >> 2;
-    const uint32_t lane_base = (quarter * 32u) << 16;
-    uint32_t chunk_it = 0, it_s = 0;
-    bool ok = true;
-    for (int tile = blockIdx.x; ok && tile < args.num_tiles; tile += gridDim.x) {
-      const int mt = tile % args.num_m_tiles, nt = tile / args.num_m_tiles;
-      const int row = mt * kBM + quarter * 32 + lane;
-      const int col0 = nt * kBN + half * 128;
-      const bool row_ok = row < M;
-      float y[128];
+  const int M = args.M, N = args.N;
+  const int groups = args.K / args.G;
+  const uint32_t quarter = warp & 3u, half = (warp - kDrainWarp0) >> 2;
+  const uint32_t lane_base = (quarter * 32u) << 16;
+  const uint32_t dt = threadIdx.x - kDrainWarp0 * 32;  // 0..255
+  const bool loader = dt < kBN / 4;                     // 64 threads move 16 bytes of scales each
+  uint32_t chunk_it = 0;
+  bool ok = true;
+  if (!kExport && loader && pr.cluster < args.num_tiles) {  // group 0 of the first tile -> slot 0
+    const int ncol = (pr.cluster / args.num_m2) * kBN + 4 * (int)dt;
+    float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
+    if (ncol < N) v = __ldg(reinterpret_cast<const float4*>(args.s_w + ncol));
+    *reinterpret_cast<float4*>(sw_smem + 4 * dt) = v;
+    mbar_arrive(&b.sw_full[0]);
+  }
+  for (int tile = pr.cluster; ok && tile < args.num_tiles; tile += pr.num_clusters) {
+    const int mt2 = tile % args.num_m2, nt = tile / args.num_m2;
+    const int row = mt2 * kPairM + (int)pr.rank * kBM + quarter * 32 + lane;
+    const int col0 = nt * kBN + half * 128;
+    const bool row_ok = row < M;
+    const float* sa_row = kExport ? nullptr : args.s_a + (int64_t)(row_ok ? row : 0) * groups;
+    float y[128];
 #pragma unroll
-      for (int i = 0; i < 128; ++i) y[i] = 0.0f;
-      for (int g = 0; g < groups; ++g) {
-        const uint32_t ab = chunk_it & 1u, s = it_s % kScaleSlots;
-        const float sa = (!kExport && row_ok) ? __ldg(args.s_a + (int64_t)row * groups + g) : 0.0f;
-        if (!(ok = mbar_wait(&full_s[s], ring_parity(it_s, kScaleSlots), abort_flag, args.status))) break;
-        if (!(ok = mbar_wait(&acc_full[ab], (chunk_it >> 1) & 1u, abort_flag, args.status))) break;
-        tc_fence_after();
-        const uint32_t taddr = tmem_base + lane_base + ab * kBN + half * 128;
-        const float* sws = sw + s * kBN + half * 128;
-        if constexpr (kExport) {
+    for (int i = 0; i < 128; ++i) y[i] = 0.0f;
+    float sa_next = (!kExport && row_ok) ? __ldg(sa_row) : 0.0f;
+    for (int g = 0; g < groups; ++g) {
+      const uint32_t ab = chunk_it & 1u;
+      const float sa = sa_next;
+      if (!kExport && row_ok && g + 1 < groups) sa_next = __ldg(sa_row + g + 1);
+      // The weight scales of the next group this CTA drains (the next group of this tile, or
+      // group 0 of the next tile) go to registers now and to shared memory after this group.
+      bool have_next = false;
+      float4 sw_next = make_float4(0.f, 0.f, 0.f, 0.f);
+      if (!kExport && loader) {
+        const int next_tile = tile + pr.num_clusters;
+        have_next = g + 1 < groups || next_tile < args.num_tiles;
+        const int ng = g + 1 < groups ? g + 1 : 0;
+        const int ncol = (g + 1 < groups ? nt : next_tile / args.num_m2) * kBN + 4 * (int)dt;
+        if (have_next && ncol < N) sw_next = __ldg(reinterpret_cast<const float4*>(args.s_w + (int64_t)ng * N + ncol));
+      }
+      // Warp-collective tcgen05.ld follows: the whole warp proceeds or none of it (a timeout in
+      // one lane must not leave the others in an aligned instruction).
+      ok = __all_sync(0xffffffffu, mbar_wait(&b.acc_full[ab], (chunk_it >> 1) & 1u, abort_flag, args.status));
+      if (!ok) break;
+      tc_fence_after();
+      const uint32_t taddr = tmem_base + lane_base + ab * kBN + half * 128;
+      if constexpr (kExport) {
 #pragma unroll 1
-          for (int cc = 0; cc < 4; ++cc) {
-            uint32_t r[32];
-            tmem_ld32(taddr + cc * 32, r);
-            tmem_ld_wait();
-            if (cc == 3) {
-              tc_fence_before();
-              mbar_arrive(&acc_empty[ab]);
-            }
-            if (row_ok) {
+        for (int cc = 0; cc < 4; ++cc) {
+          uint32_t r[32];
+          tmem_ld32(taddr + cc * 32, r);
+          tmem_ld_wait();
+          if (row_ok) {
 #pragma unroll
-              for (int j = 0; j < 32; ++j) {
-                const int col = col0 + cc * 32 + j;
-                if (col < N)
-                  args.partials[((int64_t)row * N + col) * groups + g] =
-                      static_cast<int32_t>(__uint_as_float(r[j]) * kOperandUnitInv);
-              }
-            }
-          }
-        } else {
-          const float f = sa * kOperandUnitInv;  // s_a * 2^18
-          const bool f_finite = f <= FLT_MAX;
-#pragma unroll
-          for (int cc = 0; cc < 4; ++cc) {
-            uint32_t r[32];
-            tmem_ld32(taddr + cc * 32, r);
-            tmem_ld_wait();
-            if (cc == 3) {
-              tc_fence_before();
-              mbar_arrive(&acc_empty[ab]);
-            }
-            if (f_finite) {
-#pragma unroll
-              for (int j = 0; j < 32; ++j)
-                y[cc * 32 + j] = fmaf(__uint_as_float(r[j]) * f, sws[cc * 32 + j], y[cc * 32 + j]);
-            } else {  // |s_a| > 2^110: apply 2^18 to the exact partial first
-#pragma unroll
-              for (int j = 0; j < 32; ++j)
-                y[cc * 32 + j] =
-                    fmaf((__uint_as_float(r[j]) * kOperandUnitInv) * sa, sws[cc * 32 + j], y[cc * 32 + j]);
+            for (int j = 0; j < 32; ++j) {
+              const int col = col0 + cc * 32 + j;
+              if (col < N)
+                args.partials[((int64_t)row * N + col) * groups + g] =
+                    static_cast<int32_t>(__uint_as_float(r[j]) * kOperandUnitInv);
             }
           }
         }
-        mbar_arrive(&empty_s[s]);
-        ++chunk_it;
-        ++it_s;
-      }
-      if (!ok) break;
-      if constexpr (!kExport) {
-        if (row_ok) {
-          __nv_bfloat16* yrow = args.y + (int64_t)row * N;
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive_remote_cta(leader_bar(&b.acc_empty[ab]));
+      } else {
+        const uint32_t cslot = chunk_it & 1u;
+        ok = __all_sync(0xffffffffu, mbar_wait(&b.sw_full[cslot], (chunk_it >> 1) & 1u, abort_flag, args.status));
+        if (!ok) break;
+        const float f = sa * kOperandUnitInv;  // s_a * 2^18
+        const bool f_finite = f <= FLT_MAX;
+        const float2 f2 = make_float2(f, f);
+        const float* sws = sw_smem + cslot * kBN + half * 128;
+        // y[c..c+7] += (partial * s_w) * f for one 8-column chunk already in registers
+        auto accumulate = [&](const uint32_t(&r)[8], int cc) {
+          if (f_finite) {
 #pragma unroll
-          for (int i = 0; i < 16; ++i) {
-            const int col = col0 + 8 * i;
-            if (col < N) {
-              float v[8];
-#pragma unroll
-              for (int j = 0; j < 8; ++j) v[j] = y[8 * i + j];
-              if (args.bias != nullptr) {
-                const float4 b0 = __ldg(reinterpret_cast<const float4*>(args.bias + col));
-                const float4 b1 = __ldg(reinterpret_cast<const float4*>(args.bias + col + 4));
-                v[0] += b0.x; v[1] += b0.y; v[2] += b0.z; v[3] += b0.w;
-                v[4] += b1.x; v[5] += b1.y; v[6] += b1.z; v[7] += b1.w;
-              }
-              uint4 out;
-              __nv_bfloat162 t0 = __floats2bfloat162_rn(v[0], v[1]);
-              __nv_bfloat162 t1 = __floats2bfloat162_rn(v[2], v[3]);
-              __nv_bfloat162 t2 = __floats2bfloat162_rn(v[4], v[5]);
-              __nv_bfloat162 t3 = __floats2bfloat162_rn(v[6], v[7]);
-              out.x = *reinterpret_cast<uint32_t*>(&t0);
-              out.y = *reinterpret_cast<uint32_t*>(&t1);
-              out.z = *reinterpret_cast<uint32_t*>(&t2);
-              out.w = *reinterpret_cast<uint32_t*>(&t3);
-              *reinterpret_cast<uint4*>(yrow + col) = out;
+            for (int j = 0; j < 8; j += 4) {
+              const float4 w4 = ld_shared_f4(sws + cc * 8 + j);
+              float* yy = y + cc * 8 + j;
+              const float2 t0 = __fmul2_rn(make_float2(__uint_as_float(r[j]), __uint_as_float(r[j + 1])),
+                                           make_float2(w4.x, w4.y));
+              const float2 t1 = __fmul2_rn(make_float2(__uint_as_float(r[j + 2]), __uint_as_float(r[j + 3])),
+                                           make_float2(w4.z, w4.w));
+              const float2 y0 = __ffma2_rn(t0, f2, make_float2(yy[0], yy[1]));
+              const float2 y1 = __ffma2_rn(t1, f2, make_float2(yy[2], yy[3]));
+              yy[0] = y0.x;
+              yy[1] = y0.y;
+              yy[2] = y1.x;
+              yy[3] = y1.y;
             }
+          } else {  // |s_a| > 2^110: apply 2^18 to the exact partial first so nothing overflows
+#pragma unroll
+            for (int j = 0; j < 8; ++j)
+              y[cc * 8 + j] = fmaf((__uint_as_float(r[j]) * kOperandUnitInv) * sa, sws[cc * 8 + j], y[cc * 8 + j]);
+          }
+        };
+        // 16 chunks of 8 columns; the load of chunk c+1 is in flight while chunk c is scaled
+        constexpr int kChunks = 16;
+        uint32_t ra[8], rb[8];
+        tmem_ld8(taddr, ra);
+        tmem_ld_wait();
+#pragma unroll
+        for (int cc = 0; cc < kChunks; cc += 2) {
+          tmem_ld8(taddr + (cc + 1) * 8, rb);
+          accumulate(ra, cc);
+          tmem_ld_wait();
+          if (cc + 2 < kChunks) {
+            tmem_ld8(taddr + (cc + 2) * 8, ra);
+          } else {  // every column of this accumulator is in registers: hand it back
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive_remote_cta(leader_bar(&b.acc_empty[ab]));
+          }
+          accumulate(rb, cc + 1);
+          if (cc + 2 < kChunks) tmem_ld_wait();
+        }
+        mbar_arrive(&b.sw_empty[cslot]);
+        // publish the scales prefetched at the top of this group into the other slot
+        if (loader && have_next) {
+          const uint32_t nslot = cslot ^ 1u;
+          ok = __all_sync(0xffffffffu,  // loader warps are whole warps (threads 0..63 of the drain)
+                          mbar_wait(&b.sw_empty[nslot], ring_parity(chunk_it + 1, 2) ^ 1u, abort_flag, args.status));
+          if (!ok) break;
+          *reinterpret_cast<float4*>(sw_smem + nslot * kBN + 4 * dt) = sw_next;
+          mbar_arrive(&b.sw_full[nslot]);
+        }
+      }
+      ++chunk_it;
+    }
+    if (!ok) break;
+    if constexpr (!kExport) {
+      if (row_ok) {
+        __nv_bfloat16* yrow = args.y + (int64_t)row * N;
+#pragma unroll
+        for (int i = 0; i < 16; ++i) {
+          const int col = col0 + 8 * i;
+          if (col < N) {
+            float v[8];
+#pragma unroll
+            for (int j = 0; j < 8; ++j) v[j] = y[8 * i + j];
+            if (args.bias != nullptr) {
+              const float4 b0 = __ldg(reinterpret_cast<const float4*>(args.bias + col));
+              const float4 b1 = __ldg(reinterpret_cast<const float4*>(args.bias + col + 4));
+              v[0] += b0.x; v[1] += b0.y; v[2] += b0.z; v[3] += b0.w;
+              v[4] += b1.x; v[5] += b1.y; v[6] += b1.z; v[7] += b1.w;
+            }
+            uint4 out;
+            __nv_bfloat162 t0 = __floats2bfloat162_rn(v[0], v[1]);
+            __nv_bfloat162 t1 = __floats2bfloat162_rn(v[2], v[3]);
+            __nv_bfloat162 t2 = __floats2bfloat162_rn(v[4], v[5]);
+            __nv_bfloat162 t3 = __floats2bfloat162_rn(v[6], v[7]);
+            out.x = *reinterpret_cast<uint32_t*>(&t0);
+            out.y = *reinterpret_cast<uint32_t*>(&t1);
+            out.z = *reinterpret_cast<uint32_t*>(&t2);
+            out.w = *reinterpret_cast<uint32_t*>(&t3);
+            *reinterpret_cast<uint4*>(yrow + col) = out;
           }
         }
       }
     }
+  }
+}
+
+// ------------------------------------------------------------------ A producer
+// Both CTAs load their own 128 rows of a slot's two K stages; the transfers complete on the even
+// CTA's full barrier, which the even CTA arms with the bytes of both.
+__device__ __forceinline__ void producer_a(const Args& args, const Pair& pr, const CUtensorMap* tmA, uint8_t* sA,
+                                           const Bars& b, volatile int* abort_flag) {
+  uint32_t it = 0;
+  bool ok = true;
+  for (int tile = pr.cluster; ok && tile < args.num_tiles; tile += pr.num_clusters) {
+    const int mt = (tile % args.num_m2) * 2 + (int)pr.rank;  // 128-row block of the operand image
+    for (int j = 0; j < args.slots_per_tile; ++j) {
+      const uint32_t s = it % kSlots;
+      if (!(ok = mbar_wait(&b.empty[s], ring_parity(it, kSlots) ^ 1u, abort_flag, args.status))) break;
+      if (pr.rank == 0) mbar_arrive_expect_tx(&b.full[s], 2 * kSlotABytes);
+      const int image_row = (mt * args.k_stages + j * kStagesPerSlot) * kBM;
+      tma_load_2d_pair(sA + s * kSlotABytes, tmA, leader_bar(&b.full[s]), 0, image_row);
+      ++it;
+    }
+  }
+  // Let the pair's last copies land before the CTA can leave (the even CTA sees both CTAs' bytes;
+  // on an early exit the unpack arrivals may be missing, and the bounded wait ends it).
+  if (pr.rank == 0)
+    for (uint32_t i = (it > kSlots ? it - kSlots : 0); i < it; ++i)
+      drain_wait(&b.full[i % kSlots], ring_parity(i, kSlots), args.status);
+}
+
+// ------------------------------------------------------------------ MMA issuer (even CTA)
+// The tensor core accepts only about one MMA ahead of the one it is executing, so every scalar
+// instruction or branch between two MMAs can leave it idle.  All decisions are therefore taken
+// once per K stage (a group of 128 or more elements starts and ends on stage boundaries; a
+// group of 64 is exactly half a stage), ring positions are wrapping counters, and each stage's
+// descriptors come from two precomputed bases by one add (the low field of a descriptor is the
+// shared-memory address >> 4, and no slot crosses its 14-bit range).
+struct MmaState {
+  uint32_t chunk_it = 0;  // accumulator hand-offs so far (selects buffer and parity)
+};
+
+// Opens a new accumulator: waits until the drain has emptied it.
+__device__ __forceinline__ bool mma_open_acc(const Args& args, const Bars& b, uint32_t tmem_base, MmaState& st,
+                                             uint32_t& d_tmem, volatile int* abort_flag) {
+  const uint32_t ab = st.chunk_it & 1u;
+  if (!mbar_wait_cluster(&b.acc_empty[ab], ((st.chunk_it >> 1) & 1u) ^ 1u, abort_flag, args.status)) return false;
+  tc_fence_after();
+  d_tmem = tmem_base + ab * kBN;
+  return true;
+}
+
+__device__ __forceinline__ void mma_role(const Args& args, const Pair& pr, uint32_t tmem_base, uint8_t* sA,
+                                         uint8_t* sB, const Bars& b, volatile int* abort_flag) {
+  const uint32_t idesc = idesc_e4m3_f32(kPairM, kBN);
+  constexpr uint16_t kBoth = 0x3;
+  const uint64_t adesc0 = sdesc_kmajor_sw128(smem_u32(sA));
+  const uint64_t bdesc0 = sdesc_kmajor_sw128(smem_u32(sB));
+  const int stages_per_group = args.G >= kBK ? args.G / kBK : 1;  // G = 64: two groups per stage
+  const bool half_groups = args.G < kBK;
+  const int my_tiles =
+      pr.cluster < args.num_tiles ? (args.num_tiles - 1 - pr.cluster) / pr.num_clusters + 1 : 0;
+  const uint32_t total = static_cast<uint32_t>(my_tiles) * static_cast<uint32_t>(args.slots_per_tile);
+  uint32_t slot = 0, phase = 0;
+  MmaState st;
+  uint32_t d_tmem = tmem_base;
+  int j = 0, kg = 0;  // slot within the tile, K stage within the group
+  bool ok = total > 0 && mbar_wait_cluster(&b.full[0], 0, abort_flag, args.status);
+  for (uint32_t q = 0; ok && q < total; ++q) {
+    const uint32_t nslot = slot + 1 == kSlots ? 0 : slot + 1;
+    const uint32_t nphase = slot + 1 == kSlots ? phase ^ 1u : phase;
+    const int n_st = min(kStagesPerSlot, args.k_stages - j * kStagesPerSlot);
+    bool waited_next = q + 1 >= total;  // the next slot's operands, waited for while MMAs are queued
+    for (int sub = 0; sub < n_st; ++sub) {
+      const uint64_t adesc = adesc0 + ((slot * kSlotABytes + sub * kOpABytes) >> 4);
+      const uint64_t bdesc = bdesc0 + ((slot * kSlotBBytes + sub * kOpBBytes) >> 4);
+      const bool wait_here = sub == n_st - 1 && !waited_next;
+      if (half_groups) {
+        if (!(ok = mma_open_acc(args, b, tmem_base, st, d_tmem, abort_flag))) break;
+        umma_f8f6f4_pair(d_tmem, adesc, bdesc, idesc, 0u);
+        umma_f8f6f4_pair(d_tmem, adesc + 2u, bdesc + 2u, idesc, 1u);
+        umma_commit_pair(&b.acc_full[st.chunk_it & 1u], kBoth);
+        ++st.chunk_it;
+        if (!(ok = mma_open_acc(args, b, tmem_base, st, d_tmem, abort_flag))) break;
+        umma_f8f6f4_pair(d_tmem, adesc + 4u, bdesc + 4u, idesc, 0u);
+        if (wait_here) {
+          if (!(ok = mbar_wait_cluster(&b.full[nslot], nphase, abort_flag, args.status))) break;
+          waited_next = true;
+        }
+        umma_f8f6f4_pair(d_tmem, adesc + 6u, bdesc + 6u, idesc, 1u);
+        umma_commit_pair(&b.acc_full[st.chunk_it & 1u], kBoth);
+        ++st.chunk_it;
+      } else {
+        const bool first = kg == 0;
+        if (first && !(ok = mma_open_acc(args, b, tmem_base, st, d_tmem, abort_flag))) break;
+        umma_f8f6f4_pair(d_tmem, adesc, bdesc, idesc, first ? 0u : 1u);
+        umma_f8f6f4_pair(d_tmem, adesc + 2u, bdesc + 2u, idesc, 1u);
+        if (wait_here) {
+          if (!(ok = mbar_wait_cluster(&b.full[nslot], nphase, abort_flag, args.status))) break;
+          waited_next = true;
+        }
+        umma_f8f6f4_pair(d_tmem, adesc + 4u, bdesc + 4u, idesc, 1u);
+        umma_f8f6f4_pair(d_tmem, adesc + 6u, bdesc + 6u, idesc, 1u);
+        if (++kg == stages_per_group) {
+          umma_commit_pair(&b.acc_full[st.chunk_it & 1u], kBoth);
+          ++st.chunk_it;
+          kg = 0;
+        }
+      }
+    }
+    if (!ok) break;
+    umma_commit_pair(&b.empty[slot], kBoth);
+    slot = nslot;
+    phase = nphase;
+    if (++j == args.slots_per_tile) j = 0;
+  }
+  // Every MMA this thread issued has finished once mma_done flips (in both CTAs).
+  umma_commit_pair(b.mma_done, kBoth);
+  drain_wait(b.mma_done, 0, args.status);
+}
+
+// ------------------------------------------------------------------ unpack
+// Two groups of two warps take alternate K stages.  Per stage, thread u of a group converts
+// packed chunks t = u + 64 i (i = 0..7): 16-byte chunk t % 4 of the 64 packed bytes of B row t / 4
+// (this CTA's half of the tile's columns).  Each chunk becomes two 16-byte operand chunks of the
+// 128B-swizzled row; a quarter-warp's stores cover two rows whose chunk positions differ in
+// parity, so they never share a bank.
+//
+// Each round's global loads are issued two rounds ahead.
+// Cursor over the (tile, slot) sequence of this pair; a group's stage in slot j is 2j + group.
+struct UnpackCursor {
+  int tile, j;
+};
+
+__device__ __forceinline__ void unpack_load(const Args& args, const Pair& pr, const UnpackCursor& c, uint32_t ug,
+                                            uint32_t u, uint4 (&buf)[kChunksPerThread]) {
+  const int K2 = args.K / 2;
+  const int kb = c.j * kStagesPerSlot + (int)ug;
+  if (c.tile < args.num_tiles && kb < args.k_stages) {
+    const int n0 = (c.tile / args.num_m2) * kBN + (int)pr.rank * kBNHalf;
+    const uint8_t* src = args.qw + kb * (kBK / 2) + (u & 3u) * 16;
+#pragma unroll
+    for (int i = 0; i < kChunksPerThread; ++i) {
+      const int n = n0 + (int)(u >> 2) + 16 * i;
+      buf[i] = n < args.N ? __ldg(reinterpret_cast<const uint4*>(src + (int64_t)n * K2)) : make_uint4(0u, 0u, 0u, 0u);
+    }
+  }
+}
+
+__device__ __forceinline__ void unpack_advance(const Args& args, const Pair& pr, UnpackCursor& c) {
+  if (++c.j == args.slots_per_tile) {
+    c.j = 0;
+    c.tile += pr.num_clusters;
+  }
+}
+
+// Converts this group's stage of ring slot (q % kSlots) into the slot's B half for that stage
+// (or, for the missing second stage of an odd K-stage count, only signals the slot).
+__device__ __forceinline__ bool unpack_store(const Args& args, uint8_t* sB, const Bars& b, uint32_t ug, uint32_t u,
+                                             uint32_t q, bool has_stage, const uint4 (&buf)[kChunksPerThread],
+                                             volatile int* abort_flag) {
+  const uint32_t o = q % kSlots;
+  if (!__all_sync(0xffffffffu, mbar_wait(&b.empty[o], ring_parity(q, kSlots) ^ 1u, abort_flag, args.status)))
+    return false;
+  if (has_stage) {
+    const uint32_t dst = smem_u32(sB + o * kSlotBBytes + ug * kOpBBytes);
+    const uint32_t jc = u & 3u;
+#pragma unroll
+    for (int i = 0; i < kChunksPerThread; ++i) {
+      const uint32_t r = (u >> 2) + 16u * i, r7 = r & 7u;
+      uint4 lo, hi;
+      nib32_to_operand(buf[i], lo, hi);
+      const uint32_t row_base = dst + (r >> 3) * 1024u + r7 * 128u;
+      st_shared_v4(row_base + (((2u * jc) ^ r7) << 4), lo.x, lo.y, lo.z, lo.w);
+      st_shared_v4(row_base + (((2u * jc + 1u) ^ r7) << 4), hi.x, hi.y, hi.z, hi.w);
+    }
+    // The stores went to this CTA's own shared memory.  Each thread makes its stores visible to
+    // the async proxy (the tensor core reads them there), the warp converges, and one lane
+    // arrives on the even CTA's full barrier -- the thread-producer -> pair-MMA hand-off of the
+    // SM100 pipelines: a CTA-scope release, which (unlike a cluster-scope one) does not wait for
+    // the thread's loads of later rounds that are still in flight.
+    fence_proxy_async_smem();
+  }
+  __syncwarp();
+  if ((u & 31u) == 0) mbar_arrive_remote_cta(leader_bar(&b.full[o]));
+  return true;
+}
+
+__device__ __forceinline__ void unpack_role(const Args& args, const Pair& pr, uint8_t* sB, const Bars& b,
+                                            volatile int* abort_flag) {
+  const uint32_t ut = threadIdx.x - kUnpackWarp0 * 32;
+  const uint32_t ug = ut / kUnpackGroupThreads, u = ut % kUnpackGroupThreads;
+  const int my_tiles =
+      pr.cluster < args.num_tiles ? (args.num_tiles - 1 - pr.cluster) / pr.num_clusters + 1 : 0;
+  const uint32_t total = static_cast<uint32_t>(my_tiles) * static_cast<uint32_t>(args.slots_per_tile);
+  UnpackCursor sc{pr.cluster, 0};  // the slot being stored
+  UnpackCursor lc = sc;            // the slot being loaded (two ahead)
+  uint4 b0[kChunksPerThread], b1[kChunksPerThread];
+  unpack_load(args, pr, lc, ug, u, b0);
+  unpack_advance(args, pr, lc);
+  unpack_load(args, pr, lc, ug, u, b1);
+  unpack_advance(args, pr, lc);
+  for (uint32_t q = 0; q < total; q += 2) {
+    bool has = sc.j * kStagesPerSlot + (int)ug < args.k_stages;
+    if (!unpack_store(args, sB, b, ug, u, q, has, b0, abort_flag)) return;
+    unpack_advance(args, pr, sc);
+    unpack_load(args, pr, lc, ug, u, b0);
+    unpack_advance(args, pr, lc);
+    if (q + 1 < total) {
+      has = sc.j * kStagesPerSlot + (int)ug < args.k_stages;
+      if (!unpack_store(args, sB, b, ug, u, q + 1, has, b1, abort_flag)) return;
+      unpack_advance(args, pr, sc);
+      unpack_load(args, pr, lc, ug, u, b1);
+      unpack_advance(args, pr, lc);
+    }
+  }
 }
 
 template <bool kExport>
-__global__ void __launch_bounds__(kThreads, 1)
-    w4a4_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
-                     const __grid_constant__ CUtensorMap tmS, const Args args) {
-  extern __shared__ uint8_t smem_raw[];
-  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  uint8_t* opA = smem + kOffOpA;
-  uint8_t* opB = smem + kOffOpB;
-  uint8_t* pkB = smem + kOffPkB;
-  float* sw = reinterpret_cast<float*>(smem + kOffSw);
-  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + kOffBar);
-  uint64_t* full_a = bars;                  // A operand bytes landed (TMA)
-  uint64_t* full_b = full_a + kStagesOp;    // B operand bytes written (unpack warps)
-  uint64_t* empty_op = full_b + kStagesOp;  // MMAs of the stage finished
-  uint64_t* full_pk = empty_op + kStagesOp;
-  uint64_t* empty_pk = full_pk + kStagesPk;
-  uint64_t* full_s = empty_pk + kStagesPk;
-  uint64_t* empty_s = full_s + kScaleSlots;
-  uint64_t* acc_full = empty_s + kScaleSlots;
-  uint64_t* acc_empty = acc_full + 2;
-  uint64_t* mma_done = acc_empty + 2;
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
+    w4a4_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const Args args) {
+  extern __shared__ __align__(1024) uint8_t smem_raw[];
+  if ((smem_u32(smem_raw) & 1023u) != 0) {  // uniform across the grid: nothing has been touched yet
+    if (threadIdx.x == 0 && args.status != nullptr) atomicExch(args.status, (uint32_t)kDevSmemAlign);
+    return;
+  }
+  uint8_t* smem = smem_raw;
+  uint8_t* sA = smem + kOffA;
+  uint8_t* sB = smem + kOffB;
+  uint64_t* bar = reinterpret_cast<uint64_t*>(smem + kOffBar);
+  Bars b;
+  b.full = bar;
+  b.empty = b.full + kSlots;
+  b.acc_full = b.empty + kSlots;
+  b.acc_empty = b.acc_full + 2;
+  b.mma_done = b.acc_empty + 2;
+  b.sw_full = b.mma_done + 1;
+  b.sw_empty = b.sw_full + 2;
+  float* sw_smem = reinterpret_cast<float*>(smem + kOffSw);
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + kOffMisc);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + kOffMisc + 4);
 
-  const uint32_t warp = warp_id(), lane = lane_id();
-  const int M = args.M, N = args.N, K = args.K, G = args.G;
-  const int k_stages = K / kBK;
-  const int groups = K / G;
+  Pair pr;
+  pr.rank = cluster_ctarank();
+  pr.cluster = static_cast<int>(blockIdx.x >> 1);
+  pr.num_clusters = static_cast<int>(gridDim.x >> 1);
 
+  const uint32_t warp = warp_id(), lane = lane_id();
   if (threadIdx.x == 0) {
     *abort_flag = 0;
-    for (int i = 0; i < kStagesOp; ++i) {
-      mbar_init(&full_a[i], 1);
-      mbar_init(&full_b[i], kUnpackThreads);
-      mbar_init(&empty_op[i], 1);
-    }
-    for (int i = 0; i < kStagesPk; ++i) {
-      mbar_init(&full_pk[i], 1);
-      mbar_init(&empty_pk[i], kUnpackThreads);
-    }
-    for (int i = 0; i < kScaleSlots; ++i) {
-      mbar_init(&full_s[i], 1);
-      mbar_init(&empty_s[i], kDrainThreads);
+    for (int i = 0; i < kSlots; ++i) {
+      // the even CTA's expect_tx (both CTAs' A bytes) + every unpack warp of both CTAs
+      mbar_init(&b.full[i], 1 + 2 * kUnpackGroups * kUnpackGroupWarps);
+      mbar_init(&b.empty[i], 1);  // one pair commit
     }
     for (int i = 0; i < 2; ++i) {
-      mbar_init(&acc_full[i], 1);
-      mbar_init(&acc_empty[i], kDrainThreads);
+      mbar_init(&b.acc_full[i], 1);
+      mbar_init(&b.acc_empty[i], 2 * kNumDrainWarps);  // every drain warp of both CTAs
+      mbar_init(&b.sw_full[i], kBN / 4);
+      mbar_init(&b.sw_empty[i], kDrainThreads);
     }
-    mbar_init(mma_done, 1);
+    mbar_init(b.mma_done, 1);
     fence_mbar_init();
     tma_prefetch_desc(&tmA);
-    tma_prefetch_desc(&tmB);
-    tma_prefetch_desc(&tmS);
   }
-  if (warp == 1) {
-    tmem_alloc(tmem_slot, kTmemCols);
-    tmem_relinquish();
+  if (warp == kWarpMma) {
+    tmem_alloc_pair(tmem_slot, kTmemCols);
+    tmem_relinquish_pair();
   }
   tc_fence_before();
   __syncthreads();
+  cluster_sync_all();  // the peer's barriers exist before anything signals them
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
 
+  // Register split per warpgroup (totals the 512 x 128 registers of the launch): producer and
+  // MMA (warps 0-3) 40, unpack (warps 4-7) 120, drain (warps 8-15, 128 running sums) 176.
   if (warp >= kDrainWarp0) {
-    asm volatile("setmaxnreg.inc.sync.aligned.u32 216;\n" ::: "memory");
-    drain_role<kExport>(args, tmem_base, sw, full_s, empty_s, acc_full, acc_empty, abort_flag);
+    asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;\n" ::"n"(kRegsDrain) : "memory");
+    drain_role<kExport>(args, pr, tmem_base, b, sw_smem, abort_flag);
+  } else if (warp >= kUnpackWarp0) {
+    asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;\n" ::"n"(kRegsUnpack) : "memory");
+    unpack_role(args, pr, sB, b, abort_flag);
   } else {
-    asm volatile("setmaxnreg.dec.sync.aligned.u32 40;\n" ::: "memory");
-  if (warp == 0) {
-    // ------------------------------------------------------------------ TMA producer
-    if (lane == 0) {
-      uint32_t it_op = 0, it_pk = 0, it_s = 0;
-      bool ok = true;
-      for (int tile = blockIdx.x; ok && tile < args.num_tiles; tile += gridDim.x) {
-        const int mt = tile % args.num_m_tiles, nt = tile / args.num_m_tiles;
-        for (int kb = 0; ok && kb < k_stages; ++kb) {
-          const int k0 = kb * kBK;
-          for (int kk = 0; kk < kBK; kk += (G < kBK ? G : kBK)) {
-            if ((k0 + kk) % G != 0) continue;
-            const uint32_t s = it_s % kScaleSlots;
-            if (!(ok = mbar_wait(&empty_s[s], ring_parity(it_s, kScaleSlots) ^ 1u, abort_flag, args.status))) break;
-            mbar_arrive_expect_tx(&full_s[s], kScaleBytes);
-            tma_load_2d(sw + s * kBN, &tmS, &full_s[s], nt * kBN, (k0 + kk) / G);
-            ++it_s;
-          }
-          if (!ok) break;
-          const uint32_t p = it_pk % kStagesPk;
-          if (!(ok = mbar_wait(&empty_pk[p], ring_parity(it_pk, kStagesPk) ^ 1u, abort_flag, args.status))) break;
-          mbar_arrive_expect_tx(&full_pk[p], kPkBBytes);
-          tma_load_2d(pkB + p * kPkBBytes, &tmB, &full_pk[p], kb * (kBK / 2), nt * kBN);
-          ++it_pk;
-          const uint32_t o = it_op % kStagesOp;
-          if (!(ok = mbar_wait(&empty_op[o], ring_parity(it_op, kStagesOp) ^ 1u, abort_flag, args.status))) break;
-          mbar_arrive_expect_tx(&full_a[o], kOpABytes);
-          tma_load_2d(opA + o * kOpABytes, &tmA, &full_a[o], k0, mt * kBM);
-          ++it_op;
-        }
-      }
-      // Let every issued copy land before the CTA can exit (they complete on their own).
-      for (uint32_t i = (it_s > kScaleSlots ? it_s - kScaleSlots : 0); i < it_s; ++i)
-        drain_wait(&full_s[i % kScaleSlots], ring_parity(i, kScaleSlots), args.status);
-      for (uint32_t i = (it_pk > kStagesPk ? it_pk - kStagesPk : 0); i < it_pk; ++i)
-        drain_wait(&full_pk[i % kStagesPk], ring_parity(i, kStagesPk), args.status);
-      for (uint32_t i = (it_op > kStagesOp ? it_op - kStagesOp : 0); i < it_op; ++i)
-        drain_wait(&full_a[i % kStagesOp], ring_parity(i, kStagesOp), args.status);
+    asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;\n" ::"n"(kRegsCtl) : "memory");
+    if (warp == kWarpProdA) {
+      if (lane == 0) producer_a(args, pr, &tmA, sA, b, abort_flag);
+    } else if (warp == kWarpMma && lane == 0) {
+      if (pr.rank == 0)
+        mma_role(args, pr, tmem_base, sA, sB, b, abort_flag);
+      else  // the even CTA's MMAs read this CTA's shared memory and write its TMEM until here
+        drain_wait(b.mma_done, 0, args.status);
     }
-  } else if (warp == 1) {
-    // ------------------------------------------------------------------ MMA issuer
-    if (lane == 0) {
-      const uint32_t idesc = idesc_e4m3_f32(kBM, kBN);
-      uint32_t it_op = 0, chunk_it = 0, acc_flag = 0, d_tmem = tmem_base;
-      uint32_t ab = 0;
-      bool ok = true;
-      for (int tile = blockIdx.x; ok && tile < args.num_tiles; tile += gridDim.x) {
-        for (int kb = 0; ok && kb < k_stages; ++kb) {
-          const uint32_t o = it_op % kStagesOp;
-          if (!(ok = mbar_wait(&full_a[o], ring_parity(it_op, kStagesOp), abort_flag, args.status))) break;
-          if (!(ok = mbar_wait(&full_b[o], ring_parity(it_op, kStagesOp), abort_flag, args.status))) break;
-          tc_fence_after();
-          const uint32_t a_base = smem_u32(opA + o * kOpABytes);
-          const uint32_t b_base = smem_u32(opB + o * kOpBBytes);
-#pragma unroll
-          for (int k4 = 0; k4 < kBK / 32; ++k4) {
-            const int kg = kb * kBK + k4 * 32;
-            if (kg % G == 0) {
-              ab = chunk_it & 1u;
-              if (!(ok = mbar_wait(&acc_empty[ab], ((chunk_it >> 1) & 1u) ^ 1u, abort_flag, args.status))) break;
-              tc_fence_after();
-              d_tmem = tmem_base + ab * kBN;
-              acc_flag = 0;
-            }
-            umma_f8f6f4(d_tmem, sdesc_kmajor_sw128(a_base + k4 * 32), sdesc_kmajor_sw128(b_base + k4 * 32), idesc,
-                        acc_flag);
-            acc_flag = 1;
-            if ((kg + 32) % G == 0) {
-              umma_commit(&acc_full[ab]);
-              ++chunk_it;
-            }
-          }
-          if (!ok) break;
-          umma_commit(&empty_op[o]);
-          ++it_op;
-        }
-      }
-      // Every MMA this thread issued has finished once mma_done flips.
-      umma_commit(mma_done);
-      drain_wait(mma_done, 0, args.status);
-    }
-  } else if (warp < kDrainWarp0) {
-    // ------------------------------------------------------------------ unpack
-    const uint32_t ut = threadIdx.x - kUnpackWarp0 * 32;
-    uint32_t it_pk = 0, it_op = 0;
-    bool ok = true;
-    for (int tile = blockIdx.x; ok && tile < args.num_tiles; tile += gridDim.x) {
-      for (int kb = 0; ok && kb < k_stages; ++kb) {
-        const uint32_t p = it_pk % kStagesPk, o = it_op % kStagesOp;
-        if (!(ok = mbar_wait(&full_pk[p], ring_parity(it_pk, kStagesPk), abort_flag, args.status))) break;
-        if (!(ok = mbar_wait(&empty_op[o], ring_parity(it_op, kStagesOp) ^ 1u, abort_flag, args.status))) break;
-        const uint32_t src = smem_u32(pkB + p * kPkBBytes);
-        const uint32_t dst = smem_u32(opB + o * kOpBBytes);
-        for (uint32_t c = ut; c < kBN * 4; c += kUnpackThreads) {
-          const uint32_t r = c >> 2, j = c & 3u, r7 = r & 7u;
-          const uint4 pk = ld_shared_v4(src + r * 64 + j * 16);
-          uint4 lo, hi;
-          nib32_to_operand(pk, lo, hi);
-          const uint32_t row_base = dst + (r >> 3) * 1024 + r7 * 128;
-          st_shared_v4(row_base + (((2 * j) ^ r7) << 4), lo.x, lo.y, lo.z, lo.w);
-          st_shared_v4(row_base + (((2 * j + 1) ^ r7) << 4), hi.x, hi.y, hi.z, hi.w);
-        }
-        fence_proxy_async_smem();
-        mbar_arrive(&empty_pk[p]);
-        mbar_arrive(&full_b[o]);
-        ++it_pk;
-        ++it_op;
-      }
-    }
-  }
   }
 
   tc_fence_before();
   __syncthreads();
-  if (warp == 1) {
+  cluster_sync_all();
+  if (warp == kWarpMma) {
     tc_fence_after();
-    tmem_dealloc(tmem_base, kTmemCols);
+    tmem_dealloc_pair(tmem_base, kTmemCols);
   }
 }
 
@@ -405,19 +611,32 @@ bool encode_2d(CUtensorMap* map, CUtensorMapDataType dtype, const void* base, ui
 
 template <bool kExport>
 cudaError_t launch_impl(const GemmProblem& p, cudaStream_t stream, int sms) {
-  CUtensorMap tmA, tmB, tmS;
-  if (!encode_2d(&tmA, CU_TENSOR_MAP_DATA_TYPE_UINT8, p.a_operand, p.K, p.M, p.K, kBK, kBM,
-                 CU_TENSOR_MAP_SWIZZLE_128B) ||
-      !encode_2d(&tmB, CU_TENSOR_MAP_DATA_TYPE_UINT8, p.qw, p.K / 2, p.N, p.K / 2, kBK / 2, kBN,
-                 CU_TENSOR_MAP_SWIZZLE_NONE) ||
-      !encode_2d(&tmS, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, p.s_w, p.N, p.K / p.G, (uint64_t)p.N * 4, kBN, 1,
-                 CU_TENSOR_MAP_SWIZZLE_NONE))
+  // The A-operand image seen as rows of 128 bytes: block (mt, kb) is rows (mt*k_stages + kb)*128..
+  // One box is two consecutive blocks (two K stages of one 128-row tile).  Boxes that reach past
+  // the image (the odd CTA of a pair whose rows all lie beyond M, or the second stage of an odd
+  // K-stage count at the very end) read zeros.
+  const int k_stages = p.K / kBK;
+  const uint64_t image_rows = (uint64_t)((p.M + kBM - 1) / kBM) * k_stages * kBM;
+  CUtensorMap tmA;
+  if (!encode_2d(&tmA, CU_TENSOR_MAP_DATA_TYPE_UINT8, p.a_operand, kBK, image_rows, kBK, kBK,
+                 kStagesPerSlot * kBM, CU_TENSOR_MAP_SWIZZLE_NONE))
     return cudaErrorInvalidValue;
   static bool attr_set[2] = {false, false};
+  static int max_pairs[2] = {0, 0};
   if (!attr_set[kExport]) {
     cudaError_t e = cudaFuncSetAttribute(w4a4_gemm_kernel<kExport>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          (int)kSmemBytes);
     if (e != cudaSuccess) return e;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(2 * (sms / 2), 1, 1);
+    cfg.blockDim = dim3(kThreads, 1, 1);
+    cfg.dynamicSmemBytes = kSmemBytes;
+    int clusters = 0;
+    if (cudaOccupancyMaxActiveClusters(&clusters, w4a4_gemm_kernel<kExport>, &cfg) != cudaSuccess || clusters <= 0) {
+      (void)cudaGetLastError();
+      clusters = sms / 2;
+    }
+    max_pairs[kExport] = clusters < sms / 2 ? clusters : sms / 2;
     attr_set[kExport] = true;
   }
   Args a;
@@ -425,16 +644,20 @@ cudaError_t launch_impl(const GemmProblem& p, cudaStream_t stream, int sms) {
   a.N = p.N;
   a.K = p.K;
   a.G = p.G;
-  a.num_m_tiles = (p.M + kBM - 1) / kBM;
+  a.num_m2 = (p.M + kPairM - 1) / kPairM;
   const int num_n_tiles = (p.N + kBN - 1) / kBN;
-  a.num_tiles = a.num_m_tiles * num_n_tiles;
+  a.num_tiles = a.num_m2 * num_n_tiles;
+  a.k_stages = k_stages;
+  a.slots_per_tile = (k_stages + kStagesPerSlot - 1) / kStagesPerSlot;
+  a.qw = p.qw;
   a.s_a = p.s_a;
+  a.s_w = p.s_w;
   a.bias = p.bias;
   a.y = static_cast<__nv_bfloat16*>(p.y);
   a.partials = p.partials;
   a.status = p.status;
-  const int grid = a.num_tiles < sms ? a.num_tiles : sms;
-  w4a4_gemm_kernel<kExport><<<grid, kThreads, kSmemBytes, stream>>>(tmA, tmB, tmS, a);
+  const int pairs = a.num_tiles < max_pairs[kExport] ? a.num_tiles : max_pairs[kExport];
+  w4a4_gemm_kernel<kExport><<<2 * pairs, kThreads, kSmemBytes, stream>>>(tmA, a);
   return cudaGetLastError();
 }
 

@@ -25,9 +25,10 @@ constexpr size_t kNoAllocScratchBytes = JQ_NOALLOC_MAX_SCRATCH_BYTES;
 constexpr int kMaxDevices = 64;
 constexpr int64_t kMaxK = 262016;
 
-// The scratch: the E4M3 operand image of the activations, M*K bytes.  The expansion kernel of
-// the same call writes every byte the GEMM later reads (rows past M are never read: the GEMM's
-// tensor map stops at M and fills out-of-range rows with zeros), so no byte has to start at zero.
+// The scratch: the E4M3 operand image of the activations, whole 128-row tiles of K bytes.  The
+// expansion kernel of the same call writes every row below M; rows past M in the last tile are
+// read by the GEMM but only feed accumulator rows that are never stored, so no byte of the array
+// has to start at zero.
 static __device__ __align__(256) uint8_t g_noalloc_scratch[kNoAllocScratchBytes];
 
 struct NoAllocDevice {
@@ -79,7 +80,9 @@ extern "C" jq_status jq_w4a4_linear_noalloc(const uint8_t* q, const float* s_a, 
   if (!aligned16(q) || !aligned16(s_a) || !aligned16(qw) || !aligned16(s_w) || !aligned16(y_bf16) ||
       (bias != nullptr && !aligned16(bias)))
     return JQ_ERR_MISALIGNED;
-  if (static_cast<uint64_t>(M) * static_cast<uint64_t>(K) > kNoAllocScratchBytes) return JQ_ERR_WORKSPACE;
+  // the operand image covers whole 128-row tiles
+  if ((static_cast<uint64_t>(M) + 127) / 128 * 128 * static_cast<uint64_t>(K) > kNoAllocScratchBytes)
+    return JQ_ERR_WORKSPACE;
   const NoAllocDevice* d = noalloc_device();
   if (d == nullptr) return JQ_ERR_UNSUPPORTED;
   cudaStream_t s = static_cast<cudaStream_t>(stream);

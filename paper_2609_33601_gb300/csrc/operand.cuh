@@ -23,15 +23,16 @@ namespace jq {
 
 // 8 packed nibbles (one 32-bit word, elements e0..e7) -> 8 operand bytes in operand order:
 // .x = bytes for e0,e2,e4,e6 and .y = bytes for e1,e3,e5,e7.
-// Per byte lane with nibble n (two's complement): t = n >> 3 (the sign), and
-// (n ^ (t * 0x8F)) + t  maps n < 8 to n and n >= 8 to 0x80 | (16 - n): the sign-magnitude byte.
-// No carry crosses a byte lane (every intermediate lane value stays below 0x90).
+// Per nibble n (two's complement, sign s = n >> 3): |q| = ((n & 7) ^ 7s) + s, computed for all
+// eight nibbles at once (the largest magnitude, 8, still fits a nibble, so no carry crosses
+// nibbles); then the magnitudes are spread to bytes and each sign lands on bit 7 of its byte.
 __device__ __forceinline__ uint2 nib8_to_operand(uint32_t w) {
-  const uint32_t te = (w >> 3) & 0x01010101u;
-  const uint32_t to = (w >> 7) & 0x01010101u;
-  const uint32_t ve = (w & 0x0F0F0F0Fu) ^ (te * 0x8Fu);
-  const uint32_t vo = ((w >> 4) & 0x0F0F0F0Fu) ^ (to * 0x8Fu);
-  return make_uint2(ve + te, vo + to);
+  const uint32_t s = (w >> 3) & 0x11111111u;                  // sign of each nibble, at its bit 0
+  const uint32_t s8 = s << 3;                                 // the same sign at the nibble's bit 3
+  const uint32_t mag = ((w & 0x77777777u) ^ (s8 - s)) + s;     // eight magnitudes in [0, 8]
+  const uint32_t lo = (mag & 0x0F0F0F0Fu) | ((s << 7) & 0xF0F0F0F0u);  // even elements
+  const uint32_t hi = ((mag >> 4) & 0x0F0F0F0Fu) | (s8 & 0xF0F0F0F0u);  // odd elements
+  return make_uint2(lo, hi);
 }
 
 // 32 packed codes (16 bytes) -> 32 operand bytes (two 16-byte chunks).
@@ -40,6 +41,26 @@ __device__ __forceinline__ void nib32_to_operand(uint4 p, uint4& lo, uint4& hi) 
   const uint2 c = nib8_to_operand(p.z), d = nib8_to_operand(p.w);
   lo = make_uint4(a.x, a.y, b.x, b.y);
   hi = make_uint4(c.x, c.y, d.x, d.y);
+}
+
+// A-operand image (the GEMM's activation operand in global memory): for every 128-row tile
+// mt and every 128-element K stage kb, one contiguous 16 KB block that is byte for byte the
+// shared-memory image the tensor core reads -- 128 rows of 128 operand bytes in the 128-byte
+// swizzle (16-byte chunk c of row r at chunk position c ^ (r % 8), 8-row atoms of 1024 bytes).
+// Blocks are ordered (mt, kb), so consecutive K stages of a tile are adjacent and one bulk copy
+// can fetch several.  Rows past M in the last tile are never written and never used (each output
+// row depends only on its own operand row).
+constexpr uint32_t kImageRows = 128;
+constexpr uint32_t kImageStageK = 128;
+constexpr uint32_t kImageBlockBytes = kImageRows * kImageStageK;  // 16 KB
+
+// Byte offset of the 16-byte operand chunk that holds K positions 16*c16 .. 16*c16+15 of stage
+// kb for row `row` of the operand.
+__host__ __device__ __forceinline__ uint64_t image_chunk_offset(int64_t row, uint32_t kb, uint32_t c16,
+                                                               uint32_t k_stages) {
+  const uint64_t mt = static_cast<uint64_t>(row) / kImageRows;
+  const uint32_t r = static_cast<uint32_t>(row % kImageRows);
+  return (mt * k_stages + kb) * kImageBlockBytes + (r >> 3) * 1024u + (r & 7u) * 128u + ((c16 ^ (r & 7u)) << 4);
 }
 
 // Factor that turns an fp32 sum of operand products back into the integer partial.

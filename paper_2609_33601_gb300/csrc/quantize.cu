@@ -89,17 +89,21 @@ __device__ __forceinline__ void quantize32(const float (&x)[32], float s, uint32
   }
 }
 
+// 32 codes of one row starting at K index `col` (a multiple of 32): packed codes go to the
+// row-major [rows, K/2] array; operand bytes go to the A-operand image (operand.cuh).
 template <bool kOperand>
-__device__ __forceinline__ void store32(uint8_t* out_row, int64_t col, const uint32_t (&pk)[4]) {
+__device__ __forceinline__ void store32(uint8_t* out, int64_t row, int64_t col, int64_t K, const uint32_t (&pk)[4]) {
   const uint4 p = make_uint4(pk[0], pk[1], pk[2], pk[3]);
   if constexpr (kOperand) {
     uint4 lo, hi;
     nib32_to_operand(p, lo, hi);
-    uint4* dst = reinterpret_cast<uint4*>(out_row + col);
-    dst[0] = lo;
-    dst[1] = hi;
+    const uint32_t k_stages = static_cast<uint32_t>(K / kImageStageK);
+    const uint32_t kb = static_cast<uint32_t>(col / kImageStageK);
+    const uint32_t c16 = static_cast<uint32_t>((col % kImageStageK) / 16);
+    *reinterpret_cast<uint4*>(out + image_chunk_offset(row, kb, c16, k_stages)) = lo;
+    *reinterpret_cast<uint4*>(out + image_chunk_offset(row, kb, c16 + 1, k_stages)) = hi;
   } else {
-    *reinterpret_cast<uint4*>(out_row + col / 2) = p;
+    *reinterpret_cast<uint4*>(out + row * (K / 2) + col / 2) = p;
   }
 }
 
@@ -112,7 +116,6 @@ __global__ void __launch_bounds__(256) quantize_groups_kernel(const In* __restri
   const int64_t chunks_per_row = K / 32;
   const int64_t total = M * chunks_per_row;
   const int64_t ng = K / (32 * L);
-  const int64_t out_ld = kOperand ? K : K / 2;
   for (int64_t c = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; c - (threadIdx.x & 31) < total;
        c += (int64_t)gridDim.x * blockDim.x) {
     const bool valid = c < total;
@@ -132,7 +135,7 @@ __global__ void __launch_bounds__(256) quantize_groups_kernel(const In* __restri
     if (valid) {
       uint32_t pk[4];
       quantize32(v, s, pk);
-      store32<kOperand>(out + row * out_ld, col, pk);
+      store32<kOperand>(out, row, col, K, pk);
       if ((threadIdx.x & (L - 1)) == 0) {
         const int64_t g = col / (32 * L);
         if constexpr (kScaleT) scales[g * M + row] = s;
@@ -149,7 +152,6 @@ __global__ void __launch_bounds__(128) quantize_rows_kernel(const In* __restrict
                                                             int64_t ldx, uint8_t* __restrict__ out,
                                                             float* __restrict__ scales) {
   __shared__ float red[4];
-  const int64_t out_ld = kOperand ? K : K / 2;
   for (int64_t row = blockIdx.x; row < M; row += gridDim.x) {
     const In* xr = x + row * ldx;
     float a = 0.0f;
@@ -170,7 +172,7 @@ __global__ void __launch_bounds__(128) quantize_rows_kernel(const In* __restrict
       load32(xr + col, v);
       uint32_t pk[4];
       quantize32(v, s, pk);
-      store32<kOperand>(out + row * out_ld, col, pk);
+      store32<kOperand>(out, row, col, K, pk);
     }
     if (threadIdx.x == 0) {
       if constexpr (kScaleT) scales[row] = s;  // [1, M]
@@ -179,16 +181,22 @@ __global__ void __launch_bounds__(128) quantize_rows_kernel(const In* __restrict
   }
 }
 
-// Packed codes [rows, K/2] -> operand bytes [rows, K] (16 bytes in, 32 bytes out per thread).
-__global__ void __launch_bounds__(256) expand_operand_kernel(const uint8_t* __restrict__ packed,
-                                                             int64_t chunks, uint8_t* __restrict__ op) {
+// Packed codes [rows, K/2] -> the A-operand image (16 bytes in, 32 bytes out per thread).
+__global__ void __launch_bounds__(256) expand_operand_kernel(const uint8_t* __restrict__ packed, int64_t rows,
+                                                             int64_t K, uint8_t* __restrict__ image) {
+  const int64_t per_row = K / 32;
+  const int64_t chunks = rows * per_row;
+  const uint32_t k_stages = static_cast<uint32_t>(K / kImageStageK);
   for (int64_t c = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; c < chunks; c += (int64_t)gridDim.x * blockDim.x) {
+    const int64_t row = c / per_row;
+    const int64_t col = (c % per_row) * 32;
     const uint4 p = __ldg(reinterpret_cast<const uint4*>(packed) + c);
     uint4 lo, hi;
     nib32_to_operand(p, lo, hi);
-    uint4* dst = reinterpret_cast<uint4*>(op) + 2 * c;
-    dst[0] = lo;
-    dst[1] = hi;
+    const uint32_t kb = static_cast<uint32_t>(col / kImageStageK);
+    const uint32_t c16 = static_cast<uint32_t>((col % kImageStageK) / 16);
+    *reinterpret_cast<uint4*>(image + image_chunk_offset(row, kb, c16, k_stages)) = lo;
+    *reinterpret_cast<uint4*>(image + image_chunk_offset(row, kb, c16 + 1, k_stages)) = hi;
   }
 }
 
@@ -240,7 +248,7 @@ cudaError_t launch_expand_operand(const uint8_t* packed, int64_t rows, int64_t K
                                   int sms) {
   const int64_t chunks = rows * (K / 32);
   if (chunks == 0) return cudaSuccess;
-  expand_operand_kernel<<<grid_for(chunks, 256, sms), 256, 0, stream>>>(packed, chunks, op);
+  expand_operand_kernel<<<grid_for(chunks, 256, sms), 256, 0, stream>>>(packed, rows, K, op);
   return cudaGetLastError();
 }
 

@@ -53,7 +53,7 @@ def test_workspace_size(lib):
     f.restype = ctypes.c_size_t
     assert f(1024, 12288, 4096, 128, 0) == 1024 * 4096
     assert f(1024, 12288, 4096, 128, 1) == 1024 * 4096 + 1024 * 32 * 4
-    assert f(3, 8, 256, 64, 0) == 768  # rounded up to 256
+    assert f(3, 8, 256, 64, 0) == 128 * 256  # the operand image covers whole 128-row tiles
     assert f(0, 8, 256, 64, 0) == 0
 
 

@@ -68,7 +68,7 @@ def test_noalloc_rejects_problems_beyond_its_scratch():
     small = torch.zeros(256, dtype=torch.uint8, device="cuda")
     p = ctypes.c_void_p(small.data_ptr())
     K = 4096
-    M = MAX_SCRATCH // K + 1  # one row too many
+    M = MAX_SCRATCH // K + 1  # one 128-row tile too many
     rc = lib.jq_w4a4_linear_noalloc(p, p, p, p, None, p, M, 8, K, 128, None)
     assert rc == JQ_ERR_WORKSPACE
     torch.cuda.synchronize()
