@@ -52,15 +52,14 @@ constexpr int kBK = 128;
 constexpr int kStagesPerSlot = 2;   // K stages per ring slot (one A transfer, two unpacked B stages)
 constexpr int kSlots = 3;           // operand ring: each slot holds A and B for kStagesPerSlot stages
 constexpr int kThreads = 512;
-constexpr int kWarpProdA = 0, kWarpMma = 1;
+constexpr int kWarpProdA = 0, kWarpMma = 1, kWarpScale = 2;
 constexpr int kUnpackWarp0 = 4, kUnpackThreads = 128;
 constexpr int kUnpackGroups = 2, kUnpackGroupThreads = kUnpackThreads / kUnpackGroups;  // alternate K stages
 constexpr int kUnpackGroupWarps = kUnpackGroupThreads / 32;
 constexpr int kDrainWarp0 = 8, kNumDrainWarps = 8;
-constexpr int kDrainThreads = kNumDrainWarps * 32;
 constexpr int kChunksPerThread = kBNHalf * (kBK / 2) / 16 / kUnpackGroupThreads;  // 8 packed 16-byte chunks
 constexpr uint32_t kTmemCols = 512;  // two 256-column accumulators
-constexpr int kRegsCtl = 40, kRegsUnpack = 120, kRegsDrain = 176;
+constexpr int kRegsCtl = 32, kRegsUnpack = 96, kRegsDrain = 192;
 static_assert(4 * 32 * (kRegsCtl + kRegsUnpack + 2 * kRegsDrain) == 65536, "register split must use the launch budget");
 static_assert(kChunksPerThread == 8, "unpack assumes eight chunks per thread per stage");
 
@@ -69,14 +68,23 @@ constexpr uint32_t kSlotABytes = kStagesPerSlot * kOpABytes;  // 32 KB
 constexpr uint32_t kOpBBytes = kBNHalf * kBK;                 // 16 KB per K stage per CTA
 constexpr uint32_t kSlotBBytes = kStagesPerSlot * kOpBBytes;  // 32 KB
 
+// Scale ring: each slot holds the weight scales of kScGroups groups for the tile's 256 columns
+// ([group][column] fp32) and, when they come by TMA, the activation scales of those groups for
+// this CTA's 128 rows ([row][group] fp32).
+constexpr int kScGroups = 4, kScSlots = 4;
+constexpr uint32_t kScSwBytes = kScGroups * kBN * 4;  // 4 KB
+constexpr uint32_t kScSaBytes = kScGroups * kBM * 4;  // 2 KB
+constexpr uint32_t kScSlotBytes = kScSwBytes + kScSaBytes;
+
 constexpr uint32_t kOffA = 0;
 constexpr uint32_t kOffB = kOffA + kSlots * kSlotABytes;
-constexpr uint32_t kOffBar = kOffB + kSlots * kSlotBBytes;
-constexpr uint32_t kNumBars = 2 * kSlots + 4 + 1 + 4;
+constexpr uint32_t kOffSc = kOffB + kSlots * kSlotBBytes;
+constexpr uint32_t kOffBar = kOffSc + kScSlots * kScSlotBytes;
+constexpr uint32_t kNumBars = 2 * kSlots + 4 + 1 + 2 * kScSlots;
 constexpr uint32_t kOffMisc = kOffBar + kNumBars * 8;
-constexpr uint32_t kOffSw = (kOffMisc + 16 + 127) & ~127u;  // two slots of kBN fp32 weight scales
-constexpr uint32_t kSmemBytes = kOffSw + 2 * kBN * 4;
-static_assert(kOffBar % 8 == 0 && kOffMisc % 8 == 0 && kOffSw % 16 == 0, "mbarriers need 8 bytes, v4 loads 16");
+constexpr uint32_t kSmemBytes = kOffMisc + 16;
+static_assert(kOffBar % 8 == 0 && kOffMisc % 8 == 0, "mbarriers need 8-byte alignment");
+static_assert(kOffSc % 128 == 0 && kScSlotBytes % 128 == 0 && kScSwBytes % 128 == 0, "TMA destinations need 128 bytes");
 static_assert(kOffA % 1024 == 0 && kOffB % 1024 == 0 && kOpABytes % 1024 == 0 && kOpBBytes % 1024 == 0,
               "128B-swizzled operand slots need 1024-byte alignment");
 // The rings need a 1024-byte aligned base (128B swizzle atoms); the dynamic shared memory
@@ -86,6 +94,8 @@ static_assert(kSmemBytes <= 232448, "shared memory budget");
 struct Args {
   int M, N, K, G;
   int num_m2, num_tiles, k_stages, slots_per_tile;
+  int groups, sc_boxes;  // K / G, and scale-ring slots per tile (ceil(groups / kScGroups))
+  int sa_tma;            // activation scales come through the scale ring (groups % 4 == 0)
   const uint8_t* qw;
   const float* s_a;
   const float* s_w;
@@ -98,7 +108,7 @@ struct Args {
 struct Bars {
   uint64_t *full, *empty;  // operand ring: A and B of a slot arrive on full, leave on empty
   uint64_t *acc_full, *acc_empty, *mma_done;
-  uint64_t *sw_full, *sw_empty;  // weight-scale slots of the drain (two groups)
+  uint64_t *sc_full, *sc_empty;  // scale ring
 };
 
 struct Pair {
@@ -118,172 +128,211 @@ __device__ __forceinline__ void drain_wait(uint64_t* bar, uint32_t parity, uint3
 }
 
 // ------------------------------------------------------------------ drain + epilogue
-template <bool kExport>
-__device__ __forceinline__ void drain_role(const Args& args, const Pair& pr, uint32_t tmem_base, const Bars& b,
-                                           float* sw_smem, volatile int* abort_flag) {
+// Export path (jq_w4a4_group_partials): each thread owns one TMEM lane (row) and 128 columns
+// (32x32b loads) and writes the exact integer partials of every group.
+__device__ __forceinline__ void drain_export(const Args& args, const Pair& pr, uint32_t tmem_base, const Bars& b,
+                                             volatile int* abort_flag) {
   const uint32_t warp = warp_id(), lane = lane_id();
-  const int M = args.M, N = args.N;
-  const int groups = args.K / args.G;
+  const int M = args.M, N = args.N, groups = args.groups;
   const uint32_t quarter = warp & 3u, half = (warp - kDrainWarp0) >> 2;
   const uint32_t lane_base = (quarter * 32u) << 16;
-  const uint32_t dt = threadIdx.x - kDrainWarp0 * 32;  // 0..255
-  const bool loader = dt < kBN / 4;                     // 64 threads move 16 bytes of scales each
   uint32_t chunk_it = 0;
   bool ok = true;
-  if (!kExport && loader && pr.cluster < args.num_tiles) {  // group 0 of the first tile -> slot 0
-    const int ncol = (pr.cluster / args.num_m2) * kBN + 4 * (int)dt;
-    float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
-    if (ncol < N) v = __ldg(reinterpret_cast<const float4*>(args.s_w + ncol));
-    *reinterpret_cast<float4*>(sw_smem + 4 * dt) = v;
-    mbar_arrive(&b.sw_full[0]);
-  }
   for (int tile = pr.cluster; ok && tile < args.num_tiles; tile += pr.num_clusters) {
     const int mt2 = tile % args.num_m2, nt = tile / args.num_m2;
-    const int row = mt2 * kPairM + (int)pr.rank * kBM + quarter * 32 + lane;
+    const int row = mt2 * kPairM + (int)pr.rank * kBM + (int)(quarter * 32u + lane);
     const int col0 = nt * kBN + half * 128;
     const bool row_ok = row < M;
-    const float* sa_row = kExport ? nullptr : args.s_a + (int64_t)(row_ok ? row : 0) * groups;
+    for (int g = 0; g < groups; ++g) {
+      const uint32_t ab = chunk_it & 1u;
+      // Warp-collective tcgen05.ld follows: the whole warp proceeds or none of it.
+      ok = __all_sync(0xffffffffu, mbar_wait(&b.acc_full[ab], (chunk_it >> 1) & 1u, abort_flag, args.status));
+      if (!ok) break;
+      tc_fence_after();
+      const uint32_t taddr = tmem_base + lane_base + ab * kBN + half * 128;
+#pragma unroll 1
+      for (int cc = 0; cc < 4; ++cc) {
+        uint32_t r[32];
+        tmem_ld32(taddr + cc * 32, r);
+        tmem_ld_wait();
+        if (row_ok) {
+#pragma unroll
+          for (int j = 0; j < 32; ++j) {
+            const int col = col0 + cc * 32 + j;
+            if (col < N)
+              args.partials[((int64_t)row * N + col) * groups + g] =
+                  static_cast<int32_t>(__uint_as_float(r[j]) * kOperandUnitInv);
+          }
+        }
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive_remote_cta(leader_bar(&b.acc_empty[ab]));
+      ++chunk_it;
+    }
+  }
+}
+
+// Linear path.  Warp w (drain index d = w - 8) owns TMEM lanes 32*(w%4).. (32 rows) and columns
+// 128*(d/4).. of each accumulator, read with the 16x256b shape: thread t holds rows
+// t/4 + {0, 8, 16, 24} of those 32 and columns 8j + 2(t%4) + {0, 1}, j = 0..15.  So a thread needs
+// only 32 weight scales and 4 activation scales per group; it loads all of them at the start of
+// the group (the tensor core's operand reads starve shared-memory loads issued one chunk ahead of
+// their use, but not loads issued a group ahead).
+__device__ __forceinline__ void drain_linear(const Args& args, const Pair& pr, uint32_t tmem_base, const Bars& b,
+                                             uint8_t* sSc, volatile int* abort_flag) {
+  const uint32_t warp = warp_id(), lane = lane_id();
+  const int M = args.M, N = args.N, groups = args.groups;
+  const uint32_t quarter = warp & 3u, half = (warp - kDrainWarp0) >> 2;
+  const uint32_t tq = lane & 3u, t4 = lane >> 2;
+  uint32_t chunk_it = 0, sc_it = 0;
+  bool ok = true;
+  for (int tile = pr.cluster; ok && tile < args.num_tiles; tile += pr.num_clusters) {
+    const int mt2 = tile % args.num_m2, nt = tile / args.num_m2;
+    const int row0 = mt2 * kPairM + (int)pr.rank * kBM + (int)(quarter * 32u + t4);  // + 8 * rr
+    const int col0 = nt * kBN + half * 128 + 2 * (int)tq;                              // + 8 * j
+    // y[4 * j + rr * ... ] layout: y[(rr * 16 + j) * 2 + e], rr = row index 0..3 (offset 8 * rr)
     float y[128];
 #pragma unroll
     for (int i = 0; i < 128; ++i) y[i] = 0.0f;
-    float sa_next = (!kExport && row_ok) ? __ldg(sa_row) : 0.0f;
     for (int g = 0; g < groups; ++g) {
       const uint32_t ab = chunk_it & 1u;
-      const float sa = sa_next;
-      if (!kExport && row_ok && g + 1 < groups) sa_next = __ldg(sa_row + g + 1);
-      // The weight scales of the next group this CTA drains (the next group of this tile, or
-      // group 0 of the next tile) go to registers now and to shared memory after this group.
-      bool have_next = false;
-      float4 sw_next = make_float4(0.f, 0.f, 0.f, 0.f);
-      if (!kExport && loader) {
-        const int next_tile = tile + pr.num_clusters;
-        have_next = g + 1 < groups || next_tile < args.num_tiles;
-        const int ng = g + 1 < groups ? g + 1 : 0;
-        const int ncol = (g + 1 < groups ? nt : next_tile / args.num_m2) * kBN + 4 * (int)dt;
-        if (have_next && ncol < N) sw_next = __ldg(reinterpret_cast<const float4*>(args.s_w + (int64_t)ng * N + ncol));
+      const int gi = g % kScGroups;
+      const uint32_t sslot = sc_it % kScSlots;
+      if (gi == 0) {
+        ok = __all_sync(0xffffffffu, mbar_wait(&b.sc_full[sslot], ring_parity(sc_it, kScSlots), abort_flag, args.status));
+        if (!ok) break;
+      }
+      const uint8_t* slot = sSc + sslot * kScSlotBytes;
+      const float* sws = reinterpret_cast<const float*>(slot) + gi * kBN + half * 128 + 2 * tq;
+      float2 w[16];
+#pragma unroll
+      for (int j = 0; j < 16; ++j) w[j] = *reinterpret_cast<const float2*>(sws + 8 * j);
+      float f[4];
+#pragma unroll
+      for (int rr = 0; rr < 4; ++rr) {
+        const int row = row0 + 8 * rr;
+        float sa;
+        if (args.sa_tma)
+          sa = reinterpret_cast<const float*>(slot + kScSwBytes)[(quarter * 32u + t4 + 8u * rr) * kScGroups + gi];
+        else
+          sa = row < M ? __ldg(args.s_a + (int64_t)row * groups + g) : 0.0f;
+        f[rr] = sa;
       }
       // Warp-collective tcgen05.ld follows: the whole warp proceeds or none of it (a timeout in
       // one lane must not leave the others in an aligned instruction).
       ok = __all_sync(0xffffffffu, mbar_wait(&b.acc_full[ab], (chunk_it >> 1) & 1u, abort_flag, args.status));
       if (!ok) break;
       tc_fence_after();
-      const uint32_t taddr = tmem_base + lane_base + ab * kBN + half * 128;
-      if constexpr (kExport) {
-#pragma unroll 1
-        for (int cc = 0; cc < 4; ++cc) {
-          uint32_t r[32];
-          tmem_ld32(taddr + cc * 32, r);
+      const uint32_t taddr = tmem_base + ((quarter * 32u) << 16) + ab * kBN + half * 128;
+      // The two arithmetic forms below are both exact-partial * scales in fp32; the slow one is
+      // needed when s_a * 2^18 would overflow.  The choice is made for the whole warp: both
+      // paths issue warp-collective tcgen05.ld / __syncwarp, which every lane must reach.
+      bool finite = true;
+#pragma unroll
+      for (int rr = 0; rr < 4; ++rr) finite = finite && (f[rr] * kOperandUnitInv <= FLT_MAX);
+      finite = __all_sync(0xffffffffu, finite);
+      if (finite) {
+#pragma unroll
+        for (int rr = 0; rr < 4; ++rr) f[rr] *= kOperandUnitInv;  // s_a * 2^18
+#pragma unroll
+        for (int j = 0; j < 16; ++j) {  // 8 columns per step
+          uint32_t r0[4], r1[4];        // lanes 0-15 and 16-31 of the quarter
+          tmem_ld16x256b_x1(taddr + j * 8, r0);
+          tmem_ld16x256b_x1(taddr + (16u << 16) + j * 8, r1);
           tmem_ld_wait();
-          if (row_ok) {
-#pragma unroll
-            for (int j = 0; j < 32; ++j) {
-              const int col = col0 + cc * 32 + j;
-              if (col < N)
-                args.partials[((int64_t)row * N + col) * groups + g] =
-                    static_cast<int32_t>(__uint_as_float(r[j]) * kOperandUnitInv);
-            }
-          }
-        }
-        tc_fence_before();
-        __syncwarp();
-        if (lane == 0) mbar_arrive_remote_cta(leader_bar(&b.acc_empty[ab]));
-      } else {
-        const uint32_t cslot = chunk_it & 1u;
-        ok = __all_sync(0xffffffffu, mbar_wait(&b.sw_full[cslot], (chunk_it >> 1) & 1u, abort_flag, args.status));
-        if (!ok) break;
-        const float f = sa * kOperandUnitInv;  // s_a * 2^18
-        const bool f_finite = f <= FLT_MAX;
-        const float2 f2 = make_float2(f, f);
-        const float* sws = sw_smem + cslot * kBN + half * 128;
-        // y[c..c+7] += (partial * s_w) * f for one 8-column chunk already in registers
-        auto accumulate = [&](const uint32_t(&r)[8], int cc) {
-          if (f_finite) {
-#pragma unroll
-            for (int j = 0; j < 8; j += 4) {
-              const float4 w4 = ld_shared_f4(sws + cc * 8 + j);
-              float* yy = y + cc * 8 + j;
-              const float2 t0 = __fmul2_rn(make_float2(__uint_as_float(r[j]), __uint_as_float(r[j + 1])),
-                                           make_float2(w4.x, w4.y));
-              const float2 t1 = __fmul2_rn(make_float2(__uint_as_float(r[j + 2]), __uint_as_float(r[j + 3])),
-                                           make_float2(w4.z, w4.w));
-              const float2 y0 = __ffma2_rn(t0, f2, make_float2(yy[0], yy[1]));
-              const float2 y1 = __ffma2_rn(t1, f2, make_float2(yy[2], yy[3]));
-              yy[0] = y0.x;
-              yy[1] = y0.y;
-              yy[2] = y1.x;
-              yy[3] = y1.y;
-            }
-          } else {  // |s_a| > 2^110: apply 2^18 to the exact partial first so nothing overflows
-#pragma unroll
-            for (int j = 0; j < 8; ++j)
-              y[cc * 8 + j] = fmaf((__uint_as_float(r[j]) * kOperandUnitInv) * sa, sws[cc * 8 + j], y[cc * 8 + j]);
-          }
-        };
-        // 16 chunks of 8 columns; the load of chunk c+1 is in flight while chunk c is scaled
-        constexpr int kChunks = 16;
-        uint32_t ra[8], rb[8];
-        tmem_ld8(taddr, ra);
-        tmem_ld_wait();
-#pragma unroll
-        for (int cc = 0; cc < kChunks; cc += 2) {
-          tmem_ld8(taddr + (cc + 1) * 8, rb);
-          accumulate(ra, cc);
-          tmem_ld_wait();
-          if (cc + 2 < kChunks) {
-            tmem_ld8(taddr + (cc + 2) * 8, ra);
-          } else {  // every column of this accumulator is in registers: hand it back
+          if (j == 15) {  // every column of this accumulator is in registers: hand it back
             tc_fence_before();
             __syncwarp();
             if (lane == 0) mbar_arrive_remote_cta(leader_bar(&b.acc_empty[ab]));
           }
-          accumulate(rb, cc + 1);
-          if (cc + 2 < kChunks) tmem_ld_wait();
+#pragma unroll
+          for (int rr = 0; rr < 4; ++rr) {  // r0: rows +0 / +8; r1: rows +16 / +24
+            const uint32_t* r = rr < 2 ? r0 : r1;
+            const int e = 2 * (rr & 1);
+            const float2 t = __fmul2_rn(make_float2(__uint_as_float(r[e]), __uint_as_float(r[e + 1])), w[j]);
+            float* yy = y + (rr * 16 + j) * 2;
+            const float2 v = __ffma2_rn(t, make_float2(f[rr], f[rr]), make_float2(yy[0], yy[1]));
+            yy[0] = v.x;
+            yy[1] = v.y;
+          }
         }
-        mbar_arrive(&b.sw_empty[cslot]);
-        // publish the scales prefetched at the top of this group into the other slot
-        if (loader && have_next) {
-          const uint32_t nslot = cslot ^ 1u;
-          ok = __all_sync(0xffffffffu,  // loader warps are whole warps (threads 0..63 of the drain)
-                          mbar_wait(&b.sw_empty[nslot], ring_parity(chunk_it + 1, 2) ^ 1u, abort_flag, args.status));
-          if (!ok) break;
-          *reinterpret_cast<float4*>(sw_smem + nslot * kBN + 4 * dt) = sw_next;
-          mbar_arrive(&b.sw_full[nslot]);
+      } else {  // some |s_a| > 2^110: apply 2^18 to the exact partials first so nothing overflows
+#pragma unroll
+        for (int j = 0; j < 16; ++j) {
+          uint32_t r0[4], r1[4];
+          tmem_ld16x256b_x1(taddr + j * 8, r0);
+          tmem_ld16x256b_x1(taddr + (16u << 16) + j * 8, r1);
+          tmem_ld_wait();
+          if (j == 15) {
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive_remote_cta(leader_bar(&b.acc_empty[ab]));
+          }
+#pragma unroll
+          for (int rr = 0; rr < 4; ++rr) {
+            const uint32_t* r = rr < 2 ? r0 : r1;
+            const int e = 2 * (rr & 1);
+            float* yy = y + (rr * 16 + j) * 2;
+            yy[0] = fmaf((__uint_as_float(r[e]) * kOperandUnitInv) * f[rr], w[j].x, yy[0]);
+            yy[1] = fmaf((__uint_as_float(r[e + 1]) * kOperandUnitInv) * f[rr], w[j].y, yy[1]);
+          }
         }
+      }
+      if (gi == kScGroups - 1 || g == groups - 1) {  // done with this scale slot
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&b.sc_empty[sslot]);
+        ++sc_it;
       }
       ++chunk_it;
     }
     if (!ok) break;
-    if constexpr (!kExport) {
-      if (row_ok) {
-        __nv_bfloat16* yrow = args.y + (int64_t)row * N;
+    // + bias, round to bf16, store: each (row, j) pair of columns is 4 bytes
 #pragma unroll
-        for (int i = 0; i < 16; ++i) {
-          const int col = col0 + 8 * i;
-          if (col < N) {
-            float v[8];
+    for (int j = 0; j < 16; ++j) {
+      const int col = col0 + 8 * j;
+      if (col < N) {
+        float2 bj = make_float2(0.f, 0.f);
+        if (args.bias != nullptr) bj = __ldg(reinterpret_cast<const float2*>(args.bias + col));
 #pragma unroll
-            for (int j = 0; j < 8; ++j) v[j] = y[8 * i + j];
-            if (args.bias != nullptr) {
-              const float4 b0 = __ldg(reinterpret_cast<const float4*>(args.bias + col));
-              const float4 b1 = __ldg(reinterpret_cast<const float4*>(args.bias + col + 4));
-              v[0] += b0.x; v[1] += b0.y; v[2] += b0.z; v[3] += b0.w;
-              v[4] += b1.x; v[5] += b1.y; v[6] += b1.z; v[7] += b1.w;
-            }
-            uint4 out;
-            __nv_bfloat162 t0 = __floats2bfloat162_rn(v[0], v[1]);
-            __nv_bfloat162 t1 = __floats2bfloat162_rn(v[2], v[3]);
-            __nv_bfloat162 t2 = __floats2bfloat162_rn(v[4], v[5]);
-            __nv_bfloat162 t3 = __floats2bfloat162_rn(v[6], v[7]);
-            out.x = *reinterpret_cast<uint32_t*>(&t0);
-            out.y = *reinterpret_cast<uint32_t*>(&t1);
-            out.z = *reinterpret_cast<uint32_t*>(&t2);
-            out.w = *reinterpret_cast<uint32_t*>(&t3);
-            *reinterpret_cast<uint4*>(yrow + col) = out;
+        for (int rr = 0; rr < 4; ++rr) {
+          const int row = row0 + 8 * rr;
+          if (row < M) {
+            const float* yy = y + (rr * 16 + j) * 2;
+            __nv_bfloat162 v = __floats2bfloat162_rn(yy[0] + bj.x, yy[1] + bj.y);
+            *reinterpret_cast<__nv_bfloat162*>(args.y + (int64_t)row * N + col) = v;
           }
         }
       }
     }
   }
+}
+
+// ------------------------------------------------------------------ scale producer
+// Streams the scales the drain needs into the scale ring, kScGroups groups per slot: one TMA box
+// of weight scales (kScGroups rows of 256 columns) and, when aligned, one of this CTA's
+// activation scales (128 rows of kScGroups groups).  Boxes past the tensors' ends read zeros.
+__device__ __forceinline__ void scale_producer(const Args& args, const Pair& pr, const CUtensorMap* tmSW,
+                                               const CUtensorMap* tmSA, uint8_t* sSc, const Bars& b,
+                                               volatile int* abort_flag) {
+  const uint32_t bytes = kScSwBytes + (args.sa_tma ? kScSaBytes : 0u);
+  uint32_t it = 0;
+  bool ok = true;
+  for (int tile = pr.cluster; ok && tile < args.num_tiles; tile += pr.num_clusters) {
+    const int mt2 = tile % args.num_m2, nt = tile / args.num_m2;
+    const int row0 = mt2 * kPairM + (int)pr.rank * kBM;
+    for (int bi = 0; bi < args.sc_boxes; ++bi) {
+      const uint32_t s = it % kScSlots;
+      if (!(ok = mbar_wait(&b.sc_empty[s], ring_parity(it, kScSlots) ^ 1u, abort_flag, args.status))) break;
+      uint8_t* slot = sSc + s * kScSlotBytes;
+      mbar_arrive_expect_tx(&b.sc_full[s], bytes);
+      tma_load_2d(slot, tmSW, &b.sc_full[s], nt * kBN, bi * kScGroups);
+      if (args.sa_tma) tma_load_2d(slot + kScSwBytes, tmSA, &b.sc_full[s], bi * kScGroups, row0);
+      ++it;
+    }
+  }
+  for (uint32_t i = (it > kScSlots ? it - kScSlots : 0); i < it; ++i)
+    drain_wait(&b.sc_full[i % kScSlots], ring_parity(i, kScSlots), args.status);
 }
 
 // ------------------------------------------------------------------ A producer
@@ -500,7 +549,8 @@ __device__ __forceinline__ void unpack_role(const Args& args, const Pair& pr, ui
 
 template <bool kExport>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
-    w4a4_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const Args args) {
+    w4a4_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmSW,
+                     const __grid_constant__ CUtensorMap tmSA, const Args args) {
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   if ((smem_u32(smem_raw) & 1023u) != 0) {  // uniform across the grid: nothing has been touched yet
     if (threadIdx.x == 0 && args.status != nullptr) atomicExch(args.status, (uint32_t)kDevSmemAlign);
@@ -516,9 +566,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
   b.acc_full = b.empty + kSlots;
   b.acc_empty = b.acc_full + 2;
   b.mma_done = b.acc_empty + 2;
-  b.sw_full = b.mma_done + 1;
-  b.sw_empty = b.sw_full + 2;
-  float* sw_smem = reinterpret_cast<float*>(smem + kOffSw);
+  b.sc_full = b.mma_done + 1;
+  b.sc_empty = b.sc_full + kScSlots;
+  uint8_t* sSc = smem + kOffSc;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + kOffMisc);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + kOffMisc + 4);
 
@@ -538,12 +588,18 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     for (int i = 0; i < 2; ++i) {
       mbar_init(&b.acc_full[i], 1);
       mbar_init(&b.acc_empty[i], 2 * kNumDrainWarps);  // every drain warp of both CTAs
-      mbar_init(&b.sw_full[i], kBN / 4);
-      mbar_init(&b.sw_empty[i], kDrainThreads);
     }
     mbar_init(b.mma_done, 1);
+    for (int i = 0; i < kScSlots; ++i) {
+      mbar_init(&b.sc_full[i], 1);                 // the scale producer's expect_tx
+      mbar_init(&b.sc_empty[i], kNumDrainWarps);  // every drain warp
+    }
     fence_mbar_init();
     tma_prefetch_desc(&tmA);
+    if (!kExport) {
+      tma_prefetch_desc(&tmSW);
+      if (args.sa_tma) tma_prefetch_desc(&tmSA);
+    }
   }
   if (warp == kWarpMma) {
     tmem_alloc_pair(tmem_slot, kTmemCols);
@@ -556,10 +612,13 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
   const uint32_t tmem_base = *tmem_slot;
 
   // Register split per warpgroup (totals the 512 x 128 registers of the launch): producer and
-  // MMA (warps 0-3) 40, unpack (warps 4-7) 120, drain (warps 8-15, 128 running sums) 176.
+  // MMA (warps 0-3) 32, unpack (warps 4-7) 96, drain (warps 8-15, 128 running sums) 192.
   if (warp >= kDrainWarp0) {
     asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;\n" ::"n"(kRegsDrain) : "memory");
-    drain_role<kExport>(args, pr, tmem_base, b, sw_smem, abort_flag);
+    if (kExport)
+      drain_export(args, pr, tmem_base, b, abort_flag);
+    else
+      drain_linear(args, pr, tmem_base, b, sSc, abort_flag);
   } else if (warp >= kUnpackWarp0) {
     asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;\n" ::"n"(kRegsUnpack) : "memory");
     unpack_role(args, pr, sB, b, abort_flag);
@@ -567,6 +626,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;\n" ::"n"(kRegsCtl) : "memory");
     if (warp == kWarpProdA) {
       if (lane == 0) producer_a(args, pr, &tmA, sA, b, abort_flag);
+    } else if (warp == kWarpScale) {
+      if (!kExport && lane == 0) scale_producer(args, pr, &tmSW, &tmSA, sSc, b, abort_flag);
     } else if (warp == kWarpMma && lane == 0) {
       if (pr.rank == 0)
         mma_role(args, pr, tmem_base, sA, sB, b, abort_flag);
@@ -621,6 +682,18 @@ cudaError_t launch_impl(const GemmProblem& p, cudaStream_t stream, int sms) {
   if (!encode_2d(&tmA, CU_TENSOR_MAP_DATA_TYPE_UINT8, p.a_operand, kBK, image_rows, kBK, kBK,
                  kStagesPerSlot * kBM, CU_TENSOR_MAP_SWIZZLE_NONE))
     return cudaErrorInvalidValue;
+  // Scale maps (the export path reads no scales: it passes the A map in their place, unused).
+  const int groups = p.K / p.G;
+  const bool sa_tma = !kExport && groups % kScGroups == 0;
+  CUtensorMap tmSW = tmA, tmSA = tmA;
+  if (!kExport) {
+    if (!encode_2d(&tmSW, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, p.s_w, p.N, groups, (uint64_t)p.N * 4, kBN, kScGroups,
+                   CU_TENSOR_MAP_SWIZZLE_NONE))
+      return cudaErrorInvalidValue;
+    if (sa_tma && !encode_2d(&tmSA, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, p.s_a, groups, p.M, (uint64_t)groups * 4,
+                             kScGroups, kBM, CU_TENSOR_MAP_SWIZZLE_NONE))
+      return cudaErrorInvalidValue;
+  }
   static bool attr_set[2] = {false, false};
   static int max_pairs[2] = {0, 0};
   if (!attr_set[kExport]) {
@@ -649,6 +722,9 @@ cudaError_t launch_impl(const GemmProblem& p, cudaStream_t stream, int sms) {
   a.num_tiles = a.num_m2 * num_n_tiles;
   a.k_stages = k_stages;
   a.slots_per_tile = (k_stages + kStagesPerSlot - 1) / kStagesPerSlot;
+  a.groups = groups;
+  a.sc_boxes = (groups + kScGroups - 1) / kScGroups;
+  a.sa_tma = sa_tma ? 1 : 0;
   a.qw = p.qw;
   a.s_a = p.s_a;
   a.s_w = p.s_w;
@@ -657,7 +733,7 @@ cudaError_t launch_impl(const GemmProblem& p, cudaStream_t stream, int sms) {
   a.partials = p.partials;
   a.status = p.status;
   const int pairs = a.num_tiles < max_pairs[kExport] ? a.num_tiles : max_pairs[kExport];
-  w4a4_gemm_kernel<kExport><<<2 * pairs, kThreads, kSmemBytes, stream>>>(tmA, a);
+  w4a4_gemm_kernel<kExport><<<2 * pairs, kThreads, kSmemBytes, stream>>>(tmA, tmSW, tmSA, a);
   return cudaGetLastError();
 }
 
