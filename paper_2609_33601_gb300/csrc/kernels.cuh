@@ -34,7 +34,27 @@ struct GemmProblem {
 // Device address of the library's status word on the current device, or nullptr.
 uint32_t* device_status_word();
 
+// 2-D tiled tensor map (row-major, `inner` elements per row of `row_bytes`), box
+// box_inner x box_outer; boxes past the ends read zeros.  False if the driver rejects it.
+bool encode_2d(CUtensorMap* map, CUtensorMapDataType dtype, const void* base, uint64_t inner, uint64_t outer,
+               uint64_t row_bytes, uint32_t box_inner, uint32_t box_outer, CUtensorMapSwizzle swizzle);
+
 // Encodes the tensor maps and launches the persistent tcgen05 GEMM.
 cudaError_t launch_w4a4_gemm(const GemmProblem& p, cudaStream_t stream, int sms);
+
+// Few-token linear layer (skinny.cu): reads the packed activation codes directly, needs no
+// workspace.  Used for M <= kSkinnyMaxM.
+constexpr int kSkinnyMaxM = 64;
+struct SkinnyProblem {
+  int M, N, K, G;
+  const uint8_t* q;    // [M, K/2] packed activation codes
+  const float* s_a;    // [M, K/G]
+  const uint8_t* qw;   // [N, K/2] packed weight codes
+  const float* s_w;    // [K/G, N]
+  const float* bias;   // [N] or nullptr
+  void* y;             // bf16 [M, N]
+  uint32_t* status;    // device status word
+};
+cudaError_t launch_w4a4_skinny(const SkinnyProblem& p, cudaStream_t stream, int sms);
 
 }  // namespace jq

@@ -80,6 +80,13 @@ extern "C" jq_status jq_w4a4_linear_noalloc(const uint8_t* q, const float* s_a, 
   if (!aligned16(q) || !aligned16(s_a) || !aligned16(qw) || !aligned16(s_w) || !aligned16(y_bf16) ||
       (bias != nullptr && !aligned16(bias)))
     return JQ_ERR_MISALIGNED;
+  const NoAllocDevice* d0 = nullptr;
+  if (M <= jq::kSkinnyMaxM) {  // few tokens: the weight-streaming kernel needs no scratch at all
+    if ((d0 = noalloc_device()) == nullptr) return JQ_ERR_UNSUPPORTED;
+    jq::SkinnyProblem p{static_cast<int>(M), static_cast<int>(N), static_cast<int>(K), group, q, s_a, qw, s_w, bias,
+                        y_bf16, d0->status};
+    return jq::launch_w4a4_skinny(p, static_cast<cudaStream_t>(stream), d0->sms) == cudaSuccess ? JQ_OK : JQ_ERR_CUDA;
+  }
   // the operand image covers whole 128-row tiles
   if ((static_cast<uint64_t>(M) + 127) / 128 * 128 * static_cast<uint64_t>(K) > kNoAllocScratchBytes)
     return JQ_ERR_WORKSPACE;
