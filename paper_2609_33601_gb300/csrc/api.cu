@@ -136,7 +136,7 @@ jq_status jq_w4a4_linear(const uint8_t* q, const float* s_a, const uint8_t* qw, 
   const DeviceInfo* d = current_device();
   if (d == nullptr) return JQ_ERR_UNSUPPORTED;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
-  if (M <= jq::kSkinnyMaxM) {  // few tokens: the weight-streaming kernel, no workspace needed
+  if (jq::skinny_supports(M, K, group)) {  // few tokens: the weight-streaming kernel, no workspace needed
     jq::SkinnyProblem p{static_cast<int>(M), static_cast<int>(N), static_cast<int>(K), group, q, s_a, qw, s_w, bias,
                         y_bf16, d->status};
     return from_cuda(jq::launch_w4a4_skinny(p, s, d->sms));
@@ -163,7 +163,7 @@ jq_status jq_fused_quant_linear(const void* x_bf16, int64_t ldx, const uint8_t* 
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   uint8_t* a_op = static_cast<uint8_t*>(workspace);
   float* s_a = reinterpret_cast<float*>(a_op + round_up(static_cast<size_t>(M), 128) * static_cast<size_t>(K));
-  if (M <= jq::kSkinnyMaxM) {  // few tokens: packed codes in the workspace, then the weight-streaming kernel
+  if (jq::skinny_supports(M, K, group)) {  // few tokens: packed codes in the workspace, then the weight-streaming kernel
     cudaError_t e = jq::launch_quantize_act(x_bf16, M, K, ldx, group, a_op, s_a, s, d->sms);
     if (e != cudaSuccess) return JQ_ERR_CUDA;
     jq::SkinnyProblem p{static_cast<int>(M), static_cast<int>(N), static_cast<int>(K), group, a_op, s_a, qw, s_w,

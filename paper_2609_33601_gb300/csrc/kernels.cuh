@@ -43,8 +43,14 @@ bool encode_2d(CUtensorMap* map, CUtensorMapDataType dtype, const void* base, ui
 cudaError_t launch_w4a4_gemm(const GemmProblem& p, cudaStream_t stream, int sms);
 
 // Few-token linear layer (skinny.cu): reads the packed activation codes directly, needs no
-// workspace.  Used for M <= kSkinnyMaxM.
+// workspace.  Used for M <= kSkinnyMaxM.  With one group (G = K) a CTA accumulates offset-code
+// products over its whole K range in fp32, exact while 120 * K < 2^24 (operand.cuh): larger
+// one-group problems take the GEMM.
 constexpr int kSkinnyMaxM = 64;
+constexpr int kSkinnyMaxKOneGroup = 139776;  // 1092 * 128
+inline bool skinny_supports(int64_t M, int64_t K, int32_t G) {
+  return M <= kSkinnyMaxM && (G != K || K <= kSkinnyMaxKOneGroup);
+}
 struct SkinnyProblem {
   int M, N, K, G;
   const uint8_t* q;    // [M, K/2] packed activation codes

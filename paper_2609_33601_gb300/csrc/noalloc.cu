@@ -81,7 +81,7 @@ extern "C" jq_status jq_w4a4_linear_noalloc(const uint8_t* q, const float* s_a, 
       (bias != nullptr && !aligned16(bias)))
     return JQ_ERR_MISALIGNED;
   const NoAllocDevice* d0 = nullptr;
-  if (M <= jq::kSkinnyMaxM) {  // few tokens: the weight-streaming kernel needs no scratch at all
+  if (jq::skinny_supports(M, K, group)) {  // few tokens: the weight-streaming kernel needs no scratch at all
     if ((d0 = noalloc_device()) == nullptr) return JQ_ERR_UNSUPPORTED;
     jq::SkinnyProblem p{static_cast<int>(M), static_cast<int>(N), static_cast<int>(K), group, q, s_a, qw, s_w, bias,
                         y_bf16, d0->status};

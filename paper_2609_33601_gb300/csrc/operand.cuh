@@ -43,6 +43,39 @@ __device__ __forceinline__ void nib32_to_operand(uint4 p, uint4& lo, uint4& hi) 
   hi = make_uint4(c.x, c.y, d.x, d.y);
 }
 
+// Offset operand bytes (the few-token kernel's weights): the code q becomes the byte q + 8 in
+// [0, 15], which E4M3 also reads exactly, as (q + 8) * 2^-9 (0..7 are subnormals, 8..15 have
+// exponent field 1: 2^-6 * (1 + m/8) = (8 + m) * 2^-9).  Adding 8 to a 4-bit two's complement
+// code is flipping its bit 3, so 8 codes take three operations instead of ten.  A dot product
+// with offset weights is sum (qw + 8) qa = sum qw qa + 8 sum qa: the kernel subtracts 8 times the
+// activation code sum, exactly, before any scaling.  |sum (qw + 8) qa| <= 120 per element, so a
+// run of up to 139808 elements (120 * 139808 < 2^24) accumulates exactly in fp32.
+__device__ __forceinline__ uint2 nib8_to_operand_offset(uint32_t w) {
+  return make_uint2((w & 0x0F0F0F0Fu) ^ 0x08080808u, ((w >> 4) & 0x0F0F0F0Fu) ^ 0x08080808u);
+}
+__device__ __forceinline__ void nib32_to_operand_offset(uint4 p, uint4& lo, uint4& hi) {
+  const uint2 a = nib8_to_operand_offset(p.x), b = nib8_to_operand_offset(p.y);
+  const uint2 c = nib8_to_operand_offset(p.z), d = nib8_to_operand_offset(p.w);
+  lo = make_uint4(a.x, a.y, b.x, b.y);
+  hi = make_uint4(c.x, c.y, d.x, d.y);
+}
+// Sum of the 32 signed codes of a 16-byte packed chunk: flip to offset codes q + 8, add the
+// nibble pairs of the four words bytewise (at most 4 * 30 = 120 per byte), fold the bytes into
+// 16-bit halves and the halves into one sum, and remove the 32 * 8 offset.  Plain logic and
+// adds only: the integer dot-product instruction is slow on this part.
+__device__ __forceinline__ int nib32_sum(uint4 p) {
+  const uint32_t w[4] = {p.x, p.y, p.z, p.w};
+  uint32_t bytes = 0;
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const uint32_t u = w[i] ^ 0x88888888u;
+    bytes += (u & 0x0F0F0F0Fu) + ((u >> 4) & 0x0F0F0F0Fu);
+  }
+  const uint32_t halves = (bytes & 0x00FF00FFu) + ((bytes >> 8) & 0x00FF00FFu);
+  return (int)((halves & 0xFFFFu) + (halves >> 16)) - 256;
+}
+constexpr int kOffsetMaxRun = 139808;
+
 // A-operand image (the GEMM's activation operand in global memory): for every 128-row tile
 // mt and every 128-element K stage kb, one contiguous 16 KB block that is byte for byte the
 // shared-memory image the tensor core reads -- 128 rows of 128 operand bytes in the 128-byte
@@ -63,7 +96,9 @@ __host__ __device__ __forceinline__ uint64_t image_chunk_offset(int64_t row, uin
   return (mt * k_stages + kb) * kImageBlockBytes + (r >> 3) * 1024u + (r & 7u) * 128u + ((c16 ^ (r & 7u)) << 4);
 }
 
-// Factor that turns an fp32 sum of operand products back into the integer partial.
+// Factor that turns an fp32 sum of operand products back into the integer partial, and its
+// inverse, the value of one integer unit of such a sum.
 constexpr float kOperandUnitInv = 262144.0f;  // 2^18
+constexpr float kOperandUnit = 1.0f / 262144.0f;  // 2^-18, exact
 
 }  // namespace jq

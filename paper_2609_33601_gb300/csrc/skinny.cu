@@ -3,13 +3,20 @@
 //
 // Same arithmetic as gemm.cu (Sec. 1, Appendix FAQ Q7): acc[m,n,g] = sum_{k in g} qa*qw exactly
 // (E4M3 operand bytes through tcgen05.mma kind::f8f6f4, operand.cuh), y = sum_g acc*s_a*s_w +
-// bias in fp32, rounded to bf16.  The shape of the work is different:
+// bias in fp32, rounded to bf16.  The weights enter the MMA as offset codes qw + 8 (three ALU
+// operations per 8 codes instead of ten); the MMA's sum (qw + 8) qa less 8 sum qa, formed
+// exactly from the activation codes, is acc.  The shape of the work is different:
 //   - the operands are swapped: each CTA unpacks 128 output channels of the weights into the
 //     MMA's M operand and the (at most 64) tokens are its N operand, so the MMA, the TMEM
 //     accumulators and the drain all scale with the real token count;
 //   - packed weight and activation codes stream in by TMA (two K stages per box, 128-byte
 //     swizzle) into a ring in shared memory: the TMA unit keeps far more bytes in flight per SM
 //     than per-thread loads, which is what a weight-streaming kernel needs;
+//   - the unpacked weight operand goes to tensor memory (tcgen05.st), and the MMA reads its A
+//     operand from there: a weight byte then crosses shared memory twice (the TMA write and the
+//     unpack's load of the packed code, half a byte each) instead of three times more for the
+//     operand's store and the tensor core's read, which would make shared-memory bandwidth, not
+//     HBM, the limit;
 //   - no workspace and no separate activation expansion;
 //   - K is split across the CTAs of a cluster (up to 8) so that enough SMs stream weights; the
 //     partial outputs are summed through distributed shared memory in a fixed tree order, so
@@ -17,12 +24,17 @@
 //     partials and scale once; otherwise each CTA scales its whole groups and the fp32 partial
 //     outputs are summed (the order of the fp32 sum over groups is free).
 // CTA layout, 16 warps:
-//   warp 0      TMEM owner and MMA issuer (one thread): 4 x (128 x Mp x 32) MMAs per K stage
-//   warp 1      activation scales: streams s_a into a ring for the drain, 8 groups per batch
+//   warps 0, 3  MMA issuers (one thread each) of the even / odd packed slots, each into its own
+//               accumulators: one issuing thread keeps the tensor core barely one MMA ahead, two
+//               keep it fed; 4 x (128 x Mp x 32) MMAs per K stage.  Warp 0 owns TMEM.
+//   warp 1      activation scales: s_a of every group into a ring for the drain
 //   warp 2      TMA producer (one thread): per two K stages, one box of 128 weight rows and one
 //               of the Mp token rows, 128 packed bytes each
-//   warps 4-11  unpack, two groups of four warps on alternate K stages: packed codes from the
-//               packed ring -> E4M3 operand rows (128B swizzle) in the operand ring
+//   warps 4-11  unpack, two groups of four warps on alternate packed slots (two K stages each,
+//               so that one round of waits and fences covers 32 KB of weight operand): thread =
+//               weight row (TMEM lane), packed codes -> E4M3 operand bytes in the TMEM A ring;
+//               token rows -> E4M3 operand rows (128B swizzle) in shared memory, and each
+//               token group's exact code sum (8 * sum, for the drain)
 //   warps 12-15 drain: per group, tcgen05.ld 32x32b (thread = output channel, every token
 //               column), y[m] += (acc * s_w) * (s_a[m] * 2^18)
 // Every mbarrier wait is bounded; a timeout records a status and unwinds the CTA.
@@ -43,40 +55,49 @@ namespace {
 constexpr int kRows = 128;       // output channels per CTA (the MMA's M)
 constexpr int kBK = 128;         // K elements per stage
 constexpr int kStPerSlot = 2;    // K stages per packed slot (one TMA box of 128 packed bytes per row)
-constexpr int kPkSlots = 4;      // packed ring (slots of two stages)
-constexpr int kOpSlots = 4;      // operand ring (stages)
+constexpr int kOpSlots = 4;      // operand ring (slots of two stages): weights in TMEM, tokens in shared memory
 constexpr int kThreads = 512;
-constexpr int kWarpMma = 0, kWarpScale = 1, kWarpTma = 2;
+constexpr int kWarpMma = 0, kWarpScale = 1, kWarpTma = 2, kWarpMma1 = 3;  // MMA issuers of even / odd slots
 constexpr int kUnpackWarp0 = 4, kUnpackGroups = 2, kUnpackGroupThreads = 128;
 constexpr int kUnpackGroupWarps = kUnpackGroupThreads / 32;
-constexpr int kWChunks = kRows * 4 / kUnpackGroupThreads;  // packed 16-byte weight chunks per thread per stage
 constexpr int kDrainWarp0 = 12, kNumDrainWarps = 4;
-constexpr int kSaRing = 16, kSaBatch = 8;  // activation-scale ring (groups), groups per load batch
+constexpr int kSaRing = 32;  // activation-scale ring (groups)
+// Register split per warpgroup while the roles run (totals the 512 x 128 registers of the launch):
+// warps 0-3 (MMA issuers, scales, TMA) 80, unpack 128, drain (up to 64 running sums) 176.  Every
+// warpgroup returns to 128 for the reduction that all warps take part in.
+constexpr int kRegsCtl = 80, kRegsUnpack = 128, kRegsDrain = 176, kRegsLaunch = 128;
+static_assert(kRegsCtl + 2 * kRegsUnpack + kRegsDrain == 4 * kRegsLaunch, "register split must use the launch budget");
 constexpr int kMaxSplit = 8;
-static_assert(kWChunks == 4, "unpack assumes four weight chunks per thread per stage");
 static_assert(kDrainWarp0 % 4 == 0, "drain warp w reads TMEM lanes 32 * (w % 4)");
+static_assert(kSkinnyMaxKOneGroup <= kOffsetMaxRun && kSkinnyMaxKOneGroup % kBK == 0, "exact one-group ranges");
 
 template <int kMp>
 struct Layout {
+  static constexpr int kPkSlots = kMp == 64 ? 6 : 8;      // packed ring (slots of two stages)
   static constexpr uint32_t kPkW = kRows * kBK;           // packed weights of a slot: 128 rows x 128 B
   static constexpr uint32_t kPkX = kMp * kBK;             // packed tokens of a slot: kMp rows x 128 B
   static constexpr uint32_t kPkSlot = kPkW + kPkX;
-  static constexpr uint32_t kOpA = kRows * kBK;           // weight operand bytes of a stage
   static constexpr uint32_t kOpB = kMp * kBK;             // token operand bytes of a stage
-  static constexpr uint32_t kOpSlot = kOpA + kOpB;
+  static constexpr uint32_t kOpSlot = kStPerSlot * kOpB;  // the two stages of a slot, one after the other
   static constexpr uint32_t kOffPk = 0;
   static constexpr uint32_t kOffOp = kOffPk + kPkSlots * kPkSlot;
-  static constexpr uint32_t kOffSa = kOffOp + kOpSlots * kOpSlot;  // [kSaRing][kMp] fp32
-  static constexpr uint32_t kOffBar = kOffSa + kSaRing * kMp * 4;
-  static constexpr uint32_t kNumBars = 2 * kPkSlots + 2 * kOpSlots + 4 + 1 + 2 * kSaRing;
+  static constexpr uint32_t kOffSa = kOffOp + kOpSlots * kOpSlot;  // s_a [kSaRing][kMp], then 8 sum qa [kSaRing][kMp]
+  static constexpr uint32_t kOffCorr = kOffSa + 2 * kSaRing * kMp * 4;  // G = K: 8 sum qa per unpack group [2][kMp]
+  static constexpr uint32_t kOffBar = kOffCorr + kUnpackGroups * kMp * 4;
+  static constexpr uint32_t kNumBars = 2 * kPkSlots + 2 * kOpSlots + 8 + 2 + 2 * kSaRing + 1;
   static constexpr uint32_t kOffMisc = kOffBar + kNumBars * 8;
   static constexpr uint32_t kSmemBytes = kOffMisc + 16;
-  static constexpr uint32_t kRedBytes = kMp * kRows * 4;  // fp32 partials [kMp][128], reuse the operand ring
-  static constexpr uint32_t kTmemCols = 2 * kMp < 32 ? 32 : 2 * kMp;  // two accumulators
-  static_assert(kPkW % 1024 == 0 && kPkX % 1024 == 0 && kOpA % 1024 == 0 && kOpB % 1024 == 0,
+  static constexpr uint32_t kRedBytes = kMp * kRows * 4;  // fp32 partials [kMp][128], reuse the packed ring
+  // TMEM columns: four fp32 accumulators of kMp columns at 0 (issuer e, buffer ab at column
+  // (2e + ab) kMp), the weight operand ring at kACol0 (a stage of 128 E4M3 bytes per lane is 32
+  // columns, a slot 64)
+  static constexpr uint32_t kACol0 = 256, kAStageCols = kBK / 4, kASlotCols = kStPerSlot * kAStageCols;
+  static constexpr uint32_t kTmemCols = 512;
+  static_assert(4 * kMp <= kACol0 && kACol0 + kOpSlots * kASlotCols <= kTmemCols, "TMEM columns");
+  static_assert(kPkW % 1024 == 0 && kPkX % 1024 == 0 && kOpB % 1024 == 0,
                 "128B-swizzle atoms need 1024-byte alignment");
   static_assert(kOffSa % 16 == 0 && kOffBar % 8 == 0, "alignment");
-  static_assert(kRedBytes <= kOpSlots * kOpSlot, "the reduction buffer reuses the operand ring");
+  static_assert(kRedBytes <= kPkSlots * kPkSlot, "the reduction buffer reuses the packed ring");
   static_assert(kSmemBytes <= 232448, "shared memory budget");
 };
 
@@ -95,8 +116,9 @@ struct SkArgs {
 struct SkBars {
   uint64_t *pk_full, *pk_empty;  // packed ring
   uint64_t *op_full, *op_empty;  // operand ring
-  uint64_t *acc_full, *acc_empty, *mma_done;
+  uint64_t *acc_full, *acc_empty, *mma_done;  // [2 issuers x 2 buffers], [2 issuers]
   uint64_t *sa_full, *sa_empty;  // activation-scale ring
+  uint64_t* corr_full;           // G = K: the range's code sums are in place
 };
 
 __device__ __forceinline__ uint32_t ring_parity(uint32_t it, uint32_t slots) { return (it / slots) & 1u; }
@@ -120,9 +142,6 @@ __device__ __forceinline__ int drain_groups(const SkArgs& a, const Range& r) {
 // Row r of a 128B-swizzled K-major tile at `base`: 16-byte chunk c sits at chunk c ^ (r % 8).
 __device__ __forceinline__ uint32_t sw128_row(uint32_t base, uint32_t r) { return base + (r >> 3) * 1024u + (r & 7u) * 128u; }
 
-// Within each group of 8 rows, pairs rows r and r + 4 on consecutive indices q: a quarter-warp
-// reading two such rows at the same four logical chunks hits 8 distinct physical chunks.
-__device__ __forceinline__ uint32_t row_of(uint32_t q) { return (q & ~7u) + ((q & 1u) << 2) + ((q >> 1) & 3u); }
 
 // ------------------------------------------------------------------ TMA producer
 template <int kMp>
@@ -130,6 +149,7 @@ __device__ __forceinline__ void tma_role(const SkArgs& a, const Range& rg, int n
                                          const CUtensorMap* tmX, uint8_t* smem, const SkBars& b,
                                          volatile int* abort_flag) {
   using L = Layout<kMp>;
+  constexpr int kPkSlots = L::kPkSlots;
   const int nslots = (rg.nst + kStPerSlot - 1) / kStPerSlot;
   for (int j = 0; j < nslots; ++j) {
     const uint32_t s = (uint32_t)j % kPkSlots;
@@ -148,78 +168,146 @@ __device__ __forceinline__ void tma_role(const SkArgs& a, const Range& rg, int n
 }
 
 // ------------------------------------------------------------------ unpack
-// Group ug converts stage 2j + ug of packed slot j: the 64-byte half ug of every packed row.
-// Thread u takes logical chunks t = u + 128 i: row q = t / 4 (paired by row_of), chunk t % 4.
+// Group ug converts packed slots j = ug, ug + 2, ...: both K stages of the slot.
+// Code sums: the 8 chunks of a token row sit in 8 consecutive lanes, so a group's sum (2 chunks
+// for G = 64, 4 for G = 128, all 8 and then all slots for G = K) is a butterfly over 1-3 lanes.
+// The drain removes 8 * sum qa, in the accumulator's units (2^-18), from the offset-code MMA;
+// G < K: into the scale ring next to s_a (a ring slot is full once the scale warp and the
+// group's four warps have written it); G = K: per unpack group, handed over at the end.
+// Weights: thread u is weight row u, the TMEM lane its warp may write; its 256 offset operand
+// bytes go to 64 columns of the A ring by two tcgen05.st.  Tokens: thread u takes packed chunks
+// t = u + 128 i of the token tile, row t / 8, chunk t % 8 (stage (t % 8) / 4), and stores
+// each as two operand chunks into the shared-memory operand ring.
 template <int kMp>
-__device__ __forceinline__ void unpack_role(const SkArgs& a, const Range& rg, uint8_t* smem, const SkBars& b,
-                                            volatile int* abort_flag) {
+__device__ __forceinline__ void unpack_role(const SkArgs& a, const Range& rg, uint8_t* smem, uint32_t tmem_base,
+                                            const SkBars& b, volatile int* abort_flag) {
   using L = Layout<kMp>;
-  constexpr int kXChunks = (kMp * 4 + kUnpackGroupThreads - 1) / kUnpackGroupThreads;  // token chunks per thread
+  constexpr int kPkSlots = L::kPkSlots;
+  constexpr int kXChunks = kMp * 8 / kUnpackGroupThreads;  // token chunks per thread per slot
+  static_assert(kUnpackWarp0 % 4 == 0 && kUnpackGroupThreads == kRows, "thread u of a group is TMEM lane u");
+  static_assert(kMp * 8 % kUnpackGroupThreads == 0, "token chunks divide evenly");
   const uint32_t ut = threadIdx.x - kUnpackWarp0 * 32;
   const uint32_t ug = ut / kUnpackGroupThreads, u = ut % kUnpackGroupThreads;
-  const uint32_t jc = u & 3u, lc = ug * 4u + jc;  // chunk within the stage / within the 128-byte row
+  const uint32_t r7 = u & 7u;
+  const uint32_t a_lane = tmem_base + ((u & ~31u) << 16) + L::kACol0;
   const int nslots = (rg.nst + kStPerSlot - 1) / kStPerSlot;
-  // the packed 16-byte chunk of row r in a packed tile
-  auto load = [&](uint32_t src, uint32_t r) { return ld_shared_v4(sw128_row(src, r) + ((lc ^ (r & 7u)) << 4)); };
-  // stores it as two operand chunks (rows with bit 2 set store their chunks in the other order,
-  // which keeps a quarter-warp's stores on distinct banks)
-  auto convert = [&](uint4 p, uint32_t dst, uint32_t r) {
-    uint4 lo, hi;
-    nib32_to_operand(p, lo, hi);
-    const uint32_t row_base = sw128_row(dst, r), r7 = r & 7u;
-    const uint32_t c_lo = (2u * jc) ^ r7, c_hi = (2u * jc + 1u) ^ r7;
-    if (r & 4u) {
-      st_shared_v4(row_base + (c_hi << 4), hi.x, hi.y, hi.z, hi.w);
-      st_shared_v4(row_base + (c_lo << 4), lo.x, lo.y, lo.z, lo.w);
-    } else {
-      st_shared_v4(row_base + (c_lo << 4), lo.x, lo.y, lo.z, lo.w);
-      st_shared_v4(row_base + (c_hi << 4), hi.x, hi.y, hi.z, hi.w);
-    }
-  };
-  for (int j = 0; j < nslots; ++j) {
-    const uint32_t p = (uint32_t)j % kPkSlots;
-    const int st = j * kStPerSlot + (int)ug;  // this group's stage (within the CTA's range)
+  const bool single = a.groups == 1;
+  const int gpst = groups_per_stage(a), gps = kStPerSlot * gpst;
+  const uint32_t c8 = u & 7u;  // the chunk of its token row this thread holds
+  float* c_ring = reinterpret_cast<float*>(smem + L::kOffSa) + kSaRing * kMp;
+  int tot[kXChunks];  // G = K: running code sums of this thread's token rows
+#pragma unroll
+  for (int i = 0; i < kXChunks; ++i) tot[i] = 0;
+  for (int j = (int)ug; j < nslots; j += kUnpackGroups) {
+    const int nst_j = rg.nst - j * kStPerSlot < kStPerSlot ? rg.nst - j * kStPerSlot : kStPerSlot;
+    const uint32_t p = (uint32_t)j % kPkSlots, os = (uint32_t)j % kOpSlots;
     if (!__all_sync(0xffffffffu, mbar_wait(&b.pk_full[p], ring_parity(j, kPkSlots), abort_flag, a.status))) return;
-    if (st < rg.nst) {
-      const uint32_t o = (uint32_t)st % kOpSlots;
-      if (!__all_sync(0xffffffffu, mbar_wait(&b.op_empty[o], ring_parity(st, kOpSlots) ^ 1u, abort_flag, a.status)))
+    if (!__all_sync(0xffffffffu, mbar_wait(&b.op_empty[os], ring_parity(j, kOpSlots) ^ 1u, abort_flag, a.status)))
+      return;
+    tc_fence_after();  // the MMAs that read this A slot have finished
+    const uint32_t src = smem_u32(smem + L::kOffPk + p * L::kPkSlot);
+    const uint32_t dst = smem_u32(smem + L::kOffOp + os * L::kOpSlot);
+    // loads in batches ahead of their use: the shared-memory accessors are ordered, so
+    // interleaving loads with stores would expose a load latency per chunk.  A quarter-warp reads
+    // 8 consecutive rows at one logical chunk (weights) or the 8 chunks of one row (tokens): 8
+    // distinct physical chunks.
+    uint4 pw[8], px[kXChunks];
+    const uint32_t wrow = sw128_row(src, u);
+#pragma unroll
+    for (int c = 0; c < 8; ++c) pw[c] = ld_shared_v4(wrow + (((uint32_t)c ^ r7) << 4));
+#pragma unroll
+    for (int h = 0; h < kStPerSlot; ++h) {
+      uint32_t v[32];
+#pragma unroll
+      for (int c = 0; c < 4; ++c) {
+        uint4 lo, hi;
+        nib32_to_operand_offset(pw[4 * h + c], lo, hi);
+        v[8 * c + 0] = lo.x; v[8 * c + 1] = lo.y; v[8 * c + 2] = lo.z; v[8 * c + 3] = lo.w;
+        v[8 * c + 4] = hi.x; v[8 * c + 5] = hi.y; v[8 * c + 6] = hi.z; v[8 * c + 7] = hi.w;
+      }
+      tmem_st32(a_lane + os * L::kASlotCols + (uint32_t)h * L::kAStageCols, v);
+    }
+#pragma unroll
+    for (int i = 0; i < kXChunks; ++i) {
+      const uint32_t t = u + kUnpackGroupThreads * i, r = t >> 3;
+      px[i] = ld_shared_v4(sw128_row(src + L::kPkW, r) + (((t & 7u) ^ (r & 7u)) << 4));
+    }
+    int xs[kXChunks];  // code sums of the token chunks (chunks of a stage past the range count 0)
+#pragma unroll
+    for (int i = 0; i < kXChunks; ++i) xs[i] = c8 < 4u * (uint32_t)nst_j ? nib32_sum(px[i]) : 0;
+#pragma unroll
+    for (int i = 0; i < kXChunks; ++i) {
+      const uint32_t t = u + kUnpackGroupThreads * i, r = t >> 3, h = (t >> 2) & 1u, jc = t & 3u;
+      uint4 lo, hi;
+      nib32_to_operand(px[i], lo, hi);
+      const uint32_t row_base = sw128_row(dst + h * L::kOpB, r), rr = r & 7u;
+      const uint32_t c_lo = (2u * jc) ^ rr, c_hi = (2u * jc + 1u) ^ rr;
+      // the two stage tiles sit a multiple of 128 bytes apart (same banks): the stage-1 half of
+      // the quarter-warp stores its chunks in the other order
+      if (h) {
+        st_shared_v4(row_base + (c_hi << 4), hi.x, hi.y, hi.z, hi.w);
+        st_shared_v4(row_base + (c_lo << 4), lo.x, lo.y, lo.z, lo.w);
+      } else {
+        st_shared_v4(row_base + (c_lo << 4), lo.x, lo.y, lo.z, lo.w);
+        st_shared_v4(row_base + (c_hi << 4), hi.x, hi.y, hi.z, hi.w);
+      }
+    }
+    tmem_st_wait();
+    fence_proxy_async_smem();
+    tc_fence_before();
+    __syncwarp();
+    if ((u & 31u) == 0) {
+      mbar_arrive(&b.op_full[os]);
+      mbar_arrive(&b.pk_empty[p]);
+    }
+    // group sums: lanes whose chunk opens a group hold that group's sum after the butterfly
+#pragma unroll
+    for (int i = 0; i < kXChunks; ++i) {
+      xs[i] += __shfl_xor_sync(0xffffffffu, xs[i], 1);
+      if (gpst == 1) xs[i] += __shfl_xor_sync(0xffffffffu, xs[i], 2);
+      if (single) {
+        xs[i] += __shfl_xor_sync(0xffffffffu, xs[i], 4);
+        tot[i] += xs[i];
+      }
+    }
+    if (single) continue;
+    const int cpg = 4 / gpst;  // chunks per group
+    for (int q = 0; q < nst_j * gpst; ++q) {
+      const int gi = j * gps + q;
+      const uint32_t so = (uint32_t)gi % kSaRing;
+      if (!__all_sync(0xffffffffu, mbar_wait(&b.sa_empty[so], ring_parity(gi, kSaRing) ^ 1u, abort_flag, a.status)))
         return;
-      const uint32_t src = smem_u32(smem + L::kOffPk + p * L::kPkSlot);
-      const uint32_t dst = smem_u32(smem + L::kOffOp + o * L::kOpSlot);
-      // all loads first: the shared-memory accessors are ordered, so interleaving loads with the
-      // previous chunk's stores would expose a load latency per chunk
-      uint4 pw[kWChunks], px[kXChunks];
-#pragma unroll
-      for (int i = 0; i < kWChunks; ++i) pw[i] = load(src, row_of((u + kUnpackGroupThreads * i) >> 2));
 #pragma unroll
       for (int i = 0; i < kXChunks; ++i) {
-        const uint32_t t = u + kUnpackGroupThreads * i;
-        if (t < kMp * 4) px[i] = load(src + L::kPkW, row_of(t >> 2));
+        const uint32_t r = (u + kUnpackGroupThreads * (uint32_t)i) >> 3;
+        if (c8 == (uint32_t)(q * cpg)) c_ring[so * kMp + r] = (float)(8 * xs[i]) * kOperandUnit;
       }
-#pragma unroll
-      for (int i = 0; i < kWChunks; ++i) convert(pw[i], dst, row_of((u + kUnpackGroupThreads * i) >> 2));
-#pragma unroll
-      for (int i = 0; i < kXChunks; ++i) {
-        const uint32_t t = u + kUnpackGroupThreads * i;
-        if (t < kMp * 4) convert(px[i], dst + L::kOpA, row_of(t >> 2));
-      }
-      fence_proxy_async_smem();
       __syncwarp();
-      if ((u & 31u) == 0) mbar_arrive(&b.op_full[o]);
+      if ((u & 31u) == 0) mbar_arrive(&b.sa_full[so]);
+    }
+  }
+  if (single) {  // this group's share of the range's code sums (zero if it had no slot)
+    float* corr = reinterpret_cast<float*>(smem + L::kOffCorr) + ug * kMp;
+#pragma unroll
+    for (int i = 0; i < kXChunks; ++i) {
+      const uint32_t r = (u + kUnpackGroupThreads * (uint32_t)i) >> 3;
+      if (c8 == 0u) corr[r] = (float)(8 * tot[i]) * kOperandUnit;
     }
     __syncwarp();
-    if ((u & 31u) == 0) mbar_arrive(&b.pk_empty[p]);
+    if ((u & 31u) == 0) mbar_arrive(b.corr_full);
   }
 }
 
 // ------------------------------------------------------------------ activation scales
 // One warp (lane m = token): the scales of this CTA's groups into the ring, kSaBatch groups per
-// batch of loads so that one load latency covers several groups.  Rows >= M get 0.
+// batch of loads so that one load latency covers several groups.  Rows >= M get 0.  A ring slot
+// is full once this warp and the unpack warps (the code sums) have written it.
 template <int kMp>
 __device__ __forceinline__ void scale_role(const SkArgs& a, const Range& rg, uint8_t* smem, const SkBars& b,
                                            volatile int* abort_flag) {
   using L = Layout<kMp>;
-  constexpr int kPer = kMp / 32 > 0 ? kMp / 32 : 1;  // tokens per lane
+  constexpr int kPer = kMp > 32 ? kMp / 32 : 1;  // tokens per lane
+  constexpr int kSaBatch = 8;
   const uint32_t lane = lane_id();
   float* sa_ring = reinterpret_cast<float*>(smem + L::kOffSa);
   const int ng = drain_groups(a, rg);
@@ -254,68 +342,96 @@ __device__ __forceinline__ void scale_role(const SkArgs& a, const Range& rg, uin
 }
 
 // ------------------------------------------------------------------ MMA issuer
-template <int kMp>
-__device__ __forceinline__ void mma_role(const SkArgs& a, const Range& rg, uint32_t tmem_base, uint8_t* smem,
-                                         const SkBars& b, volatile int* abort_flag) {
+// The tensor core accepts the next MMA only about one instruction ahead, so anything the issuing
+// thread executes between two MMAs (a branch, address arithmetic) leaves the pipe idle: each
+// slot's operand addresses are computed before its MMAs, which then issue straight-line, and the
+// group layout is a template parameter rather than a branch.
+//   kGroups = 0: one group over all of K (G = K), one accumulator for the CTA's whole range;
+//   kGroups = 1: one group per K stage (G = 128);  kGroups = 2: two groups per stage (G = 64).
+template <int kMp, int kGroups>
+__device__ __forceinline__ void mma_role(const SkArgs& a, const Range& rg, uint32_t e, uint32_t tmem_base,
+                                         uint8_t* smem, const SkBars& b, volatile int* abort_flag) {
   using L = Layout<kMp>;
   const uint32_t idesc = idesc_e4m3_f32(kRows, kMp);
-  const uint64_t adesc0 = sdesc_kmajor_sw128(smem_u32(smem + L::kOffOp));
-  const uint64_t bdesc0 = sdesc_kmajor_sw128(smem_u32(smem + L::kOffOp + L::kOpA));
-  const bool single = a.groups == 1;
-  const bool half_groups = a.G < kBK;
-  uint32_t chunk_it = 0, d_tmem = tmem_base;
+  const uint32_t a_tmem0 = tmem_base + L::kACol0;
+  const uint64_t bdesc0 = sdesc_kmajor_sw128(smem_u32(smem + L::kOffOp));
+  uint32_t chunk_it = 0, d_tmem = tmem_base;  // this issuer's accumulators, in order
   auto open_acc = [&]() -> bool {
-    const uint32_t ab = chunk_it & 1u;
-    if (!mbar_wait(&b.acc_empty[ab], ((chunk_it >> 1) & 1u) ^ 1u, abort_flag, a.status)) return false;
+    const uint32_t idx = 2u * e + (chunk_it & 1u);
+    if (!mbar_wait(&b.acc_empty[idx], ((chunk_it >> 1) & 1u) ^ 1u, abort_flag, a.status)) return false;
     tc_fence_after();
-    d_tmem = tmem_base + ab * kMp;
+    d_tmem = tmem_base + idx * kMp;
     return true;
   };
   auto close_acc = [&]() {
-    umma_commit(&b.acc_full[chunk_it & 1u]);
+    umma_commit(&b.acc_full[2u * e + (chunk_it & 1u)]);
     ++chunk_it;
   };
-  bool ok = rg.nst > 0 && (!single || open_acc());
-  for (int s = 0; ok && s < rg.nst; ++s) {
-    const uint32_t o = (uint32_t)s % kOpSlots;
-    if (!(ok = mbar_wait(&b.op_full[o], ring_parity(s, kOpSlots), abort_flag, a.status))) break;
-    const uint64_t ad = adesc0 + ((o * L::kOpSlot) >> 4), bd = bdesc0 + ((o * L::kOpSlot) >> 4);
-    if (single) {
-      umma_f8f6f4(d_tmem, ad, bd, idesc, s == 0 ? 0u : 1u);
-      umma_f8f6f4(d_tmem, ad + 2u, bd + 2u, idesc, 1u);
-      umma_f8f6f4(d_tmem, ad + 4u, bd + 4u, idesc, 1u);
-      umma_f8f6f4(d_tmem, ad + 6u, bd + 6u, idesc, 1u);
-    } else if (half_groups) {
+  // the four K slices of one stage: A columns +8, B descriptor +2 (32 bytes) per slice
+  auto stage4 = [&](uint32_t ad, uint64_t bd, uint32_t acc_first) {
+    umma_f8f6f4_ts(d_tmem, ad, bd, idesc, acc_first);
+    umma_f8f6f4_ts(d_tmem, ad + 8u, bd + 2u, idesc, 1u);
+    umma_f8f6f4_ts(d_tmem, ad + 16u, bd + 4u, idesc, 1u);
+    umma_f8f6f4_ts(d_tmem, ad + 24u, bd + 6u, idesc, 1u);
+  };
+  const int nslots = (rg.nst + kStPerSlot - 1) / kStPerSlot;
+  bool ok = (int)e < nslots && (kGroups != 0 || open_acc());
+  for (int j = (int)e; ok && j < nslots; j += 2) {
+    const uint32_t os = (uint32_t)j % kOpSlots;
+    const uint32_t ad0 = a_tmem0 + os * L::kASlotCols, ad1 = ad0 + L::kAStageCols;
+    const uint64_t bd0 = bdesc0 + ((os * L::kOpSlot) >> 4), bd1 = bd0 + (L::kOpB >> 4);
+    const bool both = j * kStPerSlot + 1 < rg.nst;  // false only for the last slot of an odd range
+    if (!(ok = mbar_wait(&b.op_full[os], ring_parity(j, kOpSlots), abort_flag, a.status))) break;
+    tc_fence_after();  // the unpack's tcgen05.st of this A slot is complete
+    if (kGroups == 0) {
+      const uint32_t acc0 = j > (int)e ? 1u : 0u;
+      if (both) {
+        stage4(ad0, bd0, acc0);
+        stage4(ad1, bd1, 1u);
+      } else {
+        stage4(ad0, bd0, acc0);
+      }
+    } else if (kGroups == 1) {
       if (!(ok = open_acc())) break;
-      umma_f8f6f4(d_tmem, ad, bd, idesc, 0u);
-      umma_f8f6f4(d_tmem, ad + 2u, bd + 2u, idesc, 1u);
+      stage4(ad0, bd0, 0u);
       close_acc();
-      if (!(ok = open_acc())) break;
-      umma_f8f6f4(d_tmem, ad + 4u, bd + 4u, idesc, 0u);
-      umma_f8f6f4(d_tmem, ad + 6u, bd + 6u, idesc, 1u);
-      close_acc();
+      if (both) {
+        if (!(ok = open_acc())) break;
+        stage4(ad1, bd1, 0u);
+        close_acc();
+      }
     } else {
-      if (!(ok = open_acc())) break;
-      umma_f8f6f4(d_tmem, ad, bd, idesc, 0u);
-      umma_f8f6f4(d_tmem, ad + 2u, bd + 2u, idesc, 1u);
-      umma_f8f6f4(d_tmem, ad + 4u, bd + 4u, idesc, 1u);
-      umma_f8f6f4(d_tmem, ad + 6u, bd + 6u, idesc, 1u);
-      close_acc();
+#pragma unroll
+      for (int h = 0; h < kStPerSlot; ++h) {
+        if (h == 1 && !both) break;
+        const uint32_t ad = h ? ad1 : ad0;
+        const uint64_t bd = h ? bd1 : bd0;
+        if (!(ok = open_acc())) break;
+        umma_f8f6f4_ts(d_tmem, ad, bd, idesc, 0u);
+        umma_f8f6f4_ts(d_tmem, ad + 8u, bd + 2u, idesc, 1u);
+        close_acc();
+        if (!(ok = open_acc())) break;
+        umma_f8f6f4_ts(d_tmem, ad + 16u, bd + 4u, idesc, 0u);
+        umma_f8f6f4_ts(d_tmem, ad + 24u, bd + 6u, idesc, 1u);
+        close_acc();
+      }
+      if (!ok) break;
     }
-    umma_commit(&b.op_empty[o]);
+    umma_commit(&b.op_empty[os]);
   }
-  if (ok && single && rg.nst > 0) close_acc();
-  umma_commit(b.mma_done);
+  if (ok && kGroups == 0 && (int)e < nslots) close_acc();
+  umma_commit(&b.mma_done[e]);
   int dummy = 0;
-  mbar_wait(b.mma_done, 0, &dummy, a.status);
+  mbar_wait(&b.mma_done[e], 0, &dummy, a.status);
 }
 
 // ------------------------------------------------------------------ drain
 // Warp w: TMEM lanes 32 * (w % 4).. (output channels), every token column (kH = kMp of them;
 // hf, the column-half index of a wider layout, is 0).  For G = K the accumulator is the exact
 // integer partial of this CTA's K range and is kept unscaled.  At the end the partials go to
-// the reduction buffer, which reuses the operand ring: the last group's accumulator being full
-// means every MMA has finished, and so every stage stored there has been consumed.
+// the reduction buffer, which reuses the packed ring: the last group's accumulator being full
+// means every MMA has finished, so every unpack has read its packed slot, and every TMA copy
+// into the ring has landed (the unpack waited for each one).
 template <int kMp>
 __device__ __forceinline__ void drain_role(const SkArgs& a, const Range& rg, int n0, uint32_t tmem_base, uint8_t* smem,
                                            const SkBars& b, volatile int* abort_flag) {
@@ -332,20 +448,30 @@ __device__ __forceinline__ void drain_role(const SkArgs& a, const Range& rg, int
   float y[kH];
 #pragma unroll
   for (int i = 0; i < kH; ++i) y[i] = 0.0f;
+  // Group gi was accumulated by the issuer of its slot j (e = j % 2) as that issuer's chunk
+  // (j / 2) * gps + gi % gps, gps = groups per slot.  G = K: both issuers hold a part of the one
+  // group (the second only if the range has more than one slot).
+  const int nslots = (rg.nst + kStPerSlot - 1) / kStPerSlot;
+  const int gps = kStPerSlot * groups_per_stage(a);
+  const int parts = single ? (nslots > 1 ? 2 : 1) : 1;
   float sw_next = (!single && ng > 0 && n < a.N) ? __ldg(a.s_w + (int64_t)g0 * a.N + n) : 0.0f;
-  for (int gi = 0; gi < ng; ++gi) {
-    const uint32_t ab = (uint32_t)gi & 1u;
+  for (int it = 0; it < ng * parts; ++it) {
+    const int gi = single ? 0 : it;
+    const uint32_t e = single ? (uint32_t)it : (uint32_t)(gi / gps) & 1u;
+    const uint32_t chunk = single ? 0u : (uint32_t)((gi / gps) >> 1) * (uint32_t)gps + (uint32_t)(gi % gps);
+    const uint32_t ab = 2u * e + (chunk & 1u);
     const float sw = sw_next;
     if (!single && gi + 1 < ng && n < a.N) sw_next = __ldg(a.s_w + (int64_t)(g0 + gi + 1) * a.N + n);
     const uint32_t so = (uint32_t)gi % kSaRing;
     bool ok = true;
     if (!single) ok = mbar_wait(&b.sa_full[so], ring_parity(gi, kSaRing), abort_flag, a.status);
-    ok = ok && mbar_wait(&b.acc_full[ab], ((uint32_t)gi >> 1) & 1u, abort_flag, a.status);
+    ok = ok && mbar_wait(&b.acc_full[ab], (chunk >> 1) & 1u, abort_flag, a.status);
     // warp-collective tcgen05.ld follows: the whole warp proceeds or none of it
     if (!__all_sync(0xffffffffu, ok)) break;
     tc_fence_after();
     const uint32_t taddr = tmem_base + ((quarter * 32u) << 16) + ab * kMp + hf * kH;
     const float* sas = sa_ring + so * kMp + hf * kH;
+    const float* cas = sas + kSaRing * kMp;  // 8 * sum qa of the group, per token
     // overflow-safe form needed only if some s_a * 2^18 of these columns overflows; the choice
     // is the warp's (no lane may skip the warp-collective loads below)
     bool finite = true;
@@ -374,7 +500,10 @@ __device__ __forceinline__ void drain_role(const SkArgs& a, const Range& rg, int
 #pragma unroll
         for (int i = 0; i < 8; i += 2) {
           const float2 s2 = *reinterpret_cast<const float2*>(sas + c * 8 + i);
-          const float2 t = __fmul2_rn(make_float2(__uint_as_float(r[i]), __uint_as_float(r[i + 1])), make_float2(sw, sw));
+          const float2 c2 = *reinterpret_cast<const float2*>(cas + c * 8 + i);
+          // exact: both are integers below 2^24 (in units of 2^-18)
+          const float2 d = make_float2(__uint_as_float(r[i]) - c2.x, __uint_as_float(r[i + 1]) - c2.y);
+          const float2 t = __fmul2_rn(d, make_float2(sw, sw));
           const float2 v = __ffma2_rn(t, make_float2(s2.x * kOperandUnitInv, s2.y * kOperandUnitInv),
                                       make_float2(y[c * 8 + i], y[c * 8 + i + 1]));
           y[c * 8 + i] = v.x;
@@ -383,7 +512,8 @@ __device__ __forceinline__ void drain_role(const SkArgs& a, const Range& rg, int
       } else {  // |s_a| > 2^110 somewhere: apply 2^18 to the exact partials first
 #pragma unroll
         for (int i = 0; i < 8; ++i)
-          y[c * 8 + i] = fmaf((__uint_as_float(r[i]) * kOperandUnitInv) * sas[c * 8 + i], sw, y[c * 8 + i]);
+          y[c * 8 + i] =
+              fmaf(((__uint_as_float(r[i]) - cas[c * 8 + i]) * kOperandUnitInv) * sas[c * 8 + i], sw, y[c * 8 + i]);
       }
     }
     if (!single) {
@@ -391,7 +521,14 @@ __device__ __forceinline__ void drain_role(const SkArgs& a, const Range& rg, int
       if (lane == 0) mbar_arrive(&b.sa_empty[so]);
     }
   }
-  float* red = reinterpret_cast<float*>(smem + L::kOffOp);  // [kMp][128]
+  if (single && ng > 0) {  // the exact partial: the offset-code sum less 8 * the range's code sums
+    const bool ok = mbar_wait(b.corr_full, 0, abort_flag, a.status);
+    const float* corr = reinterpret_cast<const float*>(smem + L::kOffCorr);
+#pragma unroll
+    for (int i = 0; i < kH; ++i)  // the two shares and the difference are exact integers (units 2^-18)
+      y[i] = ok ? y[i] - (corr[hf * kH + i] + corr[kMp + hf * kH + i]) : 0.0f;
+  }
+  float* red = reinterpret_cast<float*>(smem + L::kOffPk);  // [kMp][128]
 #pragma unroll
   for (int i = 0; i < kH; ++i) red[(hf * kH + i) * kRows + ch] = y[i];
 }
@@ -410,14 +547,15 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint64_t* bar = reinterpret_cast<uint64_t*>(smem + L::kOffBar);
   SkBars b;
   b.pk_full = bar;
-  b.pk_empty = b.pk_full + kPkSlots;
-  b.op_full = b.pk_empty + kPkSlots;
+  b.pk_empty = b.pk_full + L::kPkSlots;
+  b.op_full = b.pk_empty + L::kPkSlots;
   b.op_empty = b.op_full + kOpSlots;
   b.acc_full = b.op_empty + kOpSlots;
-  b.acc_empty = b.acc_full + 2;
-  b.mma_done = b.acc_empty + 2;
-  b.sa_full = b.mma_done + 1;
+  b.acc_empty = b.acc_full + 4;
+  b.mma_done = b.acc_empty + 4;
+  b.sa_full = b.mma_done + 2;
   b.sa_empty = b.sa_full + kSaRing;
+  b.corr_full = b.sa_empty + kSaRing;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + L::kOffMisc);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + L::kOffMisc + 4);
 
@@ -427,23 +565,24 @@ __global__ void __launch_bounds__(kThreads, 1)
   const uint32_t warp = warp_id(), lane = lane_id();
   if (threadIdx.x == 0) {
     *abort_flag = 0;
-    for (int i = 0; i < kPkSlots; ++i) {
+    for (int i = 0; i < L::kPkSlots; ++i) {
       mbar_init(&b.pk_full[i], 1);                                  // the producer's expect_tx
-      mbar_init(&b.pk_empty[i], kUnpackGroups * kUnpackGroupWarps);  // every unpack warp
+      mbar_init(&b.pk_empty[i], kUnpackGroupWarps);  // the slot's unpack group
     }
     for (int i = 0; i < kOpSlots; ++i) {
-      mbar_init(&b.op_full[i], kUnpackGroupWarps);  // the stage's unpack group
+      mbar_init(&b.op_full[i], kUnpackGroupWarps);  // the slot's unpack group
       mbar_init(&b.op_empty[i], 1);
     }
-    for (int i = 0; i < 2; ++i) {
+    for (int i = 0; i < 4; ++i) {
       mbar_init(&b.acc_full[i], 1);
       mbar_init(&b.acc_empty[i], kNumDrainWarps);
     }
-    mbar_init(b.mma_done, 1);
+    for (int i = 0; i < 2; ++i) mbar_init(&b.mma_done[i], 1);
     for (int i = 0; i < kSaRing; ++i) {
-      mbar_init(&b.sa_full[i], 1);
+      mbar_init(&b.sa_full[i], 1 + kUnpackGroupWarps);  // the scale warp and one unpack group
       mbar_init(&b.sa_empty[i], kNumDrainWarps);
     }
+    mbar_init(b.corr_full, kUnpackGroups * kUnpackGroupWarps);
     fence_mbar_init();
     tma_prefetch_desc(&tmW);
     tma_prefetch_desc(&tmX);
@@ -458,22 +597,37 @@ __global__ void __launch_bounds__(kThreads, 1)
   const uint32_t tmem_base = *tmem_slot;
 
   const bool drain = warp >= kDrainWarp0;
+  static_assert(kDrainWarp0 == 12 && kUnpackWarp0 == 4, "the register split is per warpgroup");
   if (drain) {
+    asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;\n" ::"n"(kRegsDrain) : "memory");
     drain_role<kMp>(a, rg, n0, tmem_base, smem, b, abort_flag);
+    __syncwarp();
+    asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;\n" ::"n"(kRegsLaunch) : "memory");
   } else if (warp >= kUnpackWarp0) {
-    unpack_role<kMp>(a, rg, smem, b, abort_flag);
-  } else if (warp == kWarpScale) {
-    scale_role<kMp>(a, rg, smem, b, abort_flag);
-  } else if (warp == kWarpTma && lane == 0) {
-    tma_role<kMp>(a, rg, n0, &tmW, &tmX, smem, b, abort_flag);
-  } else if (warp == kWarpMma && lane == 0) {
-    mma_role<kMp>(a, rg, tmem_base, smem, b, abort_flag);
+    unpack_role<kMp>(a, rg, smem, tmem_base, b, abort_flag);
+  } else {
+    asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;\n" ::"n"(kRegsCtl) : "memory");
+    if (warp == kWarpScale) {
+      scale_role<kMp>(a, rg, smem, b, abort_flag);
+    } else if (warp == kWarpTma) {
+      if (lane == 0) tma_role<kMp>(a, rg, n0, &tmW, &tmX, smem, b, abort_flag);
+    } else if (lane == 0 && (warp == kWarpMma || warp == kWarpMma1)) {
+      const uint32_t e = warp == kWarpMma ? 0u : 1u;
+      if (a.groups == 1)
+        mma_role<kMp, 0>(a, rg, e, tmem_base, smem, b, abort_flag);
+      else if (a.G >= kBK)
+        mma_role<kMp, 1>(a, rg, e, tmem_base, smem, b, abort_flag);
+      else
+        mma_role<kMp, 2>(a, rg, e, tmem_base, smem, b, abort_flag);
+    }
+    __syncwarp();
+    asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;\n" ::"n"(kRegsLaunch) : "memory");
   }
 
   // every role is done; the drain threads have written their partials to the reduction buffer
   tc_fence_before();
   __syncthreads();
-  float* red = reinterpret_cast<float*>(smem + L::kOffOp);  // [kMp][128]
+  float* red = reinterpret_cast<float*>(smem + L::kOffPk);  // [kMp][128]
   const uint32_t ch = (warp & 3u) * 32u + lane, hf = 0;
   // Fixed-order tree over the cluster: at step d, rank r (r % 2d == 0) adds rank r + d's buffer.
   for (int d = 1; d < a.split; d <<= 1) {
@@ -584,7 +738,7 @@ cudaError_t launch_mp(SkArgs a, const SkinnyProblem& p, int tiles, int sms, cuda
 
 cudaError_t launch_w4a4_skinny(const SkinnyProblem& p, cudaStream_t stream, int sms) {
   if (p.M <= 0 || p.N <= 0) return cudaSuccess;
-  if (p.M > kSkinnyMaxM) return cudaErrorInvalidValue;
+  if (!skinny_supports(p.M, p.K, p.G)) return cudaErrorInvalidValue;
   SkArgs a;
   a.M = p.M;
   a.N = p.N;

@@ -194,6 +194,32 @@ def test_full_code_range_linear():
     check_linear(host_bits(y), y64, acc, sa, sw, bias)
 
 
+@pytest.mark.parametrize("M", [1, 16, 33, 64, 200])
+@pytest.mark.parametrize("K,G", [(4096, 4096), (16384, 16384), (4096, 128), (2048, 64)])
+def test_large_partial_sums_cancel(M, K, G):
+    """Running sums climb to ~49 K/2 and fall back to a small exact integer.
+
+    Weight row n is +7 over the first half of K and -7 over the second (one code changed so that
+    the row sums to -(n % 5)); token rows are all 7 or all -8.  With unit scales y = acc exactly,
+    so an accumulation that dropped low bits of a large intermediate sum (or a mistaken code
+    offset) shows up as a wrong small integer.  M <= 64 and M > 64 take different kernels.
+    """
+    N = 264
+    qw = np.full((N, K), 7, np.int8)
+    qw[:, K // 2:] = -7
+    qw[:, 1] -= (np.arange(N) % 5).astype(np.int8)
+    qa = np.where((np.arange(M) % 2 == 0)[:, None], np.int8(7), np.int8(-8)) * np.ones((M, K), np.int8)
+    sa = np.ones((M, K // G), np.float32)
+    sw = np.ones((N, K // G), np.float32)
+    y64, _ = oracle.linear(qa, sa, qw, sw, None, G)
+    acc = oracle.group_partials(qa, qw, G).sum(axis=2)
+    assert np.abs(acc).max() <= 8 * 4 * 7  # the exact result is small; the running sums are not
+    y = jq.jq_w4a4_linear(dev(oracle.pack(qa)), dev(sa), dev(oracle.pack(qw)), dev(np.ascontiguousarray(sw.T)),
+                          None, G)
+    assert np.array_equal(wl.bf16_bits_to_f32(host_bits(y)), acc.astype(np.float32))
+    check_linear(host_bits(y), y64, oracle.group_partials(qa, qw, G), sa, sw, None)
+
+
 def test_zero_weights_and_zero_activations():
     M, N, K, G = 130, 264, 256, 128
     w = wl.make("custom", seed=2, M=M, K=K, N=N, G=G, bias=True)
