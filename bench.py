@@ -34,25 +34,39 @@ ROOT = os.path.dirname(os.path.abspath(__file__))
 sys.path.insert(0, ROOT)
 
 WORKLOADS = {
-    # name: (description, M, K, N, G, bias)
-    "dllm": ("dLLM 8B gate/up projection: M=1024 tokens x K=4096 -> N=12288, group128", 1024, 4096, 12288, 128),
-    "flux_qkv": ("FLUX 12B DiT fused QKV+MLP-in: M=4608 x K=3072 -> N=21504, group64", 4608, 3072, 21504, 64),
-    "flux_out": ("FLUX 12B DiT output projection: M=4608 x K=15360 -> N=3072, group64", 4608, 15360, 3072, 64),
+    # name: (description, M, K, N, G, generator in workloads.py)
+    "dllm": ("dLLM 8B gate/up projection: M=1024 tokens x K=4096 -> N=12288, group128", 1024, 4096, 12288, 128,
+             "dllm"),
+    "flux_qkv": ("FLUX 12B DiT fused QKV+MLP-in: M=4608 x K=3072 -> N=21504, group64", 4608, 3072, 21504, 64,
+                 "flux_qkv"),
+    "flux_out": ("FLUX 12B DiT output projection: M=4608 x K=15360 -> N=3072, group64", 4608, 15360, 3072, 64,
+                 "flux_out"),
+    # M-sweep points below the memory-to-compute crossover (per-token / per-channel: group = K);
+    # these run the few-token kernel and are bound by streaming the packed weights from HBM
+    "sweep_m1": ("M sweep: M=1 token x K=4096 -> N=12288, per-token/per-channel (group = K)", 1, 4096, 12288,
+                 4096, "sweep_a"),
+    "sweep_m16": ("M sweep: M=16 tokens x K=4096 -> N=12288, per-token/per-channel (group = K)", 16, 4096, 12288,
+                  4096, "sweep_a"),
+    "sweep_m64": ("M sweep: M=64 tokens x K=4096 -> N=12288, per-token/per-channel (group = K)", 64, 4096, 12288,
+                  4096, "sweep_a"),
 }
+FEW_TOKENS = 64  # M at or below this takes the few-token (weight-streaming) kernel
 PEAKS_PATH = os.path.join(ROOT, "MEASURED_PEAKS.json")
 FP8_PER_BF16 = 2.0  # nominal dense FP8 / BF16 tensor-core ratio on GB300 (4.5 / 2.25 PFLOP/s)
 
-# DRAM traffic of one GEMM launch (dram__bytes_read.sum + dram__bytes_write.sum) from the ncu
-# capture summarised in profiles/, keyed by the hash of the kernel source it was taken on; once
-# the kernel changes the figure no longer applies and the bench reports null.
-GEMM_TRAFFIC = {
-    ("dllm", "d598a837a9b8975a"): 31.25e6 + 0.15e6,  # profiles/w4a4_gemm_dllm_full.md
+# DRAM traffic of one launch of the dominant kernel (dram__bytes_read.sum + dram__bytes_write.sum)
+# from the ncu captures summarised in profiles/, keyed by workload and by the hash of the kernel
+# source the capture was taken on; once the kernel changes the figure no longer applies and the
+# bench reports null.
+KERNEL_TRAFFIC = {
+    ("dllm", "cf7dd0ff7f1c9c83"): 31.239e6 + 0.138e6,  # profiles/w4a4_gemm_dllm_full.md
+    ("sweep_m1", "b8c4d652385e2708"): 25.288e6,  # profiles/w4a4_skinny_sweep_m1_full.md
 }
 
 
-def kernel_hash() -> str:
+def kernel_hash(kernel_file: str) -> str:
     h = hashlib.sha256()
-    for f in ("gemm.cu", "operand.cuh", "ptx.cuh"):
+    for f in (kernel_file, "operand.cuh", "ptx.cuh"):
         with open(os.path.join(ROOT, "paper_2609_33601_gb300", "csrc", f), "rb") as fh:
             h.update(fh.read())
     return h.hexdigest()[:16]
@@ -131,8 +145,8 @@ class OracleSample:
         from paper_2609_33601_gb300 import workloads as wl
         self.oracle = oracle
         self.name = name
-        self.desc, self.M, self.K, self.N, self.G = WORKLOADS[name]
-        w = wl.make(name, seed=seed)
+        self.desc, self.M, self.K, self.N, self.G, gen = WORKLOADS[name]
+        w = wl.make(gen, seed=seed, M=self.M, G=self.G)
         self.x_bits, self.bias = w.x_bits, w.bias
         self.qw, self.sw = oracle.quantize_f32(w.w, self.G)
         self.rows = 8
@@ -201,12 +215,14 @@ def run_ours(args):
     import paper_2609_33601_gb300 as jq
     from paper_2609_33601_gb300 import workloads as wl
 
-    desc, M, K, N, G = WORKLOADS[args.workload]
+    desc, M, K, N, G, gen = WORKLOADS[args.workload]
+    few = M <= FEW_TOKENS
     dev = torch.device("cuda", local)
     sets = []
-    n_sets = args.sets
+    # rotating weight sets: together several times larger than the 126 MB L2
+    n_sets = args.sets if args.sets > 0 else max(6, -(-400_000_000 // (N * K // 2 + M * K * 2)))
     for i in range(n_sets):
-        w = wl.make(args.workload, seed=100 + 17 * rank + i)
+        w = wl.make(gen, seed=100 + 17 * rank + i, M=M, G=G)
         x = torch.from_numpy(w.x_bits.view(np.int16)).to(dev).view(torch.bfloat16)
         qw, sw = jq.jq_pack_weight(torch.from_numpy(w.w).to(dev), G)
         b = None if w.bias is None else torch.from_numpy(w.bias).to(dev)
@@ -219,14 +235,16 @@ def run_ours(args):
     ws = torch.empty(jq.jq_workspace_size(M, N, K, G, False), dtype=torch.uint8, device=dev)
     stream = torch.cuda.current_stream()
 
-    def step(i, ev=None):
-        x, qw, sw, b = sets[i % n_sets]
-        jq.jq_quantize_act(x, G, q, s_a, stream=stream)
-        if ev is not None:
-            ev[0].record(stream)
-        jq.jq_w4a4_linear(q, s_a, qw, sw, b, G, y=y, workspace=ws, stream=stream)
-        if ev is not None:
-            ev[1].record(stream)
+    def quantize(i, st):
+        jq.jq_quantize_act(sets[i % n_sets][0], G, q, s_a, stream=st)
+
+    def linear(i, st):
+        _, qw, sw, b = sets[i % n_sets]
+        jq.jq_w4a4_linear(q, s_a, qw, sw, b, G, y=y, workspace=ws, stream=st)
+
+    def step(i, st=None):
+        quantize(i, st or stream)
+        linear(i, st or stream)
 
     def barrier():
         if world > 1:
@@ -238,19 +256,42 @@ def run_ours(args):
     torch.cuda.synchronize()
     assert jq.jq_device_status() == 0, "a kernel reported a bounded-wait timeout"
 
-    gemm_ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
+    # The K timed steps are captured once into a CUDA graph and replayed: the host's per-call cost
+    # (Python, ctypes, argument checks, launch) would otherwise gate the device on the short
+    # launches of the few-token workloads.  A second graph holds the K linear launches alone, for
+    # the per-launch duration of the dominant kernel.
+    cap = torch.cuda.Stream()
+    cap.wait_stream(stream)
+    with torch.cuda.stream(cap):
+        for i in range(args.warmup):
+            step(i, cap)
+    cap.synchronize()
+    g_steps, g_linear = torch.cuda.CUDAGraph(), torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g_steps, stream=cap):
+        for i in range(args.steps):
+            step(i, cap)
+    with torch.cuda.graph(g_linear, stream=cap):
+        for i in range(args.steps):
+            linear(i, cap)
+    g_steps.replay()
+    g_linear.replay()
+    torch.cuda.synchronize()
     t_start, t_end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    l_start, l_end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     barrier()
     torch.cuda.synchronize()
     with ClockSampler(local) as clocks:
         t_start.record(stream)
-        for i in range(args.steps):
-            step(i, gemm_ev[i])
+        g_steps.replay()
         t_end.record(stream)
+        torch.cuda.synchronize()
+        l_start.record(stream)
+        g_linear.replay()
+        l_end.record(stream)
         torch.cuda.synchronize()
     barrier()
     total_ms = t_start.elapsed_time(t_end)
-    gemm_ms = sum(a.elapsed_time(b) for a, b in gemm_ev) / args.steps
+    gemm_ms = l_start.elapsed_time(l_end) / args.steps
     if world > 1:
         import torch.distributed as dist
         t = torch.tensor([total_ms, gemm_ms], device=dev)
@@ -288,10 +329,26 @@ def run_ours(args):
     ops_step = 2.0 * M * N * K
     value = world * ops_step * args.steps / (total_ms * 1e-3) / 1e12
     e2e_value = world * ops_step * args.steps / e2e_s / 1e12
-    bf16_peak, _, peak_src = measured_peaks()
+    bf16_peak, hbm_peak, peak_src = measured_peaks()
     fp8_peak = bf16_peak * FP8_PER_BF16
-    achieved = ops_step / (gemm_ms * 1e-3) / 1e12
-    traffic = GEMM_TRAFFIC.get((args.workload, kernel_hash()))
+    kernel_file = "skinny.cu" if few else "gemm.cu"
+    traffic = KERNEL_TRAFFIC.get((args.workload, kernel_hash(kernel_file)))
+    if few:
+        # algorithmic bytes of one jq_w4a4_linear: packed weights and their scales, packed
+        # activation codes and scales, bias, bf16 output
+        groups = K // G
+        alg_bytes = N * K // 2 + groups * N * 4 + M * K // 2 + M * groups * 4 + M * N * 2
+        achieved = alg_bytes / (gemm_ms * 1e-3) / 1e9
+        roofline = {"bound": "hbm", "achieved": achieved, "peak": hbm_peak, "unit": "GB/s", "frac": achieved / hbm_peak,
+                    "traffic": traffic, "algorithmic_bytes": alg_bytes,
+                    "kernel": "jq_w4a4_linear (few-token weight-streaming kernel), CUDA events around a graph of K launches",
+                    "peak_source": f"{peak_src} HBM copy bandwidth {hbm_peak} GB/s"}
+    else:
+        achieved = ops_step / (gemm_ms * 1e-3) / 1e12
+        roofline = {"bound": "tensor", "achieved": achieved, "peak": fp8_peak, "unit": "TFLOP/s",
+                    "frac": achieved / fp8_peak, "traffic": traffic,
+                    "kernel": "jq_w4a4_linear (operand expansion + tcgen05 GEMM), CUDA events around a graph of K launches",
+                    "peak_source": f"{peak_src} bf16 {bf16_peak} TFLOP/s x nominal FP8/BF16 ratio {FP8_PER_BF16}"}
 
     if rank != 0:
         if world > 1:
@@ -308,15 +365,13 @@ def run_ours(args):
         "warmup": args.warmup, "ms_per_step": total_ms / args.steps, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "int4", "data": "synthetic",
         "config": {"workload": desc, "M": M, "K": K, "N": N, "group": G,
-                   "step": "jq_quantize_act + jq_w4a4_linear", "parallelism": f"replicas x{world}",
+                   "step": "jq_quantize_act + jq_w4a4_linear", "launch": "CUDA graph of the K steps",
+                   "parallelism": f"replicas x{world}",
                    "l2": f"{n_sets} rotating input/weight sets larger than L2"},
-        "roofline": {"bound": "tensor", "achieved": achieved, "peak": fp8_peak, "unit": "TFLOP/s",
-                     "frac": achieved / fp8_peak, "traffic": traffic,
-                     "kernel": "jq_w4a4_linear (operand expansion + tcgen05 GEMM), CUDA events per launch",
-                     "peak_source": f"{peak_src} bf16 {bf16_peak} TFLOP/s x nominal FP8/BF16 ratio {FP8_PER_BF16}"},
+        "roofline": roofline,
         "cpu_baseline": cpu,
         "e2e": {"value": e2e_value, "unit": "TOPS", "h2d_bytes_per_step": M * K * 2, "d2h_bytes_per_step": M * N * 2},
-        "gpu_launches": 3 * args.steps,
+        "gpu_launches": (2 if few else 3) * args.steps,
         "clocks": clocks.summary(),
     }
     print(json.dumps(line), flush=True)
@@ -333,7 +388,7 @@ def main():
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--workload", choices=sorted(WORKLOADS), default="dllm")
-    ap.add_argument("--sets", type=int, default=6, help="rotating input/weight sets (working set > L2)")
+    ap.add_argument("--sets", type=int, default=0, help="rotating input/weight sets (0: enough for > 3x L2)")
     ap.add_argument("--ref-seconds", type=float, default=10.0, help="CPU seconds per oracle sample")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     args = ap.parse_args()
