@@ -227,17 +227,23 @@ __device__ __forceinline__ void unpack_role(const SkArgs& a, const Range& rg, ui
       }
       tmem_st32(a_lane + os * L::kASlotCols + (uint32_t)h * L::kAStageCols, v);
     }
+    // token rows: only the M real ones (rows >= M stay zero in the operand ring)
 #pragma unroll
     for (int i = 0; i < kXChunks; ++i) {
       const uint32_t t = u + kUnpackGroupThreads * i, r = t >> 3;
-      px[i] = ld_shared_v4(sw128_row(src + L::kPkW, r) + (((t & 7u) ^ (r & 7u)) << 4));
+      px[i] = r < (uint32_t)a.M ? ld_shared_v4(sw128_row(src + L::kPkW, r) + (((t & 7u) ^ (r & 7u)) << 4))
+                                : make_uint4(0x88888888u, 0x88888888u, 0x88888888u, 0x88888888u);
     }
     int xs[kXChunks];  // code sums of the token chunks (chunks of a stage past the range count 0)
 #pragma unroll
-    for (int i = 0; i < kXChunks; ++i) xs[i] = c8 < 4u * (uint32_t)nst_j ? nib32_sum(px[i]) : 0;
+    for (int i = 0; i < kXChunks; ++i) {
+      const uint32_t r = (u + kUnpackGroupThreads * (uint32_t)i) >> 3;
+      xs[i] = (r < (uint32_t)a.M && c8 < 4u * (uint32_t)nst_j) ? nib32_sum(px[i]) : 0;
+    }
 #pragma unroll
     for (int i = 0; i < kXChunks; ++i) {
       const uint32_t t = u + kUnpackGroupThreads * i, r = t >> 3, h = (t >> 2) & 1u, jc = t & 3u;
+      if (r >= (uint32_t)a.M) continue;
       uint4 lo, hi;
       nib32_to_operand(px[i], lo, hi);
       const uint32_t row_base = sw128_row(dst + h * L::kOpB, r), rr = r & 7u;
@@ -590,6 +596,16 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (warp == kWarpMma) {
     tmem_alloc(tmem_slot, L::kTmemCols);
     tmem_relinquish();
+  }
+  // Token rows >= M of the operand ring are zero codes for good: store them once here, and the
+  // unpack converts only the M real rows of every slot.
+  if (a.M < kMp) {
+    const uint32_t row_bytes = (uint32_t)(kMp - a.M) * kBK, tile0 = smem_u32(smem + L::kOffOp);
+    for (uint32_t i = threadIdx.x; i < kOpSlots * kStPerSlot * (row_bytes / 16u); i += kThreads) {
+      const uint32_t tile = i / (row_bytes / 16u), off = (uint32_t)a.M * kBK + (i % (row_bytes / 16u)) * 16u;
+      st_shared_v4(tile0 + tile * L::kOpB + off, 0u, 0u, 0u, 0u);  // whole rows: the swizzle only permutes within a row
+    }
+    fence_proxy_async_smem();
   }
   tc_fence_before();
   __syncthreads();
