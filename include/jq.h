@@ -135,13 +135,15 @@ JQ_API jq_status jq_w4a4_group_partials(const uint8_t* q, const uint8_t* qw, int
  * counterpart; this is a deployment convenience.)  jq_w4a4_linear needs a caller-provided
  * workspace; code that may not call cudaMalloc at all -- a host callback, a plug-in whose
  * framework owns every allocation, a serving loop that must not allocate after start-up --
- * cannot provide one.  This variant keeps that scratch (the activation operand bytes) in a
- * fixed device array inside the library instead, JQ_NOALLOC_MAX_SCRATCH_BYTES large, which
- * every GPU that loads the library holds until the process exits.  It allocates nothing and
+ * cannot provide one.  This variant keeps that scratch (the activation operand bytes and their
+ * per-group code sums) in a fixed device array inside the library instead,
+ * JQ_NOALLOC_MAX_SCRATCH_BYTES large, which every GPU that loads the library holds until the
+ * process exits.  It allocates nothing and
  * runs the same kernels, so its output is identical to jq_w4a4_linear's.
  *   Arguments as jq_w4a4_linear, without the workspace.
- *   Limit: ceil(M / 128) * 128 * K <= JQ_NOALLOC_MAX_SCRATCH_BYTES, else JQ_ERR_WORKSPACE
- *   (nothing launched).
+ *   Limit: ceil(M / 128) * 128 * K + ceil(4 * M * (K/group) / 256) * 256 <=
+ *   JQ_NOALLOC_MAX_SCRATCH_BYTES (the operand bytes and one fp32 per token and group), else
+ *   JQ_ERR_WORKSPACE (nothing launched); calls that take the few-token kernel need no scratch.
  *   The first call on a device looks up the array's device address (cudaGetSymbolAddress);
  *   make that first call before any stream capture.  All calls on a device share the one
  *   array, so calls whose kernels may overlap on the GPU (different streams without ordering

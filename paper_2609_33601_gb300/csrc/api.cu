@@ -104,8 +104,8 @@ size_t jq_workspace_size(int64_t M, int64_t N, int64_t K, int32_t group, int32_t
   (void)N;
   if (M <= 0 || K <= 0 || group <= 0 || K % group != 0) return 0;
   // A-operand image: whole 128-row tiles of K operand bytes (operand.cuh)
-  size_t bytes = round_up(static_cast<size_t>(M), 128) * static_cast<size_t>(K);
-  if (fused) bytes += round_up(static_cast<size_t>(M) * static_cast<size_t>(K / group) * sizeof(float), 256);
+  size_t bytes = jq::ws_image_bytes(M, K) + jq::ws_per_group_bytes(M, K, group);  // A image, corrections
+  if (fused) bytes += jq::ws_per_group_bytes(M, K, group);                           // activation scales
   return bytes;
 }
 
@@ -142,9 +142,10 @@ jq_status jq_w4a4_linear(const uint8_t* q, const float* s_a, const uint8_t* qw, 
     return from_cuda(jq::launch_w4a4_skinny(p, s, d->sms));
   }
   uint8_t* a_op = static_cast<uint8_t*>(workspace);
-  cudaError_t e = jq::launch_expand_operand(q, M, K, a_op, s, d->sms);
+  float* corr = reinterpret_cast<float*>(a_op + jq::ws_image_bytes(M, K));
+  cudaError_t e = jq::launch_expand_operand(q, M, K, group, a_op, corr, s, d->sms);
   if (e != cudaSuccess) return JQ_ERR_CUDA;
-  jq::GemmProblem p{static_cast<int>(M), static_cast<int>(N), static_cast<int>(K), group, a_op, s_a, qw, s_w, bias,
+  jq::GemmProblem p{static_cast<int>(M), static_cast<int>(N), static_cast<int>(K), group, a_op, s_a, corr, qw, s_w, bias,
                     y_bf16, nullptr, d->status};
   return from_cuda(jq::launch_w4a4_gemm(p, s, d->sms));
 }
@@ -162,7 +163,8 @@ jq_status jq_fused_quant_linear(const void* x_bf16, int64_t ldx, const uint8_t* 
   if (d == nullptr) return JQ_ERR_UNSUPPORTED;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   uint8_t* a_op = static_cast<uint8_t*>(workspace);
-  float* s_a = reinterpret_cast<float*>(a_op + round_up(static_cast<size_t>(M), 128) * static_cast<size_t>(K));
+  float* corr = reinterpret_cast<float*>(a_op + jq::ws_image_bytes(M, K));
+  float* s_a = reinterpret_cast<float*>(a_op + jq::ws_image_bytes(M, K) + jq::ws_per_group_bytes(M, K, group));
   if (jq::skinny_supports(M, K, group)) {  // few tokens: packed codes in the workspace, then the weight-streaming kernel
     cudaError_t e = jq::launch_quantize_act(x_bf16, M, K, ldx, group, a_op, s_a, s, d->sms);
     if (e != cudaSuccess) return JQ_ERR_CUDA;
@@ -170,9 +172,9 @@ jq_status jq_fused_quant_linear(const void* x_bf16, int64_t ldx, const uint8_t* 
                         bias, y_bf16, d->status};
     return from_cuda(jq::launch_w4a4_skinny(p, s, d->sms));
   }
-  cudaError_t e = jq::launch_quantize_act_operand(x_bf16, M, K, ldx, group, a_op, s_a, s, d->sms);
+  cudaError_t e = jq::launch_quantize_act_operand(x_bf16, M, K, ldx, group, a_op, s_a, corr, s, d->sms);
   if (e != cudaSuccess) return JQ_ERR_CUDA;
-  jq::GemmProblem p{static_cast<int>(M), static_cast<int>(N), static_cast<int>(K), group, a_op, s_a, qw, s_w, bias,
+  jq::GemmProblem p{static_cast<int>(M), static_cast<int>(N), static_cast<int>(K), group, a_op, s_a, corr, qw, s_w, bias,
                     y_bf16, nullptr, d->status};
   return from_cuda(jq::launch_w4a4_gemm(p, s, d->sms));
 }
@@ -189,11 +191,12 @@ jq_status jq_w4a4_group_partials(const uint8_t* q, const uint8_t* qw, int32_t* a
   if (d == nullptr) return JQ_ERR_UNSUPPORTED;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   uint8_t* a_op = static_cast<uint8_t*>(workspace);
-  cudaError_t e = jq::launch_expand_operand(q, M, K, a_op, s, d->sms);
+  float* corr = reinterpret_cast<float*>(a_op + jq::ws_image_bytes(M, K));
+  cudaError_t e = jq::launch_expand_operand(q, M, K, group, a_op, corr, s, d->sms);
   if (e != cudaSuccess) return JQ_ERR_CUDA;
   // The export path needs scale tensors only for their layout; it never reads their values,
   // but the weight-scale tensor map must point at valid memory: reuse the packed weights.
-  jq::GemmProblem p{static_cast<int>(M), static_cast<int>(N), static_cast<int>(K), group, a_op, nullptr, qw,
+  jq::GemmProblem p{static_cast<int>(M), static_cast<int>(N), static_cast<int>(K), group, a_op, nullptr, corr, qw,
                     reinterpret_cast<const float*>(qw), nullptr, nullptr, acc, d->status};
   return from_cuda(jq::launch_w4a4_gemm(p, s, d->sms));
 }

@@ -98,6 +98,7 @@ struct Args {
   int sa_tma;            // activation scales come through the scale ring (groups % 4 == 0)
   const uint8_t* qw;
   const float* s_a;
+  const float* corr;     // [M, K/G]: 8 * the group's activation code sum in 2^-18 units (offset codes)
   const float* s_w;
   const float* bias;
   __nv_bfloat16* y;
@@ -130,6 +131,7 @@ __device__ __forceinline__ void drain_wait(uint64_t* bar, uint32_t parity, uint3
 // ------------------------------------------------------------------ drain + epilogue
 // Export path (jq_w4a4_group_partials): each thread owns one TMEM lane (row) and 128 columns
 // (32x32b loads) and writes the exact integer partials of every group.
+template <bool kOffset>
 __device__ __forceinline__ void drain_export(const Args& args, const Pair& pr, uint32_t tmem_base, const Bars& b,
                                              volatile int* abort_flag) {
   const uint32_t warp = warp_id(), lane = lane_id();
@@ -145,6 +147,7 @@ __device__ __forceinline__ void drain_export(const Args& args, const Pair& pr, u
     const bool row_ok = row < M;
     for (int g = 0; g < groups; ++g) {
       const uint32_t ab = chunk_it & 1u;
+      const float cr = (kOffset && row_ok) ? -__ldg(args.corr + (int64_t)row * groups + g) : 0.0f;
       // Warp-collective tcgen05.ld follows: the whole warp proceeds or none of it.
       ok = __all_sync(0xffffffffu, mbar_wait(&b.acc_full[ab], (chunk_it >> 1) & 1u, abort_flag, args.status));
       if (!ok) break;
@@ -161,7 +164,7 @@ __device__ __forceinline__ void drain_export(const Args& args, const Pair& pr, u
             const int col = col0 + cc * 32 + j;
             if (col < N)
               args.partials[((int64_t)row * N + col) * groups + g] =
-                  static_cast<int32_t>(__uint_as_float(r[j]) * kOperandUnitInv);
+                  static_cast<int32_t>((__uint_as_float(r[j]) + cr) * kOperandUnitInv);
           }
         }
       }
@@ -179,6 +182,7 @@ __device__ __forceinline__ void drain_export(const Args& args, const Pair& pr, u
 // only 32 weight scales and 4 activation scales per group; it loads all of them at the start of
 // the group (the tensor core's operand reads starve shared-memory loads issued one chunk ahead of
 // their use, but not loads issued a group ahead).
+template <bool kOffset>
 __device__ __forceinline__ void drain_linear(const Args& args, const Pair& pr, uint32_t tmem_base, const Bars& b,
                                              uint8_t* sSc, volatile int* abort_flag) {
   const uint32_t warp = warp_id(), lane = lane_id();
@@ -208,7 +212,8 @@ __device__ __forceinline__ void drain_linear(const Args& args, const Pair& pr, u
       float2 w[16];
 #pragma unroll
       for (int j = 0; j < 16; ++j) w[j] = *reinterpret_cast<const float2*>(sws + 8 * j);
-      float f[4];
+      // per row: s_a, and (offset-code weights, one group) -8 * the activation code sum
+      float f[4], cr[4];
 #pragma unroll
       for (int rr = 0; rr < 4; ++rr) {
         const int row = row0 + 8 * rr;
@@ -218,6 +223,7 @@ __device__ __forceinline__ void drain_linear(const Args& args, const Pair& pr, u
         else
           sa = row < M ? __ldg(args.s_a + (int64_t)row * groups + g) : 0.0f;
         f[rr] = sa;
+        cr[rr] = (kOffset && row < M) ? -__ldg(args.corr + (int64_t)row * groups + g) : 0.0f;
       }
       // Warp-collective tcgen05.ld follows: the whole warp proceeds or none of it (a timeout in
       // one lane must not leave the others in an aligned instruction).
@@ -250,7 +256,10 @@ __device__ __forceinline__ void drain_linear(const Args& args, const Pair& pr, u
           for (int rr = 0; rr < 4; ++rr) {  // r0: rows +0 / +8; r1: rows +16 / +24
             const uint32_t* r = rr < 2 ? r0 : r1;
             const int e = 2 * (rr & 1);
-            const float2 t = __fmul2_rn(make_float2(__uint_as_float(r[e]), __uint_as_float(r[e + 1])), w[j]);
+            float2 d = make_float2(__uint_as_float(r[e]), __uint_as_float(r[e + 1]));
+            if (kOffset)  // the exact partial: the offset-code sum less the correction (integers < 2^24)
+              d = __fadd2_rn(d, make_float2(cr[rr], cr[rr]));
+            const float2 t = __fmul2_rn(d, w[j]);
             float* yy = y + (rr * 16 + j) * 2;
             const float2 v = __ffma2_rn(t, make_float2(f[rr], f[rr]), make_float2(yy[0], yy[1]));
             yy[0] = v.x;
@@ -274,8 +283,8 @@ __device__ __forceinline__ void drain_linear(const Args& args, const Pair& pr, u
             const uint32_t* r = rr < 2 ? r0 : r1;
             const int e = 2 * (rr & 1);
             float* yy = y + (rr * 16 + j) * 2;
-            yy[0] = fmaf((__uint_as_float(r[e]) * kOperandUnitInv) * f[rr], w[j].x, yy[0]);
-            yy[1] = fmaf((__uint_as_float(r[e + 1]) * kOperandUnitInv) * f[rr], w[j].y, yy[1]);
+            yy[0] = fmaf(((__uint_as_float(r[e]) + cr[rr]) * kOperandUnitInv) * f[rr], w[j].x, yy[0]);
+            yy[1] = fmaf(((__uint_as_float(r[e + 1]) + cr[rr]) * kOperandUnitInv) * f[rr], w[j].y, yy[1]);
           }
         }
       }
@@ -487,6 +496,7 @@ __device__ __forceinline__ void unpack_advance(const Args& args, const Pair& pr,
 
 // Converts this group's stage of ring slot (q % kSlots) into the slot's B half for that stage
 // (or, for the missing second stage of an odd K-stage count, only signals the slot).
+template <bool kOffset>
 __device__ __forceinline__ bool unpack_store(const Args& args, uint8_t* sB, const Bars& b, uint32_t ug, uint32_t u,
                                              uint32_t q, bool has_stage, const uint4 (&buf)[kChunksPerThread],
                                              volatile int* abort_flag) {
@@ -500,7 +510,10 @@ __device__ __forceinline__ bool unpack_store(const Args& args, uint8_t* sB, cons
     for (int i = 0; i < kChunksPerThread; ++i) {
       const uint32_t r = (u >> 2) + 16u * i, r7 = r & 7u;
       uint4 lo, hi;
-      nib32_to_operand(buf[i], lo, hi);
+      if (kOffset)
+        nib32_to_operand_offset(buf[i], lo, hi);  // offset weight codes (operand.cuh)
+      else
+        nib32_to_operand(buf[i], lo, hi);
       const uint32_t row_base = dst + (r >> 3) * 1024u + r7 * 128u;
       st_shared_v4(row_base + (((2u * jc) ^ r7) << 4), lo.x, lo.y, lo.z, lo.w);
       st_shared_v4(row_base + (((2u * jc + 1u) ^ r7) << 4), hi.x, hi.y, hi.z, hi.w);
@@ -517,6 +530,7 @@ __device__ __forceinline__ bool unpack_store(const Args& args, uint8_t* sB, cons
   return true;
 }
 
+template <bool kOffset>
 __device__ __forceinline__ void unpack_role(const Args& args, const Pair& pr, uint8_t* sB, const Bars& b,
                                             volatile int* abort_flag) {
   const uint32_t ut = threadIdx.x - kUnpackWarp0 * 32;
@@ -533,13 +547,13 @@ __device__ __forceinline__ void unpack_role(const Args& args, const Pair& pr, ui
   unpack_advance(args, pr, lc);
   for (uint32_t q = 0; q < total; q += 2) {
     bool has = sc.j * kStagesPerSlot + (int)ug < args.k_stages;
-    if (!unpack_store(args, sB, b, ug, u, q, has, b0, abort_flag)) return;
+    if (!unpack_store<kOffset>(args, sB, b, ug, u, q, has, b0, abort_flag)) return;
     unpack_advance(args, pr, sc);
     unpack_load(args, pr, lc, ug, u, b0);
     unpack_advance(args, pr, lc);
     if (q + 1 < total) {
       has = sc.j * kStagesPerSlot + (int)ug < args.k_stages;
-      if (!unpack_store(args, sB, b, ug, u, q + 1, has, b1, abort_flag)) return;
+      if (!unpack_store<kOffset>(args, sB, b, ug, u, q + 1, has, b1, abort_flag)) return;
       unpack_advance(args, pr, sc);
       unpack_load(args, pr, lc, ug, u, b1);
       unpack_advance(args, pr, lc);
@@ -547,7 +561,11 @@ __device__ __forceinline__ void unpack_role(const Args& args, const Pair& pr, ui
   }
 }
 
-template <bool kExport>
+// kOffset: the weights enter the MMA as offset codes (operand.cuh) and the drain removes the
+// activation-sum correction -- used for one-group problems (G = K), where the drain's exact
+// subtraction runs once per tile; with several groups the drain is the busier role and the
+// weights keep the sign-magnitude form.
+template <bool kExport, bool kOffset>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     w4a4_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmSW,
                      const __grid_constant__ CUtensorMap tmSA, const Args args) {
@@ -616,12 +634,12 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
   if (warp >= kDrainWarp0) {
     asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;\n" ::"n"(kRegsDrain) : "memory");
     if (kExport)
-      drain_export(args, pr, tmem_base, b, abort_flag);
+      drain_export<kOffset>(args, pr, tmem_base, b, abort_flag);
     else
-      drain_linear(args, pr, tmem_base, b, sSc, abort_flag);
+      drain_linear<kOffset>(args, pr, tmem_base, b, sSc, abort_flag);
   } else if (warp >= kUnpackWarp0) {
     asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;\n" ::"n"(kRegsUnpack) : "memory");
-    unpack_role(args, pr, sB, b, abort_flag);
+    unpack_role<kOffset>(args, pr, sB, b, abort_flag);
   } else {
     asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;\n" ::"n"(kRegsCtl) : "memory");
     if (warp == kWarpProdA) {
@@ -646,7 +664,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
 }
 
 // ---------------------------------------------------------------- host side
-template <bool kExport>
+template <bool kExport, bool kOffset>
 cudaError_t launch_impl(const GemmProblem& p, cudaStream_t stream, int sms) {
   // The A-operand image seen as rows of 128 bytes: block (mt, kb) is rows (mt*k_stages + kb)*128..
   // One box is two consecutive blocks (two K stages of one 128-row tile).  Boxes that reach past
@@ -670,10 +688,10 @@ cudaError_t launch_impl(const GemmProblem& p, cudaStream_t stream, int sms) {
                              kScGroups, kBM, CU_TENSOR_MAP_SWIZZLE_NONE))
       return cudaErrorInvalidValue;
   }
-  static bool attr_set[2] = {false, false};
-  static int max_pairs[2] = {0, 0};
-  if (!attr_set[kExport]) {
-    cudaError_t e = cudaFuncSetAttribute(w4a4_gemm_kernel<kExport>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+  static bool attr_set = false;
+  static int max_pairs = 0;
+  if (!attr_set) {
+    cudaError_t e = cudaFuncSetAttribute(w4a4_gemm_kernel<kExport, kOffset>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          (int)kSmemBytes);
     if (e != cudaSuccess) return e;
     cudaLaunchConfig_t cfg = {};
@@ -681,12 +699,12 @@ cudaError_t launch_impl(const GemmProblem& p, cudaStream_t stream, int sms) {
     cfg.blockDim = dim3(kThreads, 1, 1);
     cfg.dynamicSmemBytes = kSmemBytes;
     int clusters = 0;
-    if (cudaOccupancyMaxActiveClusters(&clusters, w4a4_gemm_kernel<kExport>, &cfg) != cudaSuccess || clusters <= 0) {
+    if (cudaOccupancyMaxActiveClusters(&clusters, w4a4_gemm_kernel<kExport, kOffset>, &cfg) != cudaSuccess || clusters <= 0) {
       (void)cudaGetLastError();
       clusters = sms / 2;
     }
-    max_pairs[kExport] = clusters < sms / 2 ? clusters : sms / 2;
-    attr_set[kExport] = true;
+    max_pairs = clusters < sms / 2 ? clusters : sms / 2;
+    attr_set = true;
   }
   Args a;
   a.M = p.M;
@@ -703,13 +721,14 @@ cudaError_t launch_impl(const GemmProblem& p, cudaStream_t stream, int sms) {
   a.sa_tma = sa_tma ? 1 : 0;
   a.qw = p.qw;
   a.s_a = p.s_a;
+  a.corr = p.corr;
   a.s_w = p.s_w;
   a.bias = p.bias;
   a.y = static_cast<__nv_bfloat16*>(p.y);
   a.partials = p.partials;
   a.status = p.status;
-  const int pairs = a.num_tiles < max_pairs[kExport] ? a.num_tiles : max_pairs[kExport];
-  w4a4_gemm_kernel<kExport><<<2 * pairs, kThreads, kSmemBytes, stream>>>(tmA, tmSW, tmSA, a);
+  const int pairs = a.num_tiles < max_pairs ? a.num_tiles : max_pairs;
+  w4a4_gemm_kernel<kExport, kOffset><<<2 * pairs, kThreads, kSmemBytes, stream>>>(tmA, tmSW, tmSA, a);
   return cudaGetLastError();
 }
 
@@ -743,7 +762,10 @@ bool encode_2d(CUtensorMap* map, CUtensorMapDataType dtype, const void* base, ui
 
 cudaError_t launch_w4a4_gemm(const GemmProblem& p, cudaStream_t stream, int sms) {
   if (p.M == 0 || p.N == 0) return cudaSuccess;
-  return p.partials != nullptr ? launch_impl<true>(p, stream, sms) : launch_impl<false>(p, stream, sms);
+  const bool offset = p.G == p.K;  // one group: offset-code weights (see w4a4_gemm_kernel)
+  if (p.partials != nullptr)
+    return offset ? launch_impl<true, true>(p, stream, sms) : launch_impl<true, false>(p, stream, sms);
+  return offset ? launch_impl<false, true>(p, stream, sms) : launch_impl<false, false>(p, stream, sms);
 }
 
 }  // namespace jq

@@ -9,20 +9,32 @@ namespace jq {
 // bf16 activations [M, ldx] -> packed codes [M, K/2] + scales [M, K/G].
 cudaError_t launch_quantize_act(const void* x, int64_t M, int64_t K, int64_t ldx, int G, uint8_t* q, float* s_a,
                                 cudaStream_t stream, int sms);
-// bf16 activations -> GEMM operand bytes [M, K] + scales [M, K/G] (fused path).
+// bf16 activations -> GEMM operand bytes [M, K] + scales [M, K/G] + corrections [M, K/G]
+// (fused path; the corrections are 8 * the group's code sum in 2^-18 units, operand.cuh).
 cudaError_t launch_quantize_act_operand(const void* x, int64_t M, int64_t K, int64_t ldx, int G, uint8_t* op,
-                                        float* s_a, cudaStream_t stream, int sms);
+                                        float* s_a, float* corr, cudaStream_t stream, int sms);
 // fp32 weights [N, K] -> packed codes [N, K/2] + scales [K/G, N].
 cudaError_t launch_pack_weight(const float* w, int64_t N, int64_t K, int G, uint8_t* qw, float* s_w,
                                cudaStream_t stream, int sms);
-// packed codes [rows, K/2] -> operand bytes [rows, K].
-cudaError_t launch_expand_operand(const uint8_t* packed, int64_t rows, int64_t K, uint8_t* op, cudaStream_t stream,
-                                  int sms);
+// packed codes [rows, K/2] -> operand bytes [rows, K] + corrections [rows, K/G].
+cudaError_t launch_expand_operand(const uint8_t* packed, int64_t rows, int64_t K, int G, uint8_t* op, float* corr,
+                                  cudaStream_t stream, int sms);
+
+// Workspace of the GEMM path, each part on a 256-byte boundary: the A-operand image (whole
+// 128-row tiles of K operand bytes), the corrections fp32 [M, K/G], and for the fused path the
+// activation scales fp32 [M, K/G].
+inline size_t ws_image_bytes(int64_t M, int64_t K) {
+  return static_cast<size_t>((M + 127) / 128 * 128) * static_cast<size_t>(K);
+}
+inline size_t ws_per_group_bytes(int64_t M, int64_t K, int32_t G) {
+  return (static_cast<size_t>(M) * static_cast<size_t>(K / G) * sizeof(float) + 255) / 256 * 256;
+}
 
 struct GemmProblem {
   int M, N, K, G;
   const uint8_t* a_operand;  // [M, K] operand bytes (workspace)
   const float* s_a;          // [M, K/G]
+  const float* corr;         // [M, K/G]: 8 * sum of the group's activation codes, in 2^-18 units
   const uint8_t* qw;         // [N, K/2] packed
   const float* s_w;          // [K/G, N]
   const float* bias;         // [N] or nullptr

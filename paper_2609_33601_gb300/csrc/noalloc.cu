@@ -87,14 +87,14 @@ extern "C" jq_status jq_w4a4_linear_noalloc(const uint8_t* q, const float* s_a, 
                         y_bf16, d0->status};
     return jq::launch_w4a4_skinny(p, static_cast<cudaStream_t>(stream), d0->sms) == cudaSuccess ? JQ_OK : JQ_ERR_CUDA;
   }
-  // the operand image covers whole 128-row tiles
-  if ((static_cast<uint64_t>(M) + 127) / 128 * 128 * static_cast<uint64_t>(K) > kNoAllocScratchBytes)
-    return JQ_ERR_WORKSPACE;
+  // the operand image (whole 128-row tiles) and the per-group corrections
+  if (jq::ws_image_bytes(M, K) + jq::ws_per_group_bytes(M, K, group) > kNoAllocScratchBytes) return JQ_ERR_WORKSPACE;
   const NoAllocDevice* d = noalloc_device();
   if (d == nullptr) return JQ_ERR_UNSUPPORTED;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
-  if (jq::launch_expand_operand(q, M, K, d->scratch, s, d->sms) != cudaSuccess) return JQ_ERR_CUDA;
-  jq::GemmProblem p{static_cast<int>(M), static_cast<int>(N), static_cast<int>(K), group, d->scratch, s_a, qw, s_w,
-                    bias, y_bf16, nullptr, d->status};
+  float* corr = reinterpret_cast<float*>(d->scratch + jq::ws_image_bytes(M, K));
+  if (jq::launch_expand_operand(q, M, K, group, d->scratch, corr, s, d->sms) != cudaSuccess) return JQ_ERR_CUDA;
+  jq::GemmProblem p{static_cast<int>(M), static_cast<int>(N), static_cast<int>(K), group, d->scratch, s_a, corr, qw,
+                    s_w, bias, y_bf16, nullptr, d->status};
   return jq::launch_w4a4_gemm(p, s, d->sms) == cudaSuccess ? JQ_OK : JQ_ERR_CUDA;
 }

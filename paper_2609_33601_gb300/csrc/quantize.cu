@@ -1,5 +1,7 @@
 // quantize.cu -- symmetric INT4 quantisers (activations and weights) and the conversion of
-// packed codes into the GEMM's E4M3 operand bytes.
+// packed codes into the GEMM's E4M3 operand bytes.  Both producers of the GEMM's A operand also
+// write the correction the GEMM needs for its offset-code weights (operand.cuh): per row and
+// group, corr = 8 * sum_{k in g} qa[row, k] in the accumulator's units (2^-18), exact.
 //
 // Rule (per row and per run of G consecutive K elements; group64 / group128 as the paper fixes
 // them in Sec. 4.2 "FLUX" and the Appendix experimental-detail tables, G = K for per-token):
@@ -112,7 +114,7 @@ __device__ __forceinline__ void store32(uint8_t* out, int64_t row, int64_t col, 
 template <typename In, int L, bool kOperand, bool kScaleT>
 __global__ void __launch_bounds__(256) quantize_groups_kernel(const In* __restrict__ x, int64_t M, int64_t K,
                                                               int64_t ldx, uint8_t* __restrict__ out,
-                                                              float* __restrict__ scales) {
+                                                              float* __restrict__ scales, float* __restrict__ corr) {
   const int64_t chunks_per_row = K / 32;
   const int64_t total = M * chunks_per_row;
   const int64_t ng = K / (32 * L);
@@ -132,15 +134,22 @@ __global__ void __launch_bounds__(256) quantize_groups_kernel(const In* __restri
 #pragma unroll
     for (int o = 1; o < L; o <<= 1) a = fmaxf(a, __shfl_xor_sync(0xFFFFFFFFu, a, o));
     const float s = __fdiv_rn(a, 7.0f);
+    uint32_t pk[4] = {0x88888888u, 0x88888888u, 0x88888888u, 0x88888888u};  // sums to 0 past the end
     if (valid) {
-      uint32_t pk[4];
       quantize32(v, s, pk);
       store32<kOperand>(out, row, col, K, pk);
-      if ((threadIdx.x & (L - 1)) == 0) {
-        const int64_t g = col / (32 * L);
-        if constexpr (kScaleT) scales[g * M + row] = s;
-        else scales[row * ng + g] = s;
-      }
+    }
+    int cs = 0;
+    if constexpr (kOperand) {  // the group's code sum, over its L lanes
+      cs = valid ? nib32_sum(make_uint4(pk[0], pk[1], pk[2], pk[3])) : 0;
+#pragma unroll
+      for (int o = 1; o < L; o <<= 1) cs += __shfl_xor_sync(0xFFFFFFFFu, cs, o);
+    }
+    if (valid && (threadIdx.x & (L - 1)) == 0) {
+      const int64_t g = col / (32 * L);
+      if constexpr (kScaleT) scales[g * M + row] = s;
+      else scales[row * ng + g] = s;
+      if constexpr (kOperand) corr[row * ng + g] = (float)(8 * cs) * kOperandUnit;
     }
   }
 }
@@ -150,8 +159,9 @@ __global__ void __launch_bounds__(256) quantize_groups_kernel(const In* __restri
 template <typename In, bool kOperand, bool kScaleT>
 __global__ void __launch_bounds__(128) quantize_rows_kernel(const In* __restrict__ x, int64_t M, int64_t K,
                                                             int64_t ldx, uint8_t* __restrict__ out,
-                                                            float* __restrict__ scales) {
+                                                            float* __restrict__ scales, float* __restrict__ corr) {
   __shared__ float red[4];
+  __shared__ int red_cs[4];
   for (int64_t row = blockIdx.x; row < M; row += gridDim.x) {
     const In* xr = x + row * ldx;
     float a = 0.0f;
@@ -167,36 +177,89 @@ __global__ void __launch_bounds__(128) quantize_rows_kernel(const In* __restrict
     a = fmaxf(fmaxf(red[0], red[1]), fmaxf(red[2], red[3]));
     __syncthreads();
     const float s = __fdiv_rn(a, 7.0f);
+    int cs = 0;
     for (int64_t col = threadIdx.x * 32; col < K; col += 32 * blockDim.x) {
       float v[32];
       load32(xr + col, v);
       uint32_t pk[4];
       quantize32(v, s, pk);
       store32<kOperand>(out, row, col, K, pk);
+      if constexpr (kOperand) cs += nib32_sum(make_uint4(pk[0], pk[1], pk[2], pk[3]));
+    }
+    if constexpr (kOperand) {
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) cs += __shfl_xor_sync(0xFFFFFFFFu, cs, o);
+      if ((threadIdx.x & 31) == 0) red_cs[threadIdx.x >> 5] = cs;
+      __syncthreads();
+      cs = red_cs[0] + red_cs[1] + red_cs[2] + red_cs[3];
+      __syncthreads();
     }
     if (threadIdx.x == 0) {
       if constexpr (kScaleT) scales[row] = s;  // [1, M]
       else scales[row] = s;                    // [M, 1]
+      if constexpr (kOperand) corr[row] = (float)(8 * cs) * kOperandUnit;
     }
   }
 }
 
-// Packed codes [rows, K/2] -> the A-operand image (16 bytes in, 32 bytes out per thread).
+// Packed codes [rows, K/2] -> the A-operand image (16 bytes in, 32 bytes out per thread) and
+// the per-group corrections.  G = 32 * L: a group is L adjacent lanes (a row holds a multiple of
+// L chunks, so no group straddles a warp).
+template <int L>
 __global__ void __launch_bounds__(256) expand_operand_kernel(const uint8_t* __restrict__ packed, int64_t rows,
-                                                             int64_t K, uint8_t* __restrict__ image) {
+                                                             int64_t K, uint8_t* __restrict__ image,
+                                                             float* __restrict__ corr) {
   const int64_t per_row = K / 32;
   const int64_t chunks = rows * per_row;
   const uint32_t k_stages = static_cast<uint32_t>(K / kImageStageK);
-  for (int64_t c = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; c < chunks; c += (int64_t)gridDim.x * blockDim.x) {
-    const int64_t row = c / per_row;
-    const int64_t col = (c % per_row) * 32;
-    const uint4 p = __ldg(reinterpret_cast<const uint4*>(packed) + c);
-    uint4 lo, hi;
-    nib32_to_operand(p, lo, hi);
-    const uint32_t kb = static_cast<uint32_t>(col / kImageStageK);
-    const uint32_t c16 = static_cast<uint32_t>((col % kImageStageK) / 16);
-    *reinterpret_cast<uint4*>(image + image_chunk_offset(row, kb, c16, k_stages)) = lo;
-    *reinterpret_cast<uint4*>(image + image_chunk_offset(row, kb, c16 + 1, k_stages)) = hi;
+  for (int64_t c = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; c - (threadIdx.x & 31) < chunks;
+       c += (int64_t)gridDim.x * blockDim.x) {
+    const bool valid = c < chunks;
+    const int64_t row = valid ? c / per_row : 0;
+    const int64_t col = valid ? (c % per_row) * 32 : 0;
+    const uint4 p = valid ? __ldg(reinterpret_cast<const uint4*>(packed) + c)
+                          : make_uint4(0x88888888u, 0x88888888u, 0x88888888u, 0x88888888u);
+    if (valid) {
+      uint4 lo, hi;
+      nib32_to_operand(p, lo, hi);
+      const uint32_t kb = static_cast<uint32_t>(col / kImageStageK);
+      const uint32_t c16 = static_cast<uint32_t>((col % kImageStageK) / 16);
+      *reinterpret_cast<uint4*>(image + image_chunk_offset(row, kb, c16, k_stages)) = lo;
+      *reinterpret_cast<uint4*>(image + image_chunk_offset(row, kb, c16 + 1, k_stages)) = hi;
+    }
+    int cs = valid ? nib32_sum(p) : 0;
+#pragma unroll
+    for (int o = 1; o < L; o <<= 1) cs += __shfl_xor_sync(0xFFFFFFFFu, cs, o);
+    if (valid && (threadIdx.x & (L - 1)) == 0) corr[row * (per_row / L) + col / (32 * L)] = (float)(8 * cs) * kOperandUnit;
+  }
+}
+
+// G = K: one block per row (the row's code sum is a block reduction).
+__global__ void __launch_bounds__(128) expand_operand_rows_kernel(const uint8_t* __restrict__ packed, int64_t rows,
+                                                                  int64_t K, uint8_t* __restrict__ image,
+                                                                  float* __restrict__ corr) {
+  __shared__ int red_cs[4];
+  const int64_t per_row = K / 32;
+  const uint32_t k_stages = static_cast<uint32_t>(K / kImageStageK);
+  for (int64_t row = blockIdx.x; row < rows; row += gridDim.x) {
+    int cs = 0;
+    for (int64_t i = threadIdx.x; i < per_row; i += blockDim.x) {
+      const uint4 p = __ldg(reinterpret_cast<const uint4*>(packed) + row * per_row + i);
+      uint4 lo, hi;
+      nib32_to_operand(p, lo, hi);
+      const int64_t col = i * 32;
+      const uint32_t kb = static_cast<uint32_t>(col / kImageStageK);
+      const uint32_t c16 = static_cast<uint32_t>((col % kImageStageK) / 16);
+      *reinterpret_cast<uint4*>(image + image_chunk_offset(row, kb, c16, k_stages)) = lo;
+      *reinterpret_cast<uint4*>(image + image_chunk_offset(row, kb, c16 + 1, k_stages)) = hi;
+      cs += nib32_sum(p);
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) cs += __shfl_xor_sync(0xFFFFFFFFu, cs, o);
+    if ((threadIdx.x & 31) == 0) red_cs[threadIdx.x >> 5] = cs;
+    __syncthreads();
+    if (threadIdx.x == 0) corr[row] = (float)(8 * (red_cs[0] + red_cs[1] + red_cs[2] + red_cs[3])) * kOperandUnit;
+    __syncthreads();
   }
 }
 
@@ -210,17 +273,17 @@ int grid_for(int64_t work_items, int threads, int sms) {
 
 template <typename In, bool kOperand, bool kScaleT>
 cudaError_t launch_quantize(const In* x, int64_t M, int64_t K, int64_t ldx, int G, uint8_t* out, float* scales,
-                            cudaStream_t stream, int sms) {
+                            float* corr, cudaStream_t stream, int sms) {
   if (M == 0) return cudaSuccess;
   if (G == K) {
     int blocks = static_cast<int>(M < static_cast<int64_t>(sms) * 16 ? M : static_cast<int64_t>(sms) * 16);
-    quantize_rows_kernel<In, kOperand, kScaleT><<<blocks, 128, 0, stream>>>(x, M, K, ldx, out, scales);
+    quantize_rows_kernel<In, kOperand, kScaleT><<<blocks, 128, 0, stream>>>(x, M, K, ldx, out, scales, corr);
   } else if (G == 64) {
     quantize_groups_kernel<In, 2, kOperand, kScaleT>
-        <<<grid_for(M * (K / 32), 256, sms), 256, 0, stream>>>(x, M, K, ldx, out, scales);
+        <<<grid_for(M * (K / 32), 256, sms), 256, 0, stream>>>(x, M, K, ldx, out, scales, corr);
   } else {
     quantize_groups_kernel<In, 4, kOperand, kScaleT>
-        <<<grid_for(M * (K / 32), 256, sms), 256, 0, stream>>>(x, M, K, ldx, out, scales);
+        <<<grid_for(M * (K / 32), 256, sms), 256, 0, stream>>>(x, M, K, ldx, out, scales, corr);
   }
   return cudaGetLastError();
 }
@@ -230,25 +293,32 @@ cudaError_t launch_quantize(const In* x, int64_t M, int64_t K, int64_t ldx, int 
 cudaError_t launch_quantize_act(const void* x, int64_t M, int64_t K, int64_t ldx, int G, uint8_t* q, float* s_a,
                                 cudaStream_t stream, int sms) {
   return launch_quantize<__nv_bfloat16, false, false>(static_cast<const __nv_bfloat16*>(x), M, K, ldx, G, q, s_a,
-                                                      stream, sms);
+                                                      nullptr, stream, sms);
 }
 
 cudaError_t launch_quantize_act_operand(const void* x, int64_t M, int64_t K, int64_t ldx, int G, uint8_t* op,
-                                        float* s_a, cudaStream_t stream, int sms) {
+                                        float* s_a, float* corr, cudaStream_t stream, int sms) {
   return launch_quantize<__nv_bfloat16, true, false>(static_cast<const __nv_bfloat16*>(x), M, K, ldx, G, op, s_a,
-                                                     stream, sms);
+                                                     corr, stream, sms);
 }
 
 cudaError_t launch_pack_weight(const float* w, int64_t N, int64_t K, int G, uint8_t* qw, float* s_w,
                                cudaStream_t stream, int sms) {
-  return launch_quantize<float, false, true>(w, N, K, K, G, qw, s_w, stream, sms);
+  return launch_quantize<float, false, true>(w, N, K, K, G, qw, s_w, nullptr, stream, sms);
 }
 
-cudaError_t launch_expand_operand(const uint8_t* packed, int64_t rows, int64_t K, uint8_t* op, cudaStream_t stream,
-                                  int sms) {
+cudaError_t launch_expand_operand(const uint8_t* packed, int64_t rows, int64_t K, int G, uint8_t* op, float* corr,
+                                  cudaStream_t stream, int sms) {
   const int64_t chunks = rows * (K / 32);
   if (chunks == 0) return cudaSuccess;
-  expand_operand_kernel<<<grid_for(chunks, 256, sms), 256, 0, stream>>>(packed, rows, K, op);
+  if (G == K) {
+    const int blocks = static_cast<int>(rows < static_cast<int64_t>(sms) * 16 ? rows : static_cast<int64_t>(sms) * 16);
+    expand_operand_rows_kernel<<<blocks, 128, 0, stream>>>(packed, rows, K, op, corr);
+  } else if (G == 64) {
+    expand_operand_kernel<2><<<grid_for(chunks, 256, sms), 256, 0, stream>>>(packed, rows, K, op, corr);
+  } else {
+    expand_operand_kernel<4><<<grid_for(chunks, 256, sms), 256, 0, stream>>>(packed, rows, K, op, corr);
+  }
   return cudaGetLastError();
 }
 

@@ -51,9 +51,11 @@ def test_workspace_size(lib):
     f = lib.jq_workspace_size
     f.argtypes = [ctypes.c_int64] * 3 + [ctypes.c_int32] * 2
     f.restype = ctypes.c_size_t
-    assert f(1024, 12288, 4096, 128, 0) == 1024 * 4096
-    assert f(1024, 12288, 4096, 128, 1) == 1024 * 4096 + 1024 * 32 * 4
-    assert f(3, 8, 256, 64, 0) == 128 * 256  # the operand image covers whole 128-row tiles
+    # operand image (whole 128-row tiles of K bytes), then one fp32 per token and group (the
+    # activation-sum corrections), then for the fused path the activation scales; 256-byte parts
+    assert f(1024, 12288, 4096, 128, 0) == 1024 * 4096 + 1024 * 32 * 4
+    assert f(1024, 12288, 4096, 128, 1) == 1024 * 4096 + 2 * 1024 * 32 * 4
+    assert f(3, 8, 256, 64, 0) == 128 * 256 + 256
     assert f(0, 8, 256, 64, 0) == 0
 
 
