@@ -59,7 +59,7 @@ FP8_PER_BF16 = 2.0  # nominal dense FP8 / BF16 tensor-core ratio on GB300 (4.5 /
 # source the capture was taken on; once the kernel changes the figure no longer applies and the
 # bench reports null.
 KERNEL_TRAFFIC = {
-    ("dllm", "cf7dd0ff7f1c9c83"): 31.239e6 + 0.138e6,  # profiles/w4a4_gemm_dllm_full.md
+    ("dllm", "cc6574cef178495b"): 31.244e6 + 0.123e6,  # profiles/w4a4_gemm_dllm_full.md
     ("sweep_m1", "b8c4d652385e2708"): 25.288e6,  # profiles/w4a4_skinny_sweep_m1_full.md
 }
 
