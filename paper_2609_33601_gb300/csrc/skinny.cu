@@ -82,8 +82,8 @@ struct Layout {
   static constexpr uint32_t kOffPk = 0;
   static constexpr uint32_t kOffOp = kOffPk + kPkSlots * kPkSlot;
   static constexpr uint32_t kOffSa = kOffOp + kOpSlots * kOpSlot;  // s_a [kSaRing][kMp], then 8 sum qa [kSaRing][kMp]
-  static constexpr uint32_t kOffCorr = kOffSa + 2 * kSaRing * kMp * 4;  // G = K: 8 sum qa per unpack group [2][kMp]
-  static constexpr uint32_t kOffBar = kOffCorr + kUnpackGroups * kMp * 4;
+  static constexpr uint32_t kOffCorr = kOffSa + 2 * kSaRing * kMp * 4;  // G = K: 8 sum qa per unpack group [3][kMp]
+  static constexpr uint32_t kOffBar = kOffCorr + (kUnpackGroups + 1) * kMp * 4;
   static constexpr uint32_t kNumBars = 2 * kPkSlots + 2 * kOpSlots + 8 + 2 + 2 * kSaRing + 1;
   static constexpr uint32_t kOffMisc = kOffBar + kNumBars * 8;
   static constexpr uint32_t kSmemBytes = kOffMisc + 16;
@@ -168,7 +168,8 @@ __device__ __forceinline__ void tma_role(const SkArgs& a, const Range& rg, int n
 }
 
 // ------------------------------------------------------------------ unpack
-// Group ug converts packed slots j = ug, ug + 2, ...: both K stages of the slot.
+// Group ug (of ngroups: 2, or 3 for G = K where the drain warps join in while they have nothing
+// to drain) converts packed slots j = ug, ug + ngroups, ...: both K stages of the slot.
 // Code sums: the 8 chunks of a token row sit in 8 consecutive lanes, so a group's sum (2 chunks
 // for G = 64, 4 for G = 128, all 8 and then all slots for G = K) is a butterfly over 1-3 lanes.
 // The drain removes 8 * sum qa, in the accumulator's units (2^-18), from the offset-code MMA;
@@ -180,7 +181,7 @@ __device__ __forceinline__ void tma_role(const SkArgs& a, const Range& rg, int n
 // each as two operand chunks into the shared-memory operand ring.
 template <int kMp>
 __device__ __forceinline__ void unpack_role(const SkArgs& a, const Range& rg, uint8_t* smem, uint32_t tmem_base,
-                                            const SkBars& b, volatile int* abort_flag) {
+                                            const SkBars& b, int ngroups, volatile int* abort_flag) {
   using L = Layout<kMp>;
   constexpr int kPkSlots = L::kPkSlots;
   constexpr int kXChunks = kMp * 8 / kUnpackGroupThreads;  // token chunks per thread per slot
@@ -198,7 +199,7 @@ __device__ __forceinline__ void unpack_role(const SkArgs& a, const Range& rg, ui
   int tot[kXChunks];  // G = K: running code sums of this thread's token rows
 #pragma unroll
   for (int i = 0; i < kXChunks; ++i) tot[i] = 0;
-  for (int j = (int)ug; j < nslots; j += kUnpackGroups) {
+  for (int j = (int)ug; j < nslots; j += ngroups) {
     const int nst_j = rg.nst - j * kStPerSlot < kStPerSlot ? rg.nst - j * kStPerSlot : kStPerSlot;
     const uint32_t p = (uint32_t)j % kPkSlots, os = (uint32_t)j % kOpSlots;
     if (!__all_sync(0xffffffffu, mbar_wait(&b.pk_full[p], ring_parity(j, kPkSlots), abort_flag, a.status))) return;
@@ -531,8 +532,8 @@ __device__ __forceinline__ void drain_role(const SkArgs& a, const Range& rg, int
     const bool ok = mbar_wait(b.corr_full, 0, abort_flag, a.status);
     const float* corr = reinterpret_cast<const float*>(smem + L::kOffCorr);
 #pragma unroll
-    for (int i = 0; i < kH; ++i)  // the two shares and the difference are exact integers (units 2^-18)
-      y[i] = ok ? y[i] - (corr[hf * kH + i] + corr[kMp + hf * kH + i]) : 0.0f;
+    for (int i = 0; i < kH; ++i)  // the shares and the difference are exact integers (units 2^-18)
+      y[i] = ok ? y[i] - (corr[hf * kH + i] + corr[kMp + hf * kH + i] + corr[2 * kMp + hf * kH + i]) : 0.0f;
   }
   float* red = reinterpret_cast<float*>(smem + L::kOffPk);  // [kMp][128]
 #pragma unroll
@@ -569,29 +570,33 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int n0 = (int)(blockIdx.x / a.split) * kRows;
   const Range rg = k_range(a, rank);
   const uint32_t warp = warp_id(), lane = lane_id();
-  if (threadIdx.x == 0) {
-    *abort_flag = 0;
-    for (int i = 0; i < L::kPkSlots; ++i) {
-      mbar_init(&b.pk_full[i], 1);                                  // the producer's expect_tx
+  const bool single = a.groups == 1;
+  const int ngroups = single ? kUnpackGroups + 1 : kUnpackGroups;  // G = K: the drain warps unpack too
+  if (warp == kWarpMma1) {  // barrier setup, spread over one warp
+    if (lane == 0) *abort_flag = 0;
+    for (int i = (int)lane; i < L::kPkSlots; i += 32) {
+      mbar_init(&b.pk_full[i], 1);                   // the producer's expect_tx
       mbar_init(&b.pk_empty[i], kUnpackGroupWarps);  // the slot's unpack group
     }
-    for (int i = 0; i < kOpSlots; ++i) {
+    for (int i = (int)lane; i < kOpSlots; i += 32) {
       mbar_init(&b.op_full[i], kUnpackGroupWarps);  // the slot's unpack group
       mbar_init(&b.op_empty[i], 1);
     }
-    for (int i = 0; i < 4; ++i) {
-      mbar_init(&b.acc_full[i], 1);
-      mbar_init(&b.acc_empty[i], kNumDrainWarps);
+    if (lane < 4) {
+      mbar_init(&b.acc_full[lane], 1);
+      mbar_init(&b.acc_empty[lane], kNumDrainWarps);
     }
-    for (int i = 0; i < 2; ++i) mbar_init(&b.mma_done[i], 1);
-    for (int i = 0; i < kSaRing; ++i) {
+    if (lane < 2) mbar_init(&b.mma_done[lane], 1);
+    for (int i = (int)lane; i < kSaRing; i += 32) {
       mbar_init(&b.sa_full[i], 1 + kUnpackGroupWarps);  // the scale warp and one unpack group
       mbar_init(&b.sa_empty[i], kNumDrainWarps);
     }
-    mbar_init(b.corr_full, kUnpackGroups * kUnpackGroupWarps);
+    if (lane == 0) mbar_init(b.corr_full, ngroups * kUnpackGroupWarps);
     fence_mbar_init();
-    tma_prefetch_desc(&tmW);
-    tma_prefetch_desc(&tmX);
+    if (lane == 0) {
+      tma_prefetch_desc(&tmW);
+      tma_prefetch_desc(&tmX);
+    }
   }
   if (warp == kWarpMma) {
     tmem_alloc(tmem_slot, L::kTmemCols);
@@ -616,11 +621,12 @@ __global__ void __launch_bounds__(kThreads, 1)
   static_assert(kDrainWarp0 == 12 && kUnpackWarp0 == 4, "the register split is per warpgroup");
   if (drain) {
     asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;\n" ::"n"(kRegsDrain) : "memory");
+    if (single) unpack_role<kMp>(a, rg, smem, tmem_base, b, ngroups, abort_flag);  // group 2 (warps 12-15)
     drain_role<kMp>(a, rg, n0, tmem_base, smem, b, abort_flag);
     __syncwarp();
     asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;\n" ::"n"(kRegsLaunch) : "memory");
   } else if (warp >= kUnpackWarp0) {
-    unpack_role<kMp>(a, rg, smem, tmem_base, b, abort_flag);
+    unpack_role<kMp>(a, rg, smem, tmem_base, b, ngroups, abort_flag);
   } else {
     asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;\n" ::"n"(kRegsCtl) : "memory");
     if (warp == kWarpScale) {
