@@ -81,8 +81,11 @@ struct Layout {
   static constexpr uint32_t kOpSlot = kStPerSlot * kOpB;  // the two stages of a slot, one after the other
   static constexpr uint32_t kOffPk = 0;
   static constexpr uint32_t kOffOp = kOffPk + kPkSlots * kPkSlot;
-  static constexpr uint32_t kOffSa = kOffOp + kOpSlots * kOpSlot;  // s_a [kSaRing][kMp], then 8 sum qa [kSaRing][kMp]
-  static constexpr uint32_t kOffCorr = kOffSa + 2 * kSaRing * kMp * 4;  // G = K: 8 sum qa per unpack group [3][kMp]
+  // scale ring: per group and token the pair (s_a * 2^18 -- or s_a where that overflows --,
+  // 8 sum qa in 2^-18 units) [kSaRing][kMp], then one flag per group (1: s_a * 2^18 is finite)
+  static constexpr uint32_t kOffSa = kOffOp + kOpSlots * kOpSlot;
+  static constexpr uint32_t kOffSaFlag = kOffSa + 2 * kSaRing * kMp * 4;
+  static constexpr uint32_t kOffCorr = kOffSaFlag + kSaRing * 4;  // G = K: 8 sum qa per unpack group [3][kMp]
   static constexpr uint32_t kOffBar = kOffCorr + (kUnpackGroups + 1) * kMp * 4;
   static constexpr uint32_t kNumBars = 2 * kPkSlots + 2 * kOpSlots + 8 + 2 + 2 * kSaRing + 1;
   static constexpr uint32_t kOffMisc = kOffBar + kNumBars * 8;
@@ -195,7 +198,7 @@ __device__ __forceinline__ void unpack_role(const SkArgs& a, const Range& rg, ui
   const bool single = a.groups == 1;
   const int gpst = groups_per_stage(a), gps = kStPerSlot * gpst;
   const uint32_t c8 = u & 7u;  // the chunk of its token row this thread holds
-  float* c_ring = reinterpret_cast<float*>(smem + L::kOffSa) + kSaRing * kMp;
+  float* sc_ring = reinterpret_cast<float*>(smem + L::kOffSa);  // pairs (s_a', c): c is the second
   int tot[kXChunks];  // G = K: running code sums of this thread's token rows
 #pragma unroll
   for (int i = 0; i < kXChunks; ++i) tot[i] = 0;
@@ -287,7 +290,7 @@ __device__ __forceinline__ void unpack_role(const SkArgs& a, const Range& rg, ui
 #pragma unroll
       for (int i = 0; i < kXChunks; ++i) {
         const uint32_t r = (u + kUnpackGroupThreads * (uint32_t)i) >> 3;
-        if (c8 == (uint32_t)(q * cpg)) c_ring[so * kMp + r] = (float)(8 * xs[i]) * kOperandUnit;
+        if (c8 == (uint32_t)(q * cpg)) sc_ring[2 * (so * kMp + r) + 1] = (float)(8 * xs[i]) * kOperandUnit;
       }
       __syncwarp();
       if ((u & 31u) == 0) mbar_arrive(&b.sa_full[so]);
@@ -307,8 +310,10 @@ __device__ __forceinline__ void unpack_role(const SkArgs& a, const Range& rg, ui
 
 // ------------------------------------------------------------------ activation scales
 // One warp (lane m = token): the scales of this CTA's groups into the ring, kSaBatch groups per
-// batch of loads so that one load latency covers several groups.  Rows >= M get 0.  A ring slot
-// is full once this warp and the unpack warps (the code sums) have written it.
+// batch of loads so that one load latency covers several groups.  Rows >= M get 0.  Each group's
+// s_a go in already multiplied by 2^18 unless that overflows for one of them (|s_a| > 2^110),
+// with a flag saying which, so the drain neither re-checks nor re-scales.  A ring slot is full
+// once this warp and the unpack warps (the code sums) have written it.
 template <int kMp>
 __device__ __forceinline__ void scale_role(const SkArgs& a, const Range& rg, uint8_t* smem, const SkBars& b,
                                            volatile int* abort_flag) {
@@ -316,7 +321,8 @@ __device__ __forceinline__ void scale_role(const SkArgs& a, const Range& rg, uin
   constexpr int kPer = kMp > 32 ? kMp / 32 : 1;  // tokens per lane
   constexpr int kSaBatch = 8;
   const uint32_t lane = lane_id();
-  float* sa_ring = reinterpret_cast<float*>(smem + L::kOffSa);
+  float* sc_ring = reinterpret_cast<float*>(smem + L::kOffSa);  // pairs (s_a', c): s_a' is the first
+  int* flags = reinterpret_cast<int*>(smem + L::kOffSaFlag);
   const int ng = drain_groups(a, rg);
   if (ng == 0 || a.groups == 1) return;  // G = K: the final pass reads s_a itself
   const int g0 = rg.st0 * groups_per_stage(a);
@@ -337,11 +343,16 @@ __device__ __forceinline__ void scale_role(const SkArgs& a, const Range& rg, uin
       const uint32_t it = (uint32_t)(gb + j), o = it % kSaRing;
       if (!__all_sync(0xffffffffu, mbar_wait(&b.sa_empty[o], ring_parity(it, kSaRing) ^ 1u, abort_flag, a.status)))
         return;
+      bool finite = true;
+#pragma unroll
+      for (int h = 0; h < kPer; ++h) finite = finite && fabsf(v[j][h]) * kOperandUnitInv <= FLT_MAX;
+      finite = __all_sync(0xffffffffu, finite);
 #pragma unroll
       for (int h = 0; h < kPer; ++h) {
         const int m = (int)lane + 32 * h;
-        if (m < kMp) sa_ring[o * kMp + m] = v[j][h];
+        if (m < kMp) sc_ring[2 * (o * kMp + m)] = finite ? v[j][h] * kOperandUnitInv : v[j][h];
       }
+      if (lane == 0) flags[o] = finite ? 1 : 0;
       __syncwarp();
       if (lane == 0) mbar_arrive(&b.sa_full[o]);
     }
@@ -449,7 +460,8 @@ __device__ __forceinline__ void drain_role(const SkArgs& a, const Range& rg, int
   const uint32_t ch = quarter * 32u + lane;
   const int n = n0 + (int)ch;
   const bool single = a.groups == 1;
-  const float* sa_ring = reinterpret_cast<const float*>(smem + L::kOffSa);
+  const float* sc_ring = reinterpret_cast<const float*>(smem + L::kOffSa);  // pairs (s_a', c)
+  const int* flags = reinterpret_cast<const int*>(smem + L::kOffSaFlag);
   const int ng = drain_groups(a, rg);
   const int g0 = single ? 0 : rg.st0 * groups_per_stage(a);
   float y[kH];
@@ -462,10 +474,15 @@ __device__ __forceinline__ void drain_role(const SkArgs& a, const Range& rg, int
   const int gps = kStPerSlot * groups_per_stage(a);
   const int parts = single ? (nslots > 1 ? 2 : 1) : 1;
   float sw_next = (!single && ng > 0 && n < a.N) ? __ldg(a.s_w + (int64_t)g0 * a.N + n) : 0.0f;
+  int gq = 0, js = 0;  // the group's position within its slot, and the slot (no division per group)
   for (int it = 0; it < ng * parts; ++it) {
     const int gi = single ? 0 : it;
-    const uint32_t e = single ? (uint32_t)it : (uint32_t)(gi / gps) & 1u;
-    const uint32_t chunk = single ? 0u : (uint32_t)((gi / gps) >> 1) * (uint32_t)gps + (uint32_t)(gi % gps);
+    const uint32_t e = single ? (uint32_t)it : (uint32_t)js & 1u;
+    const uint32_t chunk = single ? 0u : (uint32_t)(js >> 1) * (uint32_t)gps + (uint32_t)gq;
+    if (!single && ++gq == gps) {
+      gq = 0;
+      ++js;
+    }
     const uint32_t ab = 2u * e + (chunk & 1u);
     const float sw = sw_next;
     if (!single && gi + 1 < ng && n < a.N) sw_next = __ldg(a.s_w + (int64_t)(g0 + gi + 1) * a.N + n);
@@ -477,19 +494,10 @@ __device__ __forceinline__ void drain_role(const SkArgs& a, const Range& rg, int
     if (!__all_sync(0xffffffffu, ok)) break;
     tc_fence_after();
     const uint32_t taddr = tmem_base + ((quarter * 32u) << 16) + ab * kMp + hf * kH;
-    const float* sas = sa_ring + so * kMp + hf * kH;
-    const float* cas = sas + kSaRing * kMp;  // 8 * sum qa of the group, per token
-    // overflow-safe form needed only if some s_a * 2^18 of these columns overflows; the choice
-    // is the warp's (no lane may skip the warp-collective loads below)
-    bool finite = true;
-    if (!single) {
-#pragma unroll
-      for (int i = 0; i < kH; i += 4) {
-        const float4 s4 = *reinterpret_cast<const float4*>(sas + i);
-        finite = finite && fmaxf(fmaxf(s4.x, s4.y), fmaxf(s4.z, s4.w)) * kOperandUnitInv <= FLT_MAX;
-      }
-    }
-    finite = __all_sync(0xffffffffu, finite);
+    const float* scs = sc_ring + 2 * (so * kMp + hf * kH);  // (s_a', c) of the group's tokens
+    // the overflow-safe form is needed only if some s_a * 2^18 of the group overflows (the scale
+    // warp's flag; the same for every lane, so no lane skips the warp-collective loads below)
+    const bool finite = single || __all_sync(0xffffffffu, flags[so] != 0);
 #pragma unroll
     for (int c = 0; c < kH / 8; ++c) {
       uint32_t r[8];
@@ -506,21 +514,20 @@ __device__ __forceinline__ void drain_role(const SkArgs& a, const Range& rg, int
       } else if (finite) {
 #pragma unroll
         for (int i = 0; i < 8; i += 2) {
-          const float2 s2 = *reinterpret_cast<const float2*>(sas + c * 8 + i);
-          const float2 c2 = *reinterpret_cast<const float2*>(cas + c * 8 + i);
+          const float4 sc = *reinterpret_cast<const float4*>(scs + 2 * (c * 8 + i));  // s_a'0, c0, s_a'1, c1
           // exact: both are integers below 2^24 (in units of 2^-18)
-          const float2 d = make_float2(__uint_as_float(r[i]) - c2.x, __uint_as_float(r[i + 1]) - c2.y);
+          const float2 d = make_float2(__uint_as_float(r[i]) - sc.y, __uint_as_float(r[i + 1]) - sc.w);
           const float2 t = __fmul2_rn(d, make_float2(sw, sw));
-          const float2 v = __ffma2_rn(t, make_float2(s2.x * kOperandUnitInv, s2.y * kOperandUnitInv),
-                                      make_float2(y[c * 8 + i], y[c * 8 + i + 1]));
+          const float2 v = __ffma2_rn(t, make_float2(sc.x, sc.z), make_float2(y[c * 8 + i], y[c * 8 + i + 1]));
           y[c * 8 + i] = v.x;
           y[c * 8 + i + 1] = v.y;
         }
       } else {  // |s_a| > 2^110 somewhere: apply 2^18 to the exact partials first
 #pragma unroll
-        for (int i = 0; i < 8; ++i)
-          y[c * 8 + i] =
-              fmaf(((__uint_as_float(r[i]) - cas[c * 8 + i]) * kOperandUnitInv) * sas[c * 8 + i], sw, y[c * 8 + i]);
+        for (int i = 0; i < 8; ++i) {
+          const float2 sc = *reinterpret_cast<const float2*>(scs + 2 * (c * 8 + i));  // s_a (unscaled), c
+          y[c * 8 + i] = fmaf(((__uint_as_float(r[i]) - sc.y) * kOperandUnitInv) * sc.x, sw, y[c * 8 + i]);
+        }
       }
     }
     if (!single) {
