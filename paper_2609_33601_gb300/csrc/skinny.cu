@@ -63,10 +63,17 @@ constexpr int kUnpackGroupWarps = kUnpackGroupThreads / 32;
 constexpr int kDrainWarp0 = 12, kNumDrainWarps = 4;
 constexpr int kSaRing = 32;  // activation-scale ring (groups)
 // Register split per warpgroup while the roles run (totals the 512 x 128 registers of the launch):
-// warps 0-3 (MMA issuers, scales, TMA) 80, unpack 128, drain (up to 64 running sums) 176.  Every
-// warpgroup returns to 128 for the reduction that all warps take part in.
-constexpr int kRegsCtl = 80, kRegsUnpack = 128, kRegsDrain = 176, kRegsLaunch = 128;
-static_assert(kRegsCtl + 2 * kRegsUnpack + kRegsDrain == 4 * kRegsLaunch, "register split must use the launch budget");
+// warps 0-3 (MMA issuers, scales, TMA) 80, unpack 128, drain 176; with 64 tokens the drain's 64
+// running sums take 8 more from warps 0-3.  Every warpgroup returns to 128 for the reduction
+// that all warps take part in.
+constexpr int kRegsUnpack = 128, kRegsLaunch = 128;
+template <int kMp>
+constexpr int kRegsCtl = kMp == 64 ? 72 : 80;
+template <int kMp>
+constexpr int kRegsDrain = kMp == 64 ? 184 : 176;
+static_assert(kRegsCtl<64> + 2 * kRegsUnpack + kRegsDrain<64> == 4 * kRegsLaunch &&
+                  kRegsCtl<32> + 2 * kRegsUnpack + kRegsDrain<32> == 4 * kRegsLaunch,
+              "register split must use the launch budget");
 constexpr int kMaxSplit = 8;
 static_assert(kDrainWarp0 % 4 == 0, "drain warp w reads TMEM lanes 32 * (w % 4)");
 static_assert(kSkinnyMaxKOneGroup <= kOffsetMaxRun && kSkinnyMaxKOneGroup % kBK == 0, "exact one-group ranges");
@@ -467,72 +474,115 @@ __device__ __forceinline__ void drain_role(const SkArgs& a, const Range& rg, int
   float y[kH];
 #pragma unroll
   for (int i = 0; i < kH; ++i) y[i] = 0.0f;
-  // Group gi was accumulated by the issuer of its slot j (e = j % 2) as that issuer's chunk
-  // (j / 2) * gps + gi % gps, gps = groups per slot.  G = K: both issuers hold a part of the one
-  // group (the second only if the range has more than one slot).
+  // G = K: both issuers hold a part of the one group (the second only if the range has more
+  // than one slot), in their first accumulators.
   const int nslots = (rg.nst + kStPerSlot - 1) / kStPerSlot;
   const int gps = kStPerSlot * groups_per_stage(a);
   const int parts = single ? (nslots > 1 ? 2 : 1) : 1;
-  float sw_next = (!single && ng > 0 && n < a.N) ? __ldg(a.s_w + (int64_t)g0 * a.N + n) : 0.0f;
-  int gq = 0, js = 0;  // the group's position within its slot, and the slot (no division per group)
-  for (int it = 0; it < ng * parts; ++it) {
-    const int gi = single ? 0 : it;
-    const uint32_t e = single ? (uint32_t)it : (uint32_t)js & 1u;
-    const uint32_t chunk = single ? 0u : (uint32_t)(js >> 1) * (uint32_t)gps + (uint32_t)gq;
-    if (!single && ++gq == gps) {
-      gq = 0;
-      ++js;
-    }
-    const uint32_t ab = 2u * e + (chunk & 1u);
-    const float sw = sw_next;
-    if (!single && gi + 1 < ng && n < a.N) sw_next = __ldg(a.s_w + (int64_t)(g0 + gi + 1) * a.N + n);
-    const uint32_t so = (uint32_t)gi % kSaRing;
-    bool ok = true;
-    if (!single) ok = mbar_wait(&b.sa_full[so], ring_parity(gi, kSaRing), abort_flag, a.status);
-    ok = ok && mbar_wait(&b.acc_full[ab], (chunk >> 1) & 1u, abort_flag, a.status);
-    // warp-collective tcgen05.ld follows: the whole warp proceeds or none of it
-    if (!__all_sync(0xffffffffu, ok)) break;
-    tc_fence_after();
-    const uint32_t taddr = tmem_base + ((quarter * 32u) << 16) + ab * kMp + hf * kH;
-    const float* scs = sc_ring + 2 * (so * kMp + hf * kH);  // (s_a', c) of the group's tokens
-    // the overflow-safe form is needed only if some s_a * 2^18 of the group overflows (the scale
-    // warp's flag; the same for every lane, so no lane skips the warp-collective loads below)
-    const bool finite = single || __all_sync(0xffffffffu, flags[so] != 0);
+  if (single) {
+    for (int it = 0; ng > 0 && it < parts; ++it) {
+      const uint32_t ab = 2u * (uint32_t)it;  // issuer it's first accumulator
+      const bool ok = mbar_wait(&b.acc_full[ab], 0, abort_flag, a.status);
+      // warp-collective tcgen05.ld follows: the whole warp proceeds or none of it
+      if (!__all_sync(0xffffffffu, ok)) break;
+      tc_fence_after();
+      const uint32_t taddr = tmem_base + ((quarter * 32u) << 16) + ab * kMp + hf * kH;
 #pragma unroll
-    for (int c = 0; c < kH / 8; ++c) {
-      uint32_t r[8];
-      tmem_ld8(taddr + c * 8, r);
-      tmem_ld_wait();
-      if (c == kH / 8 - 1) {  // the accumulator is in registers: hand it back
-        tc_fence_before();
-        __syncwarp();
-        if (lane == 0) mbar_arrive(&b.acc_empty[ab]);
-      }
-      if (single) {
+      for (int c = 0; c < kH / 8; ++c) {
+        uint32_t r[8];
+        tmem_ld8(taddr + c * 8, r);
+        tmem_ld_wait();
+        if (c == kH / 8 - 1) {  // the accumulator is in registers: hand it back
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(&b.acc_empty[ab]);
+        }
 #pragma unroll
         for (int i = 0; i < 8; ++i) y[c * 8 + i] += __uint_as_float(r[i]);  // exact integer partials
-      } else if (finite) {
-#pragma unroll
-        for (int i = 0; i < 8; i += 2) {
-          const float4 sc = *reinterpret_cast<const float4*>(scs + 2 * (c * 8 + i));  // s_a'0, c0, s_a'1, c1
-          // exact: both are integers below 2^24 (in units of 2^-18)
-          const float2 d = make_float2(__uint_as_float(r[i]) - sc.y, __uint_as_float(r[i + 1]) - sc.w);
-          const float2 t = __fmul2_rn(d, make_float2(sw, sw));
-          const float2 v = __ffma2_rn(t, make_float2(sc.x, sc.z), make_float2(y[c * 8 + i], y[c * 8 + i + 1]));
-          y[c * 8 + i] = v.x;
-          y[c * 8 + i + 1] = v.y;
-        }
-      } else {  // |s_a| > 2^110 somewhere: apply 2^18 to the exact partials first
-#pragma unroll
-        for (int i = 0; i < 8; ++i) {
-          const float2 sc = *reinterpret_cast<const float2*>(scs + 2 * (c * 8 + i));  // s_a (unscaled), c
-          y[c * 8 + i] = fmaf(((__uint_as_float(r[i]) - sc.y) * kOperandUnitInv) * sc.x, sw, y[c * 8 + i]);
-        }
       }
     }
-    if (!single) {
+  } else {
+    // Two groups per round (one for Mp = 64, for registers): one round of waits and one TMEM
+    // round trip for both.  Group gi was
+    // accumulated by the issuer of its slot js (e = js % 2) as that issuer's chunk
+    // (js / 2) * gps + gi % gps (gps = groups per slot); the position is stepped, not divided.
+    int gq = 0, js = 0;
+    auto next_acc = [&](uint32_t& ab, uint32_t& parity) {
+      const uint32_t chunk = (uint32_t)(js >> 1) * (uint32_t)gps + (uint32_t)gq;
+      ab = 2u * ((uint32_t)js & 1u) + (chunk & 1u);
+      parity = (chunk >> 1) & 1u;
+      if (++gq == gps) {
+        gq = 0;
+        ++js;
+      }
+    };
+    float swa = (ng > 0 && n < a.N) ? __ldg(a.s_w + (int64_t)g0 * a.N + n) : 0.0f;
+    constexpr int kPer = kMp <= 32 ? 2 : 1;  // groups per round
+    float swb = (kPer == 2 && ng > 1 && n < a.N) ? __ldg(a.s_w + (int64_t)(g0 + 1) * a.N + n) : 0.0f;
+    for (int gi = 0; gi < ng; gi += kPer) {
+      const bool two = kPer == 2 && gi + 1 < ng;  // the same for every lane
+      uint32_t ab0, p0, ab1 = 0, p1 = 0;
+      next_acc(ab0, p0);
+      if (two) next_acc(ab1, p1);
+      const float sw0 = swa, sw1 = swb;  // and the next round's weight scales, a round early
+      if (gi + kPer < ng && n < a.N) swa = __ldg(a.s_w + (int64_t)(g0 + gi + kPer) * a.N + n);
+      if (kPer == 2 && gi + 3 < ng && n < a.N) swb = __ldg(a.s_w + (int64_t)(g0 + gi + 3) * a.N + n);
+      const uint32_t so0 = (uint32_t)gi % kSaRing, so1 = (uint32_t)(gi + 1) % kSaRing;
+      bool ok = mbar_wait(&b.sa_full[so0], ring_parity(gi, kSaRing), abort_flag, a.status);
+      if (two) ok = ok && mbar_wait(&b.sa_full[so1], ring_parity(gi + 1, kSaRing), abort_flag, a.status);
+      ok = ok && mbar_wait(&b.acc_full[ab0], p0, abort_flag, a.status);
+      if (two) ok = ok && mbar_wait(&b.acc_full[ab1], p1, abort_flag, a.status);
+      // warp-collective tcgen05.ld follows: the whole warp proceeds or none of it
+      if (!__all_sync(0xffffffffu, ok)) break;
+      tc_fence_after();
+      const uint32_t lanes = tmem_base + ((quarter * 32u) << 16) + hf * kH;
+      const float* sc0 = sc_ring + 2 * (so0 * kMp + hf * kH);  // (s_a', c) of the groups' tokens
+      const float* sc1 = sc_ring + 2 * (so1 * kMp + hf * kH);
+      // the overflow-safe form is needed only if some s_a * 2^18 of a group overflows (the scale
+      // warp's flags; the same for every lane, so no lane skips the warp-collective loads below)
+      const bool finite = __all_sync(0xffffffffu, flags[so0] != 0 && (!two || flags[so1] != 0));
+      auto accumulate = [&](const uint32_t (&r)[8], const float* scs, float sw, int c) {
+        if (finite) {
+#pragma unroll
+          for (int i = 0; i < 8; i += 2) {
+            const float4 sc = *reinterpret_cast<const float4*>(scs + 2 * (c * 8 + i));  // s_a'0, c0, s_a'1, c1
+            // exact: both are integers below 2^24 (in units of 2^-18)
+            const float2 d = make_float2(__uint_as_float(r[i]) - sc.y, __uint_as_float(r[i + 1]) - sc.w);
+            const float2 t = __fmul2_rn(d, make_float2(sw, sw));
+            const float2 v = __ffma2_rn(t, make_float2(sc.x, sc.z), make_float2(y[c * 8 + i], y[c * 8 + i + 1]));
+            y[c * 8 + i] = v.x;
+            y[c * 8 + i + 1] = v.y;
+          }
+        } else {  // |s_a| > 2^110 somewhere: apply 2^18 to the exact partials first
+#pragma unroll
+          for (int i = 0; i < 8; ++i) {
+            const float2 sc = *reinterpret_cast<const float2*>(scs + 2 * (c * 8 + i));  // s_a (unscaled), c
+            y[c * 8 + i] = fmaf(((__uint_as_float(r[i]) - sc.y) * kOperandUnitInv) * sc.x, sw, y[c * 8 + i]);
+          }
+        }
+      };
+#pragma unroll
+      for (int c = 0; c < kH / 8; ++c) {
+        uint32_t r0[8], r1[8];
+        tmem_ld8(lanes + ab0 * kMp + c * 8, r0);
+        if (two) tmem_ld8(lanes + ab1 * kMp + c * 8, r1);
+        tmem_ld_wait();
+        if (c == kH / 8 - 1) {  // both accumulators are in registers: hand them back
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) {
+            mbar_arrive(&b.acc_empty[ab0]);
+            if (two) mbar_arrive(&b.acc_empty[ab1]);
+          }
+        }
+        accumulate(r0, sc0, sw0, c);
+        if (two) accumulate(r1, sc1, sw1, c);
+      }
       __syncwarp();
-      if (lane == 0) mbar_arrive(&b.sa_empty[so]);
+      if (lane == 0) {
+        mbar_arrive(&b.sa_empty[so0]);
+        if (two) mbar_arrive(&b.sa_empty[so1]);
+      }
     }
   }
   if (single && ng > 0) {  // the exact partial: the offset-code sum less 8 * the range's code sums
@@ -627,7 +677,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   const bool drain = warp >= kDrainWarp0;
   static_assert(kDrainWarp0 == 12 && kUnpackWarp0 == 4, "the register split is per warpgroup");
   if (drain) {
-    asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;\n" ::"n"(kRegsDrain) : "memory");
+    asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;\n" ::"n"(kRegsDrain<kMp>) : "memory");
     if (single) unpack_role<kMp>(a, rg, smem, tmem_base, b, ngroups, abort_flag);  // group 2 (warps 12-15)
     drain_role<kMp>(a, rg, n0, tmem_base, smem, b, abort_flag);
     __syncwarp();
@@ -635,7 +685,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   } else if (warp >= kUnpackWarp0) {
     unpack_role<kMp>(a, rg, smem, tmem_base, b, ngroups, abort_flag);
   } else {
-    asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;\n" ::"n"(kRegsCtl) : "memory");
+    asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;\n" ::"n"(kRegsCtl<kMp>) : "memory");
     if (warp == kWarpScale) {
       scale_role<kMp>(a, rg, smem, b, abort_flag);
     } else if (warp == kWarpTma) {
