@@ -60,7 +60,7 @@ FP8_PER_BF16 = 2.0  # nominal dense FP8 / BF16 tensor-core ratio on GB300 (4.5 /
 # bench reports null.
 KERNEL_TRAFFIC = {
     ("dllm", "cc6574cef178495b"): 31.244e6 + 0.123e6,  # profiles/w4a4_gemm_dllm_full.md
-    ("sweep_m1", "b8c4d652385e2708"): 25.288e6,  # profiles/w4a4_skinny_sweep_m1_full.md
+    ("sweep_m1", "dffa0fec8c708589"): 25.294e6,  # profiles/w4a4_skinny_sweep_m1_full.md
 }
 
 
