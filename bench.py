@@ -41,6 +41,8 @@ WORKLOADS = {
                  "flux_qkv"),
     "flux_out": ("FLUX 12B DiT output projection: M=4608 x K=15360 -> N=3072, group64", 4608, 15360, 3072, 64,
                  "flux_out"),
+    "dllm_gk": ("dLLM 8B gate/up projection, per-token/per-channel scales: M=1024 x K=4096 -> N=12288, group = K",
+                1024, 4096, 12288, 4096, "dllm"),
     # M-sweep points below the memory-to-compute crossover (per-token / per-channel: group = K);
     # these run the few-token kernel and are bound by streaming the packed weights from HBM
     "sweep_m1": ("M sweep: M=1 token x K=4096 -> N=12288, per-token/per-channel (group = K)", 1, 4096, 12288,

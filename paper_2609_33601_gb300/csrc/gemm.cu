@@ -390,14 +390,60 @@ __device__ __forceinline__ bool mma_open_acc(const Args& args, const Bars& b, ui
   return true;
 }
 
+static_assert(kSlotABytes == kSlotBBytes && kOpABytes == kOpBBytes, "A and B slots share descriptor offsets");
+
+// One K stage (4 MMAs of K = 32) at descriptor offset `off` (shared-memory bytes >> 4 from the
+// rings' bases, the same for A and B).  kHalf: group64, two groups per stage, each in a fresh
+// accumulator; otherwise a group spans stages_per_group whole stages.  With `wait_next`, the wait
+// for the next ring slot's operands sits between the second and third MMA, while the tensor
+// core still has queued work.
+template <bool kHalf>
+__device__ __forceinline__ bool mma_stage(const Args& args, const Bars& b, uint32_t tmem_base, MmaState& st,
+                                          uint32_t& d_tmem, int& kg, int stages_per_group, uint64_t adesc0,
+                                          uint64_t bdesc0, uint32_t off, uint32_t idesc, bool wait_next,
+                                          uint32_t nslot, uint32_t nphase, volatile int* abort_flag) {
+  constexpr uint16_t kBoth = 0x3;
+  const uint64_t ad = adesc0 + off, bd = bdesc0 + off;
+  if (kHalf) {
+    if (!mma_open_acc(args, b, tmem_base, st, d_tmem, abort_flag)) return false;
+    umma_f8f6f4_pair(d_tmem, ad, bd, idesc, 0u);
+    umma_f8f6f4_pair(d_tmem, ad + 2u, bd + 2u, idesc, 1u);
+    umma_commit_pair(&b.acc_full[st.chunk_it & 1u], kBoth);
+    ++st.chunk_it;
+    if (!mma_open_acc(args, b, tmem_base, st, d_tmem, abort_flag)) return false;
+    umma_f8f6f4_pair(d_tmem, ad + 4u, bd + 4u, idesc, 0u);
+    if (wait_next && !mbar_wait_cluster(&b.full[nslot], nphase, abort_flag, args.status)) return false;
+    umma_f8f6f4_pair(d_tmem, ad + 6u, bd + 6u, idesc, 1u);
+    umma_commit_pair(&b.acc_full[st.chunk_it & 1u], kBoth);
+    ++st.chunk_it;
+  } else {
+    if (kg == 0 && !mma_open_acc(args, b, tmem_base, st, d_tmem, abort_flag)) return false;
+    umma_f8f6f4_pair(d_tmem, ad, bd, idesc, kg == 0 ? 0u : 1u);
+    umma_f8f6f4_pair(d_tmem, ad + 2u, bd + 2u, idesc, 1u);
+    if (wait_next && !mbar_wait_cluster(&b.full[nslot], nphase, abort_flag, args.status)) return false;
+    umma_f8f6f4_pair(d_tmem, ad + 4u, bd + 4u, idesc, 1u);
+    umma_f8f6f4_pair(d_tmem, ad + 6u, bd + 6u, idesc, 1u);
+    if (++kg == stages_per_group) {
+      umma_commit_pair(&b.acc_full[st.chunk_it & 1u], kBoth);
+      ++st.chunk_it;
+      kg = 0;
+    }
+  }
+  return true;
+}
+
+// The issue loop runs straight through each ring slot: the MMAs of its two stages, the wait for
+// the next slot in the middle of the second stage, one commit that frees the slot.  The only
+// data-dependent branch per slot is the odd K-stage tail (a slot with one stage).
+template <bool kHalf>
 __device__ __forceinline__ void mma_role(const Args& args, const Pair& pr, uint32_t tmem_base, uint8_t* sA,
                                          uint8_t* sB, const Bars& b, volatile int* abort_flag) {
   const uint32_t idesc = idesc_e4m3_f32(kPairM, kBN);
   constexpr uint16_t kBoth = 0x3;
   const uint64_t adesc0 = sdesc_kmajor_sw128(smem_u32(sA));
   const uint64_t bdesc0 = sdesc_kmajor_sw128(smem_u32(sB));
-  const int stages_per_group = args.G >= kBK ? args.G / kBK : 1;  // G = 64: two groups per stage
-  const bool half_groups = args.G < kBK;
+  const int stages_per_group = kHalf ? 1 : args.G / kBK;
+  const int odd_slot = (args.k_stages & 1) != 0 ? args.slots_per_tile - 1 : -1;  // the one-stage slot, if any
   const int my_tiles =
       pr.cluster < args.num_tiles ? (args.num_tiles - 1 - pr.cluster) / pr.num_clusters + 1 : 0;
   const uint32_t total = static_cast<uint32_t>(my_tiles) * static_cast<uint32_t>(args.slots_per_tile);
@@ -409,44 +455,16 @@ __device__ __forceinline__ void mma_role(const Args& args, const Pair& pr, uint3
   for (uint32_t q = 0; ok && q < total; ++q) {
     const uint32_t nslot = slot + 1 == kSlots ? 0 : slot + 1;
     const uint32_t nphase = slot + 1 == kSlots ? phase ^ 1u : phase;
-    const int n_st = min(kStagesPerSlot, args.k_stages - j * kStagesPerSlot);
-    bool waited_next = q + 1 >= total;  // the next slot's operands, waited for while MMAs are queued
-    for (int sub = 0; sub < n_st; ++sub) {
-      const uint64_t adesc = adesc0 + ((slot * kSlotABytes + sub * kOpABytes) >> 4);
-      const uint64_t bdesc = bdesc0 + ((slot * kSlotBBytes + sub * kOpBBytes) >> 4);
-      const bool wait_here = sub == n_st - 1 && !waited_next;
-      if (half_groups) {
-        if (!(ok = mma_open_acc(args, b, tmem_base, st, d_tmem, abort_flag))) break;
-        umma_f8f6f4_pair(d_tmem, adesc, bdesc, idesc, 0u);
-        umma_f8f6f4_pair(d_tmem, adesc + 2u, bdesc + 2u, idesc, 1u);
-        umma_commit_pair(&b.acc_full[st.chunk_it & 1u], kBoth);
-        ++st.chunk_it;
-        if (!(ok = mma_open_acc(args, b, tmem_base, st, d_tmem, abort_flag))) break;
-        umma_f8f6f4_pair(d_tmem, adesc + 4u, bdesc + 4u, idesc, 0u);
-        if (wait_here) {
-          if (!(ok = mbar_wait_cluster(&b.full[nslot], nphase, abort_flag, args.status))) break;
-          waited_next = true;
-        }
-        umma_f8f6f4_pair(d_tmem, adesc + 6u, bdesc + 6u, idesc, 1u);
-        umma_commit_pair(&b.acc_full[st.chunk_it & 1u], kBoth);
-        ++st.chunk_it;
-      } else {
-        const bool first = kg == 0;
-        if (first && !(ok = mma_open_acc(args, b, tmem_base, st, d_tmem, abort_flag))) break;
-        umma_f8f6f4_pair(d_tmem, adesc, bdesc, idesc, first ? 0u : 1u);
-        umma_f8f6f4_pair(d_tmem, adesc + 2u, bdesc + 2u, idesc, 1u);
-        if (wait_here) {
-          if (!(ok = mbar_wait_cluster(&b.full[nslot], nphase, abort_flag, args.status))) break;
-          waited_next = true;
-        }
-        umma_f8f6f4_pair(d_tmem, adesc + 4u, bdesc + 4u, idesc, 1u);
-        umma_f8f6f4_pair(d_tmem, adesc + 6u, bdesc + 6u, idesc, 1u);
-        if (++kg == stages_per_group) {
-          umma_commit_pair(&b.acc_full[st.chunk_it & 1u], kBoth);
-          ++st.chunk_it;
-          kg = 0;
-        }
-      }
+    const uint32_t off = (slot * kSlotABytes) >> 4;
+    const bool wait_next = q + 1 < total;
+    if (j != odd_slot) {
+      ok = mma_stage<kHalf>(args, b, tmem_base, st, d_tmem, kg, stages_per_group, adesc0, bdesc0, off, idesc, false,
+                            0u, 0u, abort_flag) &&
+           mma_stage<kHalf>(args, b, tmem_base, st, d_tmem, kg, stages_per_group, adesc0, bdesc0,
+                            off + (kOpABytes >> 4), idesc, wait_next, nslot, nphase, abort_flag);
+    } else {
+      ok = mma_stage<kHalf>(args, b, tmem_base, st, d_tmem, kg, stages_per_group, adesc0, bdesc0, off, idesc,
+                            wait_next, nslot, nphase, abort_flag);
     }
     if (!ok) break;
     umma_commit_pair(&b.empty[slot], kBoth);
@@ -629,6 +647,13 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
 
+  // The next kernel in the stream may launch now; it waits for this one before it touches our
+  // inputs or outputs.  Every role except the weight unpack reads data the previous kernel may
+  // write (the A operand, scales, corrections) or writes the output, so it waits for that kernel
+  // first; the unpack reads only the packed weights and starts at once.
+  pdl_launch_dependents();
+  if (warp < kUnpackWarp0 || warp >= kDrainWarp0) pdl_wait();
+
   // Register split per warpgroup (totals the 512 x 128 registers of the launch): producer and
   // MMA (warps 0-3) 32, unpack (warps 4-7) 96, drain (warps 8-15, 128 running sums) 192.
   if (warp >= kDrainWarp0) {
@@ -647,8 +672,12 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     } else if (warp == kWarpScale) {
       if (!kExport && lane == 0) scale_producer(args, pr, &tmSW, &tmSA, sSc, b, abort_flag);
     } else if (warp == kWarpMma && lane == 0) {
-      if (pr.rank == 0)
-        mma_role(args, pr, tmem_base, sA, sB, b, abort_flag);
+      if (pr.rank == 0) {
+        if (args.G < kBK)
+          mma_role<true>(args, pr, tmem_base, sA, sB, b, abort_flag);
+        else
+          mma_role<false>(args, pr, tmem_base, sA, sB, b, abort_flag);
+      }
       else  // the even CTA's MMAs read this CTA's shared memory and write its TMEM until here
         drain_wait(b.mma_done, 0, args.status);
     }
@@ -728,8 +757,8 @@ cudaError_t launch_impl(const GemmProblem& p, cudaStream_t stream, int sms) {
   a.partials = p.partials;
   a.status = p.status;
   const int pairs = a.num_tiles < max_pairs ? a.num_tiles : max_pairs;
-  w4a4_gemm_kernel<kExport, kOffset><<<2 * pairs, kThreads, kSmemBytes, stream>>>(tmA, tmSW, tmSA, a);
-  return cudaGetLastError();
+  return launch_pdl(w4a4_gemm_kernel<kExport, kOffset>, dim3(2 * pairs), dim3(kThreads), kSmemBytes, stream, tmA,
+                    tmSW, tmSA, a);
 }
 
 }  // namespace

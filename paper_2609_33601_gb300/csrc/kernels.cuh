@@ -6,6 +6,26 @@
 
 namespace jq {
 
+// Launches `kernel` with programmatic stream serialisation: it may begin while the previous
+// kernel of the stream is still running, as soon as that kernel allows it (ptx.cuh,
+// pdl_launch_dependents); the kernel itself waits (pdl_wait) before it touches anything the
+// previous kernel may write or read.
+template <typename... KArgs, typename... Args>
+cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t stream,
+                       Args... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kernel, static_cast<KArgs>(args)...);
+}
+
 // bf16 activations [M, ldx] -> packed codes [M, K/2] + scales [M, K/G].
 cudaError_t launch_quantize_act(const void* x, int64_t M, int64_t K, int64_t ldx, int G, uint8_t* q, float* s_a,
                                 cudaStream_t stream, int sms);

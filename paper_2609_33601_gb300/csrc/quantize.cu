@@ -19,6 +19,7 @@
 
 #include "kernels.cuh"
 #include "operand.cuh"
+#include "ptx.cuh"
 
 namespace jq {
 
@@ -115,6 +116,10 @@ template <typename In, int L, bool kOperand, bool kScaleT>
 __global__ void __launch_bounds__(256) quantize_groups_kernel(const In* __restrict__ x, int64_t M, int64_t K,
                                                               int64_t ldx, uint8_t* __restrict__ out,
                                                               float* __restrict__ scales, float* __restrict__ corr) {
+  // The activation quantiser lets the next kernel (the linear layer, which starts by streaming
+  // its weights) launch at once; the weight packer does not, so nothing reads weights early.
+  if (!kScaleT) pdl_launch_dependents();
+  pdl_wait();
   const int64_t chunks_per_row = K / 32;
   const int64_t total = M * chunks_per_row;
   const int64_t ng = K / (32 * L);
@@ -162,6 +167,8 @@ __global__ void __launch_bounds__(128) quantize_rows_kernel(const In* __restrict
                                                             float* __restrict__ scales, float* __restrict__ corr) {
   __shared__ float red[4];
   __shared__ int red_cs[4];
+  if (!kScaleT) pdl_launch_dependents();  // as in quantize_groups_kernel
+  pdl_wait();
   for (int64_t row = blockIdx.x; row < M; row += gridDim.x) {
     const In* xr = x + row * ldx;
     float a = 0.0f;
@@ -209,6 +216,8 @@ template <int L>
 __global__ void __launch_bounds__(256) expand_operand_kernel(const uint8_t* __restrict__ packed, int64_t rows,
                                                              int64_t K, uint8_t* __restrict__ image,
                                                              float* __restrict__ corr) {
+  pdl_launch_dependents();
+  pdl_wait();
   const int64_t per_row = K / 32;
   const int64_t chunks = rows * per_row;
   const uint32_t k_stages = static_cast<uint32_t>(K / kImageStageK);
@@ -239,6 +248,8 @@ __global__ void __launch_bounds__(128) expand_operand_rows_kernel(const uint8_t*
                                                                   int64_t K, uint8_t* __restrict__ image,
                                                                   float* __restrict__ corr) {
   __shared__ int red_cs[4];
+  pdl_launch_dependents();
+  pdl_wait();
   const int64_t per_row = K / 32;
   const uint32_t k_stages = static_cast<uint32_t>(K / kImageStageK);
   for (int64_t row = blockIdx.x; row < rows; row += gridDim.x) {
@@ -277,15 +288,15 @@ cudaError_t launch_quantize(const In* x, int64_t M, int64_t K, int64_t ldx, int 
   if (M == 0) return cudaSuccess;
   if (G == K) {
     int blocks = static_cast<int>(M < static_cast<int64_t>(sms) * 16 ? M : static_cast<int64_t>(sms) * 16);
-    quantize_rows_kernel<In, kOperand, kScaleT><<<blocks, 128, 0, stream>>>(x, M, K, ldx, out, scales, corr);
-  } else if (G == 64) {
-    quantize_groups_kernel<In, 2, kOperand, kScaleT>
-        <<<grid_for(M * (K / 32), 256, sms), 256, 0, stream>>>(x, M, K, ldx, out, scales, corr);
-  } else {
-    quantize_groups_kernel<In, 4, kOperand, kScaleT>
-        <<<grid_for(M * (K / 32), 256, sms), 256, 0, stream>>>(x, M, K, ldx, out, scales, corr);
+    return launch_pdl(quantize_rows_kernel<In, kOperand, kScaleT>, dim3(blocks), dim3(128), 0, stream, x, M, K, ldx,
+                      out, scales, corr);
   }
-  return cudaGetLastError();
+  const int grid = grid_for(M * (K / 32), 256, sms);
+  if (G == 64)
+    return launch_pdl(quantize_groups_kernel<In, 2, kOperand, kScaleT>, dim3(grid), dim3(256), 0, stream, x, M, K,
+                      ldx, out, scales, corr);
+  return launch_pdl(quantize_groups_kernel<In, 4, kOperand, kScaleT>, dim3(grid), dim3(256), 0, stream, x, M, K, ldx,
+                    out, scales, corr);
 }
 
 }  // namespace
@@ -313,13 +324,11 @@ cudaError_t launch_expand_operand(const uint8_t* packed, int64_t rows, int64_t K
   if (chunks == 0) return cudaSuccess;
   if (G == K) {
     const int blocks = static_cast<int>(rows < static_cast<int64_t>(sms) * 16 ? rows : static_cast<int64_t>(sms) * 16);
-    expand_operand_rows_kernel<<<blocks, 128, 0, stream>>>(packed, rows, K, op, corr);
-  } else if (G == 64) {
-    expand_operand_kernel<2><<<grid_for(chunks, 256, sms), 256, 0, stream>>>(packed, rows, K, op, corr);
-  } else {
-    expand_operand_kernel<4><<<grid_for(chunks, 256, sms), 256, 0, stream>>>(packed, rows, K, op, corr);
+    return launch_pdl(expand_operand_rows_kernel, dim3(blocks), dim3(128), 0, stream, packed, rows, K, op, corr);
   }
-  return cudaGetLastError();
+  const int grid = grid_for(chunks, 256, sms);
+  if (G == 64) return launch_pdl(expand_operand_kernel<2>, dim3(grid), dim3(256), 0, stream, packed, rows, K, op, corr);
+  return launch_pdl(expand_operand_kernel<4>, dim3(grid), dim3(256), 0, stream, packed, rows, K, op, corr);
 }
 
 }  // namespace jq

@@ -161,7 +161,19 @@ __device__ __forceinline__ void tma_role(const SkArgs& a, const Range& rg, int n
   using L = Layout<kMp>;
   constexpr int kPkSlots = L::kPkSlots;
   const int nslots = (rg.nst + kStPerSlot - 1) / kStPerSlot;
-  for (int j = 0; j < nslots; ++j) {
+  // The weight boxes of the ring's first pass do not depend on the previous kernel in the stream:
+  // they go out before waiting for it (programmatic launch, ptx.cuh), the token boxes after.
+  const int pre = nslots < kPkSlots ? nslots : kPkSlots;
+  for (int j = 0; j < pre; ++j) {  // a fresh ring: every slot is free
+    uint8_t* slot = smem + L::kOffPk + (uint32_t)j * L::kPkSlot;
+    mbar_arrive_expect_tx(&b.pk_full[j], L::kPkSlot);
+    tma_load_2d(slot, tmW, &b.pk_full[j], (rg.st0 + j * kStPerSlot) * (kBK / 2), n0);
+  }
+  pdl_wait();
+  for (int j = 0; j < pre; ++j)
+    tma_load_2d(smem + L::kOffPk + (uint32_t)j * L::kPkSlot + L::kPkW, tmX, &b.pk_full[j],
+                (rg.st0 + j * kStPerSlot) * (kBK / 2), 0);
+  for (int j = pre; j < nslots; ++j) {
     const uint32_t s = (uint32_t)j % kPkSlots;
     if (!mbar_wait(&b.pk_empty[s], ring_parity(j, kPkSlots) ^ 1u, abort_flag, a.status)) break;
     uint8_t* slot = smem + L::kOffPk + s * L::kPkSlot;
@@ -676,9 +688,15 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   const bool drain = warp >= kDrainWarp0;
   static_assert(kDrainWarp0 == 12 && kUnpackWarp0 == 4, "the register split is per warpgroup");
+  // The next kernel in the stream may launch now; it waits for this one before it touches our
+  // inputs or outputs.  Here the TMA producer waits for the previous kernel after its first
+  // weight boxes, the scale warp and the drain before their first access to activation data or
+  // the output; the unpack and MMA roles touch only shared and tensor memory.
+  pdl_launch_dependents();
   if (drain) {
     asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;\n" ::"n"(kRegsDrain<kMp>) : "memory");
     if (single) unpack_role<kMp>(a, rg, smem, tmem_base, b, ngroups, abort_flag);  // group 2 (warps 12-15)
+    pdl_wait();
     drain_role<kMp>(a, rg, n0, tmem_base, smem, b, abort_flag);
     __syncwarp();
     asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;\n" ::"n"(kRegsLaunch) : "memory");
@@ -687,6 +705,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   } else {
     asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;\n" ::"n"(kRegsCtl<kMp>) : "memory");
     if (warp == kWarpScale) {
+      pdl_wait();
       scale_role<kMp>(a, rg, smem, b, abort_flag);
     } else if (warp == kWarpTma) {
       if (lane == 0) tma_role<kMp>(a, rg, n0, &tmW, &tmX, smem, b, abort_flag);
@@ -758,8 +777,10 @@ cudaLaunchConfig_t make_config(int grid, int split, cudaStream_t stream, cudaLau
   attr[0].val.clusterDim.x = split;
   attr[0].val.clusterDim.y = 1;
   attr[0].val.clusterDim.z = 1;
+  attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;  // programmatic launch (ptx.cuh)
+  attr[1].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
-  cfg.numAttrs = 1;
+  cfg.numAttrs = 1;  // the cluster shape; launches add the programmatic attribute
   return cfg;
 }
 
@@ -773,7 +794,7 @@ int choose_split(int tiles, int k_stages, int sms) {
   if (!probed) {
     probed = true;
     for (int s = 1; s <= kMaxSplit; ++s) {
-      cudaLaunchAttribute attr[1];
+      cudaLaunchAttribute attr[2];
       cudaLaunchConfig_t cfg = make_config<kMp>(s * (sms / s), s, nullptr, attr);
       int n = 0;
       if (cudaOccupancyMaxActiveClusters(&n, w4a4_skinny_kernel<kMp>, &cfg) != cudaSuccess) {
@@ -808,8 +829,9 @@ cudaError_t launch_mp(SkArgs a, const SkinnyProblem& p, int tiles, int sms, cuda
       !encode_2d(&tmX, CU_TENSOR_MAP_DATA_TYPE_UINT8, p.q, p.K / 2, p.M, p.K / 2, kBK, kMp, CU_TENSOR_MAP_SWIZZLE_128B))
     return cudaErrorInvalidValue;
   a.split = choose_split<kMp>(tiles, a.k_stages, sms);
-  cudaLaunchAttribute attr[1];
+  cudaLaunchAttribute attr[2];
   cudaLaunchConfig_t cfg = make_config<kMp>(tiles * a.split, a.split, stream, attr);
+  cfg.numAttrs = 2;
   return cudaLaunchKernelEx(&cfg, w4a4_skinny_kernel<kMp>, tmW, tmX, a);
 }
 
