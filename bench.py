@@ -52,6 +52,14 @@ WORKLOADS = {
     "sweep_m64": ("M sweep: M=64 tokens x K=4096 -> N=12288, per-token/per-channel (group = K)", 64, 4096, 12288,
                   4096, "sweep_a"),
 }
+# The whole M sweep of the memory-to-compute crossover, at both shapes (per-token/per-channel
+# scales, group = K): M <= 64 runs the few-token kernel, larger M the GEMM.
+SWEEP_M = (1, 16, 64, 256, 1024, 4096, 16384)
+for _m in SWEEP_M:
+    WORKLOADS[f"sweep_a_m{_m}"] = (f"M sweep A: M={_m} x K=4096 -> N=12288, group = K", _m, 4096, 12288, 4096,
+                                   "sweep_a")
+    WORKLOADS[f"sweep_b_m{_m}"] = (f"M sweep B: M={_m} x K=3072 -> N=3072, group = K", _m, 3072, 3072, 3072,
+                                   "sweep_b")
 FEW_TOKENS = 64  # M at or below this takes the few-token (weight-streaming) kernel
 PEAKS_PATH = os.path.join(ROOT, "MEASURED_PEAKS.json")
 FP8_PER_BF16 = 2.0  # nominal dense FP8 / BF16 tensor-core ratio on GB300 (4.5 / 2.25 PFLOP/s)
@@ -61,7 +69,7 @@ FP8_PER_BF16 = 2.0  # nominal dense FP8 / BF16 tensor-core ratio on GB300 (4.5 /
 # source the capture was taken on; once the kernel changes the figure no longer applies and the
 # bench reports null.
 KERNEL_TRAFFIC = {
-    ("dllm", "cc6574cef178495b"): 31.244e6 + 0.123e6,  # profiles/w4a4_gemm_dllm_full.md
+    ("dllm", "3e8612447b6fd805"): 31.244e6 + 0.119e6,  # profiles/w4a4_gemm_dllm_full.md
     ("sweep_m1", "dffa0fec8c708589"): 25.294e6,  # profiles/w4a4_skinny_sweep_m1_full.md
 }
 
@@ -202,6 +210,45 @@ def run_reference(args):
     return 0
 
 
+# ----------------------------------------------------------------------------- context
+
+def cublas_context(torch, dev, sets, M, N, K, args, world):
+    """cuBLAS bf16 GEMM of the same shape (y = x W^T, bf16 weights), for context: rotating bf16
+    weight sets together larger than L2, K launches captured in a CUDA graph, timed with CUDA
+    events like the linear layer."""
+    wbytes = N * K * 2
+    n_w = max(2, -(-300_000_000 // wbytes))
+    if n_w * wbytes > 4_000_000_000:
+        return {"skipped": "bf16 weight sets would exceed 4 GB"}
+    gen = torch.Generator(device=dev)
+    gen.manual_seed(5)
+    ws = [(torch.randn((N, K), device=dev, generator=gen) * 0.02).to(torch.bfloat16) for _ in range(n_w)]
+    xs = [sets[i % len(sets)][0] for i in range(n_w)]
+    out = torch.empty((M, N), dtype=torch.bfloat16, device=dev)
+    cap = torch.cuda.Stream()
+    cap.wait_stream(torch.cuda.current_stream())
+    with torch.cuda.stream(cap):
+        for i in range(args.warmup):
+            torch.matmul(xs[i % n_w], ws[i % n_w].t(), out=out)
+    cap.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=cap):
+        for i in range(args.steps):
+            torch.matmul(xs[i % n_w], ws[i % n_w].t(), out=out)
+    g.replay()
+    torch.cuda.synchronize()
+    t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    t0.record()
+    g.replay()
+    t1.record()
+    torch.cuda.synchronize()
+    ms = t0.elapsed_time(t1) / args.steps
+    del ws, g
+    torch.cuda.empty_cache()
+    return {"value": world * 2.0 * M * N * K / (ms * 1e-3) / 1e12, "unit": "TFLOP/s", "ms_per_call": ms,
+            "what": "torch.matmul bf16 x[M,K] @ W[N,K]^T, same M, N, K"}
+
+
 # ----------------------------------------------------------------------------- our arm
 
 def run_ours(args):
@@ -234,18 +281,23 @@ def run_ours(args):
     q = torch.empty((M, K // 2), dtype=torch.uint8, device=dev)
     s_a = torch.empty((M, K // G), dtype=torch.float32, device=dev)
     y = torch.empty((M, N), dtype=torch.bfloat16, device=dev)
-    ws = torch.empty(jq.jq_workspace_size(M, N, K, G, False), dtype=torch.uint8, device=dev)
+    fused = args.fused
+    ws = torch.empty(max(jq.jq_workspace_size(M, N, K, G, fused), 16), dtype=torch.uint8, device=dev)
     stream = torch.cuda.current_stream()
 
     def quantize(i, st):
         jq.jq_quantize_act(sets[i % n_sets][0], G, q, s_a, stream=st)
 
     def linear(i, st):
-        _, qw, sw, b = sets[i % n_sets]
-        jq.jq_w4a4_linear(q, s_a, qw, sw, b, G, y=y, workspace=ws, stream=st)
+        x, qw, sw, b = sets[i % n_sets]
+        if fused:  # bf16 activations straight into the GEMM operand
+            jq.jq_fused_quant_linear(x, qw, sw, b, G, y=y, workspace=ws, stream=st)
+        else:
+            jq.jq_w4a4_linear(q, s_a, qw, sw, b, G, y=y, workspace=ws, stream=st)
 
     def step(i, st=None):
-        quantize(i, st or stream)
+        if not fused:
+            quantize(i, st or stream)
         linear(i, st or stream)
 
     def barrier():
@@ -309,8 +361,11 @@ def run_ours(args):
     def e2e_step(i):
         x_dev.copy_(x_host[i % len(x_host)], non_blocking=True)
         _, qw, sw, b = sets[i % n_sets]
-        jq.jq_quantize_act(x_dev, G, q, s_a, stream=stream)
-        jq.jq_w4a4_linear(q, s_a, qw, sw, b, G, y=y, workspace=ws, stream=stream)
+        if fused:
+            jq.jq_fused_quant_linear(x_dev, qw, sw, b, G, y=y, workspace=ws, stream=stream)
+        else:
+            jq.jq_quantize_act(x_dev, G, q, s_a, stream=stream)
+            jq.jq_w4a4_linear(q, s_a, qw, sw, b, G, y=y, workspace=ws, stream=stream)
         y_host.copy_(y, non_blocking=True)
 
     for i in range(args.warmup):
@@ -334,23 +389,32 @@ def run_ours(args):
     bf16_peak, hbm_peak, peak_src = measured_peaks()
     fp8_peak = bf16_peak * FP8_PER_BF16
     kernel_file = "skinny.cu" if few else "gemm.cu"
-    traffic = KERNEL_TRAFFIC.get((args.workload, kernel_hash(kernel_file)))
-    if few:
-        # algorithmic bytes of one jq_w4a4_linear: packed weights and their scales, packed
-        # activation codes and scales, bias, bf16 output
-        groups = K // G
-        alg_bytes = N * K // 2 + groups * N * 4 + M * K // 2 + M * groups * 4 + M * N * 2
+    traffic = None if fused else KERNEL_TRAFFIC.get((args.workload, kernel_hash(kernel_file)))
+    # algorithmic bytes of one linear call: packed weights and their scales, packed activation
+    # codes and scales (the fused call reads bf16 activations instead), bias, bf16 output
+    groups = K // G
+    act_bytes = M * K * 2 if fused else M * K // 2 + M * groups * 4
+    alg_bytes = N * K // 2 + groups * N * 4 + act_bytes + (0 if sets[0][3] is None else N * 4) + M * N * 2
+    # the bound is whichever of the tensor time and the HBM time is larger
+    t_tensor, t_hbm = ops_step / (fp8_peak * 1e12), alg_bytes / (hbm_peak * 1e9)
+    what = ("jq_fused_quant_linear (quantise-to-operand + tcgen05 GEMM)" if fused else
+            "jq_w4a4_linear (few-token weight-streaming kernel)" if few else
+            "jq_w4a4_linear (operand expansion + tcgen05 GEMM)")
+    if t_hbm > t_tensor:
         achieved = alg_bytes / (gemm_ms * 1e-3) / 1e9
         roofline = {"bound": "hbm", "achieved": achieved, "peak": hbm_peak, "unit": "GB/s", "frac": achieved / hbm_peak,
                     "traffic": traffic, "algorithmic_bytes": alg_bytes,
-                    "kernel": "jq_w4a4_linear (few-token weight-streaming kernel), CUDA events around a graph of K launches",
+                    "kernel": what + ", CUDA events around a graph of K launches",
                     "peak_source": f"{peak_src} HBM copy bandwidth {hbm_peak} GB/s"}
     else:
         achieved = ops_step / (gemm_ms * 1e-3) / 1e12
         roofline = {"bound": "tensor", "achieved": achieved, "peak": fp8_peak, "unit": "TFLOP/s",
-                    "frac": achieved / fp8_peak, "traffic": traffic,
-                    "kernel": "jq_w4a4_linear (operand expansion + tcgen05 GEMM), CUDA events around a graph of K launches",
+                    "frac": achieved / fp8_peak, "traffic": traffic, "algorithmic_bytes": alg_bytes,
+                    "kernel": what + ", CUDA events around a graph of K launches",
                     "peak_source": f"{peak_src} bf16 {bf16_peak} TFLOP/s x nominal FP8/BF16 ratio {FP8_PER_BF16}"}
+    context = None
+    if not args.no_context:
+        context = {"cublas_bf16": cublas_context(torch, dev, sets, M, N, K, args, world)}
 
     if rank != 0:
         if world > 1:
@@ -367,13 +431,15 @@ def run_ours(args):
         "warmup": args.warmup, "ms_per_step": total_ms / args.steps, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "int4", "data": "synthetic",
         "config": {"workload": desc, "M": M, "K": K, "N": N, "group": G,
-                   "step": "jq_quantize_act + jq_w4a4_linear", "launch": "CUDA graph of the K steps",
+                   "step": "jq_fused_quant_linear" if fused else "jq_quantize_act + jq_w4a4_linear",
+                   "launch": "CUDA graph of the K steps",
                    "parallelism": f"replicas x{world}",
                    "l2": f"{n_sets} rotating input/weight sets larger than L2"},
         "roofline": roofline,
+        "context": context,
         "cpu_baseline": cpu,
         "e2e": {"value": e2e_value, "unit": "TOPS", "h2d_bytes_per_step": M * K * 2, "d2h_bytes_per_step": M * N * 2},
-        "gpu_launches": (2 if few else 3) * args.steps,
+        "gpu_launches": (2 if (few or fused) else 3) * args.steps,
         "clocks": clocks.summary(),
     }
     print(json.dumps(line), flush=True)
@@ -393,6 +459,8 @@ def main():
     ap.add_argument("--sets", type=int, default=0, help="rotating input/weight sets (0: enough for > 3x L2)")
     ap.add_argument("--ref-seconds", type=float, default=10.0, help="CPU seconds per oracle sample")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--fused", action="store_true", help="time jq_fused_quant_linear (bf16 activations in)")
+    ap.add_argument("--no-context", action="store_true", help="skip the cuBLAS bf16 GEMM of the same shape")
     args = ap.parse_args()
     if args.warmup < 3:
         ap.error("--warmup must be at least 3")

@@ -745,18 +745,28 @@ __global__ void __launch_bounds__(kThreads, 1)
   cluster_sync_all();  // no CTA leaves while a peer may still read its buffer
   if (drain && rank == 0) {
     const int n = n0 + (int)ch;
+    // G = K: the tokens' scales, as independent loads issued together (one latency, not one
+    // per token)
+    float sa[kH];
+#pragma unroll
+    for (int i = 0; i < kH; ++i) {
+      const int m = (int)hf * kH + i;
+      sa[i] = (a.groups == 1 && m < a.M) ? __ldg(a.s_a + m) : 0.0f;
+    }
     if (n < a.N) {
       const float bn = a.bias != nullptr ? __ldg(a.bias + n) : 0.0f;
       const float swn = a.groups == 1 ? __ldg(a.s_w + n) : 0.0f;
+#pragma unroll
       for (int i = 0; i < kH; ++i) {
         const int m = (int)hf * kH + i;
-        if (m >= a.M) break;
-        float v = red[m * kRows + ch];
-        if (a.groups == 1) {  // exact integer partial: scale once
-          const float sa = __ldg(a.s_a + m), f = sa * kOperandUnitInv;
-          v = f <= FLT_MAX ? (v * swn) * f : ((v * kOperandUnitInv) * sa) * swn;
+        if (m < a.M) {
+          float v = red[m * kRows + ch];
+          if (a.groups == 1) {  // exact integer partial: scale once
+            const float f = sa[i] * kOperandUnitInv;
+            v = f <= FLT_MAX ? (v * swn) * f : ((v * kOperandUnitInv) * sa[i]) * swn;
+          }
+          a.y[(int64_t)m * a.N + n] = __float2bfloat16_rn(v + bn);
         }
-        a.y[(int64_t)m * a.N + n] = __float2bfloat16_rn(v + bn);
       }
     }
   }
