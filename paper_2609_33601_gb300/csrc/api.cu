@@ -136,13 +136,18 @@ jq_status jq_w4a4_linear(const uint8_t* q, const float* s_a, const uint8_t* qw, 
   const DeviceInfo* d = current_device();
   if (d == nullptr) return JQ_ERR_UNSUPPORTED;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
-  if (jq::skinny_supports(M, K, group)) {  // few tokens: the weight-streaming kernel, no workspace needed
-    jq::SkinnyProblem p{static_cast<int>(M), static_cast<int>(N), static_cast<int>(K), group, q, s_a, qw, s_w, bias,
-                        y_bf16, d->status};
-    return from_cuda(jq::launch_w4a4_skinny(p, s, d->sms));
-  }
   uint8_t* a_op = static_cast<uint8_t*>(workspace);
   float* corr = reinterpret_cast<float*>(a_op + jq::ws_image_bytes(M, K));
+  if (jq::skinny_supports(M, K, group)) {  // few tokens: the weight-streaming kernel
+    jq::SkinnyProblem p{static_cast<int>(M), static_cast<int>(N), static_cast<int>(K), group, q, s_a, qw, s_w, bias,
+                        y_bf16, d->status};
+    if (M > 16) {  // expand the tokens once here rather than in every CTA of the kernel
+      if (jq::launch_expand_operand(q, M, K, group, a_op, corr, s, d->sms) != cudaSuccess) return JQ_ERR_CUDA;
+      p.a_image = a_op;
+      p.corr = corr;
+    }
+    return from_cuda(jq::launch_w4a4_skinny(p, s, d->sms));
+  }
   cudaError_t e = jq::launch_expand_operand(q, M, K, group, a_op, corr, s, d->sms);
   if (e != cudaSuccess) return JQ_ERR_CUDA;
   jq::GemmProblem p{static_cast<int>(M), static_cast<int>(N), static_cast<int>(K), group, a_op, s_a, corr, qw, s_w, bias,
@@ -165,11 +170,17 @@ jq_status jq_fused_quant_linear(const void* x_bf16, int64_t ldx, const uint8_t* 
   uint8_t* a_op = static_cast<uint8_t*>(workspace);
   float* corr = reinterpret_cast<float*>(a_op + jq::ws_image_bytes(M, K));
   float* s_a = reinterpret_cast<float*>(a_op + jq::ws_image_bytes(M, K) + jq::ws_per_group_bytes(M, K, group));
-  if (jq::skinny_supports(M, K, group)) {  // few tokens: packed codes in the workspace, then the weight-streaming kernel
-    cudaError_t e = jq::launch_quantize_act(x_bf16, M, K, ldx, group, a_op, s_a, s, d->sms);
-    if (e != cudaSuccess) return JQ_ERR_CUDA;
+  if (jq::skinny_supports(M, K, group)) {  // few tokens: the weight-streaming kernel
     jq::SkinnyProblem p{static_cast<int>(M), static_cast<int>(N), static_cast<int>(K), group, a_op, s_a, qw, s_w,
                         bias, y_bf16, d->status};
+    // up to 16 tokens: packed codes in the workspace; more: the operand image and corrections
+    cudaError_t e = M > 16 ? jq::launch_quantize_act_operand(x_bf16, M, K, ldx, group, a_op, s_a, corr, s, d->sms)
+                           : jq::launch_quantize_act(x_bf16, M, K, ldx, group, a_op, s_a, s, d->sms);
+    if (e != cudaSuccess) return JQ_ERR_CUDA;
+    if (M > 16) {
+      p.a_image = a_op;
+      p.corr = corr;
+    }
     return from_cuda(jq::launch_w4a4_skinny(p, s, d->sms));
   }
   cudaError_t e = jq::launch_quantize_act_operand(x_bf16, M, K, ldx, group, a_op, s_a, corr, s, d->sms);

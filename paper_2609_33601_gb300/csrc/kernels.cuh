@@ -92,6 +92,10 @@ struct SkinnyProblem {
   const float* bias;   // [N] or nullptr
   void* y;             // bf16 [M, N]
   uint32_t* status;    // device status word
+  // Optional, for M > 16: the tokens as the A-operand image (operand.cuh) and their corrections
+  // [M, K/G] (8 * the group's code sum, 2^-18 units), as launch_expand_operand writes them.
+  const uint8_t* a_image = nullptr;
+  const float* corr = nullptr;
 };
 cudaError_t launch_w4a4_skinny(const SkinnyProblem& p, cudaStream_t stream, int sms);
 

@@ -94,7 +94,7 @@ struct Layout {
   static constexpr uint32_t kOffSaFlag = kOffSa + 2 * kSaRing * kMp * 4;
   static constexpr uint32_t kOffCorr = kOffSaFlag + kSaRing * 4;  // G = K: 8 sum qa per unpack group [3][kMp]
   static constexpr uint32_t kOffBar = kOffCorr + (kUnpackGroups + 1) * kMp * 4;
-  static constexpr uint32_t kNumBars = 2 * kPkSlots + 2 * kOpSlots + 8 + 2 + 2 * kSaRing + 1;
+  static constexpr uint32_t kNumBars = 2 * kPkSlots + 3 * kOpSlots + 8 + 2 + 2 * kSaRing + 1;
   static constexpr uint32_t kOffMisc = kOffBar + kNumBars * 8;
   static constexpr uint32_t kSmemBytes = kOffMisc + 16;
   static constexpr uint32_t kRedBytes = kMp * kRows * 4;  // fp32 partials [kMp][128], reuse the packed ring
@@ -121,6 +121,8 @@ struct SkArgs {
   const float* bias;  // [N] or nullptr
   __nv_bfloat16* y;   // [M, N]
   uint32_t* status;
+  int image;          // token operand from the pre-expanded A-operand image (see tma_role)
+  const float* corr;  // image mode: [M, K/G] 8 * the group's activation code sum, 2^-18 units
 };
 
 struct SkBars {
@@ -129,6 +131,7 @@ struct SkBars {
   uint64_t *acc_full, *acc_empty, *mma_done;  // [2 issuers x 2 buffers], [2 issuers]
   uint64_t *sa_full, *sa_empty;  // activation-scale ring
   uint64_t* corr_full;           // G = K: the range's code sums are in place
+  uint64_t* tk_full;             // image mode: the token operand of an operand-ring slot has landed
 };
 
 __device__ __forceinline__ uint32_t ring_parity(uint32_t it, uint32_t slots) { return (it / slots) & 1u; }
@@ -164,28 +167,80 @@ __device__ __forceinline__ void tma_role(const SkArgs& a, const Range& rg, int n
   // The weight boxes of the ring's first pass do not depend on the previous kernel in the stream:
   // they go out before waiting for it (programmatic launch, ptx.cuh), the token boxes after.
   const int pre = nslots < kPkSlots ? nslots : kPkSlots;
+  const uint32_t wbytes = a.image ? L::kPkW : L::kPkSlot;
   for (int j = 0; j < pre; ++j) {  // a fresh ring: every slot is free
     uint8_t* slot = smem + L::kOffPk + (uint32_t)j * L::kPkSlot;
-    mbar_arrive_expect_tx(&b.pk_full[j], L::kPkSlot);
+    mbar_arrive_expect_tx(&b.pk_full[j], wbytes);
     tma_load_2d(slot, tmW, &b.pk_full[j], (rg.st0 + j * kStPerSlot) * (kBK / 2), n0);
   }
   pdl_wait();
-  for (int j = 0; j < pre; ++j)
-    tma_load_2d(smem + L::kOffPk + (uint32_t)j * L::kPkSlot + L::kPkW, tmX, &b.pk_full[j],
-                (rg.st0 + j * kStPerSlot) * (kBK / 2), 0);
-  for (int j = pre; j < nslots; ++j) {
-    const uint32_t s = (uint32_t)j % kPkSlots;
-    if (!mbar_wait(&b.pk_empty[s], ring_parity(j, kPkSlots) ^ 1u, abort_flag, a.status)) break;
-    uint8_t* slot = smem + L::kOffPk + s * L::kPkSlot;
-    const int x = (rg.st0 + j * kStPerSlot) * (kBK / 2);  // packed byte offset along K
-    mbar_arrive_expect_tx(&b.pk_full[s], L::kPkSlot);
-    tma_load_2d(slot, tmW, &b.pk_full[s], x, n0);
-    tma_load_2d(slot + L::kPkW, tmX, &b.pk_full[s], x, 0);
+  int jt = 0, jw = pre;  // token slots issued (image mode), weight slots issued
+  if (!a.image) {
+    for (int j = 0; j < pre; ++j)
+      tma_load_2d(smem + L::kOffPk + (uint32_t)j * L::kPkSlot + L::kPkW, tmX, &b.pk_full[j],
+                  (rg.st0 + j * kStPerSlot) * (kBK / 2), 0);
+    for (; jw < nslots; ++jw) {
+      const uint32_t s = (uint32_t)jw % kPkSlots;
+      if (!mbar_wait(&b.pk_empty[s], ring_parity(jw, kPkSlots) ^ 1u, abort_flag, a.status)) break;
+      uint8_t* slot = smem + L::kOffPk + s * L::kPkSlot;
+      const int x = (rg.st0 + jw * kStPerSlot) * (kBK / 2);  // packed byte offset along K
+      mbar_arrive_expect_tx(&b.pk_full[s], L::kPkSlot);
+      tma_load_2d(slot, tmW, &b.pk_full[s], x, n0);
+      tma_load_2d(slot + L::kPkW, tmX, &b.pk_full[s], x, 0);
+    }
+  } else {
+    // Image mode: the tokens arrive as operand bytes (the A-operand image of the GEMM path: per
+    // K stage a 128-row block in the 128-byte swizzle, of which the first kMp rows are a stage of
+    // this kernel's token operand) and go straight into the operand ring, completing on tk_full;
+    // the weights keep streaming into the packed ring.  The two rings advance at different paces
+    // (the operand ring frees a slot only when its MMAs are done), so this thread polls both
+    // instead of blocking on either.
+    long long t0 = clock64();
+    while (jw < nslots || jt < nslots) {
+      bool moved = false;
+      if (jt < nslots) {
+        const uint32_t os = (uint32_t)jt % kOpSlots;
+        if (mbar_test_wait(&b.op_empty[os], ring_parity(jt, kOpSlots) ^ 1u)) {
+          const int nst_j = rg.nst - jt * kStPerSlot < kStPerSlot ? rg.nst - jt * kStPerSlot : kStPerSlot;
+          uint8_t* dst = smem + L::kOffOp + os * L::kOpSlot;
+          mbar_arrive_expect_tx(&b.tk_full[os], (uint32_t)nst_j * L::kOpB);
+          for (int h = 0; h < nst_j; ++h)
+            tma_load_2d(dst + (uint32_t)h * L::kOpB, tmX, &b.tk_full[os], 0, (rg.st0 + jt * kStPerSlot + h) * kBK);
+          ++jt;
+          moved = true;
+        }
+      }
+      if (jw < nslots) {
+        const uint32_t s = (uint32_t)jw % kPkSlots;
+        if (mbar_test_wait(&b.pk_empty[s], ring_parity(jw, kPkSlots) ^ 1u)) {
+          mbar_arrive_expect_tx(&b.pk_full[s], L::kPkW);
+          tma_load_2d(smem + L::kOffPk + s * L::kPkSlot, tmW, &b.pk_full[s], (rg.st0 + jw * kStPerSlot) * (kBK / 2),
+                      n0);
+          ++jw;
+          moved = true;
+        }
+      }
+      if (moved) {
+        t0 = clock64();
+        continue;
+      }
+      __nanosleep(32);  // leave the issue slots to the unpack warps of this SM sub-partition
+      if (*abort_flag) break;
+      if (clock64() - t0 > (1ll << 31)) {  // bounded, like every other wait here
+        *abort_flag = 1;
+        if (a.status) atomicExch(a.status, (uint32_t)kDevTimeout);
+        break;
+      }
+    }
   }
   // let the last copies land before the CTA can leave
-  for (int j = nslots > kPkSlots ? nslots - kPkSlots : 0; j < nslots; ++j) {
+  for (int j = jw > kPkSlots ? jw - kPkSlots : 0; j < jw; ++j) {
     int dummy = 0;
     mbar_wait(&b.pk_full[j % kPkSlots], ring_parity(j, kPkSlots), &dummy, a.status);
+  }
+  for (int j = jt > kOpSlots ? jt - kOpSlots : 0; j < jt; ++j) {  // image mode: the token copies
+    int dummy = 0;
+    mbar_wait(&b.tk_full[j % kOpSlots], ring_parity(j, kOpSlots), &dummy, a.status);
   }
 }
 
@@ -250,23 +305,25 @@ __device__ __forceinline__ void unpack_role(const SkArgs& a, const Range& rg, ui
       }
       tmem_st32(a_lane + os * L::kASlotCols + (uint32_t)h * L::kAStageCols, v);
     }
-    // token rows: only the M real ones (rows >= M stay zero in the operand ring)
+    // token rows: only the M real ones (rows >= M stay zero in the operand ring); in image mode
+    // the producer has copied them as operand bytes and the corrections come from global memory
+    const uint32_t mx = a.image ? 0u : (uint32_t)a.M;
 #pragma unroll
     for (int i = 0; i < kXChunks; ++i) {
       const uint32_t t = u + kUnpackGroupThreads * i, r = t >> 3;
-      px[i] = r < (uint32_t)a.M ? ld_shared_v4(sw128_row(src + L::kPkW, r) + (((t & 7u) ^ (r & 7u)) << 4))
-                                : make_uint4(0x88888888u, 0x88888888u, 0x88888888u, 0x88888888u);
+      px[i] = r < mx ? ld_shared_v4(sw128_row(src + L::kPkW, r) + (((t & 7u) ^ (r & 7u)) << 4))
+                     : make_uint4(0x88888888u, 0x88888888u, 0x88888888u, 0x88888888u);
     }
     int xs[kXChunks];  // code sums of the token chunks (chunks of a stage past the range count 0)
 #pragma unroll
     for (int i = 0; i < kXChunks; ++i) {
       const uint32_t r = (u + kUnpackGroupThreads * (uint32_t)i) >> 3;
-      xs[i] = (r < (uint32_t)a.M && c8 < 4u * (uint32_t)nst_j) ? nib32_sum(px[i]) : 0;
+      xs[i] = (r < mx && c8 < 4u * (uint32_t)nst_j) ? nib32_sum(px[i]) : 0;
     }
 #pragma unroll
     for (int i = 0; i < kXChunks; ++i) {
       const uint32_t t = u + kUnpackGroupThreads * i, r = t >> 3, h = (t >> 2) & 1u, jc = t & 3u;
-      if (r >= (uint32_t)a.M) continue;
+      if (r >= mx) continue;
       uint4 lo, hi;
       nib32_to_operand(px[i], lo, hi);
       const uint32_t row_base = sw128_row(dst + h * L::kOpB, r), rr = r & 7u;
@@ -289,6 +346,7 @@ __device__ __forceinline__ void unpack_role(const SkArgs& a, const Range& rg, ui
       mbar_arrive(&b.op_full[os]);
       mbar_arrive(&b.pk_empty[p]);
     }
+    if (a.image) continue;
     // group sums: lanes whose chunk opens a group hold that group's sum after the butterfly
 #pragma unroll
     for (int i = 0; i < kXChunks; ++i) {
@@ -315,7 +373,7 @@ __device__ __forceinline__ void unpack_role(const SkArgs& a, const Range& rg, ui
       if ((u & 31u) == 0) mbar_arrive(&b.sa_full[so]);
     }
   }
-  if (single) {  // this group's share of the range's code sums (zero if it had no slot)
+  if (single && !a.image) {  // this group's share of the range's code sums (zero if it had no slot)
     float* corr = reinterpret_cast<float*>(smem + L::kOffCorr) + ug * kMp;
 #pragma unroll
     for (int i = 0; i < kXChunks; ++i) {
@@ -347,13 +405,15 @@ __device__ __forceinline__ void scale_role(const SkArgs& a, const Range& rg, uin
   const int g0 = rg.st0 * groups_per_stage(a);
   for (int gb = 0; gb < ng; gb += kSaBatch) {
     const int nb = ng - gb < kSaBatch ? ng - gb : kSaBatch;
-    float v[kSaBatch][kPer];
+    float v[kSaBatch][kPer], cv[kSaBatch][kPer];
 #pragma unroll
     for (int j = 0; j < kSaBatch; ++j) {
 #pragma unroll
       for (int h = 0; h < kPer; ++h) {
         const int m = (int)lane + 32 * h;
-        v[j][h] = (j < nb && m < kMp && m < a.M) ? __ldg(a.s_a + (int64_t)m * a.groups + g0 + gb + j) : 0.0f;
+        const bool in = j < nb && m < kMp && m < a.M;
+        v[j][h] = in ? __ldg(a.s_a + (int64_t)m * a.groups + g0 + gb + j) : 0.0f;
+        cv[j][h] = (in && a.image) ? __ldg(a.corr + (int64_t)m * a.groups + g0 + gb + j) : 0.0f;
       }
     }
 #pragma unroll
@@ -370,6 +430,7 @@ __device__ __forceinline__ void scale_role(const SkArgs& a, const Range& rg, uin
       for (int h = 0; h < kPer; ++h) {
         const int m = (int)lane + 32 * h;
         if (m < kMp) sc_ring[2 * (o * kMp + m)] = finite ? v[j][h] * kOperandUnitInv : v[j][h];
+        if (m < kMp && a.image) sc_ring[2 * (o * kMp + m) + 1] = cv[j][h];  // 8 sum qa, 2^-18 units
       }
       if (lane == 0) flags[o] = finite ? 1 : 0;
       __syncwarp();
@@ -419,6 +480,7 @@ __device__ __forceinline__ void mma_role(const SkArgs& a, const Range& rg, uint3
     const uint64_t bd0 = bdesc0 + ((os * L::kOpSlot) >> 4), bd1 = bd0 + (L::kOpB >> 4);
     const bool both = j * kStPerSlot + 1 < rg.nst;  // false only for the last slot of an odd range
     if (!(ok = mbar_wait(&b.op_full[os], ring_parity(j, kOpSlots), abort_flag, a.status))) break;
+    if (a.image && !(ok = mbar_wait(&b.tk_full[os], ring_parity(j, kOpSlots), abort_flag, a.status))) break;
     tc_fence_after();  // the unpack's tcgen05.st of this A slot is complete
     if (kGroups == 0) {
       const uint32_t acc0 = j > (int)e ? 1u : 0u;
@@ -597,7 +659,7 @@ __device__ __forceinline__ void drain_role(const SkArgs& a, const Range& rg, int
       }
     }
   }
-  if (single && ng > 0) {  // the exact partial: the offset-code sum less 8 * the range's code sums
+  if (single && ng > 0 && !a.image) {  // the exact partial: the offset-code sum less 8 * the range's code sums
     const bool ok = mbar_wait(b.corr_full, 0, abort_flag, a.status);
     const float* corr = reinterpret_cast<const float*>(smem + L::kOffCorr);
 #pragma unroll
@@ -632,6 +694,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   b.sa_full = b.mma_done + 2;
   b.sa_empty = b.sa_full + kSaRing;
   b.corr_full = b.sa_empty + kSaRing;
+  b.tk_full = b.corr_full + 1;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + L::kOffMisc);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + L::kOffMisc + 4);
 
@@ -650,6 +713,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     for (int i = (int)lane; i < kOpSlots; i += 32) {
       mbar_init(&b.op_full[i], kUnpackGroupWarps);  // the slot's unpack group
       mbar_init(&b.op_empty[i], 1);
+      mbar_init(&b.tk_full[i], 1);  // image mode: the producer's expect_tx for the token operand
     }
     if (lane < 4) {
       mbar_init(&b.acc_full[lane], 1);
@@ -657,7 +721,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     if (lane < 2) mbar_init(&b.mma_done[lane], 1);
     for (int i = (int)lane; i < kSaRing; i += 32) {
-      mbar_init(&b.sa_full[i], 1 + kUnpackGroupWarps);  // the scale warp and one unpack group
+      // the scale warp and one unpack group (the code sums); image mode: the scale warp alone
+      mbar_init(&b.sa_full[i], a.image ? 1 : 1 + kUnpackGroupWarps);
       mbar_init(&b.sa_empty[i], kNumDrainWarps);
     }
     if (lane == 0) mbar_init(b.corr_full, ngroups * kUnpackGroupWarps);
@@ -673,7 +738,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
   // Token rows >= M of the operand ring are zero codes for good: store them once here, and the
   // unpack converts only the M real rows of every slot.
-  if (a.M < kMp) {
+  if (a.M < kMp && !a.image) {
     const uint32_t row_bytes = (uint32_t)(kMp - a.M) * kBK, tile0 = smem_u32(smem + L::kOffOp);
     for (uint32_t i = threadIdx.x; i < kOpSlots * kStPerSlot * (row_bytes / 16u); i += kThreads) {
       const uint32_t tile = i / (row_bytes / 16u), off = (uint32_t)a.M * kBK + (i % (row_bytes / 16u)) * 16u;
@@ -745,27 +810,33 @@ __global__ void __launch_bounds__(kThreads, 1)
   cluster_sync_all();  // no CTA leaves while a peer may still read its buffer
   if (drain && rank == 0) {
     const int n = n0 + (int)ch;
-    // G = K: the tokens' scales, as independent loads issued together (one latency, not one
-    // per token)
-    float sa[kH];
+    const float bn = (n < a.N && a.bias != nullptr) ? __ldg(a.bias + n) : 0.0f;
+    const float swn = (n < a.N && a.groups == 1) ? __ldg(a.s_w + n) : 0.0f;
+    // G = K: the tokens' scales (and in image mode 8 * their code sums over all of K, which the
+    // reduced offset-code sums still contain), loaded 16 tokens at a time as independent loads:
+    // one latency per batch, not one per token
+    constexpr int kB = kH < 16 ? kH : 16;
 #pragma unroll
-    for (int i = 0; i < kH; ++i) {
-      const int m = (int)hf * kH + i;
-      sa[i] = (a.groups == 1 && m < a.M) ? __ldg(a.s_a + m) : 0.0f;
-    }
-    if (n < a.N) {
-      const float bn = a.bias != nullptr ? __ldg(a.bias + n) : 0.0f;
-      const float swn = a.groups == 1 ? __ldg(a.s_w + n) : 0.0f;
+    for (int i0 = 0; i0 < kH; i0 += kB) {
+      float sa[kB], cs[kB];
 #pragma unroll
-      for (int i = 0; i < kH; ++i) {
-        const int m = (int)hf * kH + i;
-        if (m < a.M) {
-          float v = red[m * kRows + ch];
-          if (a.groups == 1) {  // exact integer partial: scale once
-            const float f = sa[i] * kOperandUnitInv;
-            v = f <= FLT_MAX ? (v * swn) * f : ((v * kOperandUnitInv) * sa[i]) * swn;
+      for (int i = 0; i < kB; ++i) {
+        const int m = (int)hf * kH + i0 + i;
+        sa[i] = (a.groups == 1 && m < a.M) ? __ldg(a.s_a + m) : 0.0f;
+        cs[i] = (a.groups == 1 && a.image && m < a.M) ? __ldg(a.corr + m) : 0.0f;
+      }
+      if (n < a.N) {
+#pragma unroll
+        for (int i = 0; i < kB; ++i) {
+          const int m = (int)hf * kH + i0 + i;
+          if (m < a.M) {
+            float v = red[m * kRows + ch] - cs[i];  // exact: integers below 2^24 (units 2^-18)
+            if (a.groups == 1) {  // exact integer partial: scale once
+              const float f = sa[i] * kOperandUnitInv;
+              v = f <= FLT_MAX ? (v * swn) * f : ((v * kOperandUnitInv) * sa[i]) * swn;
+            }
+            a.y[(int64_t)m * a.N + n] = __float2bfloat16_rn(v + bn);
           }
-          a.y[(int64_t)m * a.N + n] = __float2bfloat16_rn(v + bn);
         }
       }
     }
@@ -832,12 +903,17 @@ cudaError_t launch_mp(SkArgs a, const SkinnyProblem& p, int tiles, int sms, cuda
   }
   // Packed codes as byte matrices: weights [N, K/2], tokens [M, K/2]; one box = 128 packed bytes
   // (two K stages) x 128 weight rows or x kMp token rows, 128-byte swizzle.  Rows past N or M
-  // and columns past K/2 read zeros.
+  // and columns past K/2 read zeros.  Image mode: the tokens come from the A-operand image seen
+  // as rows of 128 bytes (block (0, kb) = rows 128 kb ..), one box = the first kMp rows of a
+  // block, copied as they are (the image is already in the 128-byte swizzle).
   CUtensorMap tmW, tmX;
-  if (!encode_2d(&tmW, CU_TENSOR_MAP_DATA_TYPE_UINT8, p.qw, p.K / 2, p.N, p.K / 2, kBK, kRows,
-                 CU_TENSOR_MAP_SWIZZLE_128B) ||
-      !encode_2d(&tmX, CU_TENSOR_MAP_DATA_TYPE_UINT8, p.q, p.K / 2, p.M, p.K / 2, kBK, kMp, CU_TENSOR_MAP_SWIZZLE_128B))
-    return cudaErrorInvalidValue;
+  const bool ok_w = encode_2d(&tmW, CU_TENSOR_MAP_DATA_TYPE_UINT8, p.qw, p.K / 2, p.N, p.K / 2, kBK, kRows,
+                              CU_TENSOR_MAP_SWIZZLE_128B);
+  const bool ok_x = a.image ? encode_2d(&tmX, CU_TENSOR_MAP_DATA_TYPE_UINT8, p.a_image, kBK,
+                                        (uint64_t)a.k_stages * kBK, kBK, kBK, kMp, CU_TENSOR_MAP_SWIZZLE_NONE)
+                            : encode_2d(&tmX, CU_TENSOR_MAP_DATA_TYPE_UINT8, p.q, p.K / 2, p.M, p.K / 2, kBK, kMp,
+                                        CU_TENSOR_MAP_SWIZZLE_128B);
+  if (!ok_w || !ok_x) return cudaErrorInvalidValue;
   a.split = choose_split<kMp>(tiles, a.k_stages, sms);
   cudaLaunchAttribute attr[2];
   cudaLaunchConfig_t cfg = make_config<kMp>(tiles * a.split, a.split, stream, attr);
@@ -863,6 +939,10 @@ cudaError_t launch_w4a4_skinny(const SkinnyProblem& p, cudaStream_t stream, int 
   a.bias = p.bias;
   a.y = static_cast<__nv_bfloat16*>(p.y);
   a.status = p.status;
+  // More than 16 tokens: converting the token rows in every CTA would cost more than the weights'
+  // conversion, so they come pre-expanded (operand image + corrections) when the caller has them.
+  a.image = (p.a_image != nullptr && p.corr != nullptr && p.M > 16) ? 1 : 0;
+  a.corr = p.corr;
   const int tiles = (p.N + kRows - 1) / kRows;
   if (p.M <= 16) return launch_mp<16>(a, p, tiles, sms, stream);
   if (p.M <= 32) return launch_mp<32>(a, p, tiles, sms, stream);

@@ -157,9 +157,13 @@ def run_linear(ref: Reference, x_bits, fused: bool):
     return jq.jq_w4a4_linear(dev(ref.packed_a), dev(ref.s_a), qw, sw, b, ref.G)
 
 
+# M <= 16: the few-token kernel converts the packed token codes itself; 16 < M <= 64: it reads
+# the tokens pre-expanded (operand image + corrections); M > 64: the GEMM
 @pytest.mark.parametrize("M,N,K,G,bias", [(300, 520, 512, 64, True), (300, 520, 512, 128, False),
                                           (300, 520, 512, 512, True), (64, 256, 256, 64, True),
-                                          (1, 8, 128, 128, True), (129, 8, 256, 64, False)])
+                                          (1, 8, 128, 128, True), (129, 8, 256, 64, False),
+                                          (17, 264, 1024, 128, True), (40, 520, 512, 512, False),
+                                          (64, 136, 2048, 2048, True), (33, 264, 768, 64, False)])
 def test_linear_matches_oracle(M, N, K, G, bias):
     w = wl.make("custom", seed=11 + M, M=M, K=K, N=N, G=G, bias=bias)
     x = act_bits(M, K, seed=3 + M, extreme=False) if M >= 8 else w.x_bits
@@ -234,9 +238,10 @@ def test_zero_weights_and_zero_activations():
     assert np.array_equal(yb[:, 9], np.full(M, wl.bf16_bits_to_f32(wl.f32_to_bf16_bits(w.bias[9:10]))[0]))
 
 
-def test_huge_activation_scale_path():
+@pytest.mark.parametrize("M", [16, 40])
+def test_huge_activation_scale_path(M):
     """s_a above 2^110 takes the epilogue's overflow-safe ordering."""
-    M, N, K, G = 16, 256, 256, 64
+    N, K, G = 256, 256, 64
     rng = np.random.default_rng(8)
     x = wl.f32_to_bf16_bits((rng.standard_normal((M, K)) * 2e35).astype(np.float32))
     w = (rng.standard_normal((N, K)) * 1e-3).astype(np.float32)
