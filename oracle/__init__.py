@@ -9,6 +9,8 @@ numpy arrays through ctypes.  Layout conventions used here:
 
 * activation codes / weight codes: ``int8 [rows, K]`` (one code per element);
 * packed codes: ``uint8 [rows, K/2]``, element 2j in the low nibble;
+* packed ternary codes (W1.58A4 weights): ``uint8 [rows, K/4]``, q + 1 in 2 bits
+  (byte layout in ``jq_oracle.c``);
 * activation scales ``s_a``: ``float32 [M, K/G]``;
 * weight scales ``s_w``: ``float32 [N, K/G]`` (per output channel);
 * bf16 values travel as their ``uint16`` bit patterns.
@@ -52,12 +54,16 @@ def _load():
             lib.oracle_bf16_rne.restype = ctypes.c_uint16
             lib.oracle_quantize_bf16.argtypes = [vp, i64, i64, i64, i64, vp, vp]
             lib.oracle_quantize_f32.argtypes = [vp, i64, i64, i64, vp, vp]
+            lib.oracle_quantize_ternary_f32.argtypes = [vp, i64, i64, i64, vp, vp]
+            lib.oracle_pack_ternary.argtypes = [vp, i64, i64, vp]
+            lib.oracle_unpack_ternary.argtypes = [vp, i64, i64, vp]
             lib.oracle_pack.argtypes = [vp, i64, i64, vp]
             lib.oracle_unpack.argtypes = [vp, i64, i64, vp]
             lib.oracle_group_partials.argtypes = [vp, vp, i64, i64, i64, i64, vp]
             lib.oracle_linear.argtypes = [vp, vp, vp, vp, vp, i64, i64, i64, i64, vp, vp]
             for f in ("oracle_quantize_bf16", "oracle_quantize_f32", "oracle_pack", "oracle_unpack",
-                      "oracle_group_partials", "oracle_linear"):
+                      "oracle_group_partials", "oracle_linear", "oracle_quantize_ternary_f32",
+                      "oracle_pack_ternary", "oracle_unpack_ternary"):
                 getattr(lib, f).restype = None
             _lib = lib
     return _lib
@@ -116,6 +122,35 @@ def unpack(packed: np.ndarray) -> np.ndarray:
     R, H = packed.shape
     out = np.empty((R, 2 * H), np.int8)
     _load().oracle_unpack(_p(packed), R, 2 * H, _p(out))
+    return out
+
+
+def quantize_ternary_f32(w: np.ndarray, group: int):
+    """fp32 weights [N, K] -> (ternary codes int8 [N,K] in {-1,0,1}, s_w f32 [N,K/G]) (absmean rule)."""
+    w = _c(w, np.float32)
+    N, K = w.shape
+    assert K % group == 0
+    codes = np.empty((N, K), np.int8)
+    scales = np.empty((N, K // group), np.float32)
+    _load().oracle_quantize_ternary_f32(_p(w), N, K, group, _p(codes), _p(scales))
+    return codes, scales
+
+
+def pack_ternary(codes: np.ndarray) -> np.ndarray:
+    """ternary codes int8 [rows, K] (K % 16 == 0) -> uint8 [rows, K/4] (2 bits per code, q + 1)."""
+    codes = _c(codes, np.int8)
+    R, K = codes.shape
+    assert K % 16 == 0 and codes.min(initial=0) >= -1 and codes.max(initial=0) <= 1
+    out = np.empty((R, K // 4), np.uint8)
+    _load().oracle_pack_ternary(_p(codes), R, K, _p(out))
+    return out
+
+
+def unpack_ternary(packed: np.ndarray) -> np.ndarray:
+    packed = _c(packed, np.uint8)
+    R, Q = packed.shape
+    out = np.empty((R, 4 * Q), np.int8)
+    _load().oracle_unpack_ternary(_p(packed), R, 4 * Q, _p(out))
     return out
 
 

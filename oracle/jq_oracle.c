@@ -163,6 +163,75 @@ void oracle_unpack(const uint8_t* packed, int64_t rows, int64_t K, int8_t* codes
     }
 }
 
+/* ---- ternary weights (W1.58A4) ----------------------------------------- */
+
+/*
+ * The W1.58A4 setting of the paper runs ternary weights with INT4 activations,
+ * group128 (Appendix table "DiT-XL/2 experimental details": "Ternary weights,
+ * INT4 activations, group128"; the ELF-B table likewise).  The paper prints no
+ * ternary rule.  The reading used here is the absmean rule of 1.58-bit weight
+ * quantisation, applied per row and per group of G consecutive reduction-axis
+ * elements (the group the paper names):
+ *     s = fl32(mean |w|)     -- the mean taken in fp64, summing the group in
+ *                               index order, then one division by G
+ *     q = clamp(rint(fl32(w / s)), -1, 1)        (round half to even)
+ * with s = 0 and q = 0 for an all-zero group.  A ternary code is an INT4 code,
+ * so the W1.58A4 linear layer is oracle_linear with these weight codes.
+ */
+void oracle_quantize_ternary_f32(const float* w, int64_t N, int64_t K, int64_t G, int8_t* codes,
+                                 float* scales) {
+#pragma omp parallel for schedule(static)
+  for (int64_t n = 0; n < N; ++n) {
+    for (int64_t g = 0; g < K / G; ++g) {
+      const float* wg = w + n * K + g * G;
+      double sum = 0.0;
+      for (int64_t k = 0; k < G; ++k) sum += fabs((double)wg[k]);
+      const float s = (float)(sum / (double)G);
+      scales[n * (K / G) + g] = s;
+      for (int64_t k = 0; k < G; ++k) {
+        int q = 0;
+        if (s != 0.0f) {
+          const float t = wg[k] / s;        /* IEEE single division */
+          const float r = rintf(t);         /* ties to even */
+          q = r > 1.0f ? 1 : (r < -1.0f ? -1 : (int)r);
+        }
+        codes[n * K + g * G + k] = (int8_t)q;
+      }
+    }
+  }
+}
+
+/*
+ * 2-bit packing of ternary codes: the code q is stored as q + 1 in {0, 1, 2}.
+ * Every 16 consecutive elements of a row fill 4 bytes; byte j (j = 0..3) holds
+ * elements 2j, 2j+1, 8+2j and 9+2j in its bits 0-1, 2-3, 4-5 and 6-7.  (Read
+ * as a little-endian 32-bit word, the four 2-bit fields at bit offsets 2i of
+ * every byte, i = 0..3, then collect elements {2j}, {2j+1}, {8+2j}, {9+2j}.)
+ */
+static int64_t ternary_bit(int64_t e) { /* bit offset of element e (0..15) within its 32-bit word */
+  const int64_t half = e / 8, r = e % 8;
+  return 8 * (r / 2) + 2 * (r % 2) + 4 * half;
+}
+
+void oracle_pack_ternary(const int8_t* codes, int64_t rows, int64_t K, uint8_t* packed) {
+  for (int64_t r = 0; r < rows; ++r)
+    for (int64_t w0 = 0; w0 < K; w0 += 16) {
+      uint32_t word = 0;
+      for (int64_t e = 0; e < 16; ++e)
+        word |= (uint32_t)(codes[r * K + w0 + e] + 1) << ternary_bit(e);
+      for (int64_t b = 0; b < 4; ++b) packed[r * (K / 4) + w0 / 4 + b] = (uint8_t)(word >> (8 * b));
+    }
+}
+
+void oracle_unpack_ternary(const uint8_t* packed, int64_t rows, int64_t K, int8_t* codes) {
+  for (int64_t r = 0; r < rows; ++r)
+    for (int64_t w0 = 0; w0 < K; w0 += 16) {
+      uint32_t word = 0;
+      for (int64_t b = 0; b < 4; ++b) word |= (uint32_t)packed[r * (K / 4) + w0 / 4 + b] << (8 * b);
+      for (int64_t e = 0; e < 16; ++e) codes[r * K + w0 + e] = (int8_t)((int)((word >> ternary_bit(e)) & 3u) - 1);
+    }
+}
+
 /* ---- integer GEMM and the dequantising epilogue ------------------------- */
 
 /* acc[m, n, g] = sum over the G elements of group g of qa[m,k] * qw[n,k]. */

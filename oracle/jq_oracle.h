@@ -13,6 +13,10 @@ void oracle_quantize_f32(const float* w, int64_t N, int64_t K, int64_t G, int8_t
                          float* scales);
 void oracle_pack(const int8_t* codes, int64_t rows, int64_t K, uint8_t* packed);
 void oracle_unpack(const uint8_t* packed, int64_t rows, int64_t K, int8_t* codes);
+void oracle_quantize_ternary_f32(const float* w, int64_t N, int64_t K, int64_t G, int8_t* codes,
+                                 float* scales);
+void oracle_pack_ternary(const int8_t* codes, int64_t rows, int64_t K, uint8_t* packed);
+void oracle_unpack_ternary(const uint8_t* packed, int64_t rows, int64_t K, int8_t* codes);
 void oracle_group_partials(const int8_t* qa, const int8_t* qw, int64_t M, int64_t N, int64_t K,
                            int64_t G, int32_t* acc);
 void oracle_linear(const int8_t* qa, const float* s_a, const int8_t* qw, const float* s_w,

@@ -320,3 +320,122 @@ def test_per_token_special_case():
 ])
 def test_bf16_rne_table(v, expect):
     assert oracle.bf16_rne(v) == expect
+
+
+# ------------------------------------------------ ternary weights (W1.58A4) ----
+
+def ternary_ref(ws):
+    """Exact-rational evaluation of the absmean ternary rule on one group: s = fl32(mean |w|)
+    with the mean taken exactly, q = clamp(round(fl32(w/s)), -1, 1).  The oracle sums the group
+    in fp64, which matches this unless the exact mean sits within ~G * 2^-53 (relative) of an
+    fp32 rounding boundary."""
+    ws = [float(np.float32(v)) for v in ws]
+    mean = sum(Fraction(abs(v)) for v in ws) / len(ws)
+    if mean == 0:
+        return [0] * len(ws), 0.0
+    s = f32_rne(mean)
+    out = []
+    for v in ws:
+        t = f32_rne(Fraction(v) / Fraction(s))
+        out.append(max(-1, min(1, round(t))))
+    return out, s
+
+
+def test_ternary_worked_example():
+    g = load_golden("ternary_example.json")
+    codes, s = oracle.quantize_ternary_f32(np.array([g["w"]], np.float32), 8)
+    assert codes[0].tolist() == g["codes"] and float(s[0, 0]) == g["scale"]
+    codes, s = oracle.quantize_ternary_f32(np.array([g["tie_w"]], np.float32), 4)
+    assert codes[0].tolist() == g["tie_codes"] and float(s[0, 0]) == g["tie_scale"]
+    packed = oracle.pack_ternary(np.array([g["pack_codes"]], np.int8))
+    assert [f"{b:02X}" for b in packed[0]] == g["packed_hex"]
+    assert oracle.unpack_ternary(packed)[0].tolist() == g["pack_codes"]
+    lin = g["linear"]
+    qw, sw = oracle.quantize_ternary_f32(np.array([g["w"]], np.float32), 8)
+    qa = np.ones((1, 8), np.int8)
+    y64, yb = oracle.linear(qa, np.array([[lin["s_a"]]], np.float32), qw, sw, np.array([lin["bias"]], np.float32), 8)
+    assert oracle.group_partials(qa, qw, 8)[0, 0, 0] == lin["acc"]
+    assert y64[0, 0] == lin["y"] and f"{int(yb[0, 0]):04X}" == lin["y_bf16_hex"]
+
+
+@pytest.mark.parametrize("seed", [0, 1, 2])
+def test_ternary_matches_exact_rational_rule(seed):
+    rng = np.random.default_rng(100 + seed)
+    G = 64
+    rows = []
+    rows.append((rng.standard_normal(G) * 0.02).astype(np.float32))             # typical weights
+    rows.append((rng.standard_normal(G) * 10.0 ** rng.uniform(-30, 30)).astype(np.float32))  # extreme magnitudes
+    r = rng.integers(-3, 4, G).astype(np.float32) * np.float32(0.5)               # many exact ties
+    r[0] = 3.0
+    rows.append(r)
+    o = (rng.standard_normal(G) * 0.02).astype(np.float32)
+    o[5] = 4.0                                                                       # one outlier
+    rows.append(o)
+    w = np.stack(rows)
+    codes, s = oracle.quantize_ternary_f32(w, G)
+    for i in range(w.shape[0]):
+        q_ref, s_ref = ternary_ref(w[i])
+        assert float(s[i, 0]) == s_ref, i
+        assert codes[i].tolist() == q_ref, i
+
+
+def test_ternary_invariants():
+    rng = np.random.default_rng(7)
+    N, K, G = 24, 384, 128
+    w = (rng.standard_normal((N, K)) * 0.02).astype(np.float32)
+    codes, s = oracle.quantize_ternary_f32(w, G)
+    assert codes.min() >= -1 and codes.max() <= 1
+    # s is the group's mean |w| (fp64 sum, then fp32): within one fp32 rounding of numpy's
+    m = np.abs(w.astype(np.float64)).reshape(N, K // G, G).mean(axis=2)
+    assert np.all(np.abs(s - m) <= m * 2.0 ** -23)
+    # sign symmetry, and scaling by a power of two moves only the scale
+    c2, s2 = oracle.quantize_ternary_f32(-w, G)
+    assert np.array_equal(c2, -codes) and np.array_equal(s2, s)
+    c3, s3 = oracle.quantize_ternary_f32(w * np.float32(8.0), G)
+    assert np.array_equal(c3, codes) and np.array_equal(s3, s * np.float32(8.0))
+    # every code is the nearest level of w/s within [-1, 1]
+    t = w.reshape(N, K // G, G) / s[:, :, None]
+    assert np.all(np.abs(np.clip(t, -1.5, 1.5) - codes.reshape(N, K // G, G)) <= 0.5 + 1e-6)
+
+
+def test_ternary_zero_and_constant_groups():
+    w = np.zeros((2, 32), np.float32)
+    w[1, :16] = -0.25
+    w[1, 16:] = 3.0
+    codes, s = oracle.quantize_ternary_f32(w, 16)
+    assert np.all(codes[0] == 0) and np.all(s[0] == 0)
+    assert s[1].tolist() == [0.25, 3.0]
+    assert codes[1].tolist() == [-1] * 16 + [1] * 16
+
+
+def test_ternary_pack_round_trip_and_layout():
+    rng = np.random.default_rng(3)
+    codes = rng.integers(-1, 2, (7, 160)).astype(np.int8)
+    packed = oracle.pack_ternary(codes)
+    assert packed.shape == (7, 40)
+    assert np.array_equal(oracle.unpack_ternary(packed), codes)
+    # every byte value a packed ternary row can hold (3^4 = 81 of them) round-trips, and a byte
+    # holds elements 2j, 2j+1, 8+2j, 9+2j of its 16-element word
+    vals = np.array([[a, b, c, d] for a in range(3) for b in range(3) for c in range(3) for d in range(3)])
+    for j in range(4):
+        row = np.zeros((len(vals), 16), np.int8)
+        row[:, 2 * j], row[:, 2 * j + 1], row[:, 8 + 2 * j], row[:, 9 + 2 * j] = (vals - 1).T
+        p = oracle.pack_ternary(row)
+        expect = vals[:, 0] | vals[:, 1] << 2 | vals[:, 2] << 4 | vals[:, 3] << 6
+        assert np.array_equal(p[:, j], expect.astype(np.uint8))
+        assert np.all(np.delete(p, j, axis=1) == 0x55)  # the other bytes: all codes 0 (q+1 = 1)
+        assert np.array_equal(oracle.unpack_ternary(p), row)
+
+
+def test_w158a4_linear_matches_numpy_fp64_dequant_matmul():
+    rng = np.random.default_rng(12)
+    M, N, K, G = 9, 40, 256, 128
+    x = wl.f32_to_bf16_bits(rng.standard_normal((M, K)).astype(np.float32))
+    qa, sa = oracle.quantize_bf16(x, G)
+    qw, sw = oracle.quantize_ternary_f32((rng.standard_normal((N, K)) * 0.02).astype(np.float32), G)
+    bias = (rng.standard_normal(N) * 0.01).astype(np.float32)
+    y64, _ = oracle.linear(qa, sa, qw, sw, bias, G)
+    a = (qa.reshape(M, K // G, G) * sa[:, :, None].astype(np.float64)).reshape(M, K)
+    w = (qw.reshape(N, K // G, G) * sw[:, :, None].astype(np.float64)).reshape(N, K)
+    ref = a @ w.T + bias.astype(np.float64)
+    assert np.allclose(y64, ref, rtol=1e-12, atol=1e-15)
