@@ -156,6 +156,44 @@ JQ_API jq_status jq_w4a4_linear_noalloc(const uint8_t* q, const float* s_a, cons
                                         int32_t group, void* stream);
 
 /*
+ * W1.58A4: ternary weights with INT4 activations (the paper's W1.58A4 setting: "Ternary
+ * weights, INT4 activations, group128", Appendix table "DiT-XL/2 experimental details"; the
+ * ELF-B table likewise).  The paper prints no ternary rule; the reading is the absmean rule per
+ * output channel and K-group:
+ *     s = fl32(mean |w|)   (fp64 sum of the group in index order, one division by group)
+ *     q = clamp(rint(fl32(w / s)), -1, 1)   (round half to even; s = q = 0 for a zero group)
+ * Packed ternary codes: q + 1 in {0, 1, 2}, 2 bits each, a row of K codes is K/4 bytes; every
+ * 16 consecutive elements fill one little-endian 32-bit word whose byte j (j = 0..3) holds
+ * elements 2j, 2j+1, 8+2j, 9+2j in bits 0-1, 2-3, 4-5, 6-7.
+ *
+ * Ternary weight packer (offline).
+ *   w   : fp32 [N, K] row-major
+ *   qw2 : uint8 [N, K/4] packed ternary codes (output)
+ *   s_w : fp32 [K/group, N] scales (output, group-major, as jq_pack_weight)
+ * Errors as jq_pack_weight.
+ */
+JQ_API jq_status jq_pack_weight_ternary(const float* w, int64_t N, int64_t K, int32_t group, uint8_t* qw2,
+                                        float* s_w, void* stream);
+
+/* Bytes of device scratch jq_w158a4_linear needs for this shape (the caller owns it). */
+JQ_API size_t jq_w158a4_workspace_size(int64_t M, int64_t N, int64_t K, int32_t group);
+
+/*
+ * W1.58A4 linear on pre-quantised activations: the linear layer above with ternary weight codes,
+ *   y = bf16( sum_g acc[m,n,g] * s_a[m,g] * s_w[g,n] + bias[n] ),  acc over qa * qw, qw in {-1,0,1}.
+ *   q, s_a    : packed INT4 activation codes and scales (jq_quantize_act)
+ *   qw2, s_w  : packed ternary weights and scales (jq_pack_weight_ternary, or any ternary codes
+ *               and finite scales in these layouts)
+ *   workspace : >= jq_w158a4_workspace_size(M, N, K, group) bytes, 16-byte aligned
+ * Up to 64 tokens the few-token kernel streams the 2-bit codes (half the bytes of INT4 weights);
+ * for more tokens the codes are rewritten as INT4 into the workspace and the INT4 GEMM runs.
+ * Other arguments, shapes and errors as jq_w4a4_linear.
+ */
+JQ_API jq_status jq_w158a4_linear(const uint8_t* q, const float* s_a, const uint8_t* qw2, const float* s_w,
+                                  const float* bias, void* y_bf16, int64_t M, int64_t N, int64_t K, int32_t group,
+                                  void* workspace, size_t workspace_bytes, void* stream);
+
+/*
  * Synchronises `stream` and returns JQ_ERR_TIMEOUT if any kernel of this library on the
  * current device gave up a bounded wait since the last reset (reset != 0 clears the flag),
  * JQ_ERR_UNSUPPORTED if a GEMM launch found its shared-memory window not 1024-byte aligned

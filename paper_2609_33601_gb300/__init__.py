@@ -62,6 +62,8 @@ def _load() -> ctypes.CDLL:
                 "jq_w4a4_group_partials": [vp, vp, vp, i64, i64, i64, i32, vp, sz, vp],
                 "jq_device_status": [vp, i32],
                 "jq_w4a4_linear_noalloc": [vp, vp, vp, vp, vp, vp, i64, i64, i64, i32, vp],
+                "jq_pack_weight_ternary": [vp, i64, i64, i32, vp, vp, vp],
+                "jq_w158a4_linear": [vp, vp, vp, vp, vp, vp, i64, i64, i64, i32, vp, sz, vp],
             }
             for name, args in sig.items():
                 f = getattr(lib, name)
@@ -69,6 +71,8 @@ def _load() -> ctypes.CDLL:
                 f.restype = ctypes.c_int
             lib.jq_workspace_size.argtypes = [i64, i64, i64, i32, i32]
             lib.jq_workspace_size.restype = ctypes.c_size_t
+            lib.jq_w158a4_workspace_size.argtypes = [i64, i64, i64, i32]
+            lib.jq_w158a4_workspace_size.restype = ctypes.c_size_t
             lib.jq_status_string.argtypes = [ctypes.c_int]
             lib.jq_status_string.restype = ctypes.c_char_p
             _lib = lib
@@ -191,6 +195,39 @@ def jq_w4a4_group_partials(q, qw, group: int, workspace=None, stream=None):
            _load().jq_w4a4_group_partials(_ptr(q), _ptr(qw), _ptr(acc), M, N, K, group, _ptr(ws), ws_bytes,
                                           _stream(stream)))
     return acc
+
+
+def jq_pack_weight_ternary(w: torch.Tensor, group: int, stream=None):
+    """fp32 weights [N, K] -> (packed ternary codes uint8 [N, K/4], scales fp32 [K/G, N])."""
+    assert w.dtype == torch.float32 and w.dim() == 2 and w.is_contiguous()
+    _need_cuda(w)
+    N, K = w.shape
+    qw2 = torch.empty((N, K // 4), dtype=torch.uint8, device=w.device)
+    s_w = torch.empty((K // group if group else 0, N), dtype=torch.float32, device=w.device)
+    _check("jq_pack_weight_ternary",
+           _load().jq_pack_weight_ternary(_ptr(w), N, K, group, _ptr(qw2), _ptr(s_w), _stream(stream)))
+    return qw2, s_w
+
+
+def jq_w158a4_workspace_size(M: int, N: int, K: int, group: int) -> int:
+    return int(_load().jq_w158a4_workspace_size(M, N, K, group))
+
+
+def jq_w158a4_linear(q, s_a, qw2, s_w, bias, group: int, y=None, workspace=None, stream=None):
+    """W1.58A4: y = bf16(sum_g acc * s_a * s_w + bias) from packed INT4 activations and packed
+    ternary weights."""
+    _need_cuda(q, s_a, qw2, s_w, bias)
+    M, K = q.shape[0], q.shape[1] * 2
+    N = qw2.shape[0]
+    if y is None:
+        y = torch.empty((M, N), dtype=torch.bfloat16, device=q.device)
+    if workspace is None:
+        workspace = torch.empty(max(jq_w158a4_workspace_size(M, N, K, group), 16), dtype=torch.uint8, device=q.device)
+    ws_bytes = workspace.numel() * workspace.element_size()
+    _check("jq_w158a4_linear",
+           _load().jq_w158a4_linear(_ptr(q), _ptr(s_a), _ptr(qw2), _ptr(s_w), _ptr(bias), _ptr(y), M, N, K, group,
+                                    _ptr(workspace), ws_bytes, _stream(stream)))
+    return y
 
 
 def jq_device_status(reset: bool = True, stream=None) -> int:

@@ -190,6 +190,60 @@ jq_status jq_fused_quant_linear(const void* x_bf16, int64_t ldx, const uint8_t* 
   return from_cuda(jq::launch_w4a4_gemm(p, s, d->sms));
 }
 
+jq_status jq_pack_weight_ternary(const float* w, int64_t N, int64_t K, int32_t group, uint8_t* qw2, float* s_w,
+                                 void* stream) {
+  if (N < 0 || !group_ok(K, group)) return JQ_ERR_INVALID_ARG;
+  if (N == 0) return JQ_OK;
+  if (w == nullptr || qw2 == nullptr || s_w == nullptr) return JQ_ERR_INVALID_ARG;
+  if (!aligned16(w) || !aligned16(qw2) || !aligned16(s_w)) return JQ_ERR_MISALIGNED;
+  const DeviceInfo* d = current_device();
+  if (d == nullptr) return JQ_ERR_UNSUPPORTED;
+  return from_cuda(jq::launch_pack_weight_ternary(w, N, K, group, qw2, s_w, static_cast<cudaStream_t>(stream),
+                                                  d->sms));
+}
+
+size_t jq_w158a4_workspace_size(int64_t M, int64_t N, int64_t K, int32_t group) {
+  if (M <= 0 || N < 0 || K <= 0 || group <= 0 || K % group != 0) return 0;
+  // as jq_w4a4_linear, + the weights rewritten as packed INT4 for the GEMM (M > 64)
+  size_t bytes = jq_workspace_size(M, N, K, group, 0);
+  if (!jq::skinny_supports(M, K, group)) bytes += round_up(static_cast<size_t>(N) * static_cast<size_t>(K / 2), 256);
+  return bytes;
+}
+
+jq_status jq_w158a4_linear(const uint8_t* q, const float* s_a, const uint8_t* qw2, const float* s_w, const float* bias,
+                           void* y_bf16, int64_t M, int64_t N, int64_t K, int32_t group, void* workspace,
+                           size_t workspace_bytes, void* stream) {
+  if (M == 0 || N == 0) return (M < 0 || N < 0) ? JQ_ERR_INVALID_ARG : JQ_OK;
+  if (q == nullptr || s_a == nullptr) return JQ_ERR_INVALID_ARG;
+  jq_status st = check_linear(M, N, K, group, qw2, s_w, bias, y_bf16, jq_w158a4_workspace_size(M, N, K, group),
+                              workspace, workspace_bytes);
+  if (st != JQ_OK) return st;
+  if (!aligned16(q) || !aligned16(s_a)) return JQ_ERR_MISALIGNED;
+  const DeviceInfo* d = current_device();
+  if (d == nullptr) return JQ_ERR_UNSUPPORTED;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  uint8_t* a_op = static_cast<uint8_t*>(workspace);
+  float* corr = reinterpret_cast<float*>(a_op + jq::ws_image_bytes(M, K));
+  if (jq::skinny_supports(M, K, group)) {  // few tokens: stream the 2-bit codes
+    jq::SkinnyProblem p{static_cast<int>(M), static_cast<int>(N), static_cast<int>(K), group, q, s_a, qw2, s_w, bias,
+                        y_bf16, d->status};
+    p.ternary = 1;
+    if (M > 16) {
+      if (jq::launch_expand_operand(q, M, K, group, a_op, corr, s, d->sms) != cudaSuccess) return JQ_ERR_CUDA;
+      p.a_image = a_op;
+      p.corr = corr;
+    }
+    return from_cuda(jq::launch_w4a4_skinny(p, s, d->sms));
+  }
+  // many tokens: the compute-bound GEMM, fed the same codes as INT4
+  uint8_t* qw4 = a_op + jq_workspace_size(M, N, K, group, 0);
+  if (jq::launch_ternary_to_int4(qw2, N, K, qw4, s, d->sms) != cudaSuccess) return JQ_ERR_CUDA;
+  if (jq::launch_expand_operand(q, M, K, group, a_op, corr, s, d->sms) != cudaSuccess) return JQ_ERR_CUDA;
+  jq::GemmProblem p{static_cast<int>(M), static_cast<int>(N), static_cast<int>(K), group, a_op, s_a, corr, qw4, s_w,
+                    bias, y_bf16, nullptr, d->status};
+  return from_cuda(jq::launch_w4a4_gemm(p, s, d->sms));
+}
+
 jq_status jq_w4a4_group_partials(const uint8_t* q, const uint8_t* qw, int32_t* acc, int64_t M, int64_t N, int64_t K,
                                  int32_t group, void* workspace, size_t workspace_bytes, void* stream) {
   if (M == 0 || N == 0) return (M < 0 || N < 0) ? JQ_ERR_INVALID_ARG : JQ_OK;

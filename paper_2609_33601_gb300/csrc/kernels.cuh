@@ -36,6 +36,12 @@ cudaError_t launch_quantize_act_operand(const void* x, int64_t M, int64_t K, int
 // fp32 weights [N, K] -> packed codes [N, K/2] + scales [K/G, N].
 cudaError_t launch_pack_weight(const float* w, int64_t N, int64_t K, int G, uint8_t* qw, float* s_w,
                                cudaStream_t stream, int sms);
+// fp32 weights [N, K] -> packed ternary codes [N, K/4] + scales [K/G, N] (ternary.cu).
+cudaError_t launch_pack_weight_ternary(const float* w, int64_t N, int64_t K, int G, uint8_t* qw, float* s_w,
+                                       cudaStream_t stream, int sms);
+// packed ternary codes [N, K/4] -> packed INT4 codes [N, K/2] (ternary.cu).
+cudaError_t launch_ternary_to_int4(const uint8_t* qw2, int64_t N, int64_t K, uint8_t* qw4, cudaStream_t stream,
+                                   int sms);
 // packed codes [rows, K/2] -> operand bytes [rows, K] + corrections [rows, K/G].
 cudaError_t launch_expand_operand(const uint8_t* packed, int64_t rows, int64_t K, int G, uint8_t* op, float* corr,
                                   cudaStream_t stream, int sms);
@@ -96,6 +102,8 @@ struct SkinnyProblem {
   // [M, K/G] (8 * the group's code sum, 2^-18 units), as launch_expand_operand writes them.
   const uint8_t* a_image = nullptr;
   const float* corr = nullptr;
+  // Ternary weights: qw is [N, K/4] in the packed ternary format (ternary.cu).
+  int ternary = 0;
 };
 cudaError_t launch_w4a4_skinny(const SkinnyProblem& p, cudaStream_t stream, int sms);
 

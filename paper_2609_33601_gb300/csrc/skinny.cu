@@ -122,6 +122,7 @@ struct SkArgs {
   __nv_bfloat16* y;   // [M, N]
   uint32_t* status;
   int image;          // token operand from the pre-expanded A-operand image (see tma_role)
+  int ternary;        // 2-bit ternary weights (ternary.cu) instead of 4-bit INT4 codes
   const float* corr;  // image mode: [M, K/G] 8 * the group's activation code sum, 2^-18 units
 };
 
@@ -167,11 +168,14 @@ __device__ __forceinline__ void tma_role(const SkArgs& a, const Range& rg, int n
   // The weight boxes of the ring's first pass do not depend on the previous kernel in the stream:
   // they go out before waiting for it (programmatic launch, ptx.cuh), the token boxes after.
   const int pre = nslots < kPkSlots ? nslots : kPkSlots;
-  const uint32_t wbytes = a.image ? L::kPkW : L::kPkSlot;
+  // packed weight bytes per K stage and per slot (2-bit ternary codes fill half the weight area)
+  const int wst = a.ternary ? kBK / 4 : kBK / 2;
+  const uint32_t wslot = a.ternary ? L::kPkW / 2 : L::kPkW;
+  const uint32_t wbytes = a.image ? wslot : wslot + L::kPkX;
   for (int j = 0; j < pre; ++j) {  // a fresh ring: every slot is free
     uint8_t* slot = smem + L::kOffPk + (uint32_t)j * L::kPkSlot;
     mbar_arrive_expect_tx(&b.pk_full[j], wbytes);
-    tma_load_2d(slot, tmW, &b.pk_full[j], (rg.st0 + j * kStPerSlot) * (kBK / 2), n0);
+    tma_load_2d(slot, tmW, &b.pk_full[j], (rg.st0 + j * kStPerSlot) * wst, n0);
   }
   pdl_wait();
   int jt = 0, jw = pre;  // token slots issued (image mode), weight slots issued
@@ -183,10 +187,10 @@ __device__ __forceinline__ void tma_role(const SkArgs& a, const Range& rg, int n
       const uint32_t s = (uint32_t)jw % kPkSlots;
       if (!mbar_wait(&b.pk_empty[s], ring_parity(jw, kPkSlots) ^ 1u, abort_flag, a.status)) break;
       uint8_t* slot = smem + L::kOffPk + s * L::kPkSlot;
-      const int x = (rg.st0 + jw * kStPerSlot) * (kBK / 2);  // packed byte offset along K
-      mbar_arrive_expect_tx(&b.pk_full[s], L::kPkSlot);
-      tma_load_2d(slot, tmW, &b.pk_full[s], x, n0);
-      tma_load_2d(slot + L::kPkW, tmX, &b.pk_full[s], x, 0);
+      const int st = rg.st0 + jw * kStPerSlot;  // first K stage of the slot
+      mbar_arrive_expect_tx(&b.pk_full[s], wbytes);
+      tma_load_2d(slot, tmW, &b.pk_full[s], st * wst, n0);
+      tma_load_2d(slot + L::kPkW, tmX, &b.pk_full[s], st * (kBK / 2), 0);
     }
   } else {
     // Image mode: the tokens arrive as operand bytes (the A-operand image of the GEMM path: per
@@ -213,9 +217,8 @@ __device__ __forceinline__ void tma_role(const SkArgs& a, const Range& rg, int n
       if (jw < nslots) {
         const uint32_t s = (uint32_t)jw % kPkSlots;
         if (mbar_test_wait(&b.pk_empty[s], ring_parity(jw, kPkSlots) ^ 1u)) {
-          mbar_arrive_expect_tx(&b.pk_full[s], L::kPkW);
-          tma_load_2d(smem + L::kOffPk + s * L::kPkSlot, tmW, &b.pk_full[s], (rg.st0 + jw * kStPerSlot) * (kBK / 2),
-                      n0);
+          mbar_arrive_expect_tx(&b.pk_full[s], wbytes);
+          tma_load_2d(smem + L::kOffPk + s * L::kPkSlot, tmW, &b.pk_full[s], (rg.st0 + jw * kStPerSlot) * wst, n0);
           ++jw;
           moved = true;
         }
@@ -273,6 +276,7 @@ __device__ __forceinline__ void unpack_role(const SkArgs& a, const Range& rg, ui
   const int gpst = groups_per_stage(a), gps = kStPerSlot * gpst;
   const uint32_t c8 = u & 7u;  // the chunk of its token row this thread holds
   float* sc_ring = reinterpret_cast<float*>(smem + L::kOffSa);  // pairs (s_a', c): c is the second
+  const int woff = a.ternary ? 1 : 8;  // the weights' operand offset: the correction is woff * sum qa
   int tot[kXChunks];  // G = K: running code sums of this thread's token rows
 #pragma unroll
   for (int i = 0; i < kXChunks; ++i) tot[i] = 0;
@@ -289,21 +293,46 @@ __device__ __forceinline__ void unpack_role(const SkArgs& a, const Range& rg, ui
     // interleaving loads with stores would expose a load latency per chunk.  A quarter-warp reads
     // 8 consecutive rows at one logical chunk (weights) or the 8 chunks of one row (tokens): 8
     // distinct physical chunks.
-    uint4 pw[8], px[kXChunks];
-    const uint32_t wrow = sw128_row(src, u);
+    uint4 px[kXChunks];
+    if (!a.ternary) {
+      uint4 pw[8];
+      const uint32_t wrow = sw128_row(src, u);
 #pragma unroll
-    for (int c = 0; c < 8; ++c) pw[c] = ld_shared_v4(wrow + (((uint32_t)c ^ r7) << 4));
+      for (int c = 0; c < 8; ++c) pw[c] = ld_shared_v4(wrow + (((uint32_t)c ^ r7) << 4));
 #pragma unroll
-    for (int h = 0; h < kStPerSlot; ++h) {
-      uint32_t v[32];
+      for (int h = 0; h < kStPerSlot; ++h) {
+        uint32_t v[32];
 #pragma unroll
-      for (int c = 0; c < 4; ++c) {
-        uint4 lo, hi;
-        nib32_to_operand_offset(pw[4 * h + c], lo, hi);
-        v[8 * c + 0] = lo.x; v[8 * c + 1] = lo.y; v[8 * c + 2] = lo.z; v[8 * c + 3] = lo.w;
-        v[8 * c + 4] = hi.x; v[8 * c + 5] = hi.y; v[8 * c + 6] = hi.z; v[8 * c + 7] = hi.w;
+        for (int c = 0; c < 4; ++c) {
+          uint4 lo, hi;
+          nib32_to_operand_offset(pw[4 * h + c], lo, hi);
+          v[8 * c + 0] = lo.x; v[8 * c + 1] = lo.y; v[8 * c + 2] = lo.z; v[8 * c + 3] = lo.w;
+          v[8 * c + 4] = hi.x; v[8 * c + 5] = hi.y; v[8 * c + 6] = hi.z; v[8 * c + 7] = hi.w;
+        }
+        tmem_st32(a_lane + os * L::kASlotCols + (uint32_t)h * L::kAStageCols, v);
       }
-      tmem_st32(a_lane + os * L::kASlotCols + (uint32_t)h * L::kAStageCols, v);
+    } else {
+      // 2-bit ternary weights: 64 packed bytes per row and slot, 64-byte swizzle (16-byte chunk c
+      // of row r at chunk c ^ ((r / 2) % 4)); each 32-bit word is 16 codes, and its four 2-bit
+      // planes are the operand bytes (q + 1) of elements {0,2,4,6}, {1,3,5,7}, {8,..,14}, {9,..,15}
+      uint4 pw[4];
+      const uint32_t wrow = src + u * 64u, sw = (u >> 1) & 3u;
+#pragma unroll
+      for (int c = 0; c < 4; ++c) pw[c] = ld_shared_v4(wrow + (((uint32_t)c ^ sw) << 4));
+#pragma unroll
+      for (int h = 0; h < kStPerSlot; ++h) {
+        uint32_t v[32];
+#pragma unroll
+        for (int c = 0; c < 2; ++c) {
+          const uint32_t wd[4] = {pw[2 * h + c].x, pw[2 * h + c].y, pw[2 * h + c].z, pw[2 * h + c].w};
+#pragma unroll
+          for (int i = 0; i < 4; ++i) {
+#pragma unroll
+            for (int k = 0; k < 4; ++k) v[16 * c + 4 * i + k] = (wd[i] >> (2 * k)) & 0x03030303u;
+          }
+        }
+        tmem_st32(a_lane + os * L::kASlotCols + (uint32_t)h * L::kAStageCols, v);
+      }
     }
     // token rows: only the M real ones (rows >= M stay zero in the operand ring); in image mode
     // the producer has copied them as operand bytes and the corrections come from global memory
@@ -367,7 +396,7 @@ __device__ __forceinline__ void unpack_role(const SkArgs& a, const Range& rg, ui
 #pragma unroll
       for (int i = 0; i < kXChunks; ++i) {
         const uint32_t r = (u + kUnpackGroupThreads * (uint32_t)i) >> 3;
-        if (c8 == (uint32_t)(q * cpg)) sc_ring[2 * (so * kMp + r) + 1] = (float)(8 * xs[i]) * kOperandUnit;
+        if (c8 == (uint32_t)(q * cpg)) sc_ring[2 * (so * kMp + r) + 1] = (float)(woff * xs[i]) * kOperandUnit;
       }
       __syncwarp();
       if ((u & 31u) == 0) mbar_arrive(&b.sa_full[so]);
@@ -378,7 +407,7 @@ __device__ __forceinline__ void unpack_role(const SkArgs& a, const Range& rg, ui
 #pragma unroll
     for (int i = 0; i < kXChunks; ++i) {
       const uint32_t r = (u + kUnpackGroupThreads * (uint32_t)i) >> 3;
-      if (c8 == 0u) corr[r] = (float)(8 * tot[i]) * kOperandUnit;
+      if (c8 == 0u) corr[r] = (float)(woff * tot[i]) * kOperandUnit;
     }
     __syncwarp();
     if ((u & 31u) == 0) mbar_arrive(b.corr_full);
@@ -430,7 +459,8 @@ __device__ __forceinline__ void scale_role(const SkArgs& a, const Range& rg, uin
       for (int h = 0; h < kPer; ++h) {
         const int m = (int)lane + 32 * h;
         if (m < kMp) sc_ring[2 * (o * kMp + m)] = finite ? v[j][h] * kOperandUnitInv : v[j][h];
-        if (m < kMp && a.image) sc_ring[2 * (o * kMp + m) + 1] = cv[j][h];  // 8 sum qa, 2^-18 units
+        // 8 sum qa in 2^-18 units; ternary weights are offset by 1, not 8: sum qa (exact)
+        if (m < kMp && a.image) sc_ring[2 * (o * kMp + m) + 1] = a.ternary ? cv[j][h] * 0.125f : cv[j][h];
       }
       if (lane == 0) flags[o] = finite ? 1 : 0;
       __syncwarp();
@@ -823,7 +853,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       for (int i = 0; i < kB; ++i) {
         const int m = (int)hf * kH + i0 + i;
         sa[i] = (a.groups == 1 && m < a.M) ? __ldg(a.s_a + m) : 0.0f;
-        cs[i] = (a.groups == 1 && a.image && m < a.M) ? __ldg(a.corr + m) : 0.0f;
+        cs[i] = (a.groups == 1 && a.image && m < a.M) ? __ldg(a.corr + m) * (a.ternary ? 0.125f : 1.0f) : 0.0f;
       }
       if (n < a.N) {
 #pragma unroll
@@ -907,8 +937,11 @@ cudaError_t launch_mp(SkArgs a, const SkinnyProblem& p, int tiles, int sms, cuda
   // as rows of 128 bytes (block (0, kb) = rows 128 kb ..), one box = the first kMp rows of a
   // block, copied as they are (the image is already in the 128-byte swizzle).
   CUtensorMap tmW, tmX;
-  const bool ok_w = encode_2d(&tmW, CU_TENSOR_MAP_DATA_TYPE_UINT8, p.qw, p.K / 2, p.N, p.K / 2, kBK, kRows,
-                              CU_TENSOR_MAP_SWIZZLE_128B);
+  // (ternary weights [N, K/4]: one box = 64 packed bytes (two K stages) x 128 rows, 64-byte swizzle)
+  const bool ok_w = a.ternary ? encode_2d(&tmW, CU_TENSOR_MAP_DATA_TYPE_UINT8, p.qw, p.K / 4, p.N, p.K / 4, kBK / 2,
+                                          kRows, CU_TENSOR_MAP_SWIZZLE_64B)
+                              : encode_2d(&tmW, CU_TENSOR_MAP_DATA_TYPE_UINT8, p.qw, p.K / 2, p.N, p.K / 2, kBK, kRows,
+                                          CU_TENSOR_MAP_SWIZZLE_128B);
   const bool ok_x = a.image ? encode_2d(&tmX, CU_TENSOR_MAP_DATA_TYPE_UINT8, p.a_image, kBK,
                                         (uint64_t)a.k_stages * kBK, kBK, kBK, kMp, CU_TENSOR_MAP_SWIZZLE_NONE)
                             : encode_2d(&tmX, CU_TENSOR_MAP_DATA_TYPE_UINT8, p.q, p.K / 2, p.M, p.K / 2, kBK, kMp,
@@ -942,6 +975,7 @@ cudaError_t launch_w4a4_skinny(const SkinnyProblem& p, cudaStream_t stream, int 
   // More than 16 tokens: converting the token rows in every CTA would cost more than the weights'
   // conversion, so they come pre-expanded (operand image + corrections) when the caller has them.
   a.image = (p.a_image != nullptr && p.corr != nullptr && p.M > 16) ? 1 : 0;
+  a.ternary = p.ternary ? 1 : 0;
   a.corr = p.corr;
   const int tiles = (p.N + kRows - 1) / kRows;
   if (p.M <= 16) return launch_mp<16>(a, p, tiles, sms, stream);

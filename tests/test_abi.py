@@ -30,7 +30,8 @@ def declared_functions():
 def test_header_declares_the_boundary():
     names = declared_functions()
     for need in ("jq_quantize_act", "jq_pack_weight", "jq_w4a4_linear", "jq_fused_quant_linear",
-                 "jq_status_string", "jq_workspace_size", "jq_w4a4_group_partials", "jq_device_status"):
+                 "jq_status_string", "jq_workspace_size", "jq_w4a4_group_partials", "jq_device_status",
+                 "jq_pack_weight_ternary", "jq_w158a4_linear", "jq_w158a4_workspace_size"):
         assert need in names
 
 
@@ -113,3 +114,32 @@ def test_binding_fails_loudly_without_cuda_tensors():
     x = torch.zeros((4, 256), dtype=torch.bfloat16)
     with pytest.raises(ValueError):
         jq.jq_quantize_act(x, 64)
+
+
+def test_w158a4_entry_points(lib):
+    i64, i32, vp, sz = ctypes.c_int64, ctypes.c_int32, ctypes.c_void_p, ctypes.c_size_t
+    lib.jq_pack_weight_ternary.argtypes = [vp, i64, i64, i32, vp, vp, vp]
+    lib.jq_w158a4_linear.argtypes = [vp, vp, vp, vp, vp, vp, i64, i64, i64, i32, vp, sz, vp]
+    lib.jq_w158a4_workspace_size.argtypes = [i64, i64, i64, i32]
+    lib.jq_w158a4_workspace_size.restype = sz
+    lib.jq_workspace_size.argtypes = [i64, i64, i64, i32, i32]
+    lib.jq_workspace_size.restype = sz
+    ws, ws4 = lib.jq_w158a4_workspace_size, lib.jq_workspace_size
+    # few tokens: as the INT4 linear; many tokens: + the weights rewritten as packed INT4
+    assert ws(64, 12288, 4096, 128) == ws4(64, 12288, 4096, 128, 0)
+    assert ws(1024, 12288, 4096, 128) == ws4(1024, 12288, 4096, 128, 0) + 12288 * 4096 // 2
+    assert ws(0, 8, 256, 64) == 0
+    A, odd = _fake(0x10000), _fake(0x10008)
+    P = lib.jq_pack_weight_ternary
+    assert P(None, 8, 256, 64, A, A, None) == INVALID
+    assert P(A, 8, 256, 100, A, A, None) == INVALID
+    assert P(A, 8, 192, 64, A, A, None) == INVALID
+    assert P(A, 8, 256, 64, odd, A, None) == MISALIGNED
+    assert P(A, 0, 256, 64, None, None, None) == OK
+    L = lib.jq_w158a4_linear
+    big = 1 << 30
+    assert L(A, A, A, A, None, A, 4, 12, 256, 64, A, big, None) == INVALID     # N % 8
+    assert L(None, A, A, A, None, A, 4, 16, 256, 64, A, big, None) == INVALID
+    assert L(A, A, odd, A, None, A, 4, 16, 256, 64, A, big, None) == MISALIGNED
+    assert L(A, A, A, A, None, A, 100, 16, 256, 64, A, 16, None) == WORKSPACE
+    assert L(A, A, A, A, None, A, 0, 16, 256, 64, None, 0, None) == OK
