@@ -82,6 +82,20 @@ def kernel_hash(kernel_file: str) -> str:
     return h.hexdigest()[:16]
 
 
+def metric_name(args) -> str:
+    return "W1.58A4 linear TOPS" if args.weights == "ternary" else "W4A4 linear TOPS"
+
+
+def launches_per_step(M: int, few: bool, fused: bool, ternary: bool) -> int:
+    """Kernels of this library per timed step: the activation quantiser (or, fused, the
+    quantise-to-operand kernel), the operand expansion when the linear kernel reads the operand
+    image (more than 16 tokens), the ternary -> INT4 rewrite (ternary weights, GEMM), and the
+    linear kernel itself."""
+    if fused:
+        return 2
+    return 1 + (1 if M > 16 else 0) + (1 if ternary and not few else 0) + 1
+
+
 def dist_env():
     rank = int(os.environ.get("RANK", "0"))
     world = int(os.environ.get("WORLD_SIZE", "1"))
@@ -150,7 +164,7 @@ class OracleSample:
     sampled activation rows and evaluate the linear layer for them (the weights are packed
     once, outside the timing, as on the GPU)."""
 
-    def __init__(self, name: str, seed: int = 7):
+    def __init__(self, name: str, seed: int = 7, ternary: bool = False):
         import oracle
         from paper_2609_33601_gb300 import workloads as wl
         self.oracle = oracle
@@ -158,7 +172,8 @@ class OracleSample:
         self.desc, self.M, self.K, self.N, self.G, gen = WORKLOADS[name]
         w = wl.make(gen, seed=seed, M=self.M, G=self.G)
         self.x_bits, self.bias = w.x_bits, w.bias
-        self.qw, self.sw = oracle.quantize_f32(w.w, self.G)
+        quant = oracle.quantize_ternary_f32 if ternary else oracle.quantize_f32
+        self.qw, self.sw = quant(w.w, self.G)
         self.rows = 8
 
     def run(self, rows: int) -> float:
@@ -191,7 +206,7 @@ def run_reference(args):
     rank, world, _ = dist_env()
     if rank != 0:
         return 0
-    o = OracleSample(args.workload)
+    o = OracleSample(args.workload, ternary=args.weights == "ternary")
     per_step = min(args.ref_seconds, 120.0 / (args.steps + args.warmup))
     o.calibrate(per_step)
     for _ in range(args.warmup):
@@ -200,7 +215,7 @@ def run_reference(args):
     mean = sum(times) / len(times)
     cb = o.describe(mean)
     value = cb["value"]
-    line = {"impl": "reference", "metric": "W4A4 linear TOPS", "value": value, "unit": "TOPS", "n_gpus": args.gpus,
+    line = {"impl": "reference", "metric": metric_name(args), "value": value, "unit": "TOPS", "n_gpus": args.gpus,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": mean * 1e3, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "int4", "data": "synthetic",
             "config": {"workload": o.desc, "M": o.M, "K": o.K, "N": o.N, "group": o.G},
@@ -273,7 +288,8 @@ def run_ours(args):
     for i in range(n_sets):
         w = wl.make(gen, seed=100 + 17 * rank + i, M=M, G=G)
         x = torch.from_numpy(w.x_bits.view(np.int16)).to(dev).view(torch.bfloat16)
-        qw, sw = jq.jq_pack_weight(torch.from_numpy(w.w).to(dev), G)
+        pack = jq.jq_pack_weight_ternary if args.weights == "ternary" else jq.jq_pack_weight
+        qw, sw = pack(torch.from_numpy(w.w).to(dev), G)
         b = None if w.bias is None else torch.from_numpy(w.bias).to(dev)
         sets.append((x, qw, sw, b))
         del w
@@ -282,7 +298,10 @@ def run_ours(args):
     s_a = torch.empty((M, K // G), dtype=torch.float32, device=dev)
     y = torch.empty((M, N), dtype=torch.bfloat16, device=dev)
     fused = args.fused
-    ws = torch.empty(max(jq.jq_workspace_size(M, N, K, G, fused), 16), dtype=torch.uint8, device=dev)
+    ternary = args.weights == "ternary"
+    need = jq.jq_w158a4_workspace_size(M, N, K, G) if ternary else jq.jq_workspace_size(M, N, K, G, fused)
+    ws = torch.empty(max(need, 16), dtype=torch.uint8, device=dev)
+    linear_call = jq.jq_w158a4_linear if ternary else jq.jq_w4a4_linear
     stream = torch.cuda.current_stream()
 
     def quantize(i, st):
@@ -293,7 +312,7 @@ def run_ours(args):
         if fused:  # bf16 activations straight into the GEMM operand
             jq.jq_fused_quant_linear(x, qw, sw, b, G, y=y, workspace=ws, stream=st)
         else:
-            jq.jq_w4a4_linear(q, s_a, qw, sw, b, G, y=y, workspace=ws, stream=st)
+            linear_call(q, s_a, qw, sw, b, G, y=y, workspace=ws, stream=st)
 
     def step(i, st=None):
         if not fused:
@@ -365,7 +384,7 @@ def run_ours(args):
             jq.jq_fused_quant_linear(x_dev, qw, sw, b, G, y=y, workspace=ws, stream=stream)
         else:
             jq.jq_quantize_act(x_dev, G, q, s_a, stream=stream)
-            jq.jq_w4a4_linear(q, s_a, qw, sw, b, G, y=y, workspace=ws, stream=stream)
+            linear_call(q, s_a, qw, sw, b, G, y=y, workspace=ws, stream=stream)
         y_host.copy_(y, non_blocking=True)
 
     for i in range(args.warmup):
@@ -389,15 +408,18 @@ def run_ours(args):
     bf16_peak, hbm_peak, peak_src = measured_peaks()
     fp8_peak = bf16_peak * FP8_PER_BF16
     kernel_file = "skinny.cu" if few else "gemm.cu"
-    traffic = None if fused else KERNEL_TRAFFIC.get((args.workload, kernel_hash(kernel_file)))
+    traffic = None if (fused or ternary) else KERNEL_TRAFFIC.get((args.workload, kernel_hash(kernel_file)))
     # algorithmic bytes of one linear call: packed weights and their scales, packed activation
     # codes and scales (the fused call reads bf16 activations instead), bias, bf16 output
     groups = K // G
     act_bytes = M * K * 2 if fused else M * K // 2 + M * groups * 4
-    alg_bytes = N * K // 2 + groups * N * 4 + act_bytes + (0 if sets[0][3] is None else N * 4) + M * N * 2
+    wbytes = N * K // 4 if ternary else N * K // 2  # 2-bit ternary or 4-bit INT4 weight codes
+    alg_bytes = wbytes + groups * N * 4 + act_bytes + (0 if sets[0][3] is None else N * 4) + M * N * 2
     # the bound is whichever of the tensor time and the HBM time is larger
     t_tensor, t_hbm = ops_step / (fp8_peak * 1e12), alg_bytes / (hbm_peak * 1e9)
-    what = ("jq_fused_quant_linear (quantise-to-operand + tcgen05 GEMM)" if fused else
+    what = ("jq_w158a4_linear (few-token kernel, 2-bit weights)" if ternary and few else
+            "jq_w158a4_linear (ternary -> INT4 rewrite + operand expansion + tcgen05 GEMM)" if ternary else
+            "jq_fused_quant_linear (quantise-to-operand + tcgen05 GEMM)" if fused else
             "jq_w4a4_linear (few-token weight-streaming kernel)" if few else
             "jq_w4a4_linear (operand expansion + tcgen05 GEMM)")
     if t_hbm > t_tensor:
@@ -423,15 +445,17 @@ def run_ours(args):
         return 0
     cpu = None
     if world == 1 and not args.no_cpu_baseline:
-        o = OracleSample(args.workload)
+        o = OracleSample(args.workload, ternary=ternary)
         o.calibrate(args.ref_seconds)
         cpu = o.describe(o.run(o.rows))
     line = {
-        "metric": "W4A4 linear TOPS", "value": value, "unit": "TOPS", "n_gpus": world, "steps": args.steps,
+        "metric": metric_name(args), "value": value, "unit": "TOPS", "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": total_ms / args.steps, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "int4", "data": "synthetic",
         "config": {"workload": desc, "M": M, "K": K, "N": N, "group": G,
-                   "step": "jq_fused_quant_linear" if fused else "jq_quantize_act + jq_w4a4_linear",
+                   "step": ("jq_fused_quant_linear" if fused else
+                            "jq_quantize_act + jq_w158a4_linear" if ternary else "jq_quantize_act + jq_w4a4_linear"),
+                   "weights": "ternary (2-bit)" if ternary else "INT4",
                    "launch": "CUDA graph of the K steps",
                    "parallelism": f"replicas x{world}",
                    "l2": f"{n_sets} rotating input/weight sets larger than L2"},
@@ -439,7 +463,7 @@ def run_ours(args):
         "context": context,
         "cpu_baseline": cpu,
         "e2e": {"value": e2e_value, "unit": "TOPS", "h2d_bytes_per_step": M * K * 2, "d2h_bytes_per_step": M * N * 2},
-        "gpu_launches": (2 if (few or fused) else 3) * args.steps,
+        "gpu_launches": launches_per_step(M, few, fused, ternary) * args.steps,
         "clocks": clocks.summary(),
     }
     print(json.dumps(line), flush=True)
@@ -460,10 +484,14 @@ def main():
     ap.add_argument("--ref-seconds", type=float, default=10.0, help="CPU seconds per oracle sample")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--fused", action="store_true", help="time jq_fused_quant_linear (bf16 activations in)")
+    ap.add_argument("--weights", choices=["int4", "ternary"], default="int4",
+                    help="ternary: the W1.58A4 layer (jq_pack_weight_ternary + jq_w158a4_linear)")
     ap.add_argument("--no-context", action="store_true", help="skip the cuBLAS bf16 GEMM of the same shape")
     args = ap.parse_args()
     if args.warmup < 3:
         ap.error("--warmup must be at least 3")
+    if args.fused and args.weights == "ternary":
+        ap.error("--fused is an INT4-weight call")
     if args.impl == "reference":
         return run_reference(args)
     return run_ours(args)
