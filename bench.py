@@ -82,6 +82,24 @@ def kernel_hash(kernel_file: str) -> str:
     return h.hexdigest()[:16]
 
 
+def max_over_ranks(values, device):
+    """Each timing's maximum over the ranks (one replica of the workload per rank): the
+    whole job is as slow as its slowest rank.  The identity on a single process."""
+    import torch
+    import torch.distributed as dist
+    if not (dist.is_available() and dist.is_initialized()) or dist.get_world_size() == 1:
+        return [float(v) for v in values]
+    t = torch.tensor([float(v) for v in values], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return [float(v) for v in t.cpu()]
+
+
+def whole_job_tops(world: int, ops_per_step: float, steps: int, seconds: float) -> float:
+    """Whole-job throughput of `world` replicas that each ran `steps` steps of `ops_per_step`
+    operations in at most `seconds` (the max over ranks)."""
+    return world * ops_per_step * steps / seconds / 1e12
+
+
 def metric_name(args) -> str:
     return "W1.58A4 linear TOPS" if args.weights == "ternary" else "W4A4 linear TOPS"
 
@@ -365,11 +383,7 @@ def run_ours(args):
     barrier()
     total_ms = t_start.elapsed_time(t_end)
     gemm_ms = l_start.elapsed_time(l_end) / args.steps
-    if world > 1:
-        import torch.distributed as dist
-        t = torch.tensor([total_ms, gemm_ms], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        total_ms, gemm_ms = float(t[0]), float(t[1])
+    total_ms, gemm_ms = max_over_ranks([total_ms, gemm_ms], dev)
     assert jq.jq_device_status() == 0, "a kernel reported a bounded-wait timeout"
 
     # end to end through the public API: pinned host activations in, host result out
@@ -396,15 +410,11 @@ def run_ours(args):
         e2e_step(i)
     torch.cuda.synchronize()
     e2e_s = time.perf_counter() - e0
-    if world > 1:
-        import torch.distributed as dist
-        t = torch.tensor([e2e_s], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        e2e_s = float(t[0])
+    (e2e_s,) = max_over_ranks([e2e_s], dev)
 
     ops_step = 2.0 * M * N * K
-    value = world * ops_step * args.steps / (total_ms * 1e-3) / 1e12
-    e2e_value = world * ops_step * args.steps / e2e_s / 1e12
+    value = whole_job_tops(world, ops_step, args.steps, total_ms * 1e-3)
+    e2e_value = whole_job_tops(world, ops_step, args.steps, e2e_s)
     bf16_peak, hbm_peak, peak_src = measured_peaks()
     fp8_peak = bf16_peak * FP8_PER_BF16
     kernel_file = "skinny.cu" if few else "gemm.cu"
