@@ -93,7 +93,10 @@ struct Layout {
   static constexpr uint32_t kOffSa = kOffOp + kOpSlots * kOpSlot;
   static constexpr uint32_t kOffSaFlag = kOffSa + 2 * kSaRing * kMp * 4;
   static constexpr uint32_t kOffCorr = kOffSaFlag + kSaRing * 4;  // G = K: 8 sum qa per unpack group [3][kMp]
-  static constexpr uint32_t kOffBar = kOffCorr + (kUnpackGroups + 1) * kMp * 4;
+  // the final pass's per-token operands (G = K), staged by the scale warp at the start: the
+  // scale and the whole-K correction [2][kMp]
+  static constexpr uint32_t kOffFin = kOffCorr + (kUnpackGroups + 1) * kMp * 4;
+  static constexpr uint32_t kOffBar = kOffFin + 2 * kMp * 4;
   static constexpr uint32_t kNumBars = 2 * kPkSlots + 3 * kOpSlots + 8 + 2 + 2 * kSaRing + 1;
   static constexpr uint32_t kOffMisc = kOffBar + kNumBars * 8;
   static constexpr uint32_t kSmemBytes = kOffMisc + 16;
@@ -159,24 +162,42 @@ __device__ __forceinline__ uint32_t sw128_row(uint32_t base, uint32_t r) { retur
 
 // ------------------------------------------------------------------ TMA producer
 template <int kMp>
+__device__ __forceinline__ int tma_pre_slots(const Range& rg) {
+  const int nslots = (rg.nst + kStPerSlot - 1) / kStPerSlot;
+  return nslots < Layout<kMp>::kPkSlots ? nslots : Layout<kMp>::kPkSlots;
+}
+// packed weight bytes per K stage and per slot (2-bit ternary codes fill half the weight area)
+__device__ __forceinline__ int weight_stage_bytes(const SkArgs& a) { return a.ternary ? kBK / 4 : kBK / 2; }
+
+// The weight boxes of the packed ring's first pass (a fresh ring: every slot is free).
+template <int kMp>
+__device__ __forceinline__ void tma_first_weights(const SkArgs& a, const Range& rg, int n0, const CUtensorMap* tmW,
+                                                  uint8_t* smem, const SkBars& b) {
+  using L = Layout<kMp>;
+  const int wst = weight_stage_bytes(a);
+  const uint32_t wslot = a.ternary ? L::kPkW / 2 : L::kPkW;
+  const uint32_t wbytes = a.image ? wslot : wslot + L::kPkX;
+  for (int j = 0; j < tma_pre_slots<kMp>(rg); ++j) {
+    mbar_arrive_expect_tx(&b.pk_full[j], wbytes);
+    tma_load_2d(smem + L::kOffPk + (uint32_t)j * L::kPkSlot, tmW, &b.pk_full[j], (rg.st0 + j * kStPerSlot) * wst,
+                n0);
+  }
+}
+
+template <int kMp>
 __device__ __forceinline__ void tma_role(const SkArgs& a, const Range& rg, int n0, const CUtensorMap* tmW,
                                          const CUtensorMap* tmX, uint8_t* smem, const SkBars& b,
                                          volatile int* abort_flag) {
   using L = Layout<kMp>;
   constexpr int kPkSlots = L::kPkSlots;
   const int nslots = (rg.nst + kStPerSlot - 1) / kStPerSlot;
-  // The weight boxes of the ring's first pass do not depend on the previous kernel in the stream:
-  // they go out before waiting for it (programmatic launch, ptx.cuh), the token boxes after.
-  const int pre = nslots < kPkSlots ? nslots : kPkSlots;
-  // packed weight bytes per K stage and per slot (2-bit ternary codes fill half the weight area)
-  const int wst = a.ternary ? kBK / 4 : kBK / 2;
+  // The weight boxes of the first pass went out during setup (tma_first_weights): they do not
+  // depend on the previous kernel in the stream (programmatic launch, ptx.cuh); the token boxes
+  // and everything after wait for it.
+  const int pre = tma_pre_slots<kMp>(rg);
+  const int wst = weight_stage_bytes(a);
   const uint32_t wslot = a.ternary ? L::kPkW / 2 : L::kPkW;
   const uint32_t wbytes = a.image ? wslot : wslot + L::kPkX;
-  for (int j = 0; j < pre; ++j) {  // a fresh ring: every slot is free
-    uint8_t* slot = smem + L::kOffPk + (uint32_t)j * L::kPkSlot;
-    mbar_arrive_expect_tx(&b.pk_full[j], wbytes);
-    tma_load_2d(slot, tmW, &b.pk_full[j], (rg.st0 + j * kStPerSlot) * wst, n0);
-  }
   pdl_wait();
   int jt = 0, jw = pre;  // token slots issued (image mode), weight slots issued
   if (!a.image) {
@@ -430,7 +451,19 @@ __device__ __forceinline__ void scale_role(const SkArgs& a, const Range& rg, uin
   float* sc_ring = reinterpret_cast<float*>(smem + L::kOffSa);  // pairs (s_a', c): s_a' is the first
   int* flags = reinterpret_cast<int*>(smem + L::kOffSaFlag);
   const int ng = drain_groups(a, rg);
-  if (ng == 0 || a.groups == 1) return;  // G = K: the final pass reads s_a itself
+  {
+    // The final pass's per-token operands, fetched at the start: under the weight stream a
+    // global load takes microseconds, which the final pass would otherwise wait for after the
+    // last MMA.  (Read after the CTA barrier that precedes the reduction.)
+    float* fin = reinterpret_cast<float*>(smem + L::kOffFin);
+    for (int m = (int)lane; m < kMp; m += 32) {
+      const bool in = a.groups == 1 && m < a.M;
+      fin[m] = in ? __ldg(a.s_a + m) : 0.0f;
+      // whole-K correction (image mode): 8 sum qa, or sum qa for ternary weights (offset 1)
+      fin[kMp + m] = (in && a.image) ? __ldg(a.corr + m) * (a.ternary ? 0.125f : 1.0f) : 0.0f;
+    }
+  }
+  if (ng == 0 || a.groups == 1) return;  // G = K: no per-group scales
   const int g0 = rg.st0 * groups_per_stage(a);
   for (int gb = 0; gb < ng; gb += kSaBatch) {
     const int nb = ng - gb < kSaBatch ? ng - gb : kSaBatch;
@@ -734,7 +767,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   const uint32_t warp = warp_id(), lane = lane_id();
   const bool single = a.groups == 1;
   const int ngroups = single ? kUnpackGroups + 1 : kUnpackGroups;  // G = K: the drain warps unpack too
-  if (warp == kWarpMma1) {  // barrier setup, spread over one warp
+  if (warp == kWarpTma) {  // barrier setup, spread over one warp: the TMA warp, which starts streaming right after
     if (lane == 0) *abort_flag = 0;
     for (int i = (int)lane; i < L::kPkSlots; i += 32) {
       mbar_init(&b.pk_full[i], 1);                   // the producer's expect_tx
@@ -757,9 +790,14 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     if (lane == 0) mbar_init(b.corr_full, ngroups * kUnpackGroupWarps);
     fence_mbar_init();
+    __syncwarp();
     if (lane == 0) {
       tma_prefetch_desc(&tmW);
       tma_prefetch_desc(&tmX);
+      // The weight boxes of the ring's first pass depend neither on the previous kernel in the
+      // stream nor on the rest of this CTA's setup (TMEM, the zeroed token rows): they go out
+      // now, before the CTA-wide barrier and before waiting for that kernel.
+      tma_first_weights<kMp>(a, rg, n0, &tmW, smem, b);
     }
   }
   if (warp == kWarpMma) {
@@ -788,6 +826,14 @@ __global__ void __launch_bounds__(kThreads, 1)
   // weight boxes, the scale warp and the drain before their first access to activation data or
   // the output; the unpack and MMA roles touch only shared and tensor memory.
   pdl_launch_dependents();
+  // drain threads: this channel's bias and (G = K) weight scale for the final pass, fetched now
+  // (weight-side data: no need to wait for the previous kernel) so that no one waits for them later
+  float fin_bn = 0.0f, fin_swn = 0.0f;
+  if (drain && rank == 0) {
+    const int n = n0 + (int)((warp & 3u) * 32u + lane);
+    fin_bn = (n < a.N && a.bias != nullptr) ? __ldg(a.bias + n) : 0.0f;
+    fin_swn = (n < a.N && a.groups == 1) ? __ldg(a.s_w + n) : 0.0f;
+  }
   if (drain) {
     asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;\n" ::"n"(kRegsDrain<kMp>) : "memory");
     if (single) unpack_role<kMp>(a, rg, smem, tmem_base, b, ngroups, abort_flag);  // group 2 (warps 12-15)
@@ -837,36 +883,22 @@ __global__ void __launch_bounds__(kThreads, 1)
       for (int i = 0; i < kH; ++i) red[(hf * kH + i) * kRows + ch] += v[i];
     }
   }
-  cluster_sync_all();  // no CTA leaves while a peer may still read its buffer
+  if (a.split > 1) cluster_sync_all();  // no CTA leaves while a peer may still read its buffer
   if (drain && rank == 0) {
     const int n = n0 + (int)ch;
-    const float bn = (n < a.N && a.bias != nullptr) ? __ldg(a.bias + n) : 0.0f;
-    const float swn = (n < a.N && a.groups == 1) ? __ldg(a.s_w + n) : 0.0f;
-    // G = K: the tokens' scales (and in image mode 8 * their code sums over all of K, which the
-    // reduced offset-code sums still contain), loaded 16 tokens at a time as independent loads:
-    // one latency per batch, not one per token
-    constexpr int kB = kH < 16 ? kH : 16;
-#pragma unroll
-    for (int i0 = 0; i0 < kH; i0 += kB) {
-      float sa[kB], cs[kB];
-#pragma unroll
-      for (int i = 0; i < kB; ++i) {
-        const int m = (int)hf * kH + i0 + i;
-        sa[i] = (a.groups == 1 && m < a.M) ? __ldg(a.s_a + m) : 0.0f;
-        cs[i] = (a.groups == 1 && a.image && m < a.M) ? __ldg(a.corr + m) * (a.ternary ? 0.125f : 1.0f) : 0.0f;
-      }
-      if (n < a.N) {
-#pragma unroll
-        for (int i = 0; i < kB; ++i) {
-          const int m = (int)hf * kH + i0 + i;
-          if (m < a.M) {
-            float v = red[m * kRows + ch] - cs[i];  // exact: integers below 2^24 (units 2^-18)
-            if (a.groups == 1) {  // exact integer partial: scale once
-              const float f = sa[i] * kOperandUnitInv;
-              v = f <= FLT_MAX ? (v * swn) * f : ((v * kOperandUnitInv) * sa[i]) * swn;
-            }
-            a.y[(int64_t)m * a.N + n] = __float2bfloat16_rn(v + bn);
+    const float* fin = reinterpret_cast<const float*>(smem + L::kOffFin);  // staged by the scale warp
+    if (n < a.N) {
+#pragma unroll 8
+      for (int i = 0; i < kH; ++i) {
+        const int m = (int)hf * kH + i;
+        if (m < a.M) {
+          float v = red[m * kRows + ch];
+          if (a.groups == 1) {  // exact integer partial (less the whole-K correction): scale once
+            v -= fin[kMp + m];  // exact: integers below 2^24 (units 2^-18)
+            const float sa = fin[m], f = sa * kOperandUnitInv;
+            v = f <= FLT_MAX ? (v * fin_swn) * f : ((v * kOperandUnitInv) * sa) * fin_swn;
           }
+          a.y[(int64_t)m * a.N + n] = __float2bfloat16_rn(v + fin_bn);
         }
       }
     }

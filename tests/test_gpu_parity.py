@@ -284,3 +284,32 @@ def test_full_size_config(name, G):
     rows = rows[rows < w.M]
     y64, _ = ref.linear(rows)
     check_linear(y_sep[rows], y64, ref.partials(rows), ref.s_a[rows], ref.s_w_rows, ref.bias, name)
+
+
+# The memory-to-compute crossover sweep at full size: both shapes (K=4096 -> N=12288 and
+# K=3072 -> N=3072, per-token/per-channel scales) at token counts that take each kernel
+# (1 and 64 tokens: the few-token kernel with and without pre-expanded tokens; 4096 and 16384:
+# the GEMM).  Every code and scale, and all N outputs of sampled rows, against the oracle.
+SWEEP_FULL = [("sweep_a", M) for M in (1, 64, 4096, 16384)] + [("sweep_b", M) for M in (1, 64, 4096, 16384)]
+
+
+@pytest.mark.parametrize("name,M", SWEEP_FULL)
+def test_sweep_full_size(name, M):
+    K = 4096 if name == "sweep_a" else 3072
+    G = K
+    w = wl.make(name, seed=2, M=M, G=G)
+    xd = dev_bf16(w.x_bits)
+    q, s = jq.jq_quantize_act(xd, G)
+    qw, sw = jq.jq_pack_weight(dev(w.w), G)
+    y = host_bits(jq.jq_w4a4_linear(q, s, qw, sw, None, G))
+    codes_a, s_a = oracle.quantize_bf16(w.x_bits, G)
+    assert np.array_equal(q.cpu().numpy(), oracle.pack(codes_a))
+    assert np.array_equal(s.cpu().numpy().view(np.uint32), s_a.view(np.uint32))
+    codes_w, s_w = oracle.quantize_f32(w.w, G)
+    assert np.array_equal(qw.cpu().numpy(), oracle.pack(codes_w))
+    assert np.array_equal(sw.cpu().numpy().view(np.uint32), np.ascontiguousarray(s_w.T).view(np.uint32))
+    rows = np.unique(np.array([0, 1, 127, 128, M // 2, M - 1]))
+    rows = rows[rows < M]
+    y64, _ = oracle.linear(codes_a[rows], s_a[rows], codes_w, s_w, None, G)
+    check_linear(y[rows], y64, oracle.group_partials(codes_a[rows], codes_w, G), s_a[rows], s_w, None,
+                 f"{name} M={M}")
