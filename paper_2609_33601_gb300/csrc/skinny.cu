@@ -75,6 +75,7 @@ static_assert(kRegsCtl<64> + 2 * kRegsUnpack + kRegsDrain<64> == 4 * kRegsLaunch
                   kRegsCtl<32> + 2 * kRegsUnpack + kRegsDrain<32> == 4 * kRegsLaunch,
               "register split must use the launch budget");
 constexpr int kMaxSplit = 8;
+constexpr int kMinSplitSlots = 6;  // K ring slots (two stages each) a CTA keeps at the least
 static_assert(kDrainWarp0 % 4 == 0, "drain warp w reads TMEM lanes 32 * (w % 4)");
 static_assert(kSkinnyMaxKOneGroup <= kOffsetMaxRun && kSkinnyMaxKOneGroup % kBK == 0, "exact one-group ranges");
 
@@ -927,9 +928,12 @@ cudaLaunchConfig_t make_config(int grid, int split, cudaStream_t stream, cudaLau
   return cfg;
 }
 
-// The split (CTAs per cluster) for `tiles` channel tiles: the largest one up to kMaxSplit, and
-// up to the K stages, for which every cluster is resident at once (one wave) and the CTAs do
-// not outnumber the SMs.  Cluster residency is asked of the runtime once per size.
+// The split (CTAs per cluster) for `tiles` channel tiles: the largest one up to kMaxSplit for
+// which every cluster is resident at once (one wave), the CTAs do not outnumber the SMs, and
+// every CTA keeps at least kMinSplitSlots ring slots of K: below that a CTA's fixed costs (setup,
+// first-byte latency, the cluster reduction) outweigh the bandwidth of the extra SMs (measured on
+// K=3072 -> N=3072, 24 tiles: split 2 beats 6 by 18 % at one token and 27 % at 64).  Cluster
+// residency is asked of the runtime once per size.
 template <int kMp>
 int choose_split(int tiles, int k_stages, int sms) {
   static int max_clusters[kMaxSplit + 1] = {0};
@@ -947,9 +951,10 @@ int choose_split(int tiles, int k_stages, int sms) {
       max_clusters[s] = n;
     }
   }
+  const int slots = (k_stages + kStPerSlot - 1) / kStPerSlot;
   int best = 1;
   for (int s = 2; s <= kMaxSplit && s <= k_stages; ++s)
-    if (tiles * s <= sms && tiles <= max_clusters[s]) best = s;
+    if (tiles * s <= sms && tiles <= max_clusters[s] && slots / s >= kMinSplitSlots) best = s;
   return best;
 }
 
