@@ -70,7 +70,7 @@ FP8_PER_BF16 = 2.0  # nominal dense FP8 / BF16 tensor-core ratio on GB300 (4.5 /
 # bench reports null.
 KERNEL_TRAFFIC = {
     ("dllm", "3e8612447b6fd805"): 31.244e6 + 0.119e6,  # profiles/w4a4_gemm_dllm_full.md
-    ("sweep_m1", "0d56d21f3b6ea46f"): 25.303e6,  # profiles/w4a4_skinny_sweep_m1_full.md
+    ("sweep_m1", "b21e1c671fb21de5"): 25.303e6,  # profiles/w4a4_skinny_sweep_m1_full.md
 }
 
 
