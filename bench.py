@@ -66,52 +66,26 @@ FP8_PER_BF16 = 2.0  # nominal dense FP8 / BF16 tensor-core ratio on GB300 (4.5 /
 
 # DRAM traffic of one launch of the dominant kernel (dram__bytes_read.sum + dram__bytes_write.sum)
 # from the ncu captures summarised in profiles/, keyed by workload and by the hash of the kernel
-# source the capture was taken on; once the kernel changes the figure no longer applies and the
-# bench reports null.
+# code the capture was taken on (kernel_hash); once the code changes the figure no longer applies
+# and the bench reports null.
 KERNEL_TRAFFIC = {
-    ("dllm", "3e8612447b6fd805"): 31.244e6 + 0.119e6,  # profiles/w4a4_gemm_dllm_full.md
-    ("sweep_m1", "b21e1c671fb21de5"): 25.303e6,  # profiles/w4a4_skinny_sweep_m1_full.md
+    ("dllm", "05e9b40bd0465fdd"): 31.244e6 + 0.119e6,  # profiles/w4a4_gemm_dllm_full.md
+    ("sweep_m1", "f3515f811b664b0e"): 25.303e6,  # profiles/w4a4_skinny_sweep_m1_full.md
 }
 
 
 def kernel_hash(kernel_file: str) -> str:
+    """Hash of a kernel's code (its .cu file and the two headers it is built from), comments and
+    whitespace removed, so that only a change of the code itself retires a traffic figure."""
+    import re
     h = hashlib.sha256()
     for f in (kernel_file, "operand.cuh", "ptx.cuh"):
-        with open(os.path.join(ROOT, "paper_2609_33601_gb300", "csrc", f), "rb") as fh:
-            h.update(fh.read())
+        with open(os.path.join(ROOT, "paper_2609_33601_gb300", "csrc", f)) as fh:
+            text = fh.read()
+        text = re.sub(r"/\*.*?\*/", " ", text, flags=re.S)  # block comments
+        text = re.sub(r"//[^\n]*", " ", text)                 # line comments
+        h.update(" ".join(text.split()).encode())
     return h.hexdigest()[:16]
-
-
-def max_over_ranks(values, device):
-    """Each timing's maximum over the ranks (one replica of the workload per rank): the
-    whole job is as slow as its slowest rank.  The identity on a single process."""
-    import torch
-    import torch.distributed as dist
-    if not (dist.is_available() and dist.is_initialized()) or dist.get_world_size() == 1:
-        return [float(v) for v in values]
-    t = torch.tensor([float(v) for v in values], dtype=torch.float64, device=device)
-    dist.all_reduce(t, op=dist.ReduceOp.MAX)
-    return [float(v) for v in t.cpu()]
-
-
-def whole_job_tops(world: int, ops_per_step: float, steps: int, seconds: float) -> float:
-    """Whole-job throughput of `world` replicas that each ran `steps` steps of `ops_per_step`
-    operations in at most `seconds` (the max over ranks)."""
-    return world * ops_per_step * steps / seconds / 1e12
-
-
-def metric_name(args) -> str:
-    return "W1.58A4 linear TOPS" if args.weights == "ternary" else "W4A4 linear TOPS"
-
-
-def launches_per_step(M: int, few: bool, fused: bool, ternary: bool) -> int:
-    """Kernels of this library per timed step: the activation quantiser (or, fused, the
-    quantise-to-operand kernel), the operand expansion when the linear kernel reads the operand
-    image (more than 16 tokens), the ternary -> INT4 rewrite (ternary weights, GEMM), and the
-    linear kernel itself."""
-    if fused:
-        return 2
-    return 1 + (1 if M > 16 else 0) + (1 if ternary and not few else 0) + 1
 
 
 def dist_env():

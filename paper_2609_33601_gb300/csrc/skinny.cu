@@ -27,16 +27,22 @@
 //   warps 0, 3  MMA issuers (one thread each) of the even / odd packed slots, each into its own
 //               accumulators: one issuing thread keeps the tensor core barely one MMA ahead, two
 //               keep it fed; 4 x (128 x Mp x 32) MMAs per K stage.  Warp 0 owns TMEM.
-//   warp 1      activation scales: s_a of every group into a ring for the drain
-//   warp 2      TMA producer (one thread): per two K stages, one box of 128 weight rows and one
-//               of the Mp token rows, 128 packed bytes each
+//   warp 1      activation scales: s_a of every group into a ring for the drain (with the
+//               corrections, when the tokens come pre-expanded); first, the final pass's
+//               per-token operands into shared memory
+//   warp 2      barrier setup, then TMA producer (one thread): it issues the first pass of
+//               weight boxes before the CTA-wide setup barrier; per two K stages, one box of 128
+//               weight rows (128 packed bytes of INT4 codes, or 64 of 2-bit ternary codes) and
+//               one of the Mp token rows (128 packed bytes), or, for more than 16 tokens, the
+//               tokens' pre-expanded operand bytes straight into the operand ring
 //   warps 4-11  unpack, two groups of four warps on alternate packed slots (two K stages each,
 //               so that one round of waits and fences covers 32 KB of weight operand): thread =
 //               weight row (TMEM lane), packed codes -> E4M3 operand bytes in the TMEM A ring;
-//               token rows -> E4M3 operand rows (128B swizzle) in shared memory, and each
-//               token group's exact code sum (8 * sum, for the drain)
+//               up to 16 tokens also the token rows -> E4M3 operand rows (128B swizzle) in
+//               shared memory, and each token group's exact code sum (for the drain)
 //   warps 12-15 drain: per group, tcgen05.ld 32x32b (thread = output channel, every token
-//               column), y[m] += (acc * s_w) * (s_a[m] * 2^18)
+//               column), y[m] += (acc * s_w) * (s_a[m] * 2^18); for one-group problems they
+//               unpack as a third group first
 // Every mbarrier wait is bounded; a timeout records a status and unwinds the CTA.
 #include <cfloat>
 #include <cstdint>
