@@ -88,6 +88,38 @@ def kernel_hash(kernel_file: str) -> str:
     return h.hexdigest()[:16]
 
 
+def max_over_ranks(values, device):
+    """Each timing's maximum over the ranks (one replica of the workload per rank): the
+    whole job is as slow as its slowest rank.  The identity on a single process."""
+    import torch
+    import torch.distributed as dist
+    if not (dist.is_available() and dist.is_initialized()) or dist.get_world_size() == 1:
+        return [float(v) for v in values]
+    t = torch.tensor([float(v) for v in values], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return [float(v) for v in t.cpu()]
+
+
+def whole_job_tops(world: int, ops_per_step: float, steps: int, seconds: float) -> float:
+    """Whole-job throughput of `world` replicas that each ran `steps` steps of `ops_per_step`
+    operations in at most `seconds` (the max over ranks)."""
+    return world * ops_per_step * steps / seconds / 1e12
+
+
+def metric_name(args) -> str:
+    return "W1.58A4 linear TOPS" if args.weights == "ternary" else "W4A4 linear TOPS"
+
+
+def launches_per_step(M: int, few: bool, fused: bool, ternary: bool) -> int:
+    """Kernels of this library per timed step: the activation quantiser (or, fused, the
+    quantise-to-operand kernel), the operand expansion when the linear kernel reads the operand
+    image (more than 16 tokens), the ternary -> INT4 rewrite (ternary weights, GEMM), and the
+    linear kernel itself."""
+    if fused:
+        return 2
+    return 1 + (1 if M > 16 else 0) + (1 if ternary and not few else 0) + 1
+
+
 def dist_env():
     rank = int(os.environ.get("RANK", "0"))
     world = int(os.environ.get("WORLD_SIZE", "1"))
