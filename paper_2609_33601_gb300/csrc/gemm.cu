@@ -21,10 +21,12 @@
 //   warp 1      TMEM owner; in the even CTA also the MMA issuer (one thread): 4 MMAs per K stage
 //               into one of two TMEM accumulators; a new accumulator starts at every group
 //               boundary and is handed to both CTAs' drain warps when the group ends
+//   warp 2      scale producer: weight (and activation) scales of 4 groups per TMA box into a
+//               ring for the drain
 //   warps 4-7   unpack: packed nibbles straight from global memory (two stages in flight in
 //               registers) -> E4M3 operand bytes in the 128B-swizzled K-major layout -> B ring
-//   warps 8-15  drain: per group, tcgen05.ld the partials (the load of the next 16 columns in
-//               flight while the previous 16 are scaled), y += (acc * s_w) * (s_a * 2^18) in fp32
+//   warps 8-15  drain: per group, the group's 36 scales from the ring, then 16 round trips of
+//               tcgen05.ld 16x256b (8 columns) and y += (acc * s_w) * (s_a * 2^18) in fp32
 //               registers (warp w owns TMEM lanes 32*(w%4).. and columns 128*((w-8)/4)..); after
 //               the last group, + bias, round to bf16, store
 // Every mbarrier wait is bounded; a timeout records a status and unwinds the CTA, and both CTAs
