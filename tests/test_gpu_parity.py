@@ -163,7 +163,12 @@ def run_linear(ref: Reference, x_bits, fused: bool):
                                           (300, 520, 512, 512, True), (64, 256, 256, 64, True),
                                           (1, 8, 128, 128, True), (129, 8, 256, 64, False),
                                           (17, 264, 1024, 128, True), (40, 520, 512, 512, False),
-                                          (64, 136, 2048, 2048, True), (33, 264, 768, 64, False)])
+                                          (64, 136, 2048, 2048, True), (33, 264, 768, 64, False),
+                                          # an odd number of 128-deep K stages (the ring's last slot
+                                          # holds one stage): DiT-XL/2's hidden size 1152 = 9 x 128
+                                          (300, 264, 384, 64, True), (300, 264, 384, 128, False),
+                                          (300, 264, 384, 384, True), (257, 520, 1152, 128, True),
+                                          (257, 136, 1152, 1152, False), (40, 264, 1152, 128, True)])
 def test_linear_matches_oracle(M, N, K, G, bias):
     w = wl.make("custom", seed=11 + M, M=M, K=K, N=N, G=G, bias=bias)
     x = act_bits(M, K, seed=3 + M, extreme=False) if M >= 8 else w.x_bits
