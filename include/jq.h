@@ -36,6 +36,11 @@
  *     crosses the ABI.
  *   - Every on-GPU wait is bounded (about a second).  A kernel that gives up records
  *     JQ_ERR_TIMEOUT in a device status word read by jq_device_status().
+ *   - Kernels are launched with programmatic dependent launch: one of this library's kernels may
+ *     start while the previous kernel on the stream is still running, when that kernel is also
+ *     one of this library's (the linear layers start streaming their weights early), and waits
+ *     for it before touching any data it writes or reads.  Stream order holds for all data;
+ *     other kernels on the stream, yours included, order with these as with any kernel.
  */
 #ifndef JQ_H
 #define JQ_H
