@@ -13,6 +13,11 @@ numpy arrays through ctypes.  Layout conventions used here:
   (byte layout in ``jq_oracle.c``);
 * activation scales ``s_a``: ``float32 [M, K/G]``;
 * weight scales ``s_w``: ``float32 [N, K/G]`` (per output channel);
+* NVFP4 (E2M1 elements, E4M3 block scales per 16 along K, one fp32 tensor
+  scale): element codes as ``int8`` holding twice the E2M1 value (integers in
+  [-12, 12]); block scales ``float32 [rows, K/16]`` (each an E4M3 value);
+  packed ``uint8 [rows, K/2]`` in the 4-bit E2M1 encoding, element 2j in the
+  low nibble;
 * bf16 values travel as their ``uint16`` bit patterns.
 """
 from __future__ import annotations
@@ -61,9 +66,17 @@ def _load():
             lib.oracle_unpack.argtypes = [vp, i64, i64, vp]
             lib.oracle_group_partials.argtypes = [vp, vp, i64, i64, i64, i64, vp]
             lib.oracle_linear.argtypes = [vp, vp, vp, vp, vp, i64, i64, i64, i64, vp, vp]
+            f32 = ctypes.c_float
+            lib.oracle_nvfp4_tensor_scale.argtypes = [vp, i64]
+            lib.oracle_nvfp4_tensor_scale.restype = f32
+            lib.oracle_quantize_nvfp4.argtypes = [vp, i64, i64, f32, vp, vp]
+            lib.oracle_pack_nvfp4.argtypes = [vp, i64, i64, vp]
+            lib.oracle_unpack_nvfp4.argtypes = [vp, i64, i64, vp]
+            lib.oracle_linear_nvfp4.argtypes = [vp, vp, f32, vp, vp, f32, vp, i64, i64, i64, vp, vp]
             for f in ("oracle_quantize_bf16", "oracle_quantize_f32", "oracle_pack", "oracle_unpack",
                       "oracle_group_partials", "oracle_linear", "oracle_quantize_ternary_f32",
-                      "oracle_pack_ternary", "oracle_unpack_ternary"):
+                      "oracle_pack_ternary", "oracle_unpack_ternary", "oracle_quantize_nvfp4",
+                      "oracle_pack_nvfp4", "oracle_unpack_nvfp4", "oracle_linear_nvfp4"):
                 getattr(lib, f).restype = None
             _lib = lib
     return _lib
@@ -176,4 +189,54 @@ def linear(qa, s_a, qw, s_w, bias, group: int):
     y64 = np.empty((M, N), np.float64)
     yb = np.empty((M, N), np.uint16)
     _load().oracle_linear(_p(qa), _p(s_a), _p(qw), _p(s_w), _p(b), M, N, K, group, _p(y64), _p(yb))
+    return y64, yb
+
+
+def nvfp4_tensor_scale(x: np.ndarray) -> float:
+    """fp32 per-tensor NVFP4 scale fl32(amax |x| / 2688) (2688 = 6 * 448)."""
+    x = _c(x, np.float32)
+    return float(_load().oracle_nvfp4_tensor_scale(_p(x), x.size))
+
+
+def quantize_nvfp4(x: np.ndarray, g: float):
+    """fp32 [rows, K] (K % 16 == 0), tensor scale g -> (2q int8 [rows,K], E4M3 block scales f32 [rows,K/16])."""
+    x = _c(x, np.float32)
+    R, K = x.shape
+    assert K % 16 == 0
+    codes2 = np.empty((R, K), np.int8)
+    scales = np.empty((R, K // 16), np.float32)
+    _load().oracle_quantize_nvfp4(_p(x), R, K, ctypes.c_float(g), _p(codes2), _p(scales))
+    return codes2, scales
+
+
+def pack_nvfp4(codes2: np.ndarray) -> np.ndarray:
+    codes2 = _c(codes2, np.int8)
+    R, K = codes2.shape
+    assert K % 2 == 0
+    assert np.isin(np.abs(codes2.astype(np.int16)), [0, 1, 2, 3, 4, 6, 8, 12]).all()
+    out = np.empty((R, K // 2), np.uint8)
+    _load().oracle_pack_nvfp4(_p(codes2), R, K, _p(out))
+    return out
+
+
+def unpack_nvfp4(packed: np.ndarray) -> np.ndarray:
+    packed = _c(packed, np.uint8)
+    R, H = packed.shape
+    out = np.empty((R, 2 * H), np.int8)
+    _load().oracle_unpack_nvfp4(_p(packed), R, 2 * H, _p(out))
+    return out
+
+
+def linear_nvfp4(qa2, sa, ga: float, qw2, sw, gw: float, bias):
+    """(y64 float64 [M,N], y_bf16 uint16 [M,N]) of the NVFP4 linear layer (block scales per 16 along K)."""
+    qa2, qw2 = _c(qa2, np.int8), _c(qw2, np.int8)
+    sa, sw = _c(sa, np.float32), _c(sw, np.float32)
+    M, K = qa2.shape
+    N = qw2.shape[0]
+    assert K % 16 == 0 and sa.shape == (M, K // 16) and sw.shape == (N, K // 16)
+    b = None if bias is None else _c(bias, np.float32)
+    y64 = np.empty((M, N), np.float64)
+    yb = np.empty((M, N), np.uint16)
+    _load().oracle_linear_nvfp4(_p(qa2), _p(sa), ctypes.c_float(ga), _p(qw2), _p(sw), ctypes.c_float(gw),
+                                _p(b), M, N, K, _p(y64), _p(yb))
     return y64, yb

@@ -232,6 +232,145 @@ void oracle_unpack_ternary(const uint8_t* packed, int64_t rows, int64_t K, int8_
     }
 }
 
+/* ---- NVFP4 (the LLaDA-8B W4A4 format) ---------------------------------- */
+
+/*
+ * The paper runs LLaDA-8B as "NVFP4 W4A4" (Appendix table "ELF-B and LLaDA-8B experimental
+ * details") and prints no definition of the format.  The reading used here is the published
+ * NVFP4 format: elements in FP4 E2M1 (magnitudes 0, 0.5, 1, 1.5, 2, 3, 4, 6), one FP8 E4M3 scale
+ * per block of 16 consecutive reduction-axis elements of a row, and one fp32 scale g per
+ * tensor.  For weights g = fl32(amax |w| / 2688) (2688 = 6 * 448: the block holding the tensor's
+ * largest magnitude gets the largest E4M3 scale); for activations g is a calibrated constant the
+ * caller supplies.  Per block b of a row:
+ *     s_b = e4m3(fl32(amax_b / fl32(6 * g)))   (nearest, ties to even mantissa, saturating at 448)
+ *     S_b = fl32(s_b * g)
+ *     q   = e2m1(fl32(x / S_b))               (nearest, ties to even mantissa, saturating at 6)
+ * and q = 0 wherever g == 0 or S_b == 0.  The codes are kept here as 2q (integers in [-12, 12]).
+ * The linear layer: y = sum_b (sum_{k in b} qa * qw) * sa_b * sw_b * ga * gw + bias, in fp64.
+ */
+
+/* Nearest E2M1 magnitude to a (finite, >= 0), ties to the even mantissa, saturating at 6;
+ * returned doubled (an integer in {0, 1, 2, 3, 4, 6, 8, 12}). */
+static int e2m1_twice(double a) {
+  static const double grid[8] = {0.0, 0.5, 1.0, 1.5, 2.0, 3.0, 4.0, 6.0};
+  static const int even[8] = {1, 0, 1, 0, 1, 0, 1, 0}; /* mantissa bit 0 */
+  if (a >= 6.0) return 12;
+  for (int i = 0; i < 7; ++i) {
+    if (a <= grid[i + 1]) {
+      const double dlo = a - grid[i], dhi = grid[i + 1] - a; /* exact: a is an fp32 value */
+      const int pick = dlo < dhi ? i : (dhi < dlo ? i + 1 : (even[i] ? i : i + 1));
+      return (int)(2.0 * grid[pick]);
+    }
+  }
+  return 12;
+}
+
+/* Nearest E4M3 value to a (finite, >= 0): 3 mantissa bits, exponent bias 7, normals down to
+ * 2^-6, subnormals in steps of 2^-9, ties to even, saturating at the largest finite 448. */
+static float e4m3_round(float a) {
+  if (a == 0.0f) return 0.0f;
+  int e;
+  (void)frexp((double)a, &e);     /* a in [2^(e-1), 2^e) */
+  int q_exp = (e - 1) - 3;        /* 3 mantissa bits */
+  if (q_exp < -9) q_exp = -9;     /* subnormal quantum */
+  const double n = rint(ldexp((double)a, -q_exp)); /* exact scaling; ties to even */
+  double r = ldexp(n, q_exp);
+  if (r > 448.0) r = 448.0;
+  return (float)r;
+}
+
+float oracle_nvfp4_tensor_scale(const float* x, int64_t n) {
+  float amax = 0.0f;
+  for (int64_t i = 0; i < n; ++i) {
+    const float a = fabsf(x[i]);
+    if (a > amax) amax = a;
+  }
+  return amax / 2688.0f;
+}
+
+void oracle_quantize_nvfp4(const float* x, int64_t rows, int64_t K, float g, int8_t* codes2,
+                           float* block_scales) {
+  const int64_t nb = K / 16;
+#pragma omp parallel for schedule(static)
+  for (int64_t r = 0; r < rows; ++r) {
+    for (int64_t b = 0; b < nb; ++b) {
+      const float* xb = x + r * K + b * 16;
+      float amax = 0.0f;
+      for (int k = 0; k < 16; ++k) {
+        const float a = fabsf(xb[k]);
+        if (a > amax) amax = a;
+      }
+      float s = 0.0f, S = 0.0f;
+      if (g != 0.0f) {
+        const float six_g = 6.0f * g;
+        s = e4m3_round(amax / six_g);
+        S = s * g;
+      }
+      block_scales[r * nb + b] = s;
+      for (int k = 0; k < 16; ++k) {
+        int q2 = 0;
+        if (S != 0.0f) {
+          const float t = xb[k] / S;  /* IEEE single division */
+          q2 = e2m1_twice(fabs((double)t));
+          if (t < 0.0f) q2 = -q2;
+        }
+        codes2[r * K + b * 16 + k] = (int8_t)q2;
+      }
+    }
+  }
+}
+
+/* Packing: E2M1 codes (bit 3 sign, bits 1-2 exponent, bit 0 mantissa), two per byte, element 2j
+ * in the low nibble of byte j.  Magnitude codes: 0 -> 0, 0.5 -> 1, 1 -> 2, 1.5 -> 3, 2 -> 4,
+ * 3 -> 5, 4 -> 6, 6 -> 7 (the code is the magnitude's index in that list). */
+static int e2m1_code(int q2) {
+  static const int twice[8] = {0, 1, 2, 3, 4, 6, 8, 12};
+  const int m = q2 < 0 ? -q2 : q2;
+  for (int i = 0; i < 8; ++i)
+    if (twice[i] == m) return (q2 < 0 ? 8 : 0) | i;
+  return -1;
+}
+
+void oracle_pack_nvfp4(const int8_t* codes2, int64_t rows, int64_t K, uint8_t* packed) {
+  for (int64_t r = 0; r < rows; ++r)
+    for (int64_t j = 0; j < K / 2; ++j)
+      packed[r * (K / 2) + j] =
+          (uint8_t)(e2m1_code(codes2[r * K + 2 * j]) | (e2m1_code(codes2[r * K + 2 * j + 1]) << 4));
+}
+
+void oracle_unpack_nvfp4(const uint8_t* packed, int64_t rows, int64_t K, int8_t* codes2) {
+  static const int twice[8] = {0, 1, 2, 3, 4, 6, 8, 12};
+  for (int64_t r = 0; r < rows; ++r)
+    for (int64_t j = 0; j < K / 2; ++j) {
+      const int b = packed[r * (K / 2) + j];
+      const int lo = b & 15, hi = b >> 4;
+      codes2[r * K + 2 * j] = (int8_t)((lo & 8) ? -twice[lo & 7] : twice[lo & 7]);
+      codes2[r * K + 2 * j + 1] = (int8_t)((hi & 8) ? -twice[hi & 7] : twice[hi & 7]);
+    }
+}
+
+/* y64[m, n] = sum_b acc4[m,n,b] / 4 * sa[m,b] * sw[n,b] * ga * gw + bias[n], in fp64, with
+ * acc4 = sum over the block of (2 qa) * (2 qw), an exact integer; ybf16 = its bf16 rounding. */
+void oracle_linear_nvfp4(const int8_t* qa2, const float* sa, float ga, const int8_t* qw2, const float* sw,
+                         float gw, const float* bias, int64_t M, int64_t N, int64_t K, double* y64,
+                         uint16_t* ybf16) {
+  const int64_t nb = K / 16;
+#pragma omp parallel for schedule(static)
+  for (int64_t m = 0; m < M; ++m)
+    for (int64_t n = 0; n < N; ++n) {
+      double y = 0.0;
+      for (int64_t b = 0; b < nb; ++b) {
+        int32_t acc4 = 0;
+        for (int k = 0; k < 16; ++k)
+          acc4 += (int32_t)qa2[m * K + b * 16 + k] * (int32_t)qw2[n * K + b * 16 + k];
+        y += (double)acc4 / 4.0 * (double)sa[m * nb + b] * (double)sw[n * nb + b];
+      }
+      y = y * (double)ga * (double)gw + (bias ? (double)bias[n] : 0.0);
+      y64[m * N + n] = y;
+      ybf16[m * N + n] = oracle_bf16_rne(y);
+    }
+}
+
 /* ---- integer GEMM and the dequantising epilogue ------------------------- */
 
 /* acc[m, n, g] = sum over the G elements of group g of qa[m,k] * qw[n,k]. */

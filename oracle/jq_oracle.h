@@ -17,6 +17,14 @@ void oracle_quantize_ternary_f32(const float* w, int64_t N, int64_t K, int64_t G
                                  float* scales);
 void oracle_pack_ternary(const int8_t* codes, int64_t rows, int64_t K, uint8_t* packed);
 void oracle_unpack_ternary(const uint8_t* packed, int64_t rows, int64_t K, int8_t* codes);
+float oracle_nvfp4_tensor_scale(const float* x, int64_t n);
+void oracle_quantize_nvfp4(const float* x, int64_t rows, int64_t K, float g, int8_t* codes2,
+                           float* block_scales);
+void oracle_pack_nvfp4(const int8_t* codes2, int64_t rows, int64_t K, uint8_t* packed);
+void oracle_unpack_nvfp4(const uint8_t* packed, int64_t rows, int64_t K, int8_t* codes2);
+void oracle_linear_nvfp4(const int8_t* qa2, const float* sa, float ga, const int8_t* qw2, const float* sw,
+                         float gw, const float* bias, int64_t M, int64_t N, int64_t K, double* y64,
+                         uint16_t* ybf16);
 void oracle_group_partials(const int8_t* qa, const int8_t* qw, int64_t M, int64_t N, int64_t K,
                            int64_t G, int32_t* acc);
 void oracle_linear(const int8_t* qa, const float* s_a, const int8_t* qw, const float* s_w,
