@@ -76,7 +76,8 @@ JQ_API const char* jq_status_string(jq_status s);
  *   x_bf16 : bf16 [M, ldx] (the first K columns are used), ldx >= K, ldx*2 % 16 == 0
  *   q      : uint8 [M, K/2] packed codes (output)
  *   s_a    : fp32 [M, K/group] scales (output)
- * Errors: JQ_ERR_INVALID_ARG (null, K/group unsupported, ldx < K), JQ_ERR_MISALIGNED.
+ * Errors: JQ_ERR_INVALID_ARG (null, K/group unsupported, ldx < K), JQ_ERR_MISALIGNED,
+ * JQ_ERR_UNSUPPORTED (the current device is not sm_103), JQ_ERR_CUDA (the launch failed).
  */
 JQ_API jq_status jq_quantize_act(const void* x_bf16, int64_t M, int64_t K, int64_t ldx, int32_t group,
                           uint8_t* q, float* s_a, void* stream);
@@ -107,7 +108,7 @@ JQ_API size_t jq_workspace_size(int64_t M, int64_t N, int64_t K, int32_t group, 
  *   bias      : fp32 [N] or NULL
  *   y_bf16    : bf16 [M, N] (output)
  *   workspace : >= jq_workspace_size(M, N, K, group, 0) bytes of device memory, 16-byte aligned
- * Errors: JQ_ERR_INVALID_ARG, JQ_ERR_MISALIGNED, JQ_ERR_WORKSPACE, JQ_ERR_CUDA.
+ * Errors: JQ_ERR_INVALID_ARG, JQ_ERR_MISALIGNED, JQ_ERR_WORKSPACE, JQ_ERR_UNSUPPORTED, JQ_ERR_CUDA.
  */
 JQ_API jq_status jq_w4a4_linear(const uint8_t* q, const float* s_a, const uint8_t* qw, const float* s_w,
                          const float* bias, void* y_bf16, int64_t M, int64_t N, int64_t K, int32_t group,
