@@ -6,6 +6,7 @@ from __future__ import annotations
 
 import concurrent.futures as cf
 import os
+import platform
 import shutil
 import subprocess
 import sys
@@ -42,9 +43,23 @@ def _stale(target: str, deps: list[str]) -> bool:
     return any(os.path.getmtime(d) > t for d in deps)
 
 
+STAMP = os.path.join(BUILD, "host.txt")  # host architecture the objects in _build were built on
+
+
+def _host_changed() -> bool:
+    """True unless the objects in _build were compiled on this host architecture (a tree copied
+    between an x86 and an Arm machine keeps newer-looking objects that cannot link)."""
+    try:
+        with open(STAMP) as f:
+            return f.read().strip() != platform.machine()
+    except OSError:
+        return True
+
+
 def build(force: bool = False, verbose: bool = False) -> str:
     nvcc = _nvcc()
     os.makedirs(BUILD, exist_ok=True)
+    force = _host_changed() or force
     hdrs = [os.path.join(CSRC, h) for h in HEADERS] + [os.path.join(INCLUDE, "jq.h")]
     jobs = []
     objs = []
@@ -68,6 +83,8 @@ def build(force: bool = False, verbose: bool = False) -> str:
         tmp = LIB + f".tmp{os.getpid()}"
         run([nvcc, "-gencode", "arch=compute_103a,code=sm_103a", "-shared", "-o", tmp, *objs])
         os.replace(tmp, LIB)
+    with open(STAMP, "w") as f:  # only after every object and the library built here
+        f.write(platform.machine() + "\n")
     return LIB
 
 
