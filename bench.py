@@ -199,6 +199,7 @@ class OracleSample:
         quant = oracle.quantize_ternary_f32 if ternary else oracle.quantize_f32
         self.qw, self.sw = quant(w.w, self.G)
         self.rows = 8
+        self.run_s = 0.0
 
     def run(self, rows: int) -> float:
         t0 = time.perf_counter()
@@ -216,14 +217,32 @@ class OracleSample:
         self.rows = rows
         return rows
 
-    def ops(self) -> float:
-        return 2.0 * self.rows * self.N * self.K
+    def ops(self, rows: int | None = None) -> float:
+        return 2.0 * (self.rows if rows is None else rows) * self.N * self.K
 
-    def describe(self, dt: float) -> dict:
-        cores = int(os.environ.get("OMP_NUM_THREADS", os.cpu_count() or 1))
-        return {"value": self.ops() / dt / 1e12, "unit": "TOPS", "cores": min(cores, self.rows), "kind": "oracle",
-                "sample": f"{self.rows} of {self.M} token rows of the {self.name} workload (all N={self.N} "
-                          f"outputs), quantise + linear, {dt:.2f} s per sample"}
+    def single_thread(self, target_s: float) -> dict:
+        """The same oracle on one host thread, on a row sample sized for about target_s."""
+        threads = self.oracle.max_threads()
+        self.oracle.set_threads(1)
+        try:
+            used = min(threads, self.rows)  # the all-cores sample ran on this many threads
+            rows = max(1, min(self.rows, int(self.rows * target_s / max(self.run_s * used, 1e-3))))
+            dt = self.run(rows)
+        finally:
+            self.oracle.set_threads(threads)
+        return {"value": self.ops(rows) / dt / 1e12, "cores": 1,
+                "sample": f"{rows} token rows, {dt:.2f} s"}
+
+    def describe(self, dt: float, single_s: float = 0.0) -> dict:
+        self.run_s = dt
+        cores = self.oracle.max_threads()
+        out = {"value": self.ops() / dt / 1e12, "unit": "TOPS", "cores": min(cores, self.rows), "kind": "oracle",
+               "host_threads": os.cpu_count(),
+               "sample": f"{self.rows} of {self.M} token rows of the {self.name} workload (all N={self.N} "
+                         f"outputs), quantise + linear, {dt:.2f} s per sample"}
+        if single_s > 0:
+            out["single_thread"] = self.single_thread(single_s)
+        return out
 
 
 def run_reference(args):
@@ -237,7 +256,7 @@ def run_reference(args):
         o.run(o.rows)
     times = [o.run(o.rows) for _ in range(args.steps)]
     mean = sum(times) / len(times)
-    cb = o.describe(mean)
+    cb = o.describe(mean, single_s=args.ref_single_seconds)
     value = cb["value"]
     line = {"impl": "reference", "metric": metric_name(args), "value": value, "unit": "TOPS", "n_gpus": args.gpus,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": mean * 1e3, "higher_is_better": True,
@@ -501,7 +520,7 @@ def run_ours(args):
     if world == 1 and not args.no_cpu_baseline:
         o = OracleSample(args.workload, ternary=ternary)
         o.calibrate(args.ref_seconds)
-        cpu = o.describe(o.run(o.rows))
+        cpu = o.describe(o.run(o.rows), single_s=args.ref_single_seconds)
     line = {
         "metric": metric_name(args), "value": value, "unit": "TOPS", "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": total_ms / args.steps, "higher_is_better": True, "scaling": "weak",
@@ -538,6 +557,8 @@ def main():
     ap.add_argument("--workload", choices=sorted(WORKLOADS), default="dllm")
     ap.add_argument("--sets", type=int, default=0, help="rotating input/weight sets (0: enough for > 3x L2)")
     ap.add_argument("--ref-seconds", type=float, default=10.0, help="CPU seconds per oracle sample")
+    ap.add_argument("--ref-single-seconds", type=float, default=5.0,
+                    help="CPU seconds for the oracle's single-thread sample (0: skip it)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--fused", action="store_true", help="time jq_fused_quant_linear (bf16 activations in)")
     ap.add_argument("--weights", choices=["int4", "ternary"], default="int4",

@@ -67,6 +67,10 @@ def _load():
             lib.oracle_group_partials.argtypes = [vp, vp, i64, i64, i64, i64, vp]
             lib.oracle_linear.argtypes = [vp, vp, vp, vp, vp, i64, i64, i64, i64, vp, vp]
             f32 = ctypes.c_float
+            lib.oracle_set_threads.argtypes = [ctypes.c_int]
+            lib.oracle_set_threads.restype = None
+            lib.oracle_max_threads.argtypes = []
+            lib.oracle_max_threads.restype = ctypes.c_int
             lib.oracle_nvfp4_tensor_scale.argtypes = [vp, i64]
             lib.oracle_nvfp4_tensor_scale.restype = f32
             lib.oracle_quantize_nvfp4.argtypes = [vp, i64, i64, f32, vp, vp]
@@ -88,6 +92,15 @@ def _p(a):
 
 def _c(a, dtype):
     return np.ascontiguousarray(a, dtype=dtype)
+
+
+def set_threads(n: int) -> None:
+    """OpenMP threads for the oracle's row-parallel loops (results do not depend on it)."""
+    _load().oracle_set_threads(int(n))
+
+
+def max_threads() -> int:
+    return int(_load().oracle_max_threads())
 
 
 def bf16_rne(v: float) -> int:

@@ -39,6 +39,13 @@
 
 #include "jq_oracle.h"
 
+#include <omp.h>
+
+/* Thread control for the timed CPU baseline (no effect on any result: every parallel loop
+ * here splits independent rows, each computed in one fixed order). */
+void oracle_set_threads(int n) { omp_set_num_threads(n > 0 ? n : 1); }
+int oracle_max_threads(void) { return omp_get_max_threads(); }
+
 /* ---- bf16 helpers ------------------------------------------------------ */
 
 /* bf16 -> fp32 is exact: a bf16 is the top half of an fp32. */

@@ -17,6 +17,8 @@ void oracle_quantize_ternary_f32(const float* w, int64_t N, int64_t K, int64_t G
                                  float* scales);
 void oracle_pack_ternary(const int8_t* codes, int64_t rows, int64_t K, uint8_t* packed);
 void oracle_unpack_ternary(const uint8_t* packed, int64_t rows, int64_t K, int8_t* codes);
+void oracle_set_threads(int n);
+int oracle_max_threads(void);
 float oracle_nvfp4_tensor_scale(const float* x, int64_t n);
 void oracle_quantize_nvfp4(const float* x, int64_t rows, int64_t K, float g, int8_t* codes2,
                            float* block_scales);

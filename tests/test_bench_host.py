@@ -1,5 +1,6 @@
 """Host-side logic of bench.py that needs no GPU: the kernel code hash that keys the recorded
-DRAM traffic, the count of this library's kernels per timed step, and the metric names."""
+DRAM traffic, the count of this library's kernels per timed step, the metric names, and the
+CPU-oracle baseline (all-cores and single-thread samples)."""
 import os
 import shutil
 
@@ -51,3 +52,37 @@ def test_metric_names():
     assert bench.metric_name(A) == "W4A4 linear TOPS"
     A.weights = "ternary"
     assert bench.metric_name(A) == "W1.58A4 linear TOPS"
+
+
+def test_oracle_results_do_not_depend_on_its_thread_count():
+    import numpy as np
+    import oracle
+    from paper_2609_33601_gb300 import workloads as wl
+    w = wl.make("tiny", seed=3)
+    qw, sw = oracle.quantize_f32(w.w, w.G)
+    threads = oracle.max_threads()
+    outs = []
+    try:
+        for n in (1, 3, max(threads, 2)):
+            oracle.set_threads(n)
+            qa, sa = oracle.quantize_bf16(w.x_bits, w.G)
+            outs.append((qa, sa) + oracle.linear(qa, sa, qw, sw, w.bias, w.G))
+    finally:
+        oracle.set_threads(threads)
+    assert oracle.max_threads() == threads
+    for o in outs[1:]:
+        assert all(np.array_equal(a, b) for a, b in zip(outs[0], o))
+
+
+def test_cpu_baseline_reports_an_all_cores_and_a_single_thread_sample(monkeypatch):
+    import oracle
+    monkeypatch.setitem(bench.WORKLOADS, "tiny", ("tiny: 64 x 256 -> 256, group64", 64, 256, 256, 64, "tiny"))
+    threads = oracle.max_threads()
+    o = bench.OracleSample("tiny")
+    o.calibrate(0.05)
+    cb = o.describe(o.run(o.rows), single_s=0.02)
+    assert cb["kind"] == "oracle" and cb["value"] > 0 and 1 <= cb["cores"] <= threads
+    st = cb["single_thread"]
+    assert st["cores"] == 1 and st["value"] > 0
+    assert oracle.max_threads() == threads  # restored
+    assert "single_thread" not in o.describe(o.run(o.rows))
