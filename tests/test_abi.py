@@ -143,3 +143,43 @@ def test_w158a4_entry_points(lib):
     assert L(A, A, odd, A, None, A, 4, 16, 256, 64, A, big, None) == MISALIGNED
     assert L(A, A, A, A, None, A, 100, 16, 256, 64, A, 16, None) == WORKSPACE
     assert L(A, A, A, A, None, A, 0, 16, 256, 64, None, 0, None) == OK
+
+
+C_CLIENT = r"""
+#include <stdio.h>
+#include <string.h>
+#include "jq.h"
+
+int main(void) {
+  int bad = 0;
+  if (strcmp(jq_status_string(JQ_ERR_WORKSPACE), "JQ_ERR_WORKSPACE") != 0) bad |= 1;
+  if (jq_workspace_size(1024, 12288, 4096, 128, 0) != (size_t)1024 * 4096 + 1024 * 32 * 4) bad |= 2;
+  /* argument checks run before any device is touched */
+  if (jq_w4a4_linear(NULL, NULL, NULL, NULL, NULL, NULL, 16, 256, 4096, 128, NULL, 0, NULL) != JQ_ERR_INVALID_ARG)
+    bad |= 4;
+  if (jq_quantize_act(NULL, 4, 100, 100, 64, NULL, NULL, NULL) != JQ_ERR_INVALID_ARG) bad |= 8;
+  if (jq_w4a4_linear(NULL, NULL, NULL, NULL, NULL, NULL, 0, 256, 4096, 128, NULL, 0, NULL) != JQ_OK) bad |= 16;
+  printf("%d\n", bad);
+  return bad;
+}
+"""
+
+
+def test_header_is_plain_c_and_links_from_a_c_program(lib, tmp_path):
+    """A C99 client compiled with gcc -pedantic -Werror against include/jq.h links to libjq.so
+    and gets the documented answers from calls that need no GPU."""
+    import shutil
+    import subprocess
+    gcc = shutil.which("gcc")
+    if gcc is None:
+        pytest.skip("gcc not available")
+    from paper_2609_33601_gb300 import build
+    libpath = build.build()
+    src = tmp_path / "client.c"
+    src.write_text(C_CLIENT)
+    exe = tmp_path / "client"
+    subprocess.run([gcc, "-std=c99", "-pedantic", "-Wall", "-Wextra", "-Werror", "-I", os.path.dirname(HEADER),
+                    str(src), "-o", str(exe), libpath, f"-Wl,-rpath,{os.path.dirname(libpath)}"],
+                   check=True, capture_output=True, text=True)
+    r = subprocess.run([str(exe)], capture_output=True, text=True, timeout=60)
+    assert r.returncode == 0 and r.stdout.strip() == "0", (r.returncode, r.stdout, r.stderr)
