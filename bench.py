@@ -69,7 +69,7 @@ FP8_PER_BF16 = 2.0  # nominal dense FP8 / BF16 tensor-core ratio on GB300 (4.5 /
 # code the capture was taken on (kernel_hash); once the code changes the figure no longer applies
 # and the bench reports null.
 KERNEL_TRAFFIC = {
-    ("dllm", "a97dcf2dca3eeebe"): 31.244e6 + 0.119e6,  # profiles/w4a4_gemm_dllm_full.md
+    ("dllm", "c9988b74e5543425"): 31.244e6 + 0.119e6,  # profiles/w4a4_gemm_dllm_full.md
     ("sweep_m1", "20541bf7a20396bf"): 25.303e6,  # profiles/w4a4_skinny_sweep_m1_full.md
 }
 

@@ -793,7 +793,10 @@ bool encode_2d(CUtensorMap* map, CUtensorMapDataType dtype, const void* base, ui
 
 cudaError_t launch_w4a4_gemm(const GemmProblem& p, cudaStream_t stream, int sms) {
   if (p.M == 0 || p.N == 0) return cudaSuccess;
-  const bool offset = p.G == p.K;  // one group: offset-code weights (see w4a4_gemm_kernel)
+  // One group: offset-code weights (see w4a4_gemm_kernel), exact while the whole K run fits the
+  // offset form's fp32 range (operand.cuh); longer one-group runs keep the sign-magnitude form,
+  // whose sums stay below 2^24 for every K the library accepts.
+  const bool offset = p.G == p.K && p.K <= kOffsetMaxRun;
   if (p.partials != nullptr)
     return offset ? launch_impl<true, true>(p, stream, sms) : launch_impl<true, false>(p, stream, sms);
   return offset ? launch_impl<false, true>(p, stream, sms) : launch_impl<false, false>(p, stream, sms);

@@ -82,9 +82,10 @@ cudaError_t launch_w4a4_gemm(const GemmProblem& p, cudaStream_t stream, int sms)
 
 // Few-token linear layer (skinny.cu): reads the packed activation codes directly and needs no
 // scratch, or, when the caller sets a_image / corr (jq_w4a4_linear does for M > 16), takes the
-// tokens pre-expanded from the caller's workspace.  Used for M <= kSkinnyMaxM.  With one group (G = K) a CTA accumulates offset-code
-// products over its whole K range in fp32, exact while 120 * K < 2^24 (operand.cuh): larger
-// one-group problems take the GEMM.
+// tokens pre-expanded from the caller's workspace.  Used for M <= kSkinnyMaxM.  With one group
+// (G = K) a CTA accumulates offset-code products over its whole K range in fp32, exact while
+// 120 * K < 2^24 (operand.cuh): larger one-group problems take the GEMM, which keeps
+// sign-magnitude weights for them.
 constexpr int kSkinnyMaxM = 64;
 constexpr int kSkinnyMaxKOneGroup = 139776;  // 1092 * 128
 inline bool skinny_supports(int64_t M, int64_t K, int32_t G) {

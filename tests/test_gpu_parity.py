@@ -229,6 +229,29 @@ def test_large_partial_sums_cancel(M, K, G):
     check_linear(host_bits(y), y64, oracle.group_partials(qa, qw, G), sa, sw, None)
 
 
+@pytest.mark.parametrize("M", [16, 200])
+def test_one_group_at_the_largest_k(M):
+    """G = K at the largest K the library accepts, 262016 (2047 K stages of 128, an odd count).
+
+    Codes in [4, 7] on both sides: the exact partial stays below 49 K < 2^24, but a sum of
+    offset-code products (q_w + 8) q_a would climb to about 74 K > 2^24, where fp32 drops odd
+    integers, so a run this long must keep the sign-magnitude form.  Both M take the GEMM (the
+    few-token kernel takes one group only up to K = 139776)."""
+    K, N = 262016, 136
+    rng = np.random.default_rng(M + 5)
+    qa = rng.integers(4, 8, (M, K), dtype=np.int8)
+    qw = rng.integers(4, 8, (N, K), dtype=np.int8)
+    ref = oracle.group_partials(qa, qw, K)
+    pa, pw = dev(oracle.pack(qa)), dev(oracle.pack(qw))
+    acc = jq.jq_w4a4_group_partials(pa, pw, K)
+    assert np.array_equal(acc.cpu().numpy(), ref)
+    sa = np.ones((M, 1), np.float32)
+    sw = np.ones((N, 1), np.float32)
+    y64, _ = oracle.linear(qa, sa, qw, sw, None, K)
+    y = jq.jq_w4a4_linear(pa, dev(sa), pw, dev(np.ascontiguousarray(sw.T)), None, K)
+    check_linear(host_bits(y), y64, ref, sa, sw, None)
+
+
 def test_zero_weights_and_zero_activations():
     M, N, K, G = 130, 264, 256, 128
     w = wl.make("custom", seed=2, M=M, K=K, N=N, G=G, bias=True)
