@@ -25,7 +25,7 @@ import torch
 __all__ = [
     "JQError", "library_path", "jq_quantize_act", "jq_pack_weight", "jq_workspace_size", "jq_w4a4_linear",
     "jq_fused_quant_linear", "jq_w4a4_group_partials", "jq_device_status", "jq_status_string",
-    "jq_w4a4_linear_noalloc",
+    "jq_w4a4_linear_noalloc", "jq_pack_weight_ternary", "jq_w158a4_workspace_size", "jq_w158a4_linear",
 ]
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
@@ -99,6 +99,52 @@ def _need_cuda(*ts):
             raise ValueError("libjq works on CUDA tensors only")
 
 
+def _groups(K: int, group: int):
+    """K/group, or None when group does not divide K (the library then rejects the call)."""
+    return K // group if group > 0 and K % group == 0 else None
+
+
+def _expect(fn: str, name: str, t, dtype, shape, device) -> None:
+    """The library receives bare pointers, so a tensor smaller than the call implies, strided,
+    of another type or on another device would be read or written out of bounds: refuse it
+    here.  shape entries of None are not checked (the scale shapes when group is invalid)."""
+    if t is None:
+        return
+    ok = (t.dtype == dtype and t.dim() == len(shape) and t.is_contiguous() and t.device == device
+          and all(want is None or have == want for have, want in zip(t.shape, shape)))
+    if not ok:
+        raise ValueError(f"{fn}: {name} must be a contiguous {dtype} tensor of shape {list(shape)} on {device}; "
+                         f"got {t.dtype} {list(t.shape)} (contiguous={t.is_contiguous()}) on {t.device}")
+
+
+def _expect_x(fn: str, x) -> None:
+    if not (x.dtype == torch.bfloat16 and x.dim() == 2 and x.stride(1) == 1):
+        raise ValueError(f"{fn}: x must be a 2-D bfloat16 tensor with unit column stride (rows may be padded); "
+                         f"got {x.dtype} {list(x.shape)} strides {list(x.stride())}")
+
+
+def _codes_shapes(fn: str, q, qw, codes_per_byte: int):
+    """(M, K, N) from packed activation codes q [M, K/2] and packed weights qw [N, K/codes_per_byte],
+    after checking both."""
+    if q.dim() != 2 or qw.dim() != 2:
+        raise ValueError(f"{fn}: q and the packed weights must be 2-D, got {list(q.shape)} and {list(qw.shape)}")
+    M, K = q.shape[0], q.shape[1] * 2
+    N = qw.shape[0]
+    _expect(fn, "q", q, torch.uint8, (M, K // 2), q.device)
+    _expect(fn, "packed weights", qw, torch.uint8, (N, K // codes_per_byte), q.device)
+    return M, K, N
+
+
+def _expect_linear(fn: str, M: int, N: int, K: int, group: int, device, s_a, s_w, bias, y, workspace) -> None:
+    ng = _groups(K, group)
+    _expect(fn, "s_a", s_a, torch.float32, (M, ng), device)
+    _expect(fn, "s_w", s_w, torch.float32, (ng, N), device)
+    _expect(fn, "bias", bias, torch.float32, (N,), device)
+    _expect(fn, "y", y, torch.bfloat16, (M, N), device)
+    if workspace is not None:
+        _expect(fn, "workspace", workspace, torch.uint8, (None,), device)
+
+
 def jq_status_string(code: int) -> str:
     return _load().jq_status_string(code).decode()
 
@@ -117,9 +163,12 @@ def _workspace(M, N, K, group, fused, device, workspace):
 def jq_quantize_act(x: torch.Tensor, group: int, q: torch.Tensor | None = None, s_a: torch.Tensor | None = None,
                     stream=None):
     """bf16 activations [M, K] (row stride >= K) -> (packed codes uint8 [M, K/2], scales fp32 [M, K/G])."""
-    assert x.dtype == torch.bfloat16 and x.dim() == 2 and x.stride(1) == 1
-    _need_cuda(x)
+    fn = "jq_quantize_act"
+    _expect_x(fn, x)
     M, K = x.shape
+    _expect(fn, "q", q, torch.uint8, (M, K // 2), x.device)
+    _expect(fn, "s_a", s_a, torch.float32, (M, _groups(K, group)), x.device)
+    _need_cuda(x)
     if q is None:
         q = torch.empty((M, K // 2), dtype=torch.uint8, device=x.device)
     if s_a is None:
@@ -131,9 +180,11 @@ def jq_quantize_act(x: torch.Tensor, group: int, q: torch.Tensor | None = None, 
 
 def jq_pack_weight(w: torch.Tensor, group: int, stream=None):
     """fp32 weights [N, K] -> (packed codes uint8 [N, K/2], scales fp32 [K/G, N])."""
-    assert w.dtype == torch.float32 and w.dim() == 2 and w.is_contiguous()
-    _need_cuda(w)
+    if w.dim() != 2:
+        raise ValueError(f"jq_pack_weight: w must be 2-D, got shape {list(w.shape)}")
     N, K = w.shape
+    _expect("jq_pack_weight", "w", w, torch.float32, (N, K), w.device)
+    _need_cuda(w)
     qw = torch.empty((N, K // 2), dtype=torch.uint8, device=w.device)
     s_w = torch.empty((K // group if group else 0, N), dtype=torch.float32, device=w.device)
     _check("jq_pack_weight", _load().jq_pack_weight(_ptr(w), N, K, group, _ptr(qw), _ptr(s_w), _stream(stream)))
@@ -142,9 +193,10 @@ def jq_pack_weight(w: torch.Tensor, group: int, stream=None):
 
 def jq_w4a4_linear(q, s_a, qw, s_w, bias, group: int, y=None, workspace=None, stream=None):
     """y = bf16(sum_g acc * s_a * s_w + bias) from packed activation and weight codes."""
+    fn = "jq_w4a4_linear"
+    M, K, N = _codes_shapes(fn, q, qw, 2)
+    _expect_linear(fn, M, N, K, group, q.device, s_a, s_w, bias, y, workspace)
     _need_cuda(q, s_a, qw, s_w, bias)
-    M, K = q.shape[0], q.shape[1] * 2
-    N = qw.shape[0]
     if y is None:
         y = torch.empty((M, N), dtype=torch.bfloat16, device=q.device)
     ws, ws_bytes = _workspace(M, N, K, group, False, q.device, workspace)
@@ -158,9 +210,10 @@ def jq_w4a4_linear_noalloc(q, s_a, qw, s_w, bias, group: int, y=None, stream=Non
     library keeps the scratch in its own fixed device array (ceil(M/128)*128*K <= 16 MiB).  Calls share that
     array, so order them on one stream.  (Only the output tensor is allocated here, by the
     caller's side, when y is None.)"""
+    fn = "jq_w4a4_linear_noalloc"
+    M, K, N = _codes_shapes(fn, q, qw, 2)
+    _expect_linear(fn, M, N, K, group, q.device, s_a, s_w, bias, y, None)
     _need_cuda(q, s_a, qw, s_w, bias)
-    M, K = q.shape[0], q.shape[1] * 2
-    N = qw.shape[0]
     if y is None:
         y = torch.empty((M, N), dtype=torch.bfloat16, device=q.device)
     _check("jq_w4a4_linear_noalloc",
@@ -171,10 +224,15 @@ def jq_w4a4_linear_noalloc(q, s_a, qw, s_w, bias, group: int, y=None, stream=Non
 
 def jq_fused_quant_linear(x, qw, s_w, bias, group: int, y=None, workspace=None, stream=None):
     """Same result as jq_w4a4_linear(*jq_quantize_act(x, group), ...), straight from bf16 x."""
-    assert x.dtype == torch.bfloat16 and x.dim() == 2 and x.stride(1) == 1
-    _need_cuda(x, qw, s_w, bias)
+    fn = "jq_fused_quant_linear"
+    _expect_x(fn, x)
     M, K = x.shape
+    if qw.dim() != 2:
+        raise ValueError(f"{fn}: qw must be 2-D, got shape {list(qw.shape)}")
     N = qw.shape[0]
+    _expect(fn, "qw", qw, torch.uint8, (N, K // 2), x.device)
+    _expect_linear(fn, M, N, K, group, x.device, None, s_w, bias, y, workspace)
+    _need_cuda(x, qw, s_w, bias)
     if y is None:
         y = torch.empty((M, N), dtype=torch.bfloat16, device=x.device)
     ws, ws_bytes = _workspace(M, N, K, group, True, x.device, workspace)
@@ -186,9 +244,13 @@ def jq_fused_quant_linear(x, qw, s_w, bias, group: int, y=None, workspace=None, 
 
 def jq_w4a4_group_partials(q, qw, group: int, workspace=None, stream=None):
     """Exact per-group integer partials int32 [M, N, K/G] (verification export)."""
+    fn = "jq_w4a4_group_partials"
+    M, K, N = _codes_shapes(fn, q, qw, 2)
+    if _groups(K, group) is None:
+        raise ValueError(f"{fn}: group {group} does not divide K = {K}")
+    if workspace is not None:
+        _expect(fn, "workspace", workspace, torch.uint8, (None,), q.device)
     _need_cuda(q, qw)
-    M, K = q.shape[0], q.shape[1] * 2
-    N = qw.shape[0]
     acc = torch.empty((M, N, K // group), dtype=torch.int32, device=q.device)
     ws, ws_bytes = _workspace(M, N, K, group, False, q.device, workspace)
     _check("jq_w4a4_group_partials",
@@ -199,9 +261,11 @@ def jq_w4a4_group_partials(q, qw, group: int, workspace=None, stream=None):
 
 def jq_pack_weight_ternary(w: torch.Tensor, group: int, stream=None):
     """fp32 weights [N, K] -> (packed ternary codes uint8 [N, K/4], scales fp32 [K/G, N])."""
-    assert w.dtype == torch.float32 and w.dim() == 2 and w.is_contiguous()
-    _need_cuda(w)
+    if w.dim() != 2:
+        raise ValueError(f"jq_pack_weight_ternary: w must be 2-D, got shape {list(w.shape)}")
     N, K = w.shape
+    _expect("jq_pack_weight_ternary", "w", w, torch.float32, (N, K), w.device)
+    _need_cuda(w)
     qw2 = torch.empty((N, K // 4), dtype=torch.uint8, device=w.device)
     s_w = torch.empty((K // group if group else 0, N), dtype=torch.float32, device=w.device)
     _check("jq_pack_weight_ternary",
@@ -216,9 +280,10 @@ def jq_w158a4_workspace_size(M: int, N: int, K: int, group: int) -> int:
 def jq_w158a4_linear(q, s_a, qw2, s_w, bias, group: int, y=None, workspace=None, stream=None):
     """W1.58A4: y = bf16(sum_g acc * s_a * s_w + bias) from packed INT4 activations and packed
     ternary weights."""
+    fn = "jq_w158a4_linear"
+    M, K, N = _codes_shapes(fn, q, qw2, 4)
+    _expect_linear(fn, M, N, K, group, q.device, s_a, s_w, bias, y, workspace)
     _need_cuda(q, s_a, qw2, s_w, bias)
-    M, K = q.shape[0], q.shape[1] * 2
-    N = qw2.shape[0]
     if y is None:
         y = torch.empty((M, N), dtype=torch.bfloat16, device=q.device)
     if workspace is None:
