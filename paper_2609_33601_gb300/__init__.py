@@ -110,11 +110,21 @@ def _expect(fn: str, name: str, t, dtype, shape, device) -> None:
     here.  shape entries of None are not checked (the scale shapes when group is invalid)."""
     if t is None:
         return
-    ok = (t.dtype == dtype and t.dim() == len(shape) and t.is_contiguous() and t.device == device
-          and all(want is None or have == want for have, want in zip(t.shape, shape)))
-    if not ok:
+    if None in shape:
+        shape_ok = t.dim() == len(shape) and all(w is None or h == w for h, w in zip(t.shape, shape))
+    else:
+        shape_ok = t.shape == shape
+    if not (shape_ok and t.dtype == dtype and t.is_contiguous() and t.device == device):
         raise ValueError(f"{fn}: {name} must be a contiguous {dtype} tensor of shape {list(shape)} on {device}; "
                          f"got {t.dtype} {list(t.shape)} (contiguous={t.is_contiguous()}) on {t.device}")
+
+
+def _expect_workspace(fn: str, ws, device) -> None:
+    """Any 1-D contiguous uint8 device buffer (the library checks its size)."""
+    if ws is not None and not (ws.dtype == torch.uint8 and ws.dim() == 1 and ws.is_contiguous()
+                               and ws.device == device):
+        raise ValueError(f"{fn}: workspace must be a contiguous 1-D uint8 tensor on {device}; "
+                         f"got {ws.dtype} {list(ws.shape)} on {ws.device}")
 
 
 def _expect_x(fn: str, x) -> None:
@@ -141,8 +151,7 @@ def _expect_linear(fn: str, M: int, N: int, K: int, group: int, device, s_a, s_w
     _expect(fn, "s_w", s_w, torch.float32, (ng, N), device)
     _expect(fn, "bias", bias, torch.float32, (N,), device)
     _expect(fn, "y", y, torch.bfloat16, (M, N), device)
-    if workspace is not None:
-        _expect(fn, "workspace", workspace, torch.uint8, (None,), device)
+    _expect_workspace(fn, workspace, device)
 
 
 def jq_status_string(code: int) -> str:
@@ -248,8 +257,7 @@ def jq_w4a4_group_partials(q, qw, group: int, workspace=None, stream=None):
     M, K, N = _codes_shapes(fn, q, qw, 2)
     if _groups(K, group) is None:
         raise ValueError(f"{fn}: group {group} does not divide K = {K}")
-    if workspace is not None:
-        _expect(fn, "workspace", workspace, torch.uint8, (None,), q.device)
+    _expect_workspace(fn, workspace, q.device)
     _need_cuda(q, qw)
     acc = torch.empty((M, N, K // group), dtype=torch.int32, device=q.device)
     ws, ws_bytes = _workspace(M, N, K, group, False, q.device, workspace)
