@@ -11,3 +11,9 @@ if ROOT not in sys.path:
 def pytest_configure(config):
     config.addinivalue_line("markers", "gpu: needs a CUDA GPU (GB300, sm_103a) and the built libjq.so")
     config.addinivalue_line("markers", "slow: long-running CPU test")
+
+
+def pytest_collection_modifyitems(config, items):
+    # Long cases run last (stable sort: the order is otherwise unchanged), so that a slow case
+    # cannot delay the rest, nor, under -x, keep them from running.
+    items.sort(key=lambda item: item.get_closest_marker("slow") is not None)

@@ -118,6 +118,32 @@ def test_quantize_act_exhaustive_bf16(G):
     assert np.array_equal(s.cpu().numpy().view(np.uint32), ref_s.view(np.uint32))
 
 
+@pytest.mark.slow
+def test_quantize_act_every_bf16_pair():
+    """Every positive finite bf16 amax with every bf16 x of magnitude up to it, both signs (about
+    1.07e9 pairs), in groups of 128 that each hold one amax: codes and scales must equal the
+    oracle's exactly.  This covers the compiled reciprocal shortcut and its fallback everywhere
+    (tests/test_fast_division_argument.py checks the argument behind it on the CPU)."""
+    G, per = 128, 127
+    allb = np.arange(1, 0x7F80, dtype=np.uint16)  # positive finite bf16, increasing in value
+    for chunk in np.array_split(np.arange(allb.size), 24):
+        blocks = []
+        for ia in chunk:
+            xs = np.concatenate([allb[: ia + 1], allb[: ia + 1] ^ np.uint16(0x8000)])
+            n = -(-xs.size // per)
+            blk = np.zeros((n, G), np.uint16)
+            blk[:, 0] = allb[ia]
+            flat = np.zeros(n * per, np.uint16)
+            flat[: xs.size] = xs
+            blk[:, 1:] = flat.reshape(n, per)
+            blocks.append(blk)
+        x = np.concatenate(blocks)
+        ref_codes, ref_s = oracle.quantize_bf16(x, G)
+        q, s = jq.jq_quantize_act(dev_bf16(x), G)
+        assert np.array_equal(q.cpu().numpy(), oracle.pack(ref_codes)), f"amax index {chunk[0]}..{chunk[-1]}"
+        assert np.array_equal(s.cpu().numpy().view(np.uint32), ref_s.view(np.uint32))
+
+
 @pytest.mark.parametrize("N,K,G", [(520, 512, 64), (264, 512, 128), (96, 1024, 1024), (8, 15360, 64)])
 def test_pack_weight_bit_exact(N, K, G):
     rng = np.random.default_rng(N + K)
