@@ -504,7 +504,8 @@ def run_ours(args):
     else:
         achieved = ops_step / (gemm_ms * 1e-3) / 1e12
         roofline = {"bound": "tensor", "achieved": achieved, "peak": fp8_peak, "unit": "TFLOP/s",
-                    "frac": achieved / fp8_peak, "traffic": traffic, "algorithmic_bytes": alg_bytes,
+                    "frac": achieved / fp8_peak, "frac_of_bf16_peak": achieved / bf16_peak,
+                    "traffic": traffic, "algorithmic_bytes": alg_bytes,
                     "kernel": what + ", CUDA events around a graph of K launches",
                     "peak_source": f"{peak_src} bf16 {bf16_peak} TFLOP/s x nominal FP8/BF16 ratio {FP8_PER_BF16}"}
     context = None
