@@ -38,7 +38,7 @@
  *     JQ_ERR_TIMEOUT in a device status word read by jq_device_status().
  *   - Devices and threads: this version sets its kernels' shared-memory attributes once per
  *     process, on the first device that launches them, so drive one GPU per process (calls on
- *     a second device of the same process return JQ_ERR_CUDA), and make the first call on a
+ *     a second device of the same process may fail with JQ_ERR_CUDA), and make the first call on a
  *     device from one thread; after that, calls from several threads are safe.
  *   - Kernels are launched with programmatic dependent launch: one of this library's kernels may
  *     start while the previous kernel on the stream is still running, when that kernel is also
