@@ -6,11 +6,17 @@
 
 #include "jq.h"
 #include "kernels.cuh"
+#include "operand.cuh"
 
 namespace {
 
 constexpr int kMaxDevices = 64;
-constexpr int64_t kMaxK = 262016;  // 64 * K < 2^24 keeps every exact group sum representable
+using jq::kMaxK;
+// The offset-code form (one group, in the few-token kernel and the GEMM) sums |(q_w + 8) q_a| <= 120
+// per element, exact in fp32 over runs of up to kOffsetMaxRun elements; the few-token kernel's
+// one-group limit stays inside that run.
+static_assert(120 * static_cast<int64_t>(jq::kOffsetMaxRun) < (int64_t{1} << 24), "offset-code runs are exact");
+static_assert(jq::kSkinnyMaxKOneGroup <= jq::kOffsetMaxRun, "one-group few-token problems are exact");
 
 // One status word per device, written by kernels that give up a bounded wait.
 __device__ uint32_t g_device_status = 0;

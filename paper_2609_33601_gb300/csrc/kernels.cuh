@@ -26,6 +26,11 @@ cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t s
   return cudaLaunchKernelEx(&cfg, kernel, static_cast<KArgs>(args)...);
 }
 
+// Largest K the library accepts: every exact group sum of sign-magnitude codes, |acc| <= 64 K,
+// stays below 2^24, so the fp32 accumulators hold it exactly (operand.cuh).
+constexpr int64_t kMaxK = 262016;  // 2047 * 128
+static_assert(64 * kMaxK < (int64_t{1} << 24) && kMaxK % 128 == 0, "exact group sums up to kMaxK");
+
 // bf16 activations [M, ldx] -> packed codes [M, K/2] + scales [M, K/G].
 cudaError_t launch_quantize_act(const void* x, int64_t M, int64_t K, int64_t ldx, int G, uint8_t* q, float* s_a,
                                 cudaStream_t stream, int sms);

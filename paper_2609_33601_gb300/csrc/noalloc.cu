@@ -23,7 +23,7 @@ namespace {
 
 constexpr size_t kNoAllocScratchBytes = JQ_NOALLOC_MAX_SCRATCH_BYTES;
 constexpr int kMaxDevices = 64;
-constexpr int64_t kMaxK = 262016;
+using jq::kMaxK;
 
 // The scratch: the E4M3 operand image of the activations, whole 128-row tiles of K bytes.  The
 // expansion kernel of the same call writes every row below M; rows past M in the last tile are
