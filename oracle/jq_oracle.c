@@ -26,6 +26,13 @@
  *   - The linear layer: acc[m,n,g] = sum_{k in g} qa[m,k]*qw[n,k] (exact
  *     integers), y[m,n] = sum_g acc*s_a[m,g]*s_w[n,g] + bias[n], evaluated
  *     here in fp64 and rounded once to bf16 (round to nearest even).
+ *   - Two further settings, each defined where its section begins below: the
+ *     ternary weights of W1.58A4 (absmean rule, 2-bit packing) and the NVFP4
+ *     format of the LLaDA-8B rows (E2M1 elements, E4M3 block scales).
+ *
+ * Every function here is pinned by tests/test_oracle_pins.py or
+ * tests/test_oracle_nvfp4_pins.py against hand-worked examples, exact
+ * rational evaluations, enumerations and invariants; none is unpinned.
  *
  * Floating point: compile with -O2 -ffp-contract=off and without fast-math,
  * so float division is the IEEE-754 single-precision correctly-rounded one
@@ -33,13 +40,12 @@
  * independent rows across threads; it never changes any arithmetic.
  */
 #include <math.h>
+#include <omp.h>
 #include <stdint.h>
 #include <stdlib.h>
 #include <string.h>
 
 #include "jq_oracle.h"
-
-#include <omp.h>
 
 /* Thread control for the timed CPU baseline (no effect on any result: every parallel loop
  * here splits independent rows, each computed in one fixed order). */
