@@ -5,7 +5,7 @@ library instead of a caller-provided workspace.
 
 Two calls in a row on different shapes, each compared with jq_w4a4_linear (which uses a
 workspace) and with the CPU oracle under the tolerance the parity tests use; then the size
-limit.  This file is collected last so that a run stopping at the first failure has already run
+limit; then 17-64 tokens, where the few-token kernel converts the tokens itself.  This file is collected last so that a run stopping at the first failure has already run
 every other test; it also passes on its own in a fresh process.
 """
 import ctypes
@@ -72,3 +72,18 @@ def test_noalloc_rejects_problems_beyond_its_scratch():
     rc = lib.jq_w4a4_linear_noalloc(p, p, p, p, None, p, M, 8, K, 128, None)
     assert rc == JQ_ERR_WORKSPACE
     torch.cuda.synchronize()
+
+
+@pytest.mark.parametrize("M,N,K,G,bias", [(17, 264, 1024, 128, True), (40, 520, 512, 64, False),
+                                          (64, 136, 2048, 2048, True)])
+def test_noalloc_few_tokens_convert_the_tokens_in_the_kernel(M, N, K, G, bias):
+    """Up to 64 tokens the no-allocation call has no workspace for pre-expanded tokens, so the
+    few-token kernel converts the packed token codes itself; with more than 16 tokens that is
+    the only caller of that form (jq_w4a4_linear hands it the tokens pre-expanded).  Same
+    result as jq_w4a4_linear, and within the oracle's tolerance."""
+    ref, args = _problem(M, N, K, G, bias, seed=M + 3)
+    y_na = _bits(jq.jq_w4a4_linear_noalloc(*args, G))
+    y_ws = _bits(jq.jq_w4a4_linear(*args, G))
+    y64, _ = ref.linear()
+    check_linear(y_na, y64, ref.partials(), ref.s_a, ref.s_w_rows, ref.bias, f"noalloc M={M}")
+    assert np.array_equal(y_na, y_ws)
