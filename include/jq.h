@@ -204,6 +204,16 @@ JQ_API jq_status jq_w158a4_linear(const uint8_t* q, const float* s_a, const uint
                                   void* workspace, size_t workspace_bytes, void* stream);
 
 /*
+ * Verification export for failure handling (computes nothing): launches one block in which one
+ * thread waits, with the bounded wait every kernel of this library uses, on an mbarrier phase
+ * that nothing completes.  After about 2^31 SM clock cycles (about a second) the wait gives up
+ * and records JQ_ERR_TIMEOUT in the device status word, which jq_device_status() then reports;
+ * nothing faults, traps or hangs, and the CUDA context stays usable.  It lets a caller test its
+ * handling of a kernel that gave up.  Errors: JQ_ERR_UNSUPPORTED, JQ_ERR_CUDA.
+ */
+JQ_API jq_status jq_debug_wait_timeout(void* stream);
+
+/*
  * Synchronises `stream` and returns JQ_ERR_TIMEOUT if any kernel of this library on the
  * current device gave up a bounded wait since the last reset (reset != 0 clears the flag),
  * JQ_ERR_UNSUPPORTED if a GEMM launch found its shared-memory window not 1024-byte aligned

@@ -26,6 +26,7 @@ __all__ = [
     "JQError", "library_path", "jq_quantize_act", "jq_pack_weight", "jq_workspace_size", "jq_w4a4_linear",
     "jq_fused_quant_linear", "jq_w4a4_group_partials", "jq_device_status", "jq_status_string",
     "jq_w4a4_linear_noalloc", "jq_pack_weight_ternary", "jq_w158a4_workspace_size", "jq_w158a4_linear",
+    "jq_debug_wait_timeout",
 ]
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
@@ -61,6 +62,7 @@ def _load() -> ctypes.CDLL:
                 "jq_fused_quant_linear": [vp, i64, vp, vp, vp, vp, i64, i64, i64, i32, vp, sz, vp],
                 "jq_w4a4_group_partials": [vp, vp, vp, i64, i64, i64, i32, vp, sz, vp],
                 "jq_device_status": [vp, i32],
+                "jq_debug_wait_timeout": [vp],
                 "jq_w4a4_linear_noalloc": [vp, vp, vp, vp, vp, vp, i64, i64, i64, i32, vp],
                 "jq_pack_weight_ternary": [vp, i64, i64, i32, vp, vp, vp],
                 "jq_w158a4_linear": [vp, vp, vp, vp, vp, vp, i64, i64, i64, i32, vp, sz, vp],
@@ -301,6 +303,12 @@ def jq_w158a4_linear(q, s_a, qw2, s_w, bias, group: int, y=None, workspace=None,
            _load().jq_w158a4_linear(_ptr(q), _ptr(s_a), _ptr(qw2), _ptr(s_w), _ptr(bias), _ptr(y), M, N, K, group,
                                     _ptr(workspace), ws_bytes, _stream(stream)))
     return y
+
+
+def jq_debug_wait_timeout(stream=None) -> None:
+    """Enqueues the failure-handling probe: a kernel whose bounded wait runs out after about a
+    second and records JQ_ERR_TIMEOUT for jq_device_status (nothing faults or hangs)."""
+    _check("jq_debug_wait_timeout", _load().jq_debug_wait_timeout(_stream(stream)))
 
 
 def jq_device_status(reset: bool = True, stream=None) -> int:

@@ -7,6 +7,7 @@
 #include "jq.h"
 #include "kernels.cuh"
 #include "operand.cuh"
+#include "ptx.cuh"
 
 namespace {
 
@@ -56,6 +57,21 @@ bool group_ok(int64_t K, int32_t group) {
 size_t round_up(size_t v, size_t a) { return (v + a - 1) / a * a; }
 
 jq_status from_cuda(cudaError_t e) { return e == cudaSuccess ? JQ_OK : JQ_ERR_CUDA; }
+
+// Failure-handling probe: one thread waits, with the bounded wait every kernel of the library
+// uses, on an mbarrier phase that nothing completes.  The wait gives up after ~2^31 cycles,
+// records kDevTimeout in the status word and the block returns: no trap, no fault, no hang.
+__global__ void __launch_bounds__(32) wait_timeout_probe_kernel(uint32_t* status) {
+  __shared__ __align__(8) uint64_t bar;
+  __shared__ int abort_flag;
+  if (threadIdx.x == 0) {
+    jq::mbar_init(&bar, 1);  // one arrival would complete phase 0; none comes
+    abort_flag = 0;
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) (void)jq::mbar_wait(&bar, 0, &abort_flag, status);
+  __syncthreads();
+}
 
 }  // namespace
 
@@ -270,6 +286,13 @@ jq_status jq_w4a4_group_partials(const uint8_t* q, const uint8_t* qw, int32_t* a
   jq::GemmProblem p{static_cast<int>(M), static_cast<int>(N), static_cast<int>(K), group, a_op, nullptr, corr, qw,
                     reinterpret_cast<const float*>(qw), nullptr, nullptr, acc, d->status};
   return from_cuda(jq::launch_w4a4_gemm(p, s, d->sms));
+}
+
+jq_status jq_debug_wait_timeout(void* stream) {
+  const DeviceInfo* d = current_device();
+  if (d == nullptr) return JQ_ERR_UNSUPPORTED;
+  wait_timeout_probe_kernel<<<1, 32, 0, static_cast<cudaStream_t>(stream)>>>(d->status);
+  return from_cuda(cudaGetLastError());
 }
 
 jq_status jq_device_status(void* stream, int32_t reset) {

@@ -107,6 +107,8 @@ def test_valid_arguments_without_a_device_report_unsupported(lib):
     lib.jq_quantize_act.argtypes = [vp, i64, i64, i64, i32, vp, vp, vp]
     A = _fake(0x10000)
     assert lib.jq_quantize_act(A, 4, 256, 256, 64, A, A, None) == UNSUPPORTED
+    lib.jq_debug_wait_timeout.argtypes = [vp]
+    assert lib.jq_debug_wait_timeout(None) == UNSUPPORTED  # the failure probe launches nothing either
 
 
 def test_binding_fails_loudly_without_cuda_tensors():
