@@ -77,7 +77,11 @@ def _load():
             lib.oracle_pack_nvfp4.argtypes = [vp, i64, i64, vp]
             lib.oracle_unpack_nvfp4.argtypes = [vp, i64, i64, vp]
             lib.oracle_linear_nvfp4.argtypes = [vp, vp, f32, vp, vp, f32, vp, i64, i64, i64, vp, vp]
-            for f in ("oracle_quantize_bf16", "oracle_quantize_f32", "oracle_pack", "oracle_unpack",
+            lib.oracle_fake_quant_bf16.argtypes = [vp, i64, i64, i64, vp, vp, vp, vp]
+            lib.oracle_fake_quant_f32.argtypes = [vp, i64, i64, i64, vp, vp, vp, vp]
+            lib.oracle_ste_backward_bf16.argtypes = [vp, vp, i64, vp]
+            for f in ("oracle_fake_quant_bf16", "oracle_fake_quant_f32", "oracle_ste_backward_bf16",
+                      "oracle_quantize_bf16", "oracle_quantize_f32", "oracle_pack", "oracle_unpack",
                       "oracle_group_partials", "oracle_linear", "oracle_quantize_ternary_f32",
                       "oracle_pack_ternary", "oracle_unpack_ternary", "oracle_quantize_nvfp4",
                       "oracle_pack_nvfp4", "oracle_unpack_nvfp4", "oracle_linear_nvfp4"):
@@ -253,3 +257,44 @@ def linear_nvfp4(qa2, sa, ga: float, qw2, sw, gw: float, bias):
     _load().oracle_linear_nvfp4(_p(qa2), _p(sa), ctypes.c_float(ga), _p(qw2), _p(sw), ctypes.c_float(gw),
                                 _p(b), M, N, K, _p(y64), _p(yb))
     return y64, yb
+
+
+def fake_quant_bf16(x_bits: np.ndarray, group: int, s_in=None):
+    """Fake quantisation of bf16 activations for training (forward of the STE reading).
+
+    x_bits uint16 [M, K] -> (xhat uint16 bf16 bits [M, K], mask uint8 [M, K], scales f32 [M, K/G]).
+    s_in: None for the amax/7 rule, else [M, K/G] positive finite scales to use instead."""
+    x_bits = _c(x_bits, np.uint16)
+    M, K = x_bits.shape
+    assert K % group == 0
+    s = None if s_in is None else _c(s_in, np.float32)
+    assert s is None or s.shape == (M, K // group)
+    xhat = np.empty((M, K), np.uint16)
+    mask = np.empty((M, K), np.uint8)
+    s_out = np.empty((M, K // group), np.float32)
+    _load().oracle_fake_quant_bf16(_p(x_bits), M, K, group, _p(s), _p(xhat), _p(mask), _p(s_out))
+    return xhat, mask, s_out
+
+
+def fake_quant_f32(w: np.ndarray, group: int, s_in=None):
+    """Fake quantisation of fp32 weights: -> (what f32 [N, K], mask uint8 [N, K], scales f32 [N, K/G])."""
+    w = _c(w, np.float32)
+    N, K = w.shape
+    assert K % group == 0
+    s = None if s_in is None else _c(s_in, np.float32)
+    assert s is None or s.shape == (N, K // group)
+    what = np.empty((N, K), np.float32)
+    mask = np.empty((N, K), np.uint8)
+    s_out = np.empty((N, K // group), np.float32)
+    _load().oracle_fake_quant_f32(_p(w), N, K, group, _p(s), _p(what), _p(mask), _p(s_out))
+    return what, mask, s_out
+
+
+def ste_backward_bf16(grad_bits: np.ndarray, mask: np.ndarray) -> np.ndarray:
+    """STE backward: bf16 gradient bits where mask is 1, +0 where it is 0 (same shape)."""
+    grad_bits = _c(grad_bits, np.uint16)
+    mask = _c(mask, np.uint8)
+    assert grad_bits.shape == mask.shape
+    out = np.empty_like(grad_bits)
+    _load().oracle_ste_backward_bf16(_p(grad_bits), _p(mask), grad_bits.size, _p(out))
+    return out

@@ -29,10 +29,13 @@
  *   - Two further settings, each defined where its section begins below: the
  *     ternary weights of W1.58A4 (absmean rule, 2-bit packing) and the NVFP4
  *     format of the LLaDA-8B rows (E2M1 elements, E4M3 block scales).
+ *   - The training side: fake quantisation with the straight-through
+ *     estimator (last section).
  *
- * Every function here is pinned by tests/test_oracle_pins.py or
- * tests/test_oracle_nvfp4_pins.py against hand-worked examples, exact
- * rational evaluations, enumerations and invariants; none is unpinned.
+ * Every function here is pinned by tests/test_oracle_pins.py,
+ * tests/test_oracle_nvfp4_pins.py or tests/test_oracle_fakequant_pins.py
+ * against hand-worked examples, exact rational evaluations, enumerations and
+ * invariants; none is unpinned.
  *
  * Floating point: compile with -O2 -ffp-contract=off and without fast-math,
  * so float division is the IEEE-754 single-precision correctly-rounded one
@@ -424,4 +427,98 @@ void oracle_linear(const int8_t* qa, const float* s_a, const int8_t* qw, const f
       if (y64) y64[m * N + n] = y;
       if (ybf16) ybf16[m * N + n] = oracle_bf16_rne(y);
     }
+}
+
+/* ---- training side: fake quantisation and the straight-through estimator ----------------
+ *
+ * Stage 1 of Theseus QAD (Sec. 3, Algorithm 1) updates the student's parameters by gradient
+ * descent through its quantised blocks, and the paper names the straight-through estimator
+ * (STE) as the gradient rule that 4-bit activations pass through (Sec. 3, "Why QAT fails";
+ * Fig. "STE instability").  It prints neither the forward nor the backward rule.  The reading
+ * computed here:
+ *   forward   xhat = q * s for every element, where q = clamp(rint(fl32(x / s)), -8, 7) is the
+ *             deployed quantiser's code and s is the group's scale: amax/7 of the group as in
+ *             the file header, or a positive finite scale the caller gives (a learned one);
+ *             q * s is formed exactly (fp64) and rounded once to the input's type (bf16 or fp32,
+ *             nearest even);
+ *   backward  dL/dx = dL/dxhat where the unclamped code rint(fl32(x / s)) lies in [-8, 7], and
+ *             +0 where the clamp acted; the scale is held constant (no gradient reaches s).
+ * With the amax scale every |x / s| is at most about 7, so no code reaches the clamp and the
+ * mask is all ones; a group whose amax is 0 has s = 0, xhat = 0 and mask 1.  A zero code gives
+ * xhat = +0 whatever the sign of x (the code, an integer, has none).
+ */
+
+/* One group of G fp32 values.  s_given: NULL for the amax rule, else the scale to use.
+ * Writes the exact products q*s (fp64) and the pass-through mask; returns the scale used. */
+static float fake_quant_group(const float* xf, int64_t G, const float* s_given, double* xhat,
+                              uint8_t* mask) {
+  float s;
+  if (s_given) {
+    s = *s_given;
+  } else {
+    float amax = 0.0f;
+    for (int64_t k = 0; k < G; ++k) {
+      float a = fabsf(xf[k]);
+      if (a > amax) amax = a;
+    }
+    if (amax == 0.0f) {
+      for (int64_t k = 0; k < G; ++k) {
+        xhat[k] = 0.0;
+        mask[k] = 1;
+      }
+      return 0.0f;
+    }
+    s = amax / 7.0f;                       /* IEEE single division */
+  }
+  for (int64_t k = 0; k < G; ++k) {
+    float r = rintf(xf[k] / s);            /* IEEE single division, then half to even */
+    mask[k] = (r >= -8.0f && r <= 7.0f) ? 1 : 0;
+    if (r > 7.0f) r = 7.0f;
+    if (r < -8.0f) r = -8.0f;
+    const int q = (int)r;                  /* the code is an integer: code 0 gives +0, never -0 */
+    xhat[k] = (double)q * (double)s;       /* exact: a 4-bit integer times a 24-bit significand */
+  }
+  return s;
+}
+
+/* Activations: bf16 [M, K] (dense rows) -> xhat bf16 [M, K], mask u8 [M, K] and the scales used
+ * [M, K/G].  s_in: NULL (amax rule) or [M, K/G] positive finite scales. */
+void oracle_fake_quant_bf16(const uint16_t* x, int64_t M, int64_t K, int64_t G, const float* s_in,
+                            uint16_t* xhat, uint8_t* mask, float* s_out) {
+  const int64_t ng = K / G;
+#pragma omp parallel for schedule(static)
+  for (int64_t m = 0; m < M; ++m) {
+    float* xf = (float*)malloc((size_t)G * sizeof(float));
+    double* e = (double*)malloc((size_t)G * sizeof(double));
+    for (int64_t g = 0; g < ng; ++g) {
+      const int64_t o = m * K + g * G;
+      for (int64_t k = 0; k < G; ++k) xf[k] = bf16_bits_to_float(x[o + k]);
+      s_out[m * ng + g] = fake_quant_group(xf, G, s_in ? s_in + m * ng + g : NULL, e, mask + o);
+      for (int64_t k = 0; k < G; ++k) xhat[o + k] = oracle_bf16_rne(e[k]);
+    }
+    free(e);
+    free(xf);
+  }
+}
+
+/* Weights: fp32 [N, K] -> xhat fp32 [N, K] (the exact product rounded once to fp32), mask and
+ * scales as above. */
+void oracle_fake_quant_f32(const float* w, int64_t N, int64_t K, int64_t G, const float* s_in,
+                           float* what, uint8_t* mask, float* s_out) {
+  const int64_t ng = K / G;
+#pragma omp parallel for schedule(static)
+  for (int64_t n = 0; n < N; ++n) {
+    double* e = (double*)malloc((size_t)G * sizeof(double));
+    for (int64_t g = 0; g < ng; ++g) {
+      const int64_t o = n * K + g * G;
+      s_out[n * ng + g] = fake_quant_group(w + o, G, s_in ? s_in + n * ng + g : NULL, e, mask + o);
+      for (int64_t k = 0; k < G; ++k) what[o + k] = (float)e[k];  /* round to nearest even */
+    }
+    free(e);
+  }
+}
+
+/* STE backward on bf16 gradients: grad_x = grad where mask is 1, +0 where it is 0. */
+void oracle_ste_backward_bf16(const uint16_t* grad, const uint8_t* mask, int64_t n, uint16_t* grad_x) {
+  for (int64_t i = 0; i < n; ++i) grad_x[i] = mask[i] ? grad[i] : (uint16_t)0;
 }

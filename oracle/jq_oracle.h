@@ -32,6 +32,11 @@ void oracle_group_partials(const int8_t* qa, const int8_t* qw, int64_t M, int64_
 void oracle_linear(const int8_t* qa, const float* s_a, const int8_t* qw, const float* s_w,
                    const float* bias, int64_t M, int64_t N, int64_t K, int64_t G, double* y64,
                    uint16_t* ybf16);
+void oracle_fake_quant_bf16(const uint16_t* x, int64_t M, int64_t K, int64_t G, const float* s_in,
+                            uint16_t* xhat, uint8_t* mask, float* s_out);
+void oracle_fake_quant_f32(const float* w, int64_t N, int64_t K, int64_t G, const float* s_in,
+                           float* what, uint8_t* mask, float* s_out);
+void oracle_ste_backward_bf16(const uint16_t* grad, const uint8_t* mask, int64_t n, uint16_t* grad_x);
 #ifdef __cplusplus
 }
 #endif
