@@ -204,6 +204,38 @@ JQ_API jq_status jq_w158a4_linear(const uint8_t* q, const float* s_a, const uint
                                   void* workspace, size_t workspace_bytes, void* stream);
 
 /*
+ * Training side: fake quantisation of bf16 activations (forward of the straight-through
+ * estimator).  Stage 1 of Theseus QAD (Sec. 3, Algorithm 1) trains the quantised student blocks
+ * by gradient descent, and Sec. 3 ("Why QAT fails") names the straight-through estimator as the
+ * gradient rule of 4-bit activations; the paper prints neither rule, and this is the reading:
+ *   xhat[m,k] = bf16( q * s )   with q = clamp(rint(fl32(x / s)), -8, 7), the deployed code,
+ *   the product formed exactly and rounded once (nearest even); a zero code gives +0;
+ *   mask[m,k] = 1 where the unclamped rint(fl32(x / s)) lies in [-8, 7], else 0.
+ *   x_bf16    : bf16 [M, K], dense rows (device)
+ *   group     : 64, 128 or K (K a multiple of 128, at most 262016)
+ *   s_in      : fp32 [M, K/group] positive finite scales with 8*s finite (e.g. learned ones), or
+ *               NULL for the quantiser's own rule s = fl32(amax/7) (then s = 0, xhat = 0 and
+ *               mask = 1 for an all-zero group, and no code is clamped)
+ *   xhat_bf16 : bf16 [M, K] (output);  mask : uint8 [M, K] (output, 0/1)
+ *   s_out     : fp32 [M, K/group] (output): the scales used
+ * All pointers 16-byte aligned; M = 0 is a no-op.  Errors: JQ_ERR_INVALID_ARG (null, K/group
+ * unsupported, M < 0), JQ_ERR_MISALIGNED, JQ_ERR_UNSUPPORTED (not sm_103), JQ_ERR_CUDA.
+ */
+JQ_API jq_status jq_fake_quant_act(const void* x_bf16, int64_t M, int64_t K, int32_t group, const float* s_in,
+                                   void* xhat_bf16, uint8_t* mask, float* s_out, void* stream);
+
+/*
+ * Training side: the straight-through backward (the reading above):
+ *   grad_x[i] = grad[i] where mask[i] != 0, else +0.
+ *   grad_bf16, grad_x_bf16 : bf16 [n] (device; grad_x may not overlap grad unless equal)
+ *   mask                   : uint8 [n] (jq_fake_quant_act's mask)
+ * Any n >= 0 (n = 0 is a no-op); pointers 16-byte aligned.  Errors: JQ_ERR_INVALID_ARG,
+ * JQ_ERR_MISALIGNED, JQ_ERR_UNSUPPORTED, JQ_ERR_CUDA.
+ */
+JQ_API jq_status jq_ste_backward(const void* grad_bf16, const uint8_t* mask, int64_t n, void* grad_x_bf16,
+                                 void* stream);
+
+/*
  * Verification export for failure handling (computes nothing): launches one block in which one
  * thread waits, with the bounded wait every kernel of this library uses, on an mbarrier phase
  * that nothing completes.  After about 2^31 SM clock cycles (about a second) the wait gives up

@@ -26,7 +26,7 @@ __all__ = [
     "JQError", "library_path", "jq_quantize_act", "jq_pack_weight", "jq_workspace_size", "jq_w4a4_linear",
     "jq_fused_quant_linear", "jq_w4a4_group_partials", "jq_device_status", "jq_status_string",
     "jq_w4a4_linear_noalloc", "jq_pack_weight_ternary", "jq_w158a4_workspace_size", "jq_w158a4_linear",
-    "jq_debug_wait_timeout",
+    "jq_debug_wait_timeout", "jq_fake_quant_act", "jq_ste_backward",
 ]
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
@@ -63,6 +63,8 @@ def _load() -> ctypes.CDLL:
                 "jq_w4a4_group_partials": [vp, vp, vp, i64, i64, i64, i32, vp, sz, vp],
                 "jq_device_status": [vp, i32],
                 "jq_debug_wait_timeout": [vp],
+                "jq_fake_quant_act": [vp, i64, i64, i32, vp, vp, vp, vp, vp],
+                "jq_ste_backward": [vp, vp, i64, vp, vp],
                 "jq_w4a4_linear_noalloc": [vp, vp, vp, vp, vp, vp, i64, i64, i64, i32, vp],
                 "jq_pack_weight_ternary": [vp, i64, i64, i32, vp, vp, vp],
                 "jq_w158a4_linear": [vp, vp, vp, vp, vp, vp, i64, i64, i64, i32, vp, sz, vp],
@@ -314,3 +316,37 @@ def jq_debug_wait_timeout(stream=None) -> None:
 def jq_device_status(reset: bool = True, stream=None) -> int:
     """Synchronises the stream; returns the library's status code (5 = a kernel timed out)."""
     return int(_load().jq_device_status(_stream(stream), 1 if reset else 0))
+
+
+def jq_fake_quant_act(x: torch.Tensor, group: int, s_in: torch.Tensor | None = None, stream=None):
+    """Training-side fake quantisation of bf16 activations [M, K] (dense rows).
+
+    Returns (xhat bf16 [M, K], mask uint8 [M, K], scales fp32 [M, K/G]); s_in, if given, is
+    [M, K/G] fp32 positive scales used in place of the amax/7 rule."""
+    fn = "jq_fake_quant_act"
+    _expect_x(fn, x)
+    M, K = x.shape
+    if not x.is_contiguous():
+        raise ValueError(f"{fn}: x must have dense rows")
+    _expect(fn, "s_in", s_in, torch.float32, (M, _groups(K, group)), x.device)
+    _need_cuda(x)
+    xhat = torch.empty((M, K), dtype=torch.bfloat16, device=x.device)
+    mask = torch.empty((M, K), dtype=torch.uint8, device=x.device)
+    s_out = torch.empty((M, K // group if group else 0), dtype=torch.float32, device=x.device)
+    _check(fn, _load().jq_fake_quant_act(_ptr(x), M, K, group, _ptr(s_in), _ptr(xhat), _ptr(mask), _ptr(s_out),
+                                         _stream(stream)))
+    return xhat, mask, s_out
+
+
+def jq_ste_backward(grad: torch.Tensor, mask: torch.Tensor, stream=None):
+    """Straight-through backward: the bf16 gradient where mask != 0, +0 elsewhere (same shape)."""
+    fn = "jq_ste_backward"
+    if grad.dtype != torch.bfloat16 or not grad.is_contiguous():
+        raise ValueError(f"{fn}: grad must be a contiguous bf16 tensor")
+    _expect(fn, "mask", mask, torch.uint8, tuple(grad.shape), grad.device)
+    if mask is None:
+        raise ValueError(f"{fn}: mask is required")
+    _need_cuda(grad)
+    out = torch.empty_like(grad)
+    _check(fn, _load().jq_ste_backward(_ptr(grad), _ptr(mask), grad.numel(), _ptr(out), _stream(stream)))
+    return out

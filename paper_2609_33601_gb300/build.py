@@ -17,7 +17,7 @@ CSRC = os.path.join(HERE, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 BUILD = os.path.join(HERE, "_build")
 LIB = os.path.join(HERE, "libjq.so")
-SOURCES = ["api.cu", "quantize.cu", "gemm.cu", "skinny.cu", "noalloc.cu", "ternary.cu"]
+SOURCES = ["api.cu", "quantize.cu", "gemm.cu", "skinny.cu", "noalloc.cu", "ternary.cu", "fakequant.cu"]
 HEADERS = ["kernels.cuh", "operand.cuh", "ptx.cuh"]
 
 NVCC_FLAGS = [

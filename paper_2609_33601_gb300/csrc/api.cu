@@ -288,6 +288,30 @@ jq_status jq_w4a4_group_partials(const uint8_t* q, const uint8_t* qw, int32_t* a
   return from_cuda(jq::launch_w4a4_gemm(p, s, d->sms));
 }
 
+jq_status jq_fake_quant_act(const void* x_bf16, int64_t M, int64_t K, int32_t group, const float* s_in,
+                            void* xhat_bf16, uint8_t* mask, float* s_out, void* stream) {
+  if (M < 0 || !group_ok(K, group)) return JQ_ERR_INVALID_ARG;
+  if (M == 0) return JQ_OK;
+  if (x_bf16 == nullptr || xhat_bf16 == nullptr || mask == nullptr || s_out == nullptr) return JQ_ERR_INVALID_ARG;
+  if (!aligned16(x_bf16) || !aligned16(xhat_bf16) || !aligned16(mask) || !aligned16(s_out) ||
+      (s_in != nullptr && !aligned16(s_in)))
+    return JQ_ERR_MISALIGNED;
+  const DeviceInfo* d = current_device();
+  if (d == nullptr) return JQ_ERR_UNSUPPORTED;
+  return from_cuda(jq::launch_fake_quant_act(x_bf16, M, K, group, s_in, xhat_bf16, mask, s_out,
+                                             static_cast<cudaStream_t>(stream), d->sms));
+}
+
+jq_status jq_ste_backward(const void* grad_bf16, const uint8_t* mask, int64_t n, void* grad_x_bf16, void* stream) {
+  if (n < 0) return JQ_ERR_INVALID_ARG;
+  if (n == 0) return JQ_OK;
+  if (grad_bf16 == nullptr || mask == nullptr || grad_x_bf16 == nullptr) return JQ_ERR_INVALID_ARG;
+  if (!aligned16(grad_bf16) || !aligned16(mask) || !aligned16(grad_x_bf16)) return JQ_ERR_MISALIGNED;
+  const DeviceInfo* d = current_device();
+  if (d == nullptr) return JQ_ERR_UNSUPPORTED;
+  return from_cuda(jq::launch_ste_backward(grad_bf16, mask, n, grad_x_bf16, static_cast<cudaStream_t>(stream), d->sms));
+}
+
 jq_status jq_debug_wait_timeout(void* stream) {
   const DeviceInfo* d = current_device();
   if (d == nullptr) return JQ_ERR_UNSUPPORTED;

@@ -1,0 +1,157 @@
+// fakequant.cu -- training side: fake quantisation of bf16 activations and the straight-through
+// backward.  Stage 1 of Theseus QAD (Sec. 3, Algorithm 1) trains the quantised student blocks by
+// gradient descent, and the paper names the straight-through estimator as the gradient rule of
+// 4-bit activations (Sec. 3, "Why QAT fails").  The forward is the deployed quantiser's code
+// dequantised, xhat = q * s, rounded once to bf16; the backward passes the gradient where the
+// unclamped code rint(fl32(x / s)) lies in [-8, 7] and writes +0 where the clamp acted.
+//
+// Both kernels stream HBM: the forward reads 2 bytes and writes 2 (xhat) + 1 (mask) per element
+// plus 4 bytes per group for the scales; the backward reads 2 + 1 and writes 2.
+#include <cstdint>
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+
+#include "kernels.cuh"
+
+namespace jq {
+namespace {
+
+constexpr int kFqThreads = 256;             // one block per row, 8 bf16 per thread per chunk
+constexpr int kFqChunk = kFqThreads * 8;    // elements of a row one pass of the block covers
+constexpr int kFqMaxGroups = kMaxK / 64;    // groups of a row at the smallest group size
+
+// bf16 of the exact product q * s, rounded once (nearest even).  The product of a 4-bit integer
+// and a 24-bit significand needs up to 28 bits; rounding it to fp32 and then to bf16 could round
+// twice.  Round to odd in fp32 instead (truncate, then set the last bit when the truncation was
+// inexact): with 24 >= 8 + 2 bits the final bf16 rounding of a round-to-odd value equals the
+// single rounding of the exact value (Boldo and Melquiond, "When double rounding is odd", 2005).
+// The fma residual q*s - rz(q*s) is exact; products here are never below the fp32 normal range
+// unless they are multiples of the subnormal quantum, hence exact.
+__device__ __forceinline__ uint16_t bf16_of_exact_product(float qf, float s) {
+  const float p = __fmul_rz(qf, s);
+  const float e = __fmaf_rn(qf, s, -p);
+  uint32_t b = __float_as_uint(p);
+  if (e != 0.0f) b |= 1u;
+  return __bfloat16_as_ushort(__float2bfloat16_rn(__uint_as_float(b)));
+}
+
+__device__ __forceinline__ float bf16_bits_to_f32(uint32_t b) { return __uint_as_float(b << 16); }
+
+__global__ void __launch_bounds__(kFqThreads) fake_quant_act_kernel(const uint16_t* __restrict__ x, int64_t M,
+                                                                     int64_t K, int G, const float* __restrict__ s_in,
+                                                                     uint16_t* __restrict__ xhat,
+                                                                     uint8_t* __restrict__ mask,
+                                                                     float* __restrict__ s_out) {
+  __shared__ float s_grp[kFqMaxGroups];  // per group of the row: amax bits, then the scale
+  const int tid = threadIdx.x;
+  const int lane = tid & 31;
+  const int ng = static_cast<int>(K / G);
+  // lanes that share a group within one 256-element warp span: G/8 for G = 64, 128; the warp
+  // for one group per row (G = K >= 256, where every lane of a warp lies in the same group)
+  const int seg = G >= 256 ? 32 : G / 8;
+  for (int64_t row = blockIdx.x; row < M; row += gridDim.x) {
+    const uint16_t* xr = x + row * K;
+    if (s_in != nullptr) {
+      for (int g = tid; g < ng; g += kFqThreads) s_grp[g] = s_in[row * ng + g];
+      __syncthreads();
+    } else {
+      for (int g = tid; g < ng; g += kFqThreads) reinterpret_cast<uint32_t*>(s_grp)[g] = 0u;
+      __syncthreads();
+      for (int64_t base = 0; base < K; base += kFqChunk) {  // uniform trip count across the block
+        const int64_t k = base + static_cast<int64_t>(tid) * 8;
+        const bool valid = k < K;
+        float m = 0.0f;
+        if (valid) {
+          const uint4 v = *reinterpret_cast<const uint4*>(xr + k);
+          const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+          for (int j = 0; j < 4; ++j) {
+            m = fmaxf(m, fabsf(bf16_bits_to_f32(w[j] & 0xFFFFu)));
+            m = fmaxf(m, fabsf(bf16_bits_to_f32(w[j] >> 16)));
+          }
+        }
+        for (int off = seg / 2; off > 0; off >>= 1) m = fmaxf(m, __shfl_xor_sync(0xFFFFFFFFu, m, off));
+        // the segment's first lane holds its smallest k: if any lane of the segment is in the row,
+        // that one is
+        if (valid && (lane % seg) == 0)
+          atomicMax(reinterpret_cast<unsigned int*>(s_grp) + k / G, __float_as_uint(m));  // m >= 0
+      }
+      __syncthreads();
+      for (int g = tid; g < ng; g += kFqThreads) {
+        const float amax = __uint_as_float(reinterpret_cast<uint32_t*>(s_grp)[g]);
+        s_grp[g] = amax == 0.0f ? 0.0f : __fdiv_rn(amax, 7.0f);
+      }
+      __syncthreads();
+    }
+    for (int g = tid; g < ng; g += kFqThreads) s_out[row * ng + g] = s_grp[g];
+    for (int64_t k = static_cast<int64_t>(tid) * 8; k < K; k += kFqChunk) {
+      const float s = s_grp[k / G];  // the 8 elements lie in one group: G % 8 == 0, k % 8 == 0
+      const uint4 v = *reinterpret_cast<const uint4*>(xr + k);
+      const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+      uint32_t out[4];
+      uint32_t mlo = 0, mhi = 0;
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
+        const float xv = bf16_bits_to_f32((w[j / 2] >> (16 * (j & 1))) & 0xFFFFu);
+        uint32_t h = 0, pass = 1;
+        if (s != 0.0f) {
+          const float r = rintf(__fdiv_rn(xv, s));  // IEEE division, then half to even
+          pass = (r >= -8.0f && r <= 7.0f) ? 1u : 0u;
+          const int q = static_cast<int>(fminf(fmaxf(r, -8.0f), 7.0f));
+          h = bf16_of_exact_product(static_cast<float>(q), s);  // code 0 gives +0
+        }
+        if (j & 1) out[j / 2] |= h << 16; else out[j / 2] = h;
+        if (j < 4) mlo |= pass << (8 * j); else mhi |= pass << (8 * (j - 4));
+      }
+      *reinterpret_cast<uint4*>(xhat + row * K + k) = make_uint4(out[0], out[1], out[2], out[3]);
+      *reinterpret_cast<uint2*>(mask + row * K + k) = make_uint2(mlo, mhi);
+    }
+    __syncthreads();  // s_grp is reused by the next row
+  }
+}
+
+__global__ void __launch_bounds__(kFqThreads) ste_backward_kernel(const uint16_t* __restrict__ grad,
+                                                                   const uint8_t* __restrict__ mask, int64_t n,
+                                                                   uint16_t* __restrict__ grad_x) {
+  const int64_t nvec = n / 8;
+  const int64_t stride = static_cast<int64_t>(gridDim.x) * kFqThreads;
+  for (int64_t i = static_cast<int64_t>(blockIdx.x) * kFqThreads + threadIdx.x; i < nvec; i += stride) {
+    const uint4 g = reinterpret_cast<const uint4*>(grad)[i];
+    const uint2 mk = reinterpret_cast<const uint2*>(mask)[i];
+    const uint32_t gw[4] = {g.x, g.y, g.z, g.w};
+    uint32_t out[4];
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      const uint32_t mb = j < 2 ? mk.x >> (16 * j) : mk.y >> (16 * (j - 2));  // two mask bytes
+      const uint32_t lo = (mb & 0xFFu) ? (gw[j] & 0xFFFFu) : 0u;
+      const uint32_t hi = ((mb >> 8) & 0xFFu) ? (gw[j] & 0xFFFF0000u) : 0u;
+      out[j] = lo | hi;
+    }
+    reinterpret_cast<uint4*>(grad_x)[i] = make_uint4(out[0], out[1], out[2], out[3]);
+  }
+  // the ragged tail (n % 8 elements), by the first threads of the grid
+  const int64_t t = nvec * 8 + static_cast<int64_t>(blockIdx.x) * kFqThreads + threadIdx.x;
+  if (t < n) grad_x[t] = mask[t] ? grad[t] : static_cast<uint16_t>(0);
+}
+
+}  // namespace
+
+cudaError_t launch_fake_quant_act(const void* x, int64_t M, int64_t K, int G, const float* s_in, void* xhat,
+                                  uint8_t* mask, float* s_out, cudaStream_t stream, int sms) {
+  const int64_t blocks = M < static_cast<int64_t>(sms) * 8 ? M : static_cast<int64_t>(sms) * 8;
+  fake_quant_act_kernel<<<static_cast<unsigned>(blocks), kFqThreads, 0, stream>>>(
+      static_cast<const uint16_t*>(x), M, K, G, s_in, static_cast<uint16_t*>(xhat), mask, s_out);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_ste_backward(const void* grad, const uint8_t* mask, int64_t n, void* grad_x, cudaStream_t stream,
+                                int sms) {
+  const int64_t want = (n / 8 + kFqThreads - 1) / kFqThreads;
+  int64_t blocks = want < static_cast<int64_t>(sms) * 8 ? want : static_cast<int64_t>(sms) * 8;
+  if (blocks < 1) blocks = 1;  // the tail alone (n < 8) still needs one block
+  ste_backward_kernel<<<static_cast<unsigned>(blocks), kFqThreads, 0, stream>>>(
+      static_cast<const uint16_t*>(grad), mask, n, static_cast<uint16_t*>(grad_x));
+  return cudaGetLastError();
+}
+
+}  // namespace jq

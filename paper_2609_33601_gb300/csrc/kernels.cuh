@@ -47,6 +47,13 @@ cudaError_t launch_pack_weight_ternary(const float* w, int64_t N, int64_t K, int
 // packed ternary codes [N, K/4] -> packed INT4 codes [N, K/2] (ternary.cu).
 cudaError_t launch_ternary_to_int4(const uint8_t* qw2, int64_t N, int64_t K, uint8_t* qw4, cudaStream_t stream,
                                    int sms);
+// bf16 activations [M, K] (dense rows) -> fake-quantised bf16 [M, K] + pass-through mask u8 [M, K]
+// + scales fp32 [M, K/G]; s_in (nullable) gives the scales instead of the amax rule (fakequant.cu).
+cudaError_t launch_fake_quant_act(const void* x, int64_t M, int64_t K, int G, const float* s_in, void* xhat,
+                                  uint8_t* mask, float* s_out, cudaStream_t stream, int sms);
+// straight-through backward: grad_x = grad where mask != 0, +0 elsewhere, n bf16 elements (fakequant.cu).
+cudaError_t launch_ste_backward(const void* grad, const uint8_t* mask, int64_t n, void* grad_x, cudaStream_t stream,
+                                int sms);
 // packed codes [rows, K/2] -> operand bytes [rows, K] + corrections [rows, K/G].
 cudaError_t launch_expand_operand(const uint8_t* packed, int64_t rows, int64_t K, int G, uint8_t* op, float* corr,
                                   cudaStream_t stream, int sms);

@@ -185,3 +185,43 @@ def test_header_is_plain_c_and_links_from_a_c_program(lib, tmp_path):
                    check=True, capture_output=True, text=True)
     r = subprocess.run([str(exe)], capture_output=True, text=True, timeout=60)
     assert r.returncode == 0 and r.stdout.strip() == "0", (r.returncode, r.stdout, r.stderr)
+
+
+def test_fake_quant_and_ste_entry_points_check_arguments(lib):
+    i64, i32, vp = ctypes.c_int64, ctypes.c_int32, ctypes.c_void_p
+    lib.jq_fake_quant_act.argtypes = [vp, i64, i64, i32, vp, vp, vp, vp, vp]
+    lib.jq_ste_backward.argtypes = [vp, vp, i64, vp, vp]
+    A = _fake(0x10000)
+    odd = _fake(0x10008)
+    fq = lib.jq_fake_quant_act
+    assert fq(None, 4, 256, 64, None, A, A, A, None) == INVALID
+    assert fq(A, 4, 256, 64, None, A, None, A, None) == INVALID      # the mask is required
+    assert fq(A, 4, 256, 32, None, A, A, A, None) == INVALID         # unsupported group
+    assert fq(A, 4, 192, 64, None, A, A, A, None) == INVALID         # K % 128 != 0
+    assert fq(A, -1, 256, 64, None, A, A, A, None) == INVALID
+    assert fq(A, 0, 256, 64, None, None, None, None, None) == OK     # M == 0 is a no-op
+    assert fq(A, 4, 256, 64, odd, A, A, A, None) == MISALIGNED       # given scales
+    assert fq(A, 4, 256, 64, None, A, odd, A, None) == MISALIGNED    # mask
+    st = lib.jq_ste_backward
+    assert st(A, A, -1, A, None) == INVALID
+    assert st(None, A, 8, A, None) == INVALID
+    assert st(A, A, 0, None, None) == OK                             # n == 0 is a no-op
+    assert st(A, odd, 8, A, None) == MISALIGNED
+    if not torch.cuda.is_available():
+        assert fq(A, 4, 256, 64, None, A, A, A, None) == UNSUPPORTED
+        assert st(A, A, 13, A, None) == UNSUPPORTED
+
+
+def test_fake_quant_binding_refuses_wrong_tensors():
+    import paper_2609_33601_gb300 as jq
+    x = torch.zeros((4, 256), dtype=torch.bfloat16)
+    with pytest.raises(ValueError, match="s_in"):
+        jq.jq_fake_quant_act(x, 64, torch.zeros((4, 3), dtype=torch.float32))
+    with pytest.raises(ValueError, match="dense rows"):
+        jq.jq_fake_quant_act(torch.zeros((4, 512), dtype=torch.bfloat16)[:, :256], 64)
+    with pytest.raises(ValueError, match="CUDA tensors only"):
+        jq.jq_fake_quant_act(x, 64)
+    with pytest.raises(ValueError, match="mask"):
+        jq.jq_ste_backward(x, torch.zeros((4, 255), dtype=torch.uint8))
+    with pytest.raises(ValueError, match="CUDA tensors only"):
+        jq.jq_ste_backward(x, torch.zeros((4, 256), dtype=torch.uint8))
