@@ -198,3 +198,15 @@ def test_fake_quant_linear_reproduces_the_deployed_layer():
     assert (np.abs(yf - y64) <= bound * 1.01 + 1e-12 * np.abs(y64)).all()
     # a dropped scale, sign or bias moves the result far outside that bound
     assert not (np.abs(-yf - y64) <= bound).all()
+
+
+def test_fp32_weight_path_rounds_to_nearest():
+    g = _golden()["fp32_rounding"]
+    s = np.float32(g["scale_numerator"] * 2.0 ** g["scale_exp2"])
+    w = np.zeros((1, 64), np.float32)
+    w[0, :2] = g["x"]
+    s_in = np.array([[s]], np.float32)
+    what, mask, _ = oracle.fake_quant_f32(w, 64, s_in)
+    assert [f"{v:08X}" for v in what[0, :2].view(np.uint32)] == g["what_f32_hex"] and mask.all()
+    xhat, _, _ = oracle.fake_quant_bf16(bf16_bits(w), 64, s_in)
+    assert [f"{v:04X}" for v in xhat[0, :2]] == g["xhat_bf16_hex"]
