@@ -225,6 +225,18 @@ JQ_API jq_status jq_fake_quant_act(const void* x_bf16, int64_t M, int64_t K, int
                                    void* xhat_bf16, uint8_t* mask, float* s_out, void* stream);
 
 /*
+ * Training side: fake quantisation of the student's fp32 weights, the same reading per output
+ * channel and K-group: what[n,k] = fl32(q * s) (one rounding of the exact product), with mask and
+ * scales as in jq_fake_quant_act.
+ *   w         : fp32 [N, K] row-major (device);  s_in : fp32 [N, K/group] or NULL (amax rule)
+ *   what      : fp32 [N, K] (output);  mask : uint8 [N, K] (output);  s_out : fp32 [N, K/group]
+ *               (output; row-major, unlike jq_pack_weight's group-major scales)
+ * Checks and errors as jq_fake_quant_act.
+ */
+JQ_API jq_status jq_fake_quant_weight(const float* w, int64_t N, int64_t K, int32_t group, const float* s_in,
+                                      float* what, uint8_t* mask, float* s_out, void* stream);
+
+/*
  * Training side: the straight-through backward (the reading above):
  *   grad_x[i] = grad[i] where mask[i] != 0, else +0.
  *   grad_bf16, grad_x_bf16 : bf16 [n] (device; grad_x may not overlap grad unless equal)

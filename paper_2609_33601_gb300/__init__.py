@@ -26,7 +26,8 @@ __all__ = [
     "JQError", "library_path", "jq_quantize_act", "jq_pack_weight", "jq_workspace_size", "jq_w4a4_linear",
     "jq_fused_quant_linear", "jq_w4a4_group_partials", "jq_device_status", "jq_status_string",
     "jq_w4a4_linear_noalloc", "jq_pack_weight_ternary", "jq_w158a4_workspace_size", "jq_w158a4_linear",
-    "jq_debug_wait_timeout", "jq_fake_quant_act", "jq_ste_backward",
+    "jq_debug_wait_timeout", "jq_fake_quant_act", "jq_fake_quant_weight",
+    "jq_ste_backward",
 ]
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
@@ -65,6 +66,7 @@ def _load() -> ctypes.CDLL:
                 "jq_debug_wait_timeout": [vp],
                 "jq_fake_quant_act": [vp, i64, i64, i32, vp, vp, vp, vp, vp],
                 "jq_ste_backward": [vp, vp, i64, vp, vp],
+                "jq_fake_quant_weight": [vp, i64, i64, i32, vp, vp, vp, vp, vp],
                 "jq_w4a4_linear_noalloc": [vp, vp, vp, vp, vp, vp, i64, i64, i64, i32, vp],
                 "jq_pack_weight_ternary": [vp, i64, i64, i32, vp, vp, vp],
                 "jq_w158a4_linear": [vp, vp, vp, vp, vp, vp, i64, i64, i64, i32, vp, sz, vp],
@@ -336,6 +338,24 @@ def jq_fake_quant_act(x: torch.Tensor, group: int, s_in: torch.Tensor | None = N
     _check(fn, _load().jq_fake_quant_act(_ptr(x), M, K, group, _ptr(s_in), _ptr(xhat), _ptr(mask), _ptr(s_out),
                                          _stream(stream)))
     return xhat, mask, s_out
+
+
+def jq_fake_quant_weight(w: torch.Tensor, group: int, s_in: torch.Tensor | None = None, stream=None):
+    """Training-side fake quantisation of fp32 weights [N, K]: (what fp32 [N, K], mask uint8 [N, K],
+    scales fp32 [N, K/G]); s_in, if given, is [N, K/G] fp32 positive scales."""
+    fn = "jq_fake_quant_weight"
+    if w.dim() != 2:
+        raise ValueError(f"{fn}: w must be 2-D, got shape {list(w.shape)}")
+    N, K = w.shape
+    _expect(fn, "w", w, torch.float32, (N, K), w.device)
+    _expect(fn, "s_in", s_in, torch.float32, (N, _groups(K, group)), w.device)
+    _need_cuda(w)
+    what = torch.empty((N, K), dtype=torch.float32, device=w.device)
+    mask = torch.empty((N, K), dtype=torch.uint8, device=w.device)
+    s_out = torch.empty((N, K // group if group else 0), dtype=torch.float32, device=w.device)
+    _check(fn, _load().jq_fake_quant_weight(_ptr(w), N, K, group, _ptr(s_in), _ptr(what), _ptr(mask), _ptr(s_out),
+                                            _stream(stream)))
+    return what, mask, s_out
 
 
 def jq_ste_backward(grad: torch.Tensor, mask: torch.Tensor, stream=None):

@@ -302,6 +302,20 @@ jq_status jq_fake_quant_act(const void* x_bf16, int64_t M, int64_t K, int32_t gr
                                              static_cast<cudaStream_t>(stream), d->sms));
 }
 
+jq_status jq_fake_quant_weight(const float* w, int64_t N, int64_t K, int32_t group, const float* s_in, float* what,
+                               uint8_t* mask, float* s_out, void* stream) {
+  if (N < 0 || !group_ok(K, group)) return JQ_ERR_INVALID_ARG;
+  if (N == 0) return JQ_OK;
+  if (w == nullptr || what == nullptr || mask == nullptr || s_out == nullptr) return JQ_ERR_INVALID_ARG;
+  if (!aligned16(w) || !aligned16(what) || !aligned16(mask) || !aligned16(s_out) ||
+      (s_in != nullptr && !aligned16(s_in)))
+    return JQ_ERR_MISALIGNED;
+  const DeviceInfo* d = current_device();
+  if (d == nullptr) return JQ_ERR_UNSUPPORTED;
+  return from_cuda(jq::launch_fake_quant_weight(w, N, K, group, s_in, what, mask, s_out,
+                                                static_cast<cudaStream_t>(stream), d->sms));
+}
+
 jq_status jq_ste_backward(const void* grad_bf16, const uint8_t* mask, int64_t n, void* grad_x_bf16, void* stream) {
   if (n < 0) return JQ_ERR_INVALID_ARG;
   if (n == 0) return JQ_OK;

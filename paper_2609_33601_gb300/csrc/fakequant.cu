@@ -5,8 +5,10 @@
 // dequantised, xhat = q * s, rounded once to bf16; the backward passes the gradient where the
 // unclamped code rint(fl32(x / s)) lies in [-8, 7] and writes +0 where the clamp acted.
 //
-// Both kernels stream HBM: the forward reads 2 bytes and writes 2 (xhat) + 1 (mask) per element
-// plus 4 bytes per group for the scales; the backward reads 2 + 1 and writes 2.
+// The same forward serves the student's fp32 weights (xhat = q * s rounded once to fp32).
+// Both kernels stream HBM: the bf16 forward reads 2 bytes and writes 2 (xhat) + 1 (mask) per
+// element plus 4 bytes per group for the scales (fp32: 4 + 4 + 1); the backward reads 2 + 1 and
+// writes 2.
 #include <cstdint>
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
@@ -37,11 +39,40 @@ __device__ __forceinline__ uint16_t bf16_of_exact_product(float qf, float s) {
 
 __device__ __forceinline__ float bf16_bits_to_f32(uint32_t b) { return __uint_as_float(b << 16); }
 
-__global__ void __launch_bounds__(kFqThreads) fake_quant_act_kernel(const uint16_t* __restrict__ x, int64_t M,
-                                                                     int64_t K, int G, const float* __restrict__ s_in,
-                                                                     uint16_t* __restrict__ xhat,
-                                                                     uint8_t* __restrict__ mask,
-                                                                     float* __restrict__ s_out) {
+// 8 consecutive elements (k % 8 == 0) widened to fp32, and xhat written back in the input's type.
+__device__ __forceinline__ void load8(const uint16_t* p, float v[8]) {
+  const uint4 u = *reinterpret_cast<const uint4*>(p);
+  const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+  for (int j = 0; j < 8; ++j) v[j] = bf16_bits_to_f32((w[j / 2] >> (16 * (j & 1))) & 0xFFFFu);
+}
+__device__ __forceinline__ void load8(const float* p, float v[8]) {
+  const float4 a = reinterpret_cast<const float4*>(p)[0], b = reinterpret_cast<const float4*>(p)[1];
+  v[0] = a.x; v[1] = a.y; v[2] = a.z; v[3] = a.w; v[4] = b.x; v[5] = b.y; v[6] = b.z; v[7] = b.w;
+}
+__device__ __forceinline__ void store8(uint16_t* p, const int q[8], float s) {
+  uint32_t out[4];
+#pragma unroll
+  for (int j = 0; j < 4; ++j)
+    out[j] = bf16_of_exact_product(static_cast<float>(q[2 * j]), s) |
+             (static_cast<uint32_t>(bf16_of_exact_product(static_cast<float>(q[2 * j + 1]), s)) << 16);
+  *reinterpret_cast<uint4*>(p) = make_uint4(out[0], out[1], out[2], out[3]);
+}
+// fp32 output: the IEEE product of the (exact) code and the scale is the single rounding of q*s.
+__device__ __forceinline__ void store8(float* p, const int q[8], float s) {
+  float o[8];
+#pragma unroll
+  for (int j = 0; j < 8; ++j) o[j] = __fmul_rn(static_cast<float>(q[j]), s);
+  reinterpret_cast<float4*>(p)[0] = make_float4(o[0], o[1], o[2], o[3]);
+  reinterpret_cast<float4*>(p)[1] = make_float4(o[4], o[5], o[6], o[7]);
+}
+
+// T = uint16_t: bf16 activations -> bf16 xhat; T = float: fp32 weights -> fp32 xhat.
+template <typename T>
+__global__ void __launch_bounds__(kFqThreads) fake_quant_kernel(const T* __restrict__ x, int64_t M, int64_t K, int G,
+                                                                 const float* __restrict__ s_in, T* __restrict__ xhat,
+                                                                 uint8_t* __restrict__ mask,
+                                                                 float* __restrict__ s_out) {
   __shared__ float s_grp[kFqMaxGroups];  // per group of the row: amax bits, then the scale
   const int tid = threadIdx.x;
   const int lane = tid & 31;
@@ -50,7 +81,7 @@ __global__ void __launch_bounds__(kFqThreads) fake_quant_act_kernel(const uint16
   // for one group per row (G = K >= 256, where every lane of a warp lies in the same group)
   const int seg = G >= 256 ? 32 : G / 8;
   for (int64_t row = blockIdx.x; row < M; row += gridDim.x) {
-    const uint16_t* xr = x + row * K;
+    const T* xr = x + row * K;
     if (s_in != nullptr) {
       for (int g = tid; g < ng; g += kFqThreads) s_grp[g] = s_in[row * ng + g];
       __syncthreads();
@@ -62,13 +93,10 @@ __global__ void __launch_bounds__(kFqThreads) fake_quant_act_kernel(const uint16
         const bool valid = k < K;
         float m = 0.0f;
         if (valid) {
-          const uint4 v = *reinterpret_cast<const uint4*>(xr + k);
-          const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+          float v[8];
+          load8(xr + k, v);
 #pragma unroll
-          for (int j = 0; j < 4; ++j) {
-            m = fmaxf(m, fabsf(bf16_bits_to_f32(w[j] & 0xFFFFu)));
-            m = fmaxf(m, fabsf(bf16_bits_to_f32(w[j] >> 16)));
-          }
+          for (int j = 0; j < 8; ++j) m = fmaxf(m, fabsf(v[j]));
         }
         for (int off = seg / 2; off > 0; off >>= 1) m = fmaxf(m, __shfl_xor_sync(0xFFFFFFFFu, m, off));
         // the segment's first lane holds its smallest k: if any lane of the segment is in the row,
@@ -86,24 +114,22 @@ __global__ void __launch_bounds__(kFqThreads) fake_quant_act_kernel(const uint16
     for (int g = tid; g < ng; g += kFqThreads) s_out[row * ng + g] = s_grp[g];
     for (int64_t k = static_cast<int64_t>(tid) * 8; k < K; k += kFqChunk) {
       const float s = s_grp[k / G];  // the 8 elements lie in one group: G % 8 == 0, k % 8 == 0
-      const uint4 v = *reinterpret_cast<const uint4*>(xr + k);
-      const uint32_t w[4] = {v.x, v.y, v.z, v.w};
-      uint32_t out[4];
+      float v[8];
+      load8(xr + k, v);
+      int q[8];
       uint32_t mlo = 0, mhi = 0;
 #pragma unroll
       for (int j = 0; j < 8; ++j) {
-        const float xv = bf16_bits_to_f32((w[j / 2] >> (16 * (j & 1))) & 0xFFFFu);
-        uint32_t h = 0, pass = 1;
+        uint32_t pass = 1;
+        q[j] = 0;  // an all-zero group (s = 0): xhat = +0, mask 1
         if (s != 0.0f) {
-          const float r = rintf(__fdiv_rn(xv, s));  // IEEE division, then half to even
+          const float r = rintf(__fdiv_rn(v[j], s));  // IEEE division, then half to even
           pass = (r >= -8.0f && r <= 7.0f) ? 1u : 0u;
-          const int q = static_cast<int>(fminf(fmaxf(r, -8.0f), 7.0f));
-          h = bf16_of_exact_product(static_cast<float>(q), s);  // code 0 gives +0
+          q[j] = static_cast<int>(fminf(fmaxf(r, -8.0f), 7.0f));  // code 0 gives +0 below
         }
-        if (j & 1) out[j / 2] |= h << 16; else out[j / 2] = h;
         if (j < 4) mlo |= pass << (8 * j); else mhi |= pass << (8 * (j - 4));
       }
-      *reinterpret_cast<uint4*>(xhat + row * K + k) = make_uint4(out[0], out[1], out[2], out[3]);
+      store8(xhat + row * K + k, q, s);
       *reinterpret_cast<uint2*>(mask + row * K + k) = make_uint2(mlo, mhi);
     }
     __syncthreads();  // s_grp is reused by the next row
@@ -139,8 +165,16 @@ __global__ void __launch_bounds__(kFqThreads) ste_backward_kernel(const uint16_t
 cudaError_t launch_fake_quant_act(const void* x, int64_t M, int64_t K, int G, const float* s_in, void* xhat,
                                   uint8_t* mask, float* s_out, cudaStream_t stream, int sms) {
   const int64_t blocks = M < static_cast<int64_t>(sms) * 8 ? M : static_cast<int64_t>(sms) * 8;
-  fake_quant_act_kernel<<<static_cast<unsigned>(blocks), kFqThreads, 0, stream>>>(
+  fake_quant_kernel<uint16_t><<<static_cast<unsigned>(blocks), kFqThreads, 0, stream>>>(
       static_cast<const uint16_t*>(x), M, K, G, s_in, static_cast<uint16_t*>(xhat), mask, s_out);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_fake_quant_weight(const float* w, int64_t N, int64_t K, int G, const float* s_in, float* what,
+                                     uint8_t* mask, float* s_out, cudaStream_t stream, int sms) {
+  const int64_t blocks = N < static_cast<int64_t>(sms) * 8 ? N : static_cast<int64_t>(sms) * 8;
+  fake_quant_kernel<float><<<static_cast<unsigned>(blocks), kFqThreads, 0, stream>>>(w, N, K, G, s_in, what, mask,
+                                                                                     s_out);
   return cudaGetLastError();
 }
 

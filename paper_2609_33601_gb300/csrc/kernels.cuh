@@ -51,6 +51,9 @@ cudaError_t launch_ternary_to_int4(const uint8_t* qw2, int64_t N, int64_t K, uin
 // + scales fp32 [M, K/G]; s_in (nullable) gives the scales instead of the amax rule (fakequant.cu).
 cudaError_t launch_fake_quant_act(const void* x, int64_t M, int64_t K, int G, const float* s_in, void* xhat,
                                   uint8_t* mask, float* s_out, cudaStream_t stream, int sms);
+// fp32 weights [N, K] -> fake-quantised fp32 [N, K] + mask u8 [N, K] + scales fp32 [N, K/G] (fakequant.cu).
+cudaError_t launch_fake_quant_weight(const float* w, int64_t N, int64_t K, int G, const float* s_in, float* what,
+                                     uint8_t* mask, float* s_out, cudaStream_t stream, int sms);
 // straight-through backward: grad_x = grad where mask != 0, +0 elsewhere, n bf16 elements (fakequant.cu).
 cudaError_t launch_ste_backward(const void* grad, const uint8_t* mask, int64_t n, void* grad_x, cudaStream_t stream,
                                 int sms);

@@ -202,6 +202,14 @@ def test_fake_quant_and_ste_entry_points_check_arguments(lib):
     assert fq(A, 0, 256, 64, None, None, None, None, None) == OK     # M == 0 is a no-op
     assert fq(A, 4, 256, 64, odd, A, A, A, None) == MISALIGNED       # given scales
     assert fq(A, 4, 256, 64, None, A, odd, A, None) == MISALIGNED    # mask
+    lib.jq_fake_quant_weight.argtypes = [vp, i64, i64, i32, vp, vp, vp, vp, vp]
+    fw = lib.jq_fake_quant_weight
+    assert fw(None, 4, 256, 64, None, A, A, A, None) == INVALID
+    assert fw(A, 4, 256, 96, None, A, A, A, None) == INVALID
+    assert fw(A, 0, 256, 64, None, None, None, None, None) == OK
+    assert fw(A, 4, 256, 64, None, odd, A, A, None) == MISALIGNED
+    if not torch.cuda.is_available():
+        assert fw(A, 4, 256, 64, None, A, A, A, None) == UNSUPPORTED
     st = lib.jq_ste_backward
     assert st(A, A, -1, A, None) == INVALID
     assert st(None, A, 8, A, None) == INVALID
@@ -221,6 +229,10 @@ def test_fake_quant_binding_refuses_wrong_tensors():
         jq.jq_fake_quant_act(torch.zeros((4, 512), dtype=torch.bfloat16)[:, :256], 64)
     with pytest.raises(ValueError, match="CUDA tensors only"):
         jq.jq_fake_quant_act(x, 64)
+    with pytest.raises(ValueError, match="s_in"):
+        jq.jq_fake_quant_weight(torch.zeros((8, 256)), 128, torch.zeros((8, 1)))
+    with pytest.raises(ValueError, match="CUDA tensors only"):
+        jq.jq_fake_quant_weight(torch.zeros((8, 256)), 128)
     with pytest.raises(ValueError, match="mask"):
         jq.jq_ste_backward(x, torch.zeros((4, 255), dtype=torch.uint8))
     with pytest.raises(ValueError, match="CUDA tensors only"):

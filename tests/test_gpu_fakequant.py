@@ -1,7 +1,7 @@
 """GPU parity of the training-side fake quantisation and straight-through backward.
 
-jq_fake_quant_act and jq_ste_backward against the oracle (oracle_fake_quant_bf16,
-oracle_ste_backward_bf16) on the same seeded inputs, bit for bit: the scales, the 0/1 mask and
+jq_fake_quant_act, jq_fake_quant_weight and jq_ste_backward against the oracle
+(oracle_fake_quant_bf16, oracle_fake_quant_f32, oracle_ste_backward_bf16) on the same seeded inputs, bit for bit: the scales, the 0/1 mask and
 the bf16 xhat (one rounding of the exact product q*s) are all decided in the same fp32 steps
 on both sides, so nothing here needs a tolerance.  Shapes cover several 2048-element row
 chunks with a ragged last chunk, one group per row with a partly filled warp (K = 384), rows
@@ -101,3 +101,19 @@ def test_forward_mask_feeds_the_backward():
     gx = jq.jq_ste_backward(grad, mask)
     keep = mask.bool()
     assert torch.equal(gx[keep], grad[keep]) and (gx[~keep].view(torch.int16) == 0).all()
+
+
+@pytest.mark.parametrize("N,K,G,given", [(256, 256, 64, False), (96, 384, 384, False), (300, 4096, 128, False),
+                                         (1300, 128, 128, False), (40, 2304, 128, True)])
+def test_weight_fake_quant_matches_the_oracle(N, K, G, given):
+    rng = np.random.default_rng(N + K)
+    w = (rng.standard_normal((N, K)) * 0.02).astype(np.float32)
+    w[1, :G] = 0  # an all-zero group
+    s_in = rng.uniform(0.001, 0.006, (N, K // G)).astype(np.float32) if given else None
+    what, mask, s = jq.jq_fake_quant_weight(torch.from_numpy(w).cuda(), G,
+                                            None if s_in is None else torch.from_numpy(s_in).cuda())
+    ow, om, os_ = oracle.fake_quant_f32(w, G, s_in)
+    assert (s.cpu().numpy().view(np.uint32) == os_.view(np.uint32)).all()
+    assert (mask.cpu().numpy() == om).all()
+    assert (what.cpu().numpy().view(np.uint32) == ow.view(np.uint32)).all()
+    assert om.all() != given  # the amax rule never clamps; these small given scales do
