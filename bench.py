@@ -1,13 +1,21 @@
 """Benchmark of the naive W4A4 linear layer (JustQuant, arxiv 2609.33601) on GB300.
 
-    python bench.py [--gpus N] [--steps K] [--warmup W] [--workload dllm] [--impl ours|reference]
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--workload flux_qkv] [--impl ours|reference]
 
 One step = one pass of the deployed hot path over one batch: the activation quantiser
 (jq_quantize_act) followed by the W4A4 GEMM with its dequantise + bias epilogue
-(jq_w4a4_linear), on the dLLM gate/up projection (M=1024 tokens x K=4096 -> N=12288,
-group128).  Weights are packed once, offline, as the paper's deployment does.  Six input/weight
-sets (about 200 MB, more than the 129 MB L2) rotate between steps, so every step streams its
-operands from HBM.  Metric: W4A4 linear TOPS (2*M*N*K per step), whole job over all ranks.
+(jq_w4a4_linear).  The default workload is the largest single-GPU configuration, the FLUX-style
+12B DiT's fused QKV+MLP-in projection (M=4608 tokens x K=3072 -> N=21504, group64, the FLUX
+setting of Sec. 4.2 and the Appendix "FLUX experimental details").  Weights are packed once,
+offline, as the paper's deployment does.  Rotating input/weight sets, together several times
+larger than the 129 MB L2, make every step stream its operands from HBM.  Metric: W4A4 linear
+TOPS (2*M*N*K per step), whole job over all ranks.
+
+Other workloads (--workload): the dLLM gate/up projection (group128), the FLUX output
+projection (also as the fused call, --fused), the M sweep of the memory-to-compute crossover,
+and, as their own lines, the memory-bound kernels alone: the activation quantiser, the
+training-side fake quantisation and the straight-through backward (GB/s against the HBM copy
+rate).
 
 Under torchrun each rank runs its own replica of the workload (the layer shards along tokens
 with no exchange), so scaling is weak and no collective sits on the data path; a barrier and a
@@ -65,13 +73,15 @@ PEAKS_PATH = os.path.join(ROOT, "MEASURED_PEAKS.json")
 FP8_PER_BF16 = 2.0  # nominal dense FP8 / BF16 tensor-core ratio on GB300 (4.5 / 2.25 PFLOP/s)
 
 # DRAM traffic of one launch of the dominant kernel (dram__bytes_read.sum + dram__bytes_write.sum)
-# from the ncu captures summarised in profiles/, keyed by workload and by the hash of the kernel
-# code the capture was taken on (kernel_hash); once the code changes the figure no longer applies
-# and the bench reports null.
-KERNEL_TRAFFIC = {
-    ("dllm", "c9988b74e5543425"): 31.244e6 + 0.119e6,  # profiles/w4a4_gemm_dllm_full.md
-    ("sweep_m1", "20541bf7a20396bf"): 25.303e6,  # profiles/w4a4_skinny_sweep_m1_full.md
-}
+# from an ncu capture of that kernel, keyed by workload and by the hash of the kernel code the
+# capture was taken on (kernel_hash); once the code changes the figure no longer applies and the
+# bench reports null until a new capture is recorded here.
+KERNEL_TRAFFIC: dict = {}
+
+
+def recorded_traffic(workload: str, kernel_file: str):
+    """The captured DRAM bytes per launch for this workload on the current kernel code, or None."""
+    return KERNEL_TRAFFIC.get((workload, kernel_hash(kernel_file)))
 
 
 def kernel_hash(kernel_file: str) -> str:
@@ -268,6 +278,23 @@ def run_reference(args):
     return 0
 
 
+def run_stream_reference(args):
+    """The reference arm of a memory-bound kernel line: the oracle's version on the host cores."""
+    rank, world, _ = dist_env()
+    if rank != 0:
+        return 0
+    o = StreamOracle(args.workload)
+    cb = o.baseline(min(args.ref_seconds, 120.0 / (args.steps + args.warmup)))
+    line = {"impl": "reference", "metric": STREAM_METRIC[o.op], "value": cb["value"], "unit": "GB/s",
+            "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "bf16" if o.op != "fq_weight" else "f32",
+            "data": "synthetic", "config": {"workload": o.desc, "rows": o.M, "K": o.K, "group": o.G},
+            "cpu_baseline": cb, "e2e": {"value": cb["value"], "unit": "GB/s", "h2d_bytes_per_step": 0,
+                                        "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+    return 0
+
+
 # ----------------------------------------------------------------------------- context
 
 def cublas_context(torch, dev, sets, M, N, K, args, world):
@@ -305,6 +332,235 @@ def cublas_context(torch, dev, sets, M, N, K, args, world):
     torch.cuda.empty_cache()
     return {"value": world * 2.0 * M * N * K / (ms * 1e-3) / 1e12, "unit": "TFLOP/s", "ms_per_call": ms,
             "what": "torch.matmul bf16 x[M,K] @ W[N,K]^T, same M, N, K"}
+
+
+# ----------------------------------------------------------------------------- memory-bound kernels
+
+# The HBM-bound kernels of the library timed alone: name -> (description, op, rows, K, G, generator).
+# op: "quantize" (jq_quantize_act), "fq_act" (jq_fake_quant_act), "fq_weight"
+# (jq_fake_quant_weight, fp32 rows), "ste" (jq_ste_backward over rows x K gradients).
+STREAM_WORKLOADS = {
+    "quant_dllm": ("activation quantiser on the dLLM activations: 1024 x 4096 bf16, group128", "quantize", 1024,
+                   4096, 128, "dllm"),
+    "quant_flux_out": ("activation quantiser on the FLUX output projection's input: 4608 x 15360 bf16, group64",
+                       "quantize", 4608, 15360, 64, "flux_out"),
+    "fq_act_dllm": ("training-side fake quantisation of activations: 1024 x 4096 bf16, group128", "fq_act", 1024,
+                    4096, 128, "dllm"),
+    "fq_act_flux_out": ("training-side fake quantisation of activations: 4608 x 15360 bf16, group64", "fq_act",
+                        4608, 15360, 64, "flux_out"),
+    "fq_w_flux_qkv": ("training-side fake quantisation of the student's fp32 weights: 21504 x 3072, group64",
+                      "fq_weight", 21504, 3072, 64, "flux_qkv"),
+    "ste_dllm": ("straight-through backward: 1024 x 4096 bf16 gradients and their pass-through mask", "ste", 1024,
+                 4096, 128, "dllm"),
+    "ste_flux_out": ("straight-through backward: 4608 x 15360 bf16 gradients and their pass-through mask", "ste",
+                     4608, 15360, 64, "flux_out"),
+}
+STREAM_METRIC = {"quantize": "activation quantiser GB/s", "fq_act": "fake-quant (activations) GB/s",
+                 "fq_weight": "fake-quant (weights) GB/s", "ste": "STE backward GB/s"}
+
+
+def stream_bytes(op: str, rows: int, K: int, G: int) -> float:
+    """Algorithmic HBM bytes of one launch: every input read once, every output written once."""
+    n = rows * K
+    if op == "quantize":
+        return 2 * n + n / 2 + 4 * n / G      # bf16 in; packed codes, scales out
+    if op == "fq_act":
+        return 2 * n + 2 * n + n + 4 * n / G  # bf16 in; bf16 x-hat, mask, scales out
+    if op == "fq_weight":
+        return 4 * n + 4 * n + n + 4 * n / G  # fp32 in; fp32 w-hat, mask, scales out
+    if op == "ste":
+        return 2 * n + n + 2 * n              # bf16 gradient and mask in; bf16 gradient out
+    raise KeyError(op)
+
+
+class StreamOracle:
+    """The CPU oracle's version of a memory-bound kernel on a bounded row sample."""
+
+    def __init__(self, name: str, seed: int = 7):
+        import oracle
+        from paper_2609_33601_gb300 import workloads as wl
+        self.oracle = oracle
+        self.desc, self.op, self.M, self.K, self.G, gen = STREAM_WORKLOADS[name]
+        rows = min(self.M, 512)
+        if self.op == "fq_weight":
+            self.x = wl.make(gen, seed=seed, M=1, N=rows, K=self.K, G=self.G).w
+        else:
+            self.x = wl.make(gen, seed=seed, M=rows, K=self.K, G=self.G, with_weights=False).x_bits
+        self.mask = (np.arange(self.x.size).reshape(self.x.shape) % 7 != 0).astype(np.uint8)
+        self.rows = 8
+
+    def run(self, rows: int) -> float:
+        t0 = time.perf_counter()
+        x = self.x[:rows]
+        if self.op == "quantize":
+            self.oracle.quantize_bf16(x, self.G)
+        elif self.op == "fq_act":
+            self.oracle.fake_quant_bf16(x, self.G)
+        elif self.op == "fq_weight":
+            self.oracle.fake_quant_f32(x, self.G)
+        else:
+            self.oracle.ste_backward_bf16(x, self.mask[:rows])
+        return time.perf_counter() - t0
+
+    def baseline(self, target_s: float) -> dict:
+        rows = 8
+        while True:
+            dt = self.run(rows)
+            if dt >= 0.8 * target_s or rows >= len(self.x):
+                break
+            rows = min(len(self.x), max(rows * 2, int(rows * target_s / max(dt, 1e-4))))
+        reps = max(1, int(target_s / max(dt, 1e-4)))
+        t = sum(self.run(rows) for _ in range(reps)) / reps
+        return {"value": stream_bytes(self.op, rows, self.K, self.G) / t / 1e9, "unit": "GB/s",
+                "cores": min(self.oracle.max_threads(), rows), "kind": "oracle", "host_threads": os.cpu_count(),
+                "sample": f"{rows} of {self.M} rows, {reps} repetition(s) of {t:.3f} s"}
+
+
+def run_stream(args):
+    """Times one memory-bound kernel alone: a CUDA graph of K launches over rotating buffers that
+    together exceed L2 several times over, so every launch reads and writes HBM."""
+    import torch
+
+    rank, world, local = dist_env()
+    torch.cuda.set_device(local)
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    from paper_2609_33601_gb300 import build as jq_build
+    jq_build.build()
+    import paper_2609_33601_gb300 as jq
+    from paper_2609_33601_gb300 import workloads as wl
+
+    desc, op, M, K, G, gen = STREAM_WORKLOADS[args.workload]
+    dev = torch.device("cuda", local)
+    alg = stream_bytes(op, M, K, G)
+    n_sets = max(3, -(-int(1.2e9) // int(alg)))
+    if op == "fq_weight":
+        base = torch.from_numpy(wl.make(gen, seed=100 + rank, M=1, N=M, K=K, G=G).w).to(dev)
+    else:
+        base = torch.from_numpy(wl.make(gen, seed=100 + rank, M=M, K=K, G=G, with_weights=False).x_bits
+                                .view(np.int16)).to(dev).view(torch.bfloat16)
+    mask0 = (torch.arange(M * K, device=dev).reshape(M, K) % 7 != 0).to(torch.uint8)
+    sets = []
+    for i in range(n_sets):
+        # each set its own inputs and outputs (the row order rolled, so no two sets share lines)
+        x = torch.roll(base, shifts=i * 37, dims=0).contiguous()
+        if op == "quantize":
+            outs = (torch.empty((M, K // 2), dtype=torch.uint8, device=dev),
+                    torch.empty((M, K // G), dtype=torch.float32, device=dev))
+        elif op == "ste":
+            outs = (torch.roll(mask0, shifts=i, dims=0).contiguous(),)
+        else:
+            outs = ()
+        sets.append((x, outs))
+    torch.cuda.synchronize()
+
+    def launch(i, st):
+        x, outs = sets[i % n_sets]
+        if op == "quantize":
+            jq.jq_quantize_act(x, G, outs[0], outs[1], stream=st)
+        elif op == "fq_act":
+            jq.jq_fake_quant_act(x, G, stream=st)
+        elif op == "fq_weight":
+            jq.jq_fake_quant_weight(x, G, stream=st)
+        else:
+            jq.jq_ste_backward(x, outs[0], stream=st)
+
+    stream = torch.cuda.current_stream()
+    for i in range(args.warmup):
+        launch(i, stream)
+    torch.cuda.synchronize()
+    # the fake-quant calls allocate their outputs: capture them in the graph's private pool
+    cap = torch.cuda.Stream()
+    cap.wait_stream(stream)
+    with torch.cuda.stream(cap):
+        for i in range(args.warmup):
+            launch(i, cap)
+    cap.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=cap):
+        for i in range(args.steps):
+            launch(i, cap)
+    g.replay()
+    torch.cuda.synchronize()
+    t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+    torch.cuda.synchronize()
+    with ClockSampler(local) as clocks:
+        t0.record(stream)
+        g.replay()
+        t1.record(stream)
+        torch.cuda.synchronize()
+    (ms,) = max_over_ranks([t0.elapsed_time(t1)], dev)
+    assert jq.jq_device_status() == 0, "a kernel reported a bounded-wait timeout"
+
+    # end to end through the public API: host input copied in and the outputs copied out per step
+    x_host = sets[0][0].cpu().pin_memory()
+    x_dev = torch.empty_like(sets[0][0])
+    host_outs = {}
+
+    def e2e_step(i):
+        x_dev.copy_(x_host, non_blocking=True)
+        if op == "quantize":
+            q, sa = jq.jq_quantize_act(x_dev, G)
+            res = (q, sa)
+        elif op == "fq_act":
+            res = jq.jq_fake_quant_act(x_dev, G)
+        elif op == "fq_weight":
+            res = jq.jq_fake_quant_weight(x_dev, G)
+        else:
+            res = (jq.jq_ste_backward(x_dev, sets[0][1][0]),)
+        for j, r in enumerate(res):
+            if j not in host_outs:
+                host_outs[j] = torch.empty(r.shape, dtype=r.dtype).pin_memory()
+            host_outs[j].copy_(r, non_blocking=True)
+
+    for i in range(args.warmup):
+        e2e_step(i)
+    torch.cuda.synchronize()
+    e0 = time.perf_counter()
+    for i in range(args.steps):
+        e2e_step(i)
+    torch.cuda.synchronize()
+    (e2e_s,) = max_over_ranks([time.perf_counter() - e0], dev)
+    h2d = sets[0][0].numel() * sets[0][0].element_size()
+    d2h = sum(t.numel() * t.element_size() for t in host_outs.values())
+
+    _, hbm_peak, peak_src = measured_peaks()
+    gbs = world * alg * args.steps / (ms * 1e-3) / 1e9
+    per_launch = alg / (ms / args.steps * 1e-3) / 1e9
+    if rank != 0:
+        if world > 1:
+            import torch.distributed as dist
+            dist.destroy_process_group()
+        return 0
+    cpu = None
+    if world == 1 and not args.no_cpu_baseline:
+        cpu = StreamOracle(args.workload).baseline(args.ref_seconds)
+    line = {
+        "metric": STREAM_METRIC[op], "value": gbs, "unit": "GB/s", "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": ms / args.steps, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "bf16" if op != "fq_weight" else "f32", "data": "synthetic",
+        "config": {"workload": desc, "rows": M, "K": K, "group": G, "launch": "CUDA graph of the K launches",
+                   "parallelism": f"replicas x{world}",
+                   "l2": f"{n_sets} rotating input/output sets, {n_sets * alg / 1e9:.2f} GB in all"},
+        "roofline": {"bound": "hbm", "achieved": per_launch, "peak": hbm_peak, "unit": "GB/s",
+                     "frac": per_launch / hbm_peak, "traffic": None, "algorithmic_bytes": alg,
+                     "kernel": f"{op} kernel alone, CUDA events around a graph of K launches",
+                     "peak_source": f"{peak_src} HBM copy bandwidth {hbm_peak} GB/s"},
+        "cpu_baseline": cpu,
+        "e2e": {"value": world * alg * args.steps / e2e_s / 1e9, "unit": "GB/s", "h2d_bytes_per_step": h2d,
+                "d2h_bytes_per_step": d2h, "copies": "pinned host buffers, on the compute stream around the kernel"},
+        "gpu_launches": args.steps,
+        "clocks": clocks.summary(),
+    }
+    print(json.dumps(line), flush=True)
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+    return 0
 
 
 # ----------------------------------------------------------------------------- our arm
@@ -481,7 +737,7 @@ def run_ours(args):
     bf16_peak, hbm_peak, peak_src = measured_peaks()
     fp8_peak = bf16_peak * FP8_PER_BF16
     kernel_file = "skinny.cu" if few else "gemm.cu"
-    traffic = None if (fused or ternary) else KERNEL_TRAFFIC.get((args.workload, kernel_hash(kernel_file)))
+    traffic = None if (fused or ternary) else recorded_traffic(args.workload, kernel_file)
     # algorithmic bytes of one linear call: packed weights and their scales, packed activation
     # codes and scales (the fused call reads bf16 activations instead), bias, bf16 output
     groups = K // G
@@ -555,7 +811,7 @@ def main():
     ap.add_argument("--steps", type=int, default=50)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
-    ap.add_argument("--workload", choices=sorted(WORKLOADS), default="dllm")
+    ap.add_argument("--workload", choices=sorted(WORKLOADS) + sorted(STREAM_WORKLOADS), default="flux_qkv")
     ap.add_argument("--sets", type=int, default=0, help="rotating input/weight sets (0: enough for > 3x L2)")
     ap.add_argument("--ref-seconds", type=float, default=10.0, help="CPU seconds per oracle sample")
     ap.add_argument("--ref-single-seconds", type=float, default=5.0,
@@ -570,6 +826,10 @@ def main():
         ap.error("--warmup must be at least 3")
     if args.fused and args.weights == "ternary":
         ap.error("--fused is an INT4-weight call")
+    if args.workload in STREAM_WORKLOADS:
+        if args.impl == "reference":
+            return run_stream_reference(args)
+        return run_stream(args)
     if args.impl == "reference":
         return run_reference(args)
     return run_ours(args)

@@ -99,10 +99,31 @@ def _stream(stream=None):
     return ctypes.c_void_p(s.cuda_stream)
 
 
-def _need_cuda(*ts):
+def _device_mismatch(device, current: int, stream_device=None) -> str | None:
+    """Why tensors on `device` cannot go to a library call made with CUDA device `current` and a
+    stream of `stream_device`, or None when they can.  The C calls launch on the current device
+    and address its memory, so tensors of another GPU would be read there as foreign pointers."""
+    if device.index is not None and device.index != current:
+        return (f"the tensors are on {device} but the current CUDA device is cuda:{current}; "
+                f"call inside `with torch.cuda.device({device.index}):`")
+    if stream_device is not None and stream_device != device:
+        return f"the stream belongs to {stream_device}, the tensors to {device}"
+    return None
+
+
+def _need_cuda(*ts, stream=None):
+    """Every tensor is a CUDA tensor on the current device, and the stream (if given) is one of
+    that device (the tensors' agreement with one another is checked by _expect)."""
+    dev = None
     for t in ts:
         if t is not None and not t.is_cuda:
             raise ValueError("libjq works on CUDA tensors only")
+        if t is not None and dev is None:
+            dev = t.device
+    if dev is not None:
+        why = _device_mismatch(dev, torch.cuda.current_device(), None if stream is None else stream.device)
+        if why is not None:
+            raise ValueError(f"libjq: {why}")
 
 
 def _groups(K: int, group: int):
@@ -183,7 +204,7 @@ def jq_quantize_act(x: torch.Tensor, group: int, q: torch.Tensor | None = None, 
     M, K = x.shape
     _expect(fn, "q", q, torch.uint8, (M, K // 2), x.device)
     _expect(fn, "s_a", s_a, torch.float32, (M, _groups(K, group)), x.device)
-    _need_cuda(x)
+    _need_cuda(x, stream=stream)
     if q is None:
         q = torch.empty((M, K // 2), dtype=torch.uint8, device=x.device)
     if s_a is None:
@@ -199,7 +220,7 @@ def jq_pack_weight(w: torch.Tensor, group: int, stream=None):
         raise ValueError(f"jq_pack_weight: w must be 2-D, got shape {list(w.shape)}")
     N, K = w.shape
     _expect("jq_pack_weight", "w", w, torch.float32, (N, K), w.device)
-    _need_cuda(w)
+    _need_cuda(w, stream=stream)
     qw = torch.empty((N, K // 2), dtype=torch.uint8, device=w.device)
     s_w = torch.empty((K // group if group else 0, N), dtype=torch.float32, device=w.device)
     _check("jq_pack_weight", _load().jq_pack_weight(_ptr(w), N, K, group, _ptr(qw), _ptr(s_w), _stream(stream)))
@@ -211,7 +232,7 @@ def jq_w4a4_linear(q, s_a, qw, s_w, bias, group: int, y=None, workspace=None, st
     fn = "jq_w4a4_linear"
     M, K, N = _codes_shapes(fn, q, qw, 2)
     _expect_linear(fn, M, N, K, group, q.device, s_a, s_w, bias, y, workspace)
-    _need_cuda(q, s_a, qw, s_w, bias)
+    _need_cuda(q, s_a, qw, s_w, bias, stream=stream)
     if y is None:
         y = torch.empty((M, N), dtype=torch.bfloat16, device=q.device)
     ws, ws_bytes = _workspace(M, N, K, group, False, q.device, workspace)
@@ -222,13 +243,16 @@ def jq_w4a4_linear(q, s_a, qw, s_w, bias, group: int, y=None, workspace=None, st
 
 def jq_w4a4_linear_noalloc(q, s_a, qw, s_w, bias, group: int, y=None, stream=None):
     """jq_w4a4_linear without a workspace, for callers that cannot allocate device memory: the
-    library keeps the scratch in its own fixed device array (ceil(M/128)*128*K <= 16 MiB).  Calls share that
-    array, so order them on one stream.  (Only the output tensor is allocated here, by the
-    caller's side, when y is None.)"""
+    library keeps the scratch in its own fixed 16 MiB device array.  More than 64 tokens (and
+    one-group problems with K above 139776) need
+    ceil(M/128)*128*K + round_up(4*M*(K/G), 256) <= 16 MiB
+    (the operand image, then one fp32 correction per token and group); larger calls raise
+    JQError(JQ_ERR_WORKSPACE).  Calls share that array, so order them on one stream.  (Only the
+    output tensor is allocated here, by the caller's side, when y is None.)"""
     fn = "jq_w4a4_linear_noalloc"
     M, K, N = _codes_shapes(fn, q, qw, 2)
     _expect_linear(fn, M, N, K, group, q.device, s_a, s_w, bias, y, None)
-    _need_cuda(q, s_a, qw, s_w, bias)
+    _need_cuda(q, s_a, qw, s_w, bias, stream=stream)
     if y is None:
         y = torch.empty((M, N), dtype=torch.bfloat16, device=q.device)
     _check("jq_w4a4_linear_noalloc",
@@ -247,7 +271,7 @@ def jq_fused_quant_linear(x, qw, s_w, bias, group: int, y=None, workspace=None, 
     N = qw.shape[0]
     _expect(fn, "qw", qw, torch.uint8, (N, K // 2), x.device)
     _expect_linear(fn, M, N, K, group, x.device, None, s_w, bias, y, workspace)
-    _need_cuda(x, qw, s_w, bias)
+    _need_cuda(x, qw, s_w, bias, stream=stream)
     if y is None:
         y = torch.empty((M, N), dtype=torch.bfloat16, device=x.device)
     ws, ws_bytes = _workspace(M, N, K, group, True, x.device, workspace)
@@ -264,7 +288,7 @@ def jq_w4a4_group_partials(q, qw, group: int, workspace=None, stream=None):
     if _groups(K, group) is None:
         raise ValueError(f"{fn}: group {group} does not divide K = {K}")
     _expect_workspace(fn, workspace, q.device)
-    _need_cuda(q, qw)
+    _need_cuda(q, qw, stream=stream)
     acc = torch.empty((M, N, K // group), dtype=torch.int32, device=q.device)
     ws, ws_bytes = _workspace(M, N, K, group, False, q.device, workspace)
     _check("jq_w4a4_group_partials",
@@ -279,7 +303,7 @@ def jq_pack_weight_ternary(w: torch.Tensor, group: int, stream=None):
         raise ValueError(f"jq_pack_weight_ternary: w must be 2-D, got shape {list(w.shape)}")
     N, K = w.shape
     _expect("jq_pack_weight_ternary", "w", w, torch.float32, (N, K), w.device)
-    _need_cuda(w)
+    _need_cuda(w, stream=stream)
     qw2 = torch.empty((N, K // 4), dtype=torch.uint8, device=w.device)
     s_w = torch.empty((K // group if group else 0, N), dtype=torch.float32, device=w.device)
     _check("jq_pack_weight_ternary",
@@ -297,7 +321,7 @@ def jq_w158a4_linear(q, s_a, qw2, s_w, bias, group: int, y=None, workspace=None,
     fn = "jq_w158a4_linear"
     M, K, N = _codes_shapes(fn, q, qw2, 4)
     _expect_linear(fn, M, N, K, group, q.device, s_a, s_w, bias, y, workspace)
-    _need_cuda(q, s_a, qw2, s_w, bias)
+    _need_cuda(q, s_a, qw2, s_w, bias, stream=stream)
     if y is None:
         y = torch.empty((M, N), dtype=torch.bfloat16, device=q.device)
     if workspace is None:
@@ -331,7 +355,7 @@ def jq_fake_quant_act(x: torch.Tensor, group: int, s_in: torch.Tensor | None = N
     if not x.is_contiguous():
         raise ValueError(f"{fn}: x must have dense rows")
     _expect(fn, "s_in", s_in, torch.float32, (M, _groups(K, group)), x.device)
-    _need_cuda(x)
+    _need_cuda(x, stream=stream)
     xhat = torch.empty((M, K), dtype=torch.bfloat16, device=x.device)
     mask = torch.empty((M, K), dtype=torch.uint8, device=x.device)
     s_out = torch.empty((M, K // group if group else 0), dtype=torch.float32, device=x.device)
@@ -349,7 +373,7 @@ def jq_fake_quant_weight(w: torch.Tensor, group: int, s_in: torch.Tensor | None 
     N, K = w.shape
     _expect(fn, "w", w, torch.float32, (N, K), w.device)
     _expect(fn, "s_in", s_in, torch.float32, (N, _groups(K, group)), w.device)
-    _need_cuda(w)
+    _need_cuda(w, stream=stream)
     what = torch.empty((N, K), dtype=torch.float32, device=w.device)
     mask = torch.empty((N, K), dtype=torch.uint8, device=w.device)
     s_out = torch.empty((N, K // group if group else 0), dtype=torch.float32, device=w.device)
@@ -366,7 +390,7 @@ def jq_ste_backward(grad: torch.Tensor, mask: torch.Tensor, stream=None):
     _expect(fn, "mask", mask, torch.uint8, tuple(grad.shape), grad.device)
     if mask is None:
         raise ValueError(f"{fn}: mask is required")
-    _need_cuda(grad)
+    _need_cuda(grad, mask, stream=stream)
     out = torch.empty_like(grad)
     _check(fn, _load().jq_ste_backward(_ptr(grad), _ptr(mask), grad.numel(), _ptr(out), _stream(stream)))
     return out

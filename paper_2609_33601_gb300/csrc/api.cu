@@ -2,6 +2,8 @@
 // launches on the caller's stream.  No allocation, no synchronisation (except in
 // jq_device_status), no exceptions.
 #include <cstdint>
+#include <mutex>
+
 #include <cuda_runtime.h>
 
 #include "jq.h"
@@ -11,7 +13,7 @@
 
 namespace {
 
-constexpr int kMaxDevices = 64;
+using jq::kMaxDevices;
 using jq::kMaxK;
 // The offset-code form (one group, in the few-token kernel and the GEMM) sums |(q_w + 8) q_a| <= 120
 // per element, exact in fp32 over runs of up to kOffsetMaxRun elements; the few-token kernel's
@@ -29,20 +31,26 @@ struct DeviceInfo {
   uint32_t* status = nullptr;
 };
 DeviceInfo g_devices[kMaxDevices];
+std::mutex g_devices_mutex;
 
-// Resolves the current device once: it must be an sm_103 part.
+// Resolves the current device once: it must be an sm_103 part.  The probe runs under a mutex and
+// is recorded only once it has an answer, so a first call from several host threads at once sees
+// either the finished probe or runs it itself, never a half-written entry.
 const DeviceInfo* current_device() {
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return nullptr;
+  std::lock_guard<std::mutex> lock(g_devices_mutex);
   DeviceInfo& d = g_devices[dev];
   if (!d.probed) {
-    d.probed = true;
     cudaDeviceProp prop;
-    if (cudaGetDeviceProperties(&prop, dev) != cudaSuccess) return nullptr;
-    d.sms = prop.multiProcessorCount;
+    if (cudaGetDeviceProperties(&prop, dev) != cudaSuccess) return nullptr;  // not recorded: asked again
     void* p = nullptr;
-    d.ok = (prop.major == 10 && prop.minor == 3) && cudaGetSymbolAddress(&p, g_device_status) == cudaSuccess;
+    const bool sm103 = prop.major == 10 && prop.minor == 3;
+    if (sm103 && cudaGetSymbolAddress(&p, g_device_status) != cudaSuccess) return nullptr;
+    d.sms = prop.multiProcessorCount;
     d.status = static_cast<uint32_t*>(p);
+    d.ok = sm103 && p != nullptr;
+    d.probed = true;
   }
   return d.ok ? &d : nullptr;
 }

@@ -719,24 +719,29 @@ cudaError_t launch_impl(const GemmProblem& p, cudaStream_t stream, int sms) {
                              kScGroups, kBM, CU_TENSOR_MAP_SWIZZLE_NONE))
       return cudaErrorInvalidValue;
   }
-  static bool attr_set = false;
-  static int max_pairs = 0;
-  if (!attr_set) {
-    cudaError_t e = cudaFuncSetAttribute(w4a4_gemm_kernel<kExport, kOffset>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         (int)kSmemBytes);
-    if (e != cudaSuccess) return e;
-    cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3(2 * (sms / 2), 1, 1);
-    cfg.blockDim = dim3(kThreads, 1, 1);
-    cfg.dynamicSmemBytes = kSmemBytes;
-    int clusters = 0;
-    if (cudaOccupancyMaxActiveClusters(&clusters, w4a4_gemm_kernel<kExport, kOffset>, &cfg) != cudaSuccess || clusters <= 0) {
-      (void)cudaGetLastError();
-      clusters = sms / 2;
-    }
-    max_pairs = clusters < sms / 2 ? clusters : sms / 2;
-    attr_set = true;
-  }
+  // Once per device: the shared-memory attribute, and how many pairs can be resident at once.
+  static PerDevice<int> setup;
+  int max_pairs = 0;
+  cudaError_t se = setup.get(
+      [sms](int& pairs) {
+        cudaError_t e = cudaFuncSetAttribute(w4a4_gemm_kernel<kExport, kOffset>,
+                                             cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemBytes);
+        if (e != cudaSuccess) return e;
+        cudaLaunchConfig_t cfg = {};
+        cfg.gridDim = dim3(2 * (sms / 2), 1, 1);
+        cfg.blockDim = dim3(kThreads, 1, 1);
+        cfg.dynamicSmemBytes = kSmemBytes;
+        int clusters = 0;
+        if (cudaOccupancyMaxActiveClusters(&clusters, w4a4_gemm_kernel<kExport, kOffset>, &cfg) != cudaSuccess ||
+            clusters <= 0) {
+          (void)cudaGetLastError();
+          clusters = sms / 2;
+        }
+        pairs = clusters < sms / 2 ? clusters : sms / 2;
+        return cudaSuccess;
+      },
+      max_pairs);
+  if (se != cudaSuccess) return se;
   Args a;
   a.M = p.M;
   a.N = p.N;
@@ -766,15 +771,17 @@ cudaError_t launch_impl(const GemmProblem& p, cudaStream_t stream, int sms) {
 }  // namespace
 
 namespace {
+// The driver's tensor-map encoder (one entry point per process; the initialisation of a
+// function-local static is thread-safe).
 PFN_cuTensorMapEncodeTiled_v12000 tensor_map_encoder() {
-  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
-  if (fn == nullptr) {
+  static const PFN_cuTensorMapEncodeTiled_v12000 fn = []() -> PFN_cuTensorMapEncodeTiled_v12000 {
     void* p = nullptr;
     cudaDriverEntryPointQueryResult q;
     if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) == cudaSuccess &&
         q == cudaDriverEntryPointSuccess)
-      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
-  }
+      return reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+    return nullptr;
+  }();
   return fn;
 }
 }  // namespace

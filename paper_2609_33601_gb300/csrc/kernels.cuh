@@ -1,10 +1,47 @@
 // kernels.cuh -- internal launchers behind the C ABI (no argument checking here; api.cu does it).
 #pragma once
 #include <cstdint>
+#include <mutex>
+
 #include <cuda.h>
 #include <cuda_runtime.h>
 
 namespace jq {
+
+// Highest device ordinal (+1) the library serves in one process.
+constexpr int kMaxDevices = 64;
+
+// Launch set-up that has to happen once per device: kernel attributes (the dynamic shared-memory
+// size) and occupancy probes are properties of a kernel on one device, so a value found with
+// device 0 current says nothing about device 1.  get() runs `init` for the current device the
+// first time that device asks, under a mutex, and records the result only when `init` succeeded
+// (a failed set-up is retried on the next call).  Safe to call from several host threads.
+template <typename T>
+class PerDevice {
+ public:
+  template <typename F>
+  cudaError_t get(F&& init, T& out) {
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    if (dev < 0 || dev >= kMaxDevices) return cudaErrorInvalidDevice;
+    std::lock_guard<std::mutex> lock(mu_);
+    if (!done_[dev]) {
+      T v{};
+      e = init(v);
+      if (e != cudaSuccess) return e;
+      vals_[dev] = v;
+      done_[dev] = true;
+    }
+    out = vals_[dev];
+    return cudaSuccess;
+  }
+
+ private:
+  std::mutex mu_;
+  bool done_[kMaxDevices] = {};
+  T vals_[kMaxDevices] = {};
+};
 
 // Launches `kernel` with programmatic stream serialisation: it may begin while the previous
 // kernel of the stream is still running, as soon as that kernel allows it (ptx.cuh,

@@ -22,7 +22,7 @@
 namespace {
 
 constexpr size_t kNoAllocScratchBytes = JQ_NOALLOC_MAX_SCRATCH_BYTES;
-constexpr int kMaxDevices = 64;
+using jq::kMaxDevices;
 using jq::kMaxK;
 
 // The scratch: the E4M3 operand image of the activations, whole 128-row tiles of K bytes.  The

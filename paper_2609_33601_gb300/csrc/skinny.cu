@@ -939,41 +939,55 @@ cudaLaunchConfig_t make_config(int grid, int split, cudaStream_t stream, cudaLau
 // every CTA keeps at least kMinSplitSlots ring slots of K: below that a CTA's fixed costs (setup,
 // first-byte latency, the cluster reduction) outweigh the bandwidth of the extra SMs (measured on
 // K=3072 -> N=3072, 24 tiles: split 2 beats 6 by 18 % at one token and 27 % at 64).  Cluster
-// residency is asked of the runtime once per size.
+// residency is asked of the runtime once per device and size.
+struct SplitProbe {
+  int max_clusters[kMaxSplit + 1];
+};
+
 template <int kMp>
-int choose_split(int tiles, int k_stages, int sms) {
-  static int max_clusters[kMaxSplit + 1] = {0};
-  static bool probed = false;
-  if (!probed) {
-    probed = true;
-    for (int s = 1; s <= kMaxSplit; ++s) {
-      cudaLaunchAttribute attr[2];
-      cudaLaunchConfig_t cfg = make_config<kMp>(s * (sms / s), s, nullptr, attr);
-      int n = 0;
-      if (cudaOccupancyMaxActiveClusters(&n, w4a4_skinny_kernel<kMp>, &cfg) != cudaSuccess) {
-        (void)cudaGetLastError();
-        n = 0;
-      }
-      max_clusters[s] = n;
-    }
-  }
+cudaError_t choose_split(int tiles, int k_stages, int sms, int& best) {
+  // Cluster residency per split, asked of the runtime once per device and tile height.
+  static PerDevice<SplitProbe> probes;
+  SplitProbe pr;
+  cudaError_t e = probes.get(
+      [sms](SplitProbe& v) {
+        v.max_clusters[0] = 0;
+        for (int s = 1; s <= kMaxSplit; ++s) {
+          cudaLaunchAttribute attr[2];
+          cudaLaunchConfig_t cfg = make_config<kMp>(s * (sms / s), s, nullptr, attr);
+          int n = 0;
+          if (cudaOccupancyMaxActiveClusters(&n, w4a4_skinny_kernel<kMp>, &cfg) != cudaSuccess) {
+            (void)cudaGetLastError();
+            n = 0;
+          }
+          v.max_clusters[s] = n;
+        }
+        return cudaSuccess;
+      },
+      pr);
+  if (e != cudaSuccess) return e;
   const int slots = (k_stages + kStPerSlot - 1) / kStPerSlot;
-  int best = 1;
+  best = 1;
   for (int s = 2; s <= kMaxSplit && s <= k_stages; ++s)
-    if (tiles * s <= sms && tiles <= max_clusters[s] && slots / s >= kMinSplitSlots) best = s;
-  return best;
+    if (tiles * s <= sms && tiles <= pr.max_clusters[s] && slots / s >= kMinSplitSlots) best = s;
+  return cudaSuccess;
 }
 
 template <int kMp>
 cudaError_t launch_mp(SkArgs a, const SkinnyProblem& p, int tiles, int sms, cudaStream_t stream) {
   using L = Layout<kMp>;
-  static bool attr_set = false;
-  if (!attr_set) {
-    cudaError_t e = cudaFuncSetAttribute(w4a4_skinny_kernel<kMp>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         (int)L::kSmemBytes);
-    if (e != cudaSuccess) return e;
-    attr_set = true;
-  }
+  // The shared-memory attribute is per device: set once for each device, before its first
+  // occupancy probe (choose_split) and launch.
+  static PerDevice<bool> smem_attr;
+  bool attr_ok = false;
+  cudaError_t ae = smem_attr.get(
+      [](bool& v) {
+        v = true;
+        return cudaFuncSetAttribute(w4a4_skinny_kernel<kMp>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                    (int)L::kSmemBytes);
+      },
+      attr_ok);
+  if (ae != cudaSuccess) return ae;
   // Packed codes as byte matrices: weights [N, K/2], tokens [M, K/2]; one box = 128 packed bytes
   // (two K stages) x 128 weight rows or x kMp token rows, 128-byte swizzle.  Rows past N or M
   // and columns past K/2 read zeros.  Image mode: the tokens come from the A-operand image seen
@@ -990,7 +1004,8 @@ cudaError_t launch_mp(SkArgs a, const SkinnyProblem& p, int tiles, int sms, cuda
                             : encode_2d(&tmX, CU_TENSOR_MAP_DATA_TYPE_UINT8, p.q, p.K / 2, p.M, p.K / 2, kBK, kMp,
                                         CU_TENSOR_MAP_SWIZZLE_128B);
   if (!ok_w || !ok_x) return cudaErrorInvalidValue;
-  a.split = choose_split<kMp>(tiles, a.k_stages, sms);
+  cudaError_t se = choose_split<kMp>(tiles, a.k_stages, sms, a.split);
+  if (se != cudaSuccess) return se;
   cudaLaunchAttribute attr[2];
   cudaLaunchConfig_t cfg = make_config<kMp>(tiles * a.split, a.split, stream, attr);
   cfg.numAttrs = 2;

@@ -26,10 +26,14 @@ def test_kernel_hash_ignores_comments_and_whitespace_but_not_code(tmp_path, monk
     assert bench.kernel_hash("k.cu") != h0
 
 
-def test_recorded_traffic_matches_the_current_kernels():
-    # the traffic figures in bench.py were taken on the current kernel code (profiles/)
-    assert ("dllm", bench.kernel_hash("gemm.cu")) in bench.KERNEL_TRAFFIC
-    assert ("sweep_m1", bench.kernel_hash("skinny.cu")) in bench.KERNEL_TRAFFIC
+def test_recorded_traffic_applies_only_to_the_code_it_was_captured_on(monkeypatch):
+    # a DRAM-traffic figure is keyed by workload and kernel code hash: it is reported for that
+    # exact code, and null once the code changes (until a new ncu capture is recorded)
+    h = bench.kernel_hash("gemm.cu")
+    monkeypatch.setattr(bench, "KERNEL_TRAFFIC", {("flux_qkv", h): 123.0, ("dllm", "0" * 16): 5.0})
+    assert bench.recorded_traffic("flux_qkv", "gemm.cu") == 123.0
+    assert bench.recorded_traffic("dllm", "gemm.cu") is None
+    assert bench.recorded_traffic("flux_out", "gemm.cu") is None
 
 
 @pytest.mark.parametrize("M,few,fused,ternary,expect", [

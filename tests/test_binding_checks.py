@@ -125,3 +125,15 @@ def test_tensors_on_different_devices_are_refused():
     with pytest.raises(ValueError) as e:
         call_linear(a)
     assert "s_w" in str(e.value) and CUDA_ONLY not in str(e.value)
+
+
+def test_tensors_of_another_gpu_than_the_current_one_are_refused():
+    """The C calls launch on the current CUDA device; tensors (or a stream) of another device
+    would be addressed there as foreign pointers, so the binding names the mismatch first."""
+    cuda1 = torch.device("cuda", 1)
+    assert jq._device_mismatch(torch.device("cuda", 0), 0) is None
+    assert jq._device_mismatch(cuda1, 1, cuda1) is None
+    why = jq._device_mismatch(cuda1, 0)
+    assert why is not None and "cuda:1" in why and "current CUDA device is cuda:0" in why
+    why = jq._device_mismatch(torch.device("cuda", 0), 0, cuda1)
+    assert why is not None and "stream" in why

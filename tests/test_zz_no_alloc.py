@@ -87,3 +87,26 @@ def test_noalloc_few_tokens_convert_the_tokens_in_the_kernel(M, N, K, G, bias):
     y64, _ = ref.linear()
     check_linear(y_na, y64, ref.partials(), ref.s_a, ref.s_w_rows, ref.bias, f"noalloc M={M}")
     assert np.array_equal(y_na, y_ws)
+
+
+def test_noalloc_largest_accepted_problem_fills_the_scratch():
+    """At K = 4096, group128 the scratch holds the operand image (whole 128-row tiles of K bytes)
+    and then one fp32 correction per token and group, rounded up to 256 bytes: M = 3968 needs
+    16,760,832 of the 16,777,216 bytes, so the corrections end within 17 KB of the array's last
+    byte.  That call must give the same bits as jq_w4a4_linear; one more token (M = 3969 starts a
+    32nd image tile) must be refused before any launch."""
+    K, G, N = 4096, 128, 264
+    M = 3968
+    assert -(-M // 128) * 128 * K + -(-(4 * M * (K // G)) // 256) * 256 == 16_760_832 <= MAX_SCRATCH
+    ref, args = _problem(M, N, K, G, True, seed=9)
+    y_na = _bits(jq.jq_w4a4_linear_noalloc(*args, G))
+    y_ws = _bits(jq.jq_w4a4_linear(*args, G))
+    assert np.array_equal(y_na, y_ws)
+    rows = np.array([0, 1, 2047, 3840, M - 1])
+    y64, _ = ref.linear(rows)
+    check_linear(y_na[rows], y64, ref.partials(rows), ref.s_a[rows], ref.s_w_rows, ref.bias, "noalloc M=3968")
+    lib = jq._load()
+    small = torch.zeros(256, dtype=torch.uint8, device="cuda")
+    p = ctypes.c_void_p(small.data_ptr())
+    assert lib.jq_w4a4_linear_noalloc(p, p, p, p, None, p, M + 1, N, K, G, None) == JQ_ERR_WORKSPACE
+    torch.cuda.synchronize()
