@@ -10,25 +10,29 @@
 // so the fp32 TMEM accumulator holds acc[m,n,g] * 2^-18 exactly.
 //
 // Persistent kernel on CTA pairs (clusters of two SMs, tcgen05 cta_group::2).  A pair owns a
-// 256x256 output tile at a time: CTA r of the pair holds A rows 128r..128r+127 and B rows (output
-// columns) 128r..128r+127 of the tile, and the even CTA issues 256x256x32 MMAs that read both
-// CTAs' shared memory and write 128 rows x 256 columns into each CTA's TMEM.  Per SM this halves
-// the B bytes the tensor core reads and the B nibbles each SM unpacks, against a one-SM 128x256
-// tile.  K stages of 128; 16 warps per CTA:
+// 256 x kBN output tile at a time (kBN = 256): CTA r of the pair holds A rows 128r..128r+127 and B
+// rows (output columns) r*kBN/2.. of the tile, and the even CTA issues 256 x kBN x 32 MMAs that
+// read both CTAs' shared memory and write 128 rows x kBN columns into each CTA's TMEM (two
+// accumulators fill its 512 columns).  Per SM this halves the B bytes the tensor core reads and
+// the B nibbles each SM unpacks, against a one-SM tile.  The tile width is a parameter of the
+// layout (Tile): a 128-column tile with four accumulators was built and measured for the group
+// modes, and ran at half this tile's rate -- the per-group rescale costs about the same time per
+// group at either width, so the wider tile does twice the work per rescale.  K stages of 128;
+// 16 warps per CTA:
 //   warp 0      A producer: one 2-D TMA per two K stages (256 rows x 128 bytes of the
 //               pre-swizzled A-operand image, 32 KB) -> A ring, completing on the even CTA's
 //               barrier
 //   warp 1      TMEM owner; in the even CTA also the MMA issuer (one thread): 4 MMAs per K stage
-//               into one of two TMEM accumulators; a new accumulator starts at every group
+//               into one of the TMEM accumulators; a new accumulator starts at every group
 //               boundary and is handed to both CTAs' drain warps when the group ends
 //   warp 2      scale producer: weight (and activation) scales of 4 groups per TMA box into a
 //               ring for the drain
 //   warps 4-7   unpack: packed nibbles straight from global memory (two stages in flight in
 //               registers) -> E4M3 operand bytes in the 128B-swizzled K-major layout -> B ring
-//   warps 8-15  drain: per group, the group's 36 scales from the ring, then 16 round trips of
-//               tcgen05.ld 16x256b (8 columns) and y += (acc * s_w) * (s_a * 2^18) in fp32
-//               registers (warp w owns TMEM lanes 32*(w%4).. and columns 128*((w-8)/4)..); after
-//               the last group, + bias, round to bf16, store
+//   warps 8-15  drain: per group, the group's scales, then the accumulator from TMEM and
+//               y += (acc * s_w) * (s_a * 2^18) in fp32 registers (warp w owns TMEM lanes
+//               32*(w%4).. and columns (kBN/2)*((w-8)/4)..); after the last group, + bias, round to
+//               bf16, store
 // Every mbarrier wait is bounded; a timeout records a status and unwinds the CTA, and both CTAs
 // of a pair meet at a final cluster barrier before the pair's TMEM is released.
 #include <cfloat>
@@ -48,50 +52,58 @@ namespace {
 
 constexpr int kBM = 128;            // A rows per CTA (a pair covers 256)
 constexpr int kPairM = 2 * kBM;
-constexpr int kBN = 256;            // output columns per pair tile
-constexpr int kBNHalf = kBN / 2;    // B rows per CTA
 constexpr int kBK = 128;
 constexpr int kStagesPerSlot = 2;   // K stages per ring slot (one A transfer, two unpacked B stages)
-constexpr int kSlots = 3;           // operand ring: each slot holds A and B for kStagesPerSlot stages
 constexpr int kThreads = 512;
 constexpr int kWarpProdA = 0, kWarpMma = 1, kWarpScale = 2;
 constexpr int kUnpackWarp0 = 4, kUnpackThreads = 128;
 constexpr int kUnpackGroups = 2, kUnpackGroupThreads = kUnpackThreads / kUnpackGroups;  // alternate K stages
 constexpr int kUnpackGroupWarps = kUnpackGroupThreads / 32;
 constexpr int kDrainWarp0 = 8, kNumDrainWarps = 8;
-constexpr int kChunksPerThread = kBNHalf * (kBK / 2) / 16 / kUnpackGroupThreads;  // 8 packed 16-byte chunks
-constexpr uint32_t kTmemCols = 512;  // two 256-column accumulators
+constexpr uint32_t kTmemCols = 512;
 constexpr int kRegsCtl = 32, kRegsUnpack = 96, kRegsDrain = 192;
 static_assert(4 * 32 * (kRegsCtl + kRegsUnpack + 2 * kRegsDrain) == 65536, "register split must use the launch budget");
-static_assert(kChunksPerThread == 8, "unpack assumes eight chunks per thread per stage");
 
 constexpr uint32_t kOpABytes = kBM * kBK;                     // 16 KB per K stage per CTA
 constexpr uint32_t kSlotABytes = kStagesPerSlot * kOpABytes;  // 32 KB
-constexpr uint32_t kOpBBytes = kBNHalf * kBK;                 // 16 KB per K stage per CTA
-constexpr uint32_t kSlotBBytes = kStagesPerSlot * kOpBBytes;  // 32 KB
 
-// Scale ring: each slot holds the weight scales of kScGroups groups for the tile's 256 columns
+// Scale ring: each slot holds the weight scales of kScGroups groups for the tile's kBN columns
 // ([group][column] fp32) and, when they come by TMA, the activation scales of those groups for
 // this CTA's 128 rows ([row][group] fp32).
 constexpr int kScGroups = 4, kScSlots = 4;
-constexpr uint32_t kScSwBytes = kScGroups * kBN * 4;  // 4 KB
 constexpr uint32_t kScSaBytes = kScGroups * kBM * 4;  // 2 KB
-constexpr uint32_t kScSlotBytes = kScSwBytes + kScSaBytes;
 
-constexpr uint32_t kOffA = 0;
-constexpr uint32_t kOffB = kOffA + kSlots * kSlotABytes;
-constexpr uint32_t kOffSc = kOffB + kSlots * kSlotBBytes;
-constexpr uint32_t kOffBar = kOffSc + kScSlots * kScSlotBytes;
-constexpr uint32_t kNumBars = 2 * kSlots + 4 + 1 + 2 * kScSlots;
-constexpr uint32_t kOffMisc = kOffBar + kNumBars * 8;
-constexpr uint32_t kSmemBytes = kOffMisc + 16;
-static_assert(kOffBar % 8 == 0 && kOffMisc % 8 == 0, "mbarriers need 8-byte alignment");
-static_assert(kOffSc % 128 == 0 && kScSlotBytes % 128 == 0 && kScSwBytes % 128 == 0, "TMA destinations need 128 bytes");
-static_assert(kOffA % 1024 == 0 && kOffB % 1024 == 0 && kOpABytes % 1024 == 0 && kOpBBytes % 1024 == 0,
-              "128B-swizzled operand slots need 1024-byte alignment");
-// The rings need a 1024-byte aligned base (128B swizzle atoms); the dynamic shared memory
-// window is declared with that alignment and the kernel checks it before touching anything.
-static_assert(kSmemBytes <= 232448, "shared memory budget");
+// Everything that depends on the tile width kBN (output columns per pair tile).
+template <int kBN_>
+struct Tile {
+  static constexpr int kBN = kBN_;
+  static constexpr int kBNHalf = kBN / 2;                    // B rows per CTA
+  static constexpr int kAccBufs = kTmemCols / kBN;           // TMEM accumulators (2 or 4)
+  static constexpr int kDrainCols = kBN / 2;                 // accumulator columns per drain warp
+  static constexpr int kSlots = kBN == 256 ? 3 : 4;          // operand ring slots (what fits in shared memory)
+  static constexpr uint32_t kOpBBytes = kBNHalf * kBK;       // B bytes per K stage per CTA
+  static constexpr uint32_t kSlotBBytes = kStagesPerSlot * kOpBBytes;
+  static constexpr int kChunksPerThread = kBNHalf * (kBK / 2) / 16 / kUnpackGroupThreads;  // packed 16-byte chunks
+  static constexpr uint32_t kScSwBytes = kScGroups * kBN * 4;
+  static constexpr uint32_t kScSlotBytes = kScSwBytes + kScSaBytes;
+  static constexpr uint32_t kOffA = 0;
+  static constexpr uint32_t kOffB = kOffA + kSlots * kSlotABytes;
+  static constexpr uint32_t kOffSc = kOffB + kSlots * kSlotBBytes;
+  static constexpr uint32_t kOffBar = kOffSc + kScSlots * kScSlotBytes;
+  static constexpr uint32_t kNumBars = 2 * kSlots + 2 * kAccBufs + 1 + 2 * kScSlots;
+  static constexpr uint32_t kOffMisc = kOffBar + kNumBars * 8;
+  static constexpr uint32_t kSmemBytes = kOffMisc + 16;
+  static_assert(kBN == 128 || kBN == 256, "tile widths");
+  static_assert(kChunksPerThread * kUnpackGroupThreads * 16 == kBNHalf * (kBK / 2), "unpack covers the B half");
+  static_assert(kOffBar % 8 == 0 && kOffMisc % 8 == 0, "mbarriers need 8-byte alignment");
+  static_assert(kOffSc % 128 == 0 && kScSlotBytes % 128 == 0 && kScSwBytes % 128 == 0,
+                "TMA destinations need 128 bytes");
+  static_assert(kOffA % 1024 == 0 && kOffB % 1024 == 0 && kOpABytes % 1024 == 0 && kOpBBytes % 1024 == 0,
+                "128B-swizzled operand slots need 1024-byte alignment");
+  // The rings need a 1024-byte aligned base (128B swizzle atoms); the dynamic shared memory
+  // window is declared with that alignment and the kernel checks it before touching anything.
+  static_assert(kSmemBytes <= 232448, "shared memory budget");
+};
 
 struct Args {
   int M, N, K, G;
@@ -110,9 +122,16 @@ struct Args {
 
 struct Bars {
   uint64_t *full, *empty;  // operand ring: A and B of a slot arrive on full, leave on empty
-  uint64_t *acc_full, *acc_empty, *mma_done;
+  uint64_t *acc_full, *acc_empty, *mma_done;  // TMEM accumulators (T::kAccBufs of each)
   uint64_t *sc_full, *sc_empty;  // scale ring
 };
+
+// Accumulator hand-offs: the i-th group accumulated by the pair uses buffer i % kAccBufs, and
+// that buffer's phase parity is (i / kAccBufs) & 1.
+template <class T>
+__device__ __forceinline__ uint32_t acc_buf(uint32_t i) { return i % T::kAccBufs; }
+template <class T>
+__device__ __forceinline__ uint32_t acc_parity(uint32_t i) { return (i / T::kAccBufs) & 1u; }
 
 struct Pair {
   uint32_t rank;     // 0 = the CTA that issues the MMAs
@@ -131,9 +150,9 @@ __device__ __forceinline__ void drain_wait(uint64_t* bar, uint32_t parity, uint3
 }
 
 // ------------------------------------------------------------------ drain + epilogue
-// Export path (jq_w4a4_group_partials): each thread owns one TMEM lane (row) and 128 columns
-// (32x32b loads) and writes the exact integer partials of every group.
-template <bool kOffset>
+// Export path (jq_w4a4_group_partials, 256-column tiles): each thread owns one TMEM lane (row) and
+// 128 columns (32x32b loads) and writes the exact integer partials of every group.
+template <class T, bool kOffset>
 __device__ __forceinline__ void drain_export(const Args& args, const Pair& pr, uint32_t tmem_base, const Bars& b,
                                              volatile int* abort_flag) {
   const uint32_t warp = warp_id(), lane = lane_id();
@@ -145,18 +164,18 @@ __device__ __forceinline__ void drain_export(const Args& args, const Pair& pr, u
   for (int tile = pr.cluster; ok && tile < args.num_tiles; tile += pr.num_clusters) {
     const int mt2 = tile % args.num_m2, nt = tile / args.num_m2;
     const int row = mt2 * kPairM + (int)pr.rank * kBM + (int)(quarter * 32u + lane);
-    const int col0 = nt * kBN + half * 128;
+    const int col0 = nt * T::kBN + half * T::kDrainCols;
     const bool row_ok = row < M;
     for (int g = 0; g < groups; ++g) {
-      const uint32_t ab = chunk_it & 1u;
+      const uint32_t ab = acc_buf<T>(chunk_it);
       const float cr = (kOffset && row_ok) ? -__ldg(args.corr + (int64_t)row * groups + g) : 0.0f;
       // Warp-collective tcgen05.ld follows: the whole warp proceeds or none of it.
-      ok = __all_sync(0xffffffffu, mbar_wait(&b.acc_full[ab], (chunk_it >> 1) & 1u, abort_flag, args.status));
+      ok = __all_sync(0xffffffffu, mbar_wait(&b.acc_full[ab], acc_parity<T>(chunk_it), abort_flag, args.status));
       if (!ok) break;
       tc_fence_after();
-      const uint32_t taddr = tmem_base + lane_base + ab * kBN + half * 128;
+      const uint32_t taddr = tmem_base + lane_base + ab * T::kBN + half * T::kDrainCols;
 #pragma unroll 1
-      for (int cc = 0; cc < 4; ++cc) {
+      for (int cc = 0; cc < T::kDrainCols / 32; ++cc) {
         uint32_t r[32];
         tmem_ld32(taddr + cc * 32, r);
         tmem_ld_wait();
@@ -178,15 +197,16 @@ __device__ __forceinline__ void drain_export(const Args& args, const Pair& pr, u
   }
 }
 
-// Linear path.  Warp w (drain index d = w - 8) owns TMEM lanes 32*(w%4).. (32 rows) and columns
-// 128*(d/4).. of each accumulator, read with the 16x256b shape: thread t holds rows
-// t/4 + {0, 8, 16, 24} of those 32 and columns 8j + 2(t%4) + {0, 1}, j = 0..15.  So a thread needs
-// only 32 weight scales and 4 activation scales per group; it loads all of them at the start of
-// the group (the tensor core's operand reads starve shared-memory loads issued one chunk ahead of
-// their use, but not loads issued a group ahead).
-template <bool kOffset>
+// Linear path, 256-column tiles (one-group problems).  Warp w (drain index d = w - 8) owns TMEM
+// lanes 32*(w%4).. (32 rows) and columns 128*(d/4).. of each accumulator, read with the 16x256b
+// shape: thread t holds rows t/4 + {0, 8, 16, 24} of those 32 and columns 8j + 2(t%4) + {0, 1},
+// j = 0..15.  So a thread needs only 32 weight scales and 4 activation scales per group; it loads
+// all of them at the start of the group (the tensor core's operand reads starve shared-memory
+// loads issued one chunk ahead of their use, but not loads issued a group ahead).
+template <class T, bool kOffset>
 __device__ __forceinline__ void drain_linear(const Args& args, const Pair& pr, uint32_t tmem_base, const Bars& b,
                                              uint8_t* sSc, volatile int* abort_flag) {
+  static_assert(T::kBN == 256, "the 128-column tiles drain in drain_linear128");
   const uint32_t warp = warp_id(), lane = lane_id();
   const int M = args.M, N = args.N, groups = args.groups;
   const uint32_t quarter = warp & 3u, half = (warp - kDrainWarp0) >> 2;
@@ -196,21 +216,21 @@ __device__ __forceinline__ void drain_linear(const Args& args, const Pair& pr, u
   for (int tile = pr.cluster; ok && tile < args.num_tiles; tile += pr.num_clusters) {
     const int mt2 = tile % args.num_m2, nt = tile / args.num_m2;
     const int row0 = mt2 * kPairM + (int)pr.rank * kBM + (int)(quarter * 32u + t4);  // + 8 * rr
-    const int col0 = nt * kBN + half * 128 + 2 * (int)tq;                              // + 8 * j
-    // y[4 * j + rr * ... ] layout: y[(rr * 16 + j) * 2 + e], rr = row index 0..3 (offset 8 * rr)
+    const int col0 = nt * T::kBN + half * 128 + 2 * (int)tq;                           // + 8 * j
+    // y layout: y[(rr * 16 + j) * 2 + e], rr = row index 0..3 (offset 8 * rr)
     float y[128];
 #pragma unroll
     for (int i = 0; i < 128; ++i) y[i] = 0.0f;
     for (int g = 0; g < groups; ++g) {
-      const uint32_t ab = chunk_it & 1u;
+      const uint32_t ab = acc_buf<T>(chunk_it);
       const int gi = g % kScGroups;
       const uint32_t sslot = sc_it % kScSlots;
       if (gi == 0) {
         ok = __all_sync(0xffffffffu, mbar_wait(&b.sc_full[sslot], ring_parity(sc_it, kScSlots), abort_flag, args.status));
         if (!ok) break;
       }
-      const uint8_t* slot = sSc + sslot * kScSlotBytes;
-      const float* sws = reinterpret_cast<const float*>(slot) + gi * kBN + half * 128 + 2 * tq;
+      const uint8_t* slot = sSc + sslot * T::kScSlotBytes;
+      const float* sws = reinterpret_cast<const float*>(slot) + gi * T::kBN + half * 128 + 2 * tq;
       float2 w[16];
 #pragma unroll
       for (int j = 0; j < 16; ++j) w[j] = *reinterpret_cast<const float2*>(sws + 8 * j);
@@ -221,7 +241,7 @@ __device__ __forceinline__ void drain_linear(const Args& args, const Pair& pr, u
         const int row = row0 + 8 * rr;
         float sa;
         if (args.sa_tma)
-          sa = reinterpret_cast<const float*>(slot + kScSwBytes)[(quarter * 32u + t4 + 8u * rr) * kScGroups + gi];
+          sa = reinterpret_cast<const float*>(slot + T::kScSwBytes)[(quarter * 32u + t4 + 8u * rr) * kScGroups + gi];
         else
           sa = row < M ? __ldg(args.s_a + (int64_t)row * groups + g) : 0.0f;
         f[rr] = sa;
@@ -229,10 +249,10 @@ __device__ __forceinline__ void drain_linear(const Args& args, const Pair& pr, u
       }
       // Warp-collective tcgen05.ld follows: the whole warp proceeds or none of it (a timeout in
       // one lane must not leave the others in an aligned instruction).
-      ok = __all_sync(0xffffffffu, mbar_wait(&b.acc_full[ab], (chunk_it >> 1) & 1u, abort_flag, args.status));
+      ok = __all_sync(0xffffffffu, mbar_wait(&b.acc_full[ab], acc_parity<T>(chunk_it), abort_flag, args.status));
       if (!ok) break;
       tc_fence_after();
-      const uint32_t taddr = tmem_base + ((quarter * 32u) << 16) + ab * kBN + half * 128;
+      const uint32_t taddr = tmem_base + ((quarter * 32u) << 16) + ab * T::kBN + half * 128;
       // The two arithmetic forms below are both exact-partial * scales in fp32; the slow one is
       // needed when s_a * 2^18 would overflow.  The choice is made for the whole warp: both
       // paths issue warp-collective tcgen05.ld / __syncwarp, which every lane must reach.
@@ -321,12 +341,13 @@ __device__ __forceinline__ void drain_linear(const Args& args, const Pair& pr, u
 
 // ------------------------------------------------------------------ scale producer
 // Streams the scales the drain needs into the scale ring, kScGroups groups per slot: one TMA box
-// of weight scales (kScGroups rows of 256 columns) and, when aligned, one of this CTA's
+// of weight scales (kScGroups rows of kBN columns) and, when aligned, one of this CTA's
 // activation scales (128 rows of kScGroups groups).  Boxes past the tensors' ends read zeros.
+template <class T>
 __device__ __forceinline__ void scale_producer(const Args& args, const Pair& pr, const CUtensorMap* tmSW,
                                                const CUtensorMap* tmSA, uint8_t* sSc, const Bars& b,
                                                volatile int* abort_flag) {
-  const uint32_t bytes = kScSwBytes + (args.sa_tma ? kScSaBytes : 0u);
+  const uint32_t bytes = T::kScSwBytes + (args.sa_tma ? kScSaBytes : 0u);
   uint32_t it = 0;
   bool ok = true;
   for (int tile = pr.cluster; ok && tile < args.num_tiles; tile += pr.num_clusters) {
@@ -335,10 +356,10 @@ __device__ __forceinline__ void scale_producer(const Args& args, const Pair& pr,
     for (int bi = 0; bi < args.sc_boxes; ++bi) {
       const uint32_t s = it % kScSlots;
       if (!(ok = mbar_wait(&b.sc_empty[s], ring_parity(it, kScSlots) ^ 1u, abort_flag, args.status))) break;
-      uint8_t* slot = sSc + s * kScSlotBytes;
+      uint8_t* slot = sSc + s * T::kScSlotBytes;
       mbar_arrive_expect_tx(&b.sc_full[s], bytes);
-      tma_load_2d(slot, tmSW, &b.sc_full[s], nt * kBN, bi * kScGroups);
-      if (args.sa_tma) tma_load_2d(slot + kScSwBytes, tmSA, &b.sc_full[s], bi * kScGroups, row0);
+      tma_load_2d(slot, tmSW, &b.sc_full[s], nt * T::kBN, bi * kScGroups);
+      if (args.sa_tma) tma_load_2d(slot + T::kScSwBytes, tmSA, &b.sc_full[s], bi * kScGroups, row0);
       ++it;
     }
   }
@@ -349,6 +370,7 @@ __device__ __forceinline__ void scale_producer(const Args& args, const Pair& pr,
 // ------------------------------------------------------------------ A producer
 // Both CTAs load their own 128 rows of a slot's two K stages; the transfers complete on the even
 // CTA's full barrier, which the even CTA arms with the bytes of both.
+template <class T>
 __device__ __forceinline__ void producer_a(const Args& args, const Pair& pr, const CUtensorMap* tmA, uint8_t* sA,
                                            const Bars& b, volatile int* abort_flag) {
   uint32_t it = 0;
@@ -356,8 +378,8 @@ __device__ __forceinline__ void producer_a(const Args& args, const Pair& pr, con
   for (int tile = pr.cluster; ok && tile < args.num_tiles; tile += pr.num_clusters) {
     const int mt = (tile % args.num_m2) * 2 + (int)pr.rank;  // 128-row block of the operand image
     for (int j = 0; j < args.slots_per_tile; ++j) {
-      const uint32_t s = it % kSlots;
-      if (!(ok = mbar_wait(&b.empty[s], ring_parity(it, kSlots) ^ 1u, abort_flag, args.status))) break;
+      const uint32_t s = it % T::kSlots;
+      if (!(ok = mbar_wait(&b.empty[s], ring_parity(it, T::kSlots) ^ 1u, abort_flag, args.status))) break;
       if (pr.rank == 0) mbar_arrive_expect_tx(&b.full[s], 2 * kSlotABytes);
       const int image_row = (mt * args.k_stages + j * kStagesPerSlot) * kBM;
       tma_load_2d_pair(sA + s * kSlotABytes, tmA, leader_bar(&b.full[s]), 0, image_row);
@@ -367,8 +389,8 @@ __device__ __forceinline__ void producer_a(const Args& args, const Pair& pr, con
   // Let the pair's last copies land before the CTA can leave (the even CTA sees both CTAs' bytes;
   // on an early exit the unpack arrivals may be missing, and the bounded wait ends it).
   if (pr.rank == 0)
-    for (uint32_t i = (it > kSlots ? it - kSlots : 0); i < it; ++i)
-      drain_wait(&b.full[i % kSlots], ring_parity(i, kSlots), args.status);
+    for (uint32_t i = (it > T::kSlots ? it - T::kSlots : 0); i < it; ++i)
+      drain_wait(&b.full[i % T::kSlots], ring_parity(i, T::kSlots), args.status);
 }
 
 // ------------------------------------------------------------------ MMA issuer (even CTA)
@@ -383,50 +405,49 @@ struct MmaState {
 };
 
 // Opens a new accumulator: waits until the drain has emptied it.
+template <class T>
 __device__ __forceinline__ bool mma_open_acc(const Args& args, const Bars& b, uint32_t tmem_base, MmaState& st,
                                              uint32_t& d_tmem, volatile int* abort_flag) {
-  const uint32_t ab = st.chunk_it & 1u;
-  if (!mbar_wait_cluster(&b.acc_empty[ab], ((st.chunk_it >> 1) & 1u) ^ 1u, abort_flag, args.status)) return false;
+  const uint32_t ab = acc_buf<T>(st.chunk_it);
+  if (!mbar_wait_cluster(&b.acc_empty[ab], acc_parity<T>(st.chunk_it) ^ 1u, abort_flag, args.status)) return false;
   tc_fence_after();
-  d_tmem = tmem_base + ab * kBN;
+  d_tmem = tmem_base + ab * T::kBN;
   return true;
 }
 
-static_assert(kSlotABytes == kSlotBBytes && kOpABytes == kOpBBytes, "A and B slots share descriptor offsets");
-
-// One K stage (4 MMAs of K = 32) at descriptor offset `off` (shared-memory bytes >> 4 from the
-// rings' bases, the same for A and B).  kHalf: group64, two groups per stage, each in a fresh
-// accumulator; otherwise a group spans stages_per_group whole stages.  With `wait_next`, the wait
-// for the next ring slot's operands sits between the second and third MMA, while the tensor
-// core still has queued work.
-template <bool kHalf>
+// One K stage (4 MMAs of K = 32) at descriptor offsets aoff / boff (shared-memory bytes >> 4
+// from the rings' bases).  kHalf: group64, two groups per stage, each in a fresh accumulator;
+// otherwise a group spans stages_per_group whole stages.  With `wait_next`, the wait for the next
+// ring slot's operands sits between the second and third MMA, while the tensor core still has
+// queued work.
+template <class T, bool kHalf>
 __device__ __forceinline__ bool mma_stage(const Args& args, const Bars& b, uint32_t tmem_base, MmaState& st,
                                           uint32_t& d_tmem, int& kg, int stages_per_group, uint64_t adesc0,
-                                          uint64_t bdesc0, uint32_t off, uint32_t idesc, bool wait_next,
-                                          uint32_t nslot, uint32_t nphase, volatile int* abort_flag) {
+                                          uint64_t bdesc0, uint32_t aoff, uint32_t boff, uint32_t idesc,
+                                          bool wait_next, uint32_t nslot, uint32_t nphase, volatile int* abort_flag) {
   constexpr uint16_t kBoth = 0x3;
-  const uint64_t ad = adesc0 + off, bd = bdesc0 + off;
+  const uint64_t ad = adesc0 + aoff, bd = bdesc0 + boff;
   if (kHalf) {
-    if (!mma_open_acc(args, b, tmem_base, st, d_tmem, abort_flag)) return false;
+    if (!mma_open_acc<T>(args, b, tmem_base, st, d_tmem, abort_flag)) return false;
     umma_f8f6f4_pair(d_tmem, ad, bd, idesc, 0u);
     umma_f8f6f4_pair(d_tmem, ad + 2u, bd + 2u, idesc, 1u);
-    umma_commit_pair(&b.acc_full[st.chunk_it & 1u], kBoth);
+    umma_commit_pair(&b.acc_full[acc_buf<T>(st.chunk_it)], kBoth);
     ++st.chunk_it;
-    if (!mma_open_acc(args, b, tmem_base, st, d_tmem, abort_flag)) return false;
+    if (!mma_open_acc<T>(args, b, tmem_base, st, d_tmem, abort_flag)) return false;
     umma_f8f6f4_pair(d_tmem, ad + 4u, bd + 4u, idesc, 0u);
     if (wait_next && !mbar_wait_cluster(&b.full[nslot], nphase, abort_flag, args.status)) return false;
     umma_f8f6f4_pair(d_tmem, ad + 6u, bd + 6u, idesc, 1u);
-    umma_commit_pair(&b.acc_full[st.chunk_it & 1u], kBoth);
+    umma_commit_pair(&b.acc_full[acc_buf<T>(st.chunk_it)], kBoth);
     ++st.chunk_it;
   } else {
-    if (kg == 0 && !mma_open_acc(args, b, tmem_base, st, d_tmem, abort_flag)) return false;
+    if (kg == 0 && !mma_open_acc<T>(args, b, tmem_base, st, d_tmem, abort_flag)) return false;
     umma_f8f6f4_pair(d_tmem, ad, bd, idesc, kg == 0 ? 0u : 1u);
     umma_f8f6f4_pair(d_tmem, ad + 2u, bd + 2u, idesc, 1u);
     if (wait_next && !mbar_wait_cluster(&b.full[nslot], nphase, abort_flag, args.status)) return false;
     umma_f8f6f4_pair(d_tmem, ad + 4u, bd + 4u, idesc, 1u);
     umma_f8f6f4_pair(d_tmem, ad + 6u, bd + 6u, idesc, 1u);
     if (++kg == stages_per_group) {
-      umma_commit_pair(&b.acc_full[st.chunk_it & 1u], kBoth);
+      umma_commit_pair(&b.acc_full[acc_buf<T>(st.chunk_it)], kBoth);
       ++st.chunk_it;
       kg = 0;
     }
@@ -437,10 +458,10 @@ __device__ __forceinline__ bool mma_stage(const Args& args, const Bars& b, uint3
 // The issue loop runs straight through each ring slot: the MMAs of its two stages, the wait for
 // the next slot in the middle of the second stage, one commit that frees the slot.  The only
 // data-dependent branch per slot is the odd K-stage tail (a slot with one stage).
-template <bool kHalf>
+template <class T, bool kHalf>
 __device__ __forceinline__ void mma_role(const Args& args, const Pair& pr, uint32_t tmem_base, uint8_t* sA,
                                          uint8_t* sB, const Bars& b, volatile int* abort_flag) {
-  const uint32_t idesc = idesc_e4m3_f32(kPairM, kBN);
+  const uint32_t idesc = idesc_e4m3_f32(kPairM, T::kBN);
   constexpr uint16_t kBoth = 0x3;
   const uint64_t adesc0 = sdesc_kmajor_sw128(smem_u32(sA));
   const uint64_t bdesc0 = sdesc_kmajor_sw128(smem_u32(sB));
@@ -455,18 +476,19 @@ __device__ __forceinline__ void mma_role(const Args& args, const Pair& pr, uint3
   int j = 0, kg = 0;  // slot within the tile, K stage within the group
   bool ok = total > 0 && mbar_wait_cluster(&b.full[0], 0, abort_flag, args.status);
   for (uint32_t q = 0; ok && q < total; ++q) {
-    const uint32_t nslot = slot + 1 == kSlots ? 0 : slot + 1;
-    const uint32_t nphase = slot + 1 == kSlots ? phase ^ 1u : phase;
-    const uint32_t off = (slot * kSlotABytes) >> 4;
+    const uint32_t nslot = slot + 1 == (uint32_t)T::kSlots ? 0 : slot + 1;
+    const uint32_t nphase = slot + 1 == (uint32_t)T::kSlots ? phase ^ 1u : phase;
+    const uint32_t aoff = (slot * kSlotABytes) >> 4, boff = (slot * T::kSlotBBytes) >> 4;
     const bool wait_next = q + 1 < total;
     if (j != odd_slot) {
-      ok = mma_stage<kHalf>(args, b, tmem_base, st, d_tmem, kg, stages_per_group, adesc0, bdesc0, off, idesc, false,
-                            0u, 0u, abort_flag) &&
-           mma_stage<kHalf>(args, b, tmem_base, st, d_tmem, kg, stages_per_group, adesc0, bdesc0,
-                            off + (kOpABytes >> 4), idesc, wait_next, nslot, nphase, abort_flag);
+      ok = mma_stage<T, kHalf>(args, b, tmem_base, st, d_tmem, kg, stages_per_group, adesc0, bdesc0, aoff, boff, idesc,
+                               false, 0u, 0u, abort_flag) &&
+           mma_stage<T, kHalf>(args, b, tmem_base, st, d_tmem, kg, stages_per_group, adesc0, bdesc0,
+                               aoff + (kOpABytes >> 4), boff + (T::kOpBBytes >> 4), idesc, wait_next, nslot, nphase,
+                               abort_flag);
     } else {
-      ok = mma_stage<kHalf>(args, b, tmem_base, st, d_tmem, kg, stages_per_group, adesc0, bdesc0, off, idesc,
-                            wait_next, nslot, nphase, abort_flag);
+      ok = mma_stage<T, kHalf>(args, b, tmem_base, st, d_tmem, kg, stages_per_group, adesc0, bdesc0, aoff, boff, idesc,
+                               wait_next, nslot, nphase, abort_flag);
     }
     if (!ok) break;
     umma_commit_pair(&b.empty[slot], kBoth);
@@ -481,10 +503,10 @@ __device__ __forceinline__ void mma_role(const Args& args, const Pair& pr, uint3
 
 // ------------------------------------------------------------------ unpack
 // Two groups of two warps take alternate K stages.  Per stage, thread u of a group converts
-// packed chunks t = u + 64 i (i = 0..7): 16-byte chunk t % 4 of the 64 packed bytes of B row t / 4
-// (this CTA's half of the tile's columns).  Each chunk becomes two 16-byte operand chunks of the
-// 128B-swizzled row; a quarter-warp's stores cover two rows whose chunk positions differ in
-// parity, so they never share a bank.
+// packed chunks t = u + 64 i (i < kChunksPerThread): 16-byte chunk t % 4 of the 64 packed bytes
+// of B row t / 4 (this CTA's half of the tile's columns).  Each chunk becomes two 16-byte operand
+// chunks of the 128B-swizzled row; a quarter-warp's stores cover two rows whose chunk positions
+// differ in parity, so they never share a bank.
 //
 // Each round's global loads are issued two rounds ahead.
 // Cursor over the (tile, slot) sequence of this pair; a group's stage in slot j is 2j + group.
@@ -492,15 +514,16 @@ struct UnpackCursor {
   int tile, j;
 };
 
+template <class T>
 __device__ __forceinline__ void unpack_load(const Args& args, const Pair& pr, const UnpackCursor& c, uint32_t ug,
-                                            uint32_t u, uint4 (&buf)[kChunksPerThread]) {
+                                            uint32_t u, uint4 (&buf)[T::kChunksPerThread]) {
   const int K2 = args.K / 2;
   const int kb = c.j * kStagesPerSlot + (int)ug;
   if (c.tile < args.num_tiles && kb < args.k_stages) {
-    const int n0 = (c.tile / args.num_m2) * kBN + (int)pr.rank * kBNHalf;
+    const int n0 = (c.tile / args.num_m2) * T::kBN + (int)pr.rank * T::kBNHalf;
     const uint8_t* src = args.qw + kb * (kBK / 2) + (u & 3u) * 16;
 #pragma unroll
-    for (int i = 0; i < kChunksPerThread; ++i) {
+    for (int i = 0; i < T::kChunksPerThread; ++i) {
       const int n = n0 + (int)(u >> 2) + 16 * i;
       buf[i] = n < args.N ? __ldg(reinterpret_cast<const uint4*>(src + (int64_t)n * K2)) : make_uint4(0u, 0u, 0u, 0u);
     }
@@ -516,18 +539,18 @@ __device__ __forceinline__ void unpack_advance(const Args& args, const Pair& pr,
 
 // Converts this group's stage of ring slot (q % kSlots) into the slot's B half for that stage
 // (or, for the missing second stage of an odd K-stage count, only signals the slot).
-template <bool kOffset>
+template <class T, bool kOffset>
 __device__ __forceinline__ bool unpack_store(const Args& args, uint8_t* sB, const Bars& b, uint32_t ug, uint32_t u,
-                                             uint32_t q, bool has_stage, const uint4 (&buf)[kChunksPerThread],
+                                             uint32_t q, bool has_stage, const uint4 (&buf)[T::kChunksPerThread],
                                              volatile int* abort_flag) {
-  const uint32_t o = q % kSlots;
-  if (!__all_sync(0xffffffffu, mbar_wait(&b.empty[o], ring_parity(q, kSlots) ^ 1u, abort_flag, args.status)))
+  const uint32_t o = q % T::kSlots;
+  if (!__all_sync(0xffffffffu, mbar_wait(&b.empty[o], ring_parity(q, T::kSlots) ^ 1u, abort_flag, args.status)))
     return false;
   if (has_stage) {
-    const uint32_t dst = smem_u32(sB + o * kSlotBBytes + ug * kOpBBytes);
+    const uint32_t dst = smem_u32(sB + o * T::kSlotBBytes + ug * T::kOpBBytes);
     const uint32_t jc = u & 3u;
 #pragma unroll
-    for (int i = 0; i < kChunksPerThread; ++i) {
+    for (int i = 0; i < T::kChunksPerThread; ++i) {
       const uint32_t r = (u >> 2) + 16u * i, r7 = r & 7u;
       uint4 lo, hi;
       if (kOffset)
@@ -550,7 +573,7 @@ __device__ __forceinline__ bool unpack_store(const Args& args, uint8_t* sB, cons
   return true;
 }
 
-template <bool kOffset>
+template <class T, bool kOffset>
 __device__ __forceinline__ void unpack_role(const Args& args, const Pair& pr, uint8_t* sB, const Bars& b,
                                             volatile int* abort_flag) {
   const uint32_t ut = threadIdx.x - kUnpackWarp0 * 32;
@@ -560,22 +583,22 @@ __device__ __forceinline__ void unpack_role(const Args& args, const Pair& pr, ui
   const uint32_t total = static_cast<uint32_t>(my_tiles) * static_cast<uint32_t>(args.slots_per_tile);
   UnpackCursor sc{pr.cluster, 0};  // the slot being stored
   UnpackCursor lc = sc;            // the slot being loaded (two ahead)
-  uint4 b0[kChunksPerThread], b1[kChunksPerThread];
-  unpack_load(args, pr, lc, ug, u, b0);
+  uint4 b0[T::kChunksPerThread], b1[T::kChunksPerThread];
+  unpack_load<T>(args, pr, lc, ug, u, b0);
   unpack_advance(args, pr, lc);
-  unpack_load(args, pr, lc, ug, u, b1);
+  unpack_load<T>(args, pr, lc, ug, u, b1);
   unpack_advance(args, pr, lc);
   for (uint32_t q = 0; q < total; q += 2) {
     bool has = sc.j * kStagesPerSlot + (int)ug < args.k_stages;
-    if (!unpack_store<kOffset>(args, sB, b, ug, u, q, has, b0, abort_flag)) return;
+    if (!unpack_store<T, kOffset>(args, sB, b, ug, u, q, has, b0, abort_flag)) return;
     unpack_advance(args, pr, sc);
-    unpack_load(args, pr, lc, ug, u, b0);
+    unpack_load<T>(args, pr, lc, ug, u, b0);
     unpack_advance(args, pr, lc);
     if (q + 1 < total) {
       has = sc.j * kStagesPerSlot + (int)ug < args.k_stages;
-      if (!unpack_store<kOffset>(args, sB, b, ug, u, q + 1, has, b1, abort_flag)) return;
+      if (!unpack_store<T, kOffset>(args, sB, b, ug, u, q + 1, has, b1, abort_flag)) return;
       unpack_advance(args, pr, sc);
-      unpack_load(args, pr, lc, ug, u, b1);
+      unpack_load<T>(args, pr, lc, ug, u, b1);
       unpack_advance(args, pr, lc);
     }
   }
@@ -585,30 +608,31 @@ __device__ __forceinline__ void unpack_role(const Args& args, const Pair& pr, ui
 // activation-sum correction -- used for one-group problems (G = K), where the drain's exact
 // subtraction runs once per tile; with several groups the drain is the busier role and the
 // weights keep the sign-magnitude form.
-template <bool kExport, bool kOffset>
+template <bool kExport, bool kOffset, int kBN>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     w4a4_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmSW,
                      const __grid_constant__ CUtensorMap tmSA, const Args args) {
+  using T = Tile<kBN>;
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   if ((smem_u32(smem_raw) & 1023u) != 0) {  // uniform across the grid: nothing has been touched yet
     if (threadIdx.x == 0 && args.status != nullptr) atomicExch(args.status, (uint32_t)kDevSmemAlign);
     return;
   }
   uint8_t* smem = smem_raw;
-  uint8_t* sA = smem + kOffA;
-  uint8_t* sB = smem + kOffB;
-  uint64_t* bar = reinterpret_cast<uint64_t*>(smem + kOffBar);
+  uint8_t* sA = smem + T::kOffA;
+  uint8_t* sB = smem + T::kOffB;
+  uint64_t* bar = reinterpret_cast<uint64_t*>(smem + T::kOffBar);
   Bars b;
   b.full = bar;
-  b.empty = b.full + kSlots;
-  b.acc_full = b.empty + kSlots;
-  b.acc_empty = b.acc_full + 2;
-  b.mma_done = b.acc_empty + 2;
+  b.empty = b.full + T::kSlots;
+  b.acc_full = b.empty + T::kSlots;
+  b.acc_empty = b.acc_full + T::kAccBufs;
+  b.mma_done = b.acc_empty + T::kAccBufs;
   b.sc_full = b.mma_done + 1;
   b.sc_empty = b.sc_full + kScSlots;
-  uint8_t* sSc = smem + kOffSc;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + kOffMisc);
-  volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + kOffMisc + 4);
+  uint8_t* sSc = smem + T::kOffSc;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + T::kOffMisc);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + T::kOffMisc + 4);
 
   Pair pr;
   pr.rank = cluster_ctarank();
@@ -618,12 +642,12 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
   const uint32_t warp = warp_id(), lane = lane_id();
   if (threadIdx.x == 0) {
     *abort_flag = 0;
-    for (int i = 0; i < kSlots; ++i) {
+    for (int i = 0; i < T::kSlots; ++i) {
       // the even CTA's expect_tx (both CTAs' A bytes) + every unpack warp of both CTAs
       mbar_init(&b.full[i], 1 + 2 * kUnpackGroups * kUnpackGroupWarps);
       mbar_init(&b.empty[i], 1);  // one pair commit
     }
-    for (int i = 0; i < 2; ++i) {
+    for (int i = 0; i < T::kAccBufs; ++i) {
       mbar_init(&b.acc_full[i], 1);
       mbar_init(&b.acc_empty[i], 2 * kNumDrainWarps);  // every drain warp of both CTAs
     }
@@ -657,28 +681,28 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
   if (warp < kUnpackWarp0 || warp >= kDrainWarp0) pdl_wait();
 
   // Register split per warpgroup (totals the 512 x 128 registers of the launch): producer and
-  // MMA (warps 0-3) 32, unpack (warps 4-7) 96, drain (warps 8-15, 128 running sums) 192.
+  // MMA (warps 0-3) 32, unpack (warps 4-7) 96, drain (warps 8-15, the running sums) 192.
   if (warp >= kDrainWarp0) {
     asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;\n" ::"n"(kRegsDrain) : "memory");
     if (kExport)
-      drain_export<kOffset>(args, pr, tmem_base, b, abort_flag);
+      drain_export<T, kOffset>(args, pr, tmem_base, b, abort_flag);
     else
-      drain_linear<kOffset>(args, pr, tmem_base, b, sSc, abort_flag);
+      drain_linear<T, kOffset>(args, pr, tmem_base, b, sSc, abort_flag);
   } else if (warp >= kUnpackWarp0) {
     asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;\n" ::"n"(kRegsUnpack) : "memory");
-    unpack_role<kOffset>(args, pr, sB, b, abort_flag);
+    unpack_role<T, kOffset>(args, pr, sB, b, abort_flag);
   } else {
     asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;\n" ::"n"(kRegsCtl) : "memory");
     if (warp == kWarpProdA) {
-      if (lane == 0) producer_a(args, pr, &tmA, sA, b, abort_flag);
+      if (lane == 0) producer_a<T>(args, pr, &tmA, sA, b, abort_flag);
     } else if (warp == kWarpScale) {
-      if (!kExport && lane == 0) scale_producer(args, pr, &tmSW, &tmSA, sSc, b, abort_flag);
+      if (!kExport && lane == 0) scale_producer<T>(args, pr, &tmSW, &tmSA, sSc, b, abort_flag);
     } else if (warp == kWarpMma && lane == 0) {
       if (pr.rank == 0) {
         if (args.G < kBK)
-          mma_role<true>(args, pr, tmem_base, sA, sB, b, abort_flag);
+          mma_role<T, true>(args, pr, tmem_base, sA, sB, b, abort_flag);
         else
-          mma_role<false>(args, pr, tmem_base, sA, sB, b, abort_flag);
+          mma_role<T, false>(args, pr, tmem_base, sA, sB, b, abort_flag);
       }
       else  // the even CTA's MMAs read this CTA's shared memory and write its TMEM until here
         drain_wait(b.mma_done, 0, args.status);
@@ -695,8 +719,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
 }
 
 // ---------------------------------------------------------------- host side
-template <bool kExport, bool kOffset>
+template <bool kExport, bool kOffset, int kBN>
 cudaError_t launch_impl(const GemmProblem& p, cudaStream_t stream, int sms) {
+  using T = Tile<kBN>;
   // The A-operand image seen as rows of 128 bytes: block (mt, kb) is rows (mt*k_stages + kb)*128..
   // One box is two consecutive blocks (two K stages of one 128-row tile).  Boxes that reach past
   // the image (the odd CTA of a pair whose rows all lie beyond M, or the second stage of an odd
@@ -724,15 +749,16 @@ cudaError_t launch_impl(const GemmProblem& p, cudaStream_t stream, int sms) {
   int max_pairs = 0;
   cudaError_t se = setup.get(
       [sms](int& pairs) {
-        cudaError_t e = cudaFuncSetAttribute(w4a4_gemm_kernel<kExport, kOffset>,
-                                             cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemBytes);
+        cudaError_t e = cudaFuncSetAttribute(w4a4_gemm_kernel<kExport, kOffset, kBN>,
+                                             cudaFuncAttributeMaxDynamicSharedMemorySize, (int)T::kSmemBytes);
         if (e != cudaSuccess) return e;
         cudaLaunchConfig_t cfg = {};
         cfg.gridDim = dim3(2 * (sms / 2), 1, 1);
         cfg.blockDim = dim3(kThreads, 1, 1);
-        cfg.dynamicSmemBytes = kSmemBytes;
+        cfg.dynamicSmemBytes = T::kSmemBytes;
         int clusters = 0;
-        if (cudaOccupancyMaxActiveClusters(&clusters, w4a4_gemm_kernel<kExport, kOffset>, &cfg) != cudaSuccess ||
+        if (cudaOccupancyMaxActiveClusters(&clusters, w4a4_gemm_kernel<kExport, kOffset, kBN>, &cfg) !=
+                cudaSuccess ||
             clusters <= 0) {
           (void)cudaGetLastError();
           clusters = sms / 2;
@@ -764,8 +790,8 @@ cudaError_t launch_impl(const GemmProblem& p, cudaStream_t stream, int sms) {
   a.partials = p.partials;
   a.status = p.status;
   const int pairs = a.num_tiles < max_pairs ? a.num_tiles : max_pairs;
-  return launch_pdl(w4a4_gemm_kernel<kExport, kOffset>, dim3(2 * pairs), dim3(kThreads), kSmemBytes, stream, tmA,
-                    tmSW, tmSA, a);
+  return launch_pdl(w4a4_gemm_kernel<kExport, kOffset, kBN>, dim3(2 * pairs), dim3(kThreads), T::kSmemBytes, stream,
+                    tmA, tmSW, tmSA, a);
 }
 
 }  // namespace
@@ -802,11 +828,11 @@ cudaError_t launch_w4a4_gemm(const GemmProblem& p, cudaStream_t stream, int sms)
   if (p.M == 0 || p.N == 0) return cudaSuccess;
   // One group: offset-code weights (see w4a4_gemm_kernel), exact while the whole K run fits the
   // offset form's fp32 range (operand.cuh); longer one-group runs keep the sign-magnitude form,
-  // whose sums stay below 2^24 for every K the library accepts.
+  // whose sums stay below 2^24 for every K the library accepts.  Group scales: 128-column tiles.
   const bool offset = p.G == p.K && p.K <= kOffsetMaxRun;
   if (p.partials != nullptr)
-    return offset ? launch_impl<true, true>(p, stream, sms) : launch_impl<true, false>(p, stream, sms);
-  return offset ? launch_impl<false, true>(p, stream, sms) : launch_impl<false, false>(p, stream, sms);
+    return offset ? launch_impl<true, true, 256>(p, stream, sms) : launch_impl<true, false, 256>(p, stream, sms);
+  return offset ? launch_impl<false, true, 256>(p, stream, sms) : launch_impl<false, false, 256>(p, stream, sms);
 }
 
 }  // namespace jq
