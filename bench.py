@@ -60,6 +60,23 @@ WORKLOADS = {
     "sweep_m64": ("M sweep: M=64 tokens x K=4096 -> N=12288, per-token/per-channel (group = K)", 64, 4096, 12288,
                   4096, "sweep_a"),
 }
+# DiT-XL/2 block linears (16 images of 256 tokens, group128) with the neighbour operation that
+# feeds each one fused into the activation quantiser: the adaLN modulation before the attention's
+# QKV projection and the MLP's first linear, the tanh GELU before the MLP's second linear; the
+# attention output projection takes the plain quantiser.
+DIT = {
+    "dit_qkv": ("DiT-XL/2 attention QKV: 16 images x 256 tokens = 4096 x 1152 -> 3456, group128, "
+                "modulation fused into the quantiser", 4096, 1152, 3456, 128, "dit", "modulate"),
+    "dit_proj": ("DiT-XL/2 attention output projection: 4096 x 1152 -> 1152, group128", 4096, 1152, 1152, 128, "dit",
+                 None),
+    "dit_fc1": ("DiT-XL/2 MLP in: 4096 x 1152 -> 4608, group128, modulation fused into the quantiser", 4096, 1152,
+                4608, 128, "dit", "modulate"),
+    "dit_fc2": ("DiT-XL/2 MLP out: 4096 x 4608 -> 1152, group128, tanh GELU fused into the quantiser", 4096, 4608,
+                1152, 128, "dit", "gelu"),
+}
+for _n, _v in DIT.items():
+    WORKLOADS[_n] = _v[:6]
+DIT_PROLOGUE = {n: v[6] for n, v in DIT.items()}
 # The whole M sweep of the memory-to-compute crossover, at both shapes (per-token/per-channel
 # scales, group = K): M <= 64 runs the few-token kernel, larger M the GEMM.
 SWEEP_M = (1, 16, 64, 256, 1024, 4096, 16384)
@@ -76,7 +93,10 @@ FP8_PER_BF16 = 2.0  # nominal dense FP8 / BF16 tensor-core ratio on GB300 (4.5 /
 # from an ncu capture of that kernel, keyed by workload and by the hash of the kernel code the
 # capture was taken on (kernel_hash); once the code changes the figure no longer applies and the
 # bench reports null until a new capture is recorded here.
-KERNEL_TRAFFIC: dict = {}
+KERNEL_TRAFFIC: dict = {
+    ("flux_qkv", "d0d1b1f0f83343fb"): 54.647296e6 + 143.780096e6,
+    ("dllm", "d0d1b1f0f83343fb"): 31.236864e6 + 0.134656e6,
+}
 
 
 def recorded_traffic(workload: str, kernel_file: str):
@@ -204,16 +224,25 @@ class OracleSample:
         self.oracle = oracle
         self.name = name
         self.desc, self.M, self.K, self.N, self.G, gen = WORKLOADS[name]
-        w = wl.make(gen, seed=seed, M=self.M, G=self.G)
+        w = wl.make(gen, seed=seed, M=self.M, K=self.K, N=self.N, G=self.G)
         self.x_bits, self.bias = w.x_bits, w.bias
         quant = oracle.quantize_ternary_f32 if ternary else oracle.quantize_f32
         self.qw, self.sw = quant(w.w, self.G)
         self.rows = 8
         self.run_s = 0.0
+        self.tokens_per_sample = wl.DIT_TOKENS_PER_IMAGE
+        self.mod = wl.dit_modulation(seed, -(-self.M // self.tokens_per_sample), self.K)
 
     def run(self, rows: int) -> float:
         t0 = time.perf_counter()
-        qa, sa = self.oracle.quantize_bf16(self.x_bits[:rows], self.G)
+        prologue = DIT_PROLOGUE.get(self.name)
+        if prologue == "modulate":
+            _, qa, sa = self.oracle.modulate_quantize_bf16(self.x_bits[:rows], self.mod[0], self.mod[1],
+                                                           self.tokens_per_sample, self.G)
+        elif prologue == "gelu":
+            _, qa, sa = self.oracle.gelu_quantize_bf16(self.x_bits[:rows], self.G)
+        else:
+            qa, sa = self.oracle.quantize_bf16(self.x_bits[:rows], self.G)
         self.oracle.linear(qa, sa, self.qw, self.sw, self.bias, self.G)
         return time.perf_counter() - t0
 
@@ -332,6 +361,56 @@ def cublas_context(torch, dev, sets, M, N, K, args, world):
     torch.cuda.empty_cache()
     return {"value": world * 2.0 * M * N * K / (ms * 1e-3) / 1e12, "unit": "TFLOP/s", "ms_per_call": ms,
             "what": "torch.matmul bf16 x[M,K] @ W[N,K]^T, same M, N, K"}
+
+
+def prologue_context(torch, jq, sets, mods, prologue, G, T, q, s_a, args):
+    """The DiT neighbour operation fused into the quantiser against the same operation done
+    separately (PyTorch bf16 ops writing the activation, then jq_quantize_act reading it back),
+    each as a CUDA graph of K launches over the rotating inputs."""
+    n = len(sets)
+
+    def graph_ms(fn):
+        cap = torch.cuda.Stream()
+        cap.wait_stream(torch.cuda.current_stream())
+        with torch.cuda.stream(cap):
+            for i in range(args.warmup):
+                fn(i, cap)
+        cap.synchronize()
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=cap):
+            for i in range(args.steps):
+                fn(i, cap)
+        g.replay()
+        torch.cuda.synchronize()
+        t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        t0.record()
+        g.replay()
+        t1.record()
+        torch.cuda.synchronize()
+        return t0.elapsed_time(t1) / args.steps
+
+    def fused(i, st):
+        x = sets[i % n][0]
+        if prologue == "modulate":
+            jq.jq_modulate_quantize_act(x, mods[i % n][0], mods[i % n][1], T, G, q, s_a, stream=st)
+        else:
+            jq.jq_gelu_quantize_act(x, G, q, s_a, stream=st)
+
+    def separate(i, st):
+        x = sets[i % n][0]
+        M = x.shape[0]
+        if prologue == "modulate":
+            sh, sc = mods[i % n]
+            rows = torch.arange(M, device=x.device) // T
+            z = (x.float() * (1.0 + sc[rows]) + sh[rows]).to(torch.bfloat16)
+        else:
+            z = torch.nn.functional.gelu(x, approximate="tanh")
+        jq.jq_quantize_act(z, G, q, s_a, stream=st)
+
+    f, sep = graph_ms(fused), graph_ms(separate)
+    return {"fused_us": f * 1e3, "separate_us": sep * 1e3,
+            "what": f"{prologue} fused into the activation quantiser vs the PyTorch {prologue} writing bf16 "
+                    "followed by jq_quantize_act (per launch, CUDA graph)"}
 
 
 # ----------------------------------------------------------------------------- memory-bound kernels
@@ -585,7 +664,7 @@ def run_ours(args):
     # rotating weight sets: together several times larger than the 126 MB L2
     n_sets = args.sets if args.sets > 0 else max(6, -(-400_000_000 // (N * K // 2 + M * K * 2)))
     for i in range(n_sets):
-        w = wl.make(gen, seed=100 + 17 * rank + i, M=M, G=G)
+        w = wl.make(gen, seed=100 + 17 * rank + i, M=M, K=K, N=N, G=G)
         x = torch.from_numpy(w.x_bits.view(np.int16)).to(dev).view(torch.bfloat16)
         pack = jq.jq_pack_weight_ternary if args.weights == "ternary" else jq.jq_pack_weight
         qw, sw = pack(torch.from_numpy(w.w).to(dev), G)
@@ -603,8 +682,21 @@ def run_ours(args):
     linear_call = jq.jq_w158a4_linear if ternary else jq.jq_w4a4_linear
     stream = torch.cuda.current_stream()
 
+    prologue = DIT_PROLOGUE.get(args.workload)
+    T = wl.DIT_TOKENS_PER_IMAGE
+    if prologue == "modulate":
+        mods = [tuple(torch.from_numpy(a).to(dev) for a in wl.dit_modulation(300 + 31 * rank + i, -(-M // T), K))
+                for i in range(n_sets)]
+
     def quantize(i, st):
-        jq.jq_quantize_act(sets[i % n_sets][0], G, q, s_a, stream=st)
+        x = sets[i % n_sets][0]
+        if prologue == "modulate":
+            sh, sc = mods[i % n_sets]
+            jq.jq_modulate_quantize_act(x, sh, sc, T, G, q, s_a, stream=st)
+        elif prologue == "gelu":
+            jq.jq_gelu_quantize_act(x, G, q, s_a, stream=st)
+        else:
+            jq.jq_quantize_act(x, G, q, s_a, stream=st)
 
     def linear(i, st):
         x, qw, sw, b = sets[i % n_sets]
@@ -683,6 +775,15 @@ def run_ours(args):
     x_free = [None] * nb  # the kernels that read x_dev[k] are done
     y_free = [None] * nb  # the copy out of y_dev[k] is done
 
+    def quantize_x(x, i, st):
+        if prologue == "modulate":
+            sh, sc = mods[i % n_sets]
+            jq.jq_modulate_quantize_act(x, sh, sc, T, G, q, s_a, stream=st)
+        elif prologue == "gelu":
+            jq.jq_gelu_quantize_act(x, G, q, s_a, stream=st)
+        else:
+            jq.jq_quantize_act(x, G, q, s_a, stream=st)
+
     def e2e_step(i):
         k = i % nb
         if not pipelined:
@@ -691,7 +792,7 @@ def run_ours(args):
             if fused:
                 jq.jq_fused_quant_linear(x_dev[0], qw, sw, b, G, y=y_dev[0], workspace=ws, stream=stream)
             else:
-                jq.jq_quantize_act(x_dev[0], G, q, s_a, stream=stream)
+                quantize_x(x_dev[0], i, stream)
                 linear_call(q, s_a, qw, sw, b, G, y=y_dev[0], workspace=ws, stream=stream)
             y_host[0].copy_(y_dev[0], non_blocking=True)
             return
@@ -708,7 +809,7 @@ def run_ours(args):
         if fused:
             jq.jq_fused_quant_linear(x_dev[k], qw, sw, b, G, y=y_dev[k], workspace=ws, stream=stream)
         else:
-            jq.jq_quantize_act(x_dev[k], G, q, s_a, stream=stream)
+            quantize_x(x_dev[k], i, stream)
             linear_call(q, s_a, qw, sw, b, G, y=y_dev[k], workspace=ws, stream=stream)
         done = torch.cuda.Event()
         done.record(stream)
@@ -767,6 +868,9 @@ def run_ours(args):
     context = None
     if not args.no_context:
         context = {"cublas_bf16": cublas_context(torch, dev, sets, M, N, K, args, world)}
+        if prologue is not None:
+            context["prologue"] = prologue_context(torch, jq, sets, mods if prologue == "modulate" else None, prologue,
+                                                   G, T, q, s_a, args)
 
     if rank != 0:
         if world > 1:
@@ -784,7 +888,10 @@ def run_ours(args):
         "vs_baseline": None, "dtype": "int4", "data": "synthetic",
         "config": {"workload": desc, "M": M, "K": K, "N": N, "group": G,
                    "step": ("jq_fused_quant_linear" if fused else
-                            "jq_quantize_act + jq_w158a4_linear" if ternary else "jq_quantize_act + jq_w4a4_linear"),
+                            "jq_quantize_act + jq_w158a4_linear" if ternary else
+                            "jq_modulate_quantize_act + jq_w4a4_linear" if prologue == "modulate" else
+                            "jq_gelu_quantize_act + jq_w4a4_linear" if prologue == "gelu" else
+                            "jq_quantize_act + jq_w4a4_linear"),
                    "weights": "ternary (2-bit)" if ternary else "INT4",
                    "launch": "CUDA graph of the K steps",
                    "parallelism": f"replicas x{world}",

@@ -36,10 +36,10 @@
  *     crosses the ABI.
  *   - Every on-GPU wait is bounded (about a second).  A kernel that gives up records
  *     JQ_ERR_TIMEOUT in a device status word read by jq_device_status().
- *   - Devices and threads: this version sets its kernels' shared-memory attributes once per
- *     process, on the first device that launches them, so drive one GPU per process (calls on
- *     a second device of the same process may fail with JQ_ERR_CUDA), and make the first call on a
- *     device from one thread; after that, calls from several threads are safe.
+ *   - Devices and threads: kernels launch on the CURRENT device (cudaGetDevice) and all
+ *     pointers must belong to it.  Per-device launch set-up (kernel attributes, occupancy
+ *     probes, the device status word) happens on a device's first call, under a mutex, so a
+ *     process may drive several GPUs and call from several host threads, first calls included.
  *   - Kernels are launched with programmatic dependent launch: one of this library's kernels may
  *     start while the previous kernel on the stream is still running, when that kernel is also
  *     one of this library's (the linear layers start streaming their weights early), and waits
@@ -72,11 +72,14 @@ typedef enum {
   JQ_ERR_WORKSPACE = 6     /* workspace pointer NULL/misaligned or smaller than required */
 } jq_status;
 
-/* Human-readable name of a status code (static string, never NULL). */
+/* Human-readable name of a status code (static string, never NULL; no counterpart in the paper). */
 JQ_API const char* jq_status_string(jq_status s);
 
 /*
- * Activation quantiser (per token and K-group; rule above).
+ * Activation quantiser (per token and K-group; rule above).  The paper quantises the activations
+ * of the transformer-block linears to INT4 with group64 (Sec. 4.2 "FLUX"; Appendix "FLUX
+ * experimental details") or group128 (Appendix "DiT-XL/2 experimental details", "ELF-B and
+ * LLaDA-8B experimental details"); the formula is the reading above.
  *   x_bf16 : bf16 [M, ldx] (the first K columns are used), ldx >= K, ldx*2 % 16 == 0
  *   q      : uint8 [M, K/2] packed codes (output)
  *   s_a    : fp32 [M, K/group] scales (output)
@@ -87,7 +90,9 @@ JQ_API jq_status jq_quantize_act(const void* x_bf16, int64_t M, int64_t K, int64
                           uint8_t* q, float* s_a, void* stream);
 
 /*
- * Weight packer (offline; the same rule per output channel and K-group).
+ * Weight packer (offline; the same rule per output channel and K-group).  INT4 weights with the
+ * activations' group size (the same Appendix tables); packing is one of the kernels the deployed
+ * graph needs (Appendix FAQ Q7).
  *   w   : fp32 [N, K] row-major
  *   qw  : uint8 [N, K/2] packed codes (output)
  *   s_w : fp32 [K/group, N] scales (output, group-major)
@@ -97,14 +102,49 @@ JQ_API jq_status jq_pack_weight(const float* w, int64_t N, int64_t K, int32_t gr
                          void* stream);
 
 /*
+ * DiT neighbour operations fused with the activation quantiser.  The paper's deployment remark
+ * (Sec. 1, the figure on naive W1.58A4 deployment) concerns a 0.6B DiT, DiT-XL/2, where small
+ * matrices and non-GEMM time limit the speed-up; its W4A4 / W1.58A4 setting there is group128
+ * (Appendix "DiT-XL/2 experimental details").  In a DiT-XL/2 block the inputs of the linears
+ * come from the adaLN modulation (before the attention's QKV projection and the MLP's first
+ * linear) and from the MLP's tanh GELU (before its second linear); these calls read that
+ * operation's input and write the quantised codes of its output, so the bf16 activation between
+ * the two never goes to memory.  The paper prints neither operation; the readings:
+ *   modulation: token m of sample b = m / tokens_per_sample, channel k:
+ *     z = bf16( fl32( fl32( x * fl32(1 + scale[b,k]) ) + shift[b,k] ) )
+ *     (IEEE single steps, no fused multiply-add, one rounding to bf16, nearest even);
+ *   GELU: z = bf16( 0.5 h (1 + tanh(sqrt(2/pi) (h + 0.044715 h^3))) ), the exact value rounded
+ *     once to bf16 (nearest even; +-0 stays +-0);
+ * then the activation rule above on z.  Codes and scales are exactly those of
+ * jq_quantize_act applied to z.
+ *   x_bf16 / h_bf16 : bf16 [M, ldx] (ldx >= K, ldx*2 % 16 == 0)
+ *   shift, scale    : fp32 [ceil(M / tokens_per_sample), K], dense rows (modulation)
+ *   tokens_per_sample > 0
+ *   q, s_a          : outputs as jq_quantize_act
+ * Errors as jq_quantize_act (JQ_ERR_INVALID_ARG also for tokens_per_sample <= 0 or a NULL
+ * shift / scale).
+ */
+JQ_API jq_status jq_modulate_quantize_act(const void* x_bf16, int64_t M, int64_t K, int64_t ldx, const float* shift,
+                                          const float* scale, int64_t tokens_per_sample, int32_t group, uint8_t* q,
+                                          float* s_a, void* stream);
+JQ_API jq_status jq_gelu_quantize_act(const void* h_bf16, int64_t M, int64_t K, int64_t ldh, int32_t group,
+                                      uint8_t* q, float* s_a, void* stream);
+
+/*
  * Bytes of device scratch the two linear entry points need for this shape
- * (fused != 0: jq_fused_quant_linear, else jq_w4a4_linear).  The caller owns it.
+ * (fused != 0: jq_fused_quant_linear, else jq_w4a4_linear).  The caller owns it.  (The paper has
+ * no counterpart: the scratch holds the activations in the GEMM's operand layout, the library's
+ * own design, so that the library itself never allocates.)
  */
 JQ_API size_t jq_workspace_size(int64_t M, int64_t N, int64_t K, int32_t group, int32_t fused);
 
 /*
- * W4A4 linear on pre-quantised activations:
+ * W4A4 linear on pre-quantised activations -- the deployed "naive W4A4" linear layer, a plain
+ * low-bit GEMM with no smoothing, rotation or SVD branch (Sec. 1; Appendix FAQ Q7), with group
+ * scales (Sec. 4.2; Appendix experimental-detail tables):
  *   y = bf16( sum_g acc[m,n,g] * s_a[m,g] * s_w[g,n] + bias[n] ).
+ *   (The weight scales are group-major [K/group, N] so that one group's channel scales are
+ *   contiguous for the GEMM's scale loads; the workspace keeps allocation with the caller.)
  *   q         : uint8 [M, K/2] packed activation codes (jq_quantize_act)
  *   s_a       : fp32 [M, K/group]
  *   qw, s_w   : packed weights and scales (jq_pack_weight, or any codes/finite scales in
@@ -119,8 +159,9 @@ JQ_API jq_status jq_w4a4_linear(const uint8_t* q, const float* s_a, const uint8_
                          void* workspace, size_t workspace_bytes, void* stream);
 
 /*
- * W4A4 linear straight from bf16 activations: quantises x (rule above, per token and
- * K-group) directly into the GEMM's operand layout, then runs the same GEMM.  Results are
+ * W4A4 linear straight from bf16 activations (the quantise + low-bit GEMM pair of Appendix FAQ
+ * Q7 in one call): quantises x (rule above, per token and K-group) directly into the GEMM's
+ * operand layout, then runs the same GEMM.  Results are
  * bit-identical to jq_quantize_act followed by jq_w4a4_linear.
  *   x_bf16    : bf16 [M, ldx]
  *   workspace : >= jq_workspace_size(M, N, K, group, 1) bytes
@@ -131,7 +172,8 @@ JQ_API jq_status jq_fused_quant_linear(const void* x_bf16, int64_t ldx, const ui
                                 int32_t group, void* workspace, size_t workspace_bytes, void* stream);
 
 /*
- * Verification export of the exact per-group integer partials of the GEMM:
+ * Verification export of the exact per-group integer partials of the GEMM (no counterpart in the
+ * paper; it exposes the exact integer sums of the linear layer above for testing):
  *   acc : int32 [M, N, K/group], acc[m,n,g] = sum_{k in g} qa[m,k] * qw[n,k].
  * Runs the same mainloop as jq_w4a4_linear with the dequantising epilogue replaced by an
  * integer store; meant for small shapes.  workspace as jq_w4a4_linear.
@@ -185,7 +227,8 @@ JQ_API jq_status jq_w4a4_linear_noalloc(const uint8_t* q, const float* s_a, cons
 JQ_API jq_status jq_pack_weight_ternary(const float* w, int64_t N, int64_t K, int32_t group, uint8_t* qw2,
                                         float* s_w, void* stream);
 
-/* Bytes of device scratch jq_w158a4_linear needs for this shape (the caller owns it). */
+/* Bytes of device scratch jq_w158a4_linear needs for this shape (the caller owns it; as
+ * jq_workspace_size, the paper has no counterpart). */
 JQ_API size_t jq_w158a4_workspace_size(int64_t M, int64_t N, int64_t K, int32_t group);
 
 /*
@@ -248,7 +291,8 @@ JQ_API jq_status jq_ste_backward(const void* grad_bf16, const uint8_t* mask, int
                                  void* stream);
 
 /*
- * Verification export for failure handling (computes nothing): launches one block in which one
+ * Verification export for failure handling (computes nothing; no counterpart in the paper):
+ * launches one block in which one
  * thread waits, with the bounded wait every kernel of this library uses, on an mbarrier phase
  * that nothing completes.  After about 2^31 SM clock cycles (about a second) the wait gives up
  * and records JQ_ERR_TIMEOUT in the device status word, which jq_device_status() then reports;
@@ -258,6 +302,7 @@ JQ_API jq_status jq_ste_backward(const void* grad_bf16, const uint8_t* mask, int
 JQ_API jq_status jq_debug_wait_timeout(void* stream);
 
 /*
+ * (No counterpart in the paper; the library's failure reporting.)
  * Synchronises `stream` and returns JQ_ERR_TIMEOUT if any kernel of this library on the
  * current device gave up a bounded wait since the last reset (reset != 0 clears the flag),
  * JQ_ERR_UNSUPPORTED if a GEMM launch found its shared-memory window not 1024-byte aligned

@@ -18,7 +18,9 @@ numpy arrays through ctypes.  Layout conventions used here:
   [-12, 12]); block scales ``float32 [rows, K/16]`` (each an E4M3 value);
   packed ``uint8 [rows, K/2]`` in the 4-bit E2M1 encoding, element 2j in the
   low nibble;
-* bf16 values travel as their ``uint16`` bit patterns.
+* bf16 values travel as their ``uint16`` bit patterns;
+* DiT neighbour operations fused with the quantiser (adaLN modulation, tanh
+  GELU): the modulated / activated bf16 bits come back beside the codes.
 """
 from __future__ import annotations
 
@@ -80,11 +82,16 @@ def _load():
             lib.oracle_fake_quant_bf16.argtypes = [vp, i64, i64, i64, vp, vp, vp, vp]
             lib.oracle_fake_quant_f32.argtypes = [vp, i64, i64, i64, vp, vp, vp, vp]
             lib.oracle_ste_backward_bf16.argtypes = [vp, vp, i64, vp]
+            lib.oracle_gelu_tanh_f32.argtypes = [ctypes.c_float]
+            lib.oracle_gelu_tanh_f32.restype = ctypes.c_float
+            lib.oracle_modulate_quantize_bf16.argtypes = [vp, i64, i64, i64, vp, vp, i64, i64, vp, vp, vp]
+            lib.oracle_gelu_quantize_bf16.argtypes = [vp, i64, i64, i64, i64, vp, vp, vp]
             for f in ("oracle_fake_quant_bf16", "oracle_fake_quant_f32", "oracle_ste_backward_bf16",
                       "oracle_quantize_bf16", "oracle_quantize_f32", "oracle_pack", "oracle_unpack",
                       "oracle_group_partials", "oracle_linear", "oracle_quantize_ternary_f32",
                       "oracle_pack_ternary", "oracle_unpack_ternary", "oracle_quantize_nvfp4",
-                      "oracle_pack_nvfp4", "oracle_unpack_nvfp4", "oracle_linear_nvfp4"):
+                      "oracle_pack_nvfp4", "oracle_unpack_nvfp4", "oracle_linear_nvfp4",
+                      "oracle_modulate_quantize_bf16", "oracle_gelu_quantize_bf16"):
                 getattr(lib, f).restype = None
             _lib = lib
     return _lib
@@ -298,3 +305,50 @@ def ste_backward_bf16(grad_bits: np.ndarray, mask: np.ndarray) -> np.ndarray:
     out = np.empty_like(grad_bits)
     _load().oracle_ste_backward_bf16(_p(grad_bits), _p(mask), grad_bits.size, _p(out))
     return out
+
+
+def gelu_tanh_f32(h: float) -> float:
+    """The tanh-approximate GELU of one fp32 value, in the oracle's fp32 steps."""
+    return float(_load().oracle_gelu_tanh_f32(ctypes.c_float(h)))
+
+
+def _rows(a):
+    a = np.asarray(a)
+    assert a.dtype == np.uint16 and a.ndim == 2
+    if a.strides[1] != 2 or a.strides[0] % 2:
+        a = np.ascontiguousarray(a)
+    return a, a.strides[0] // 2
+
+
+def modulate_quantize_bf16(x_bits: np.ndarray, shift: np.ndarray, scale: np.ndarray, tokens_per_sample: int,
+                           group: int):
+    """adaLN modulation fused with the activation quantiser (DiT-XL/2 block linears).
+
+    x_bits uint16 [M, K] (bf16 bits, rows may be strided); shift, scale f32 [B, K] with
+    B = ceil(M / tokens_per_sample) -> (z uint16 [M, K] the modulated bf16 bits,
+    codes int8 [M, K], scales f32 [M, K/G])."""
+    x_bits, ldx = _rows(x_bits)
+    M, K = x_bits.shape
+    assert K % group == 0 and tokens_per_sample > 0
+    sh, sc = _c(shift, np.float32), _c(scale, np.float32)
+    assert sh.shape == sc.shape and sh.shape[1] == K and sh.shape[0] * tokens_per_sample >= M
+    z = np.empty((M, K), np.uint16)
+    codes = np.empty((M, K), np.int8)
+    scales = np.empty((M, K // group), np.float32)
+    _load().oracle_modulate_quantize_bf16(_p(x_bits), M, K, ldx, _p(sh), _p(sc), tokens_per_sample, group, _p(z),
+                                          _p(codes), _p(scales))
+    return z, codes, scales
+
+
+def gelu_quantize_bf16(h_bits: np.ndarray, group: int):
+    """tanh-approximate GELU fused with the activation quantiser (the input of a DiT MLP's second
+    linear): h_bits uint16 [M, K] -> (z uint16 [M, K] = bf16 of the fp32-evaluated GELU(h),
+    codes int8 [M, K], scales f32 [M, K/G])."""
+    h_bits, ldh = _rows(h_bits)
+    M, K = h_bits.shape
+    assert K % group == 0
+    z = np.empty((M, K), np.uint16)
+    codes = np.empty((M, K), np.int8)
+    scales = np.empty((M, K // group), np.float32)
+    _load().oracle_gelu_quantize_bf16(_p(h_bits), M, K, ldh, group, _p(z), _p(codes), _p(scales))
+    return z, codes, scales

@@ -522,3 +522,125 @@ void oracle_fake_quant_f32(const float* w, int64_t N, int64_t K, int64_t G, cons
 void oracle_ste_backward_bf16(const uint16_t* grad, const uint8_t* mask, int64_t n, uint16_t* grad_x) {
   for (int64_t i = 0; i < n; ++i) grad_x[i] = mask[i] ? grad[i] : (uint16_t)0;
 }
+
+/* ---- DiT-XL/2 neighbour operations fused with the activation quantiser ---
+ *
+ * In a DiT-XL/2 block (the 0.6B model of the paper's Sec. 1 deployment remark
+ * and of its W4A4 / W1.58A4 group128 experiments, Appendix table "DiT-XL/2
+ * experimental details") the inputs of the block linears come from small
+ * elementwise operations: the adaLN modulation x (1 + scale) + shift of the
+ * normalised tokens feeds the attention's QKV projection and the MLP's first
+ * linear, and the MLP's GELU (tanh approximation) feeds its second linear.
+ * The paper prints neither operation; these are the readings:
+ *   - modulation: per token m of sample b = m / T (T tokens per sample) and
+ *     channel k, the bf16 value the linear layer receives is
+ *         z = bf16( fl32( fl32( x * fl32(1 + scale[b,k]) ) + shift[b,k] ) ),
+ *     each step an IEEE single operation (no fused multiply-add), rounded
+ *     once to bf16 (nearest even);
+ *   - GELU: the tanh approximation 0.5 h (1 + tanh(sqrt(2/pi) (h + 0.044715 h^3)))
+ *     evaluated in fp32 by a fully specified sequence of IEEE single operations
+ *     (oracle_gelu_tanh_f32: 1 + tanh(u) as 2 sigma(2u), the logistic through
+ *     an exponential of Cody and Waite's reduction and a degree-8 Taylor
+ *     polynomial), then rounded to bf16, as a bf16 model evaluates it (in fp32,
+ *     then stored in bf16).  The kernels execute the same operations, so the
+ *     two agree bit for bit; the fp32 value is within a few ulps of the exact
+ *     GELU where h >= -9 (below that the logistic underflows: |GELU| < 2^-105).
+ * Then z is quantised by the activation rule of the file header.  The
+ * functions also return z, so that the two steps can be checked apart.
+ */
+
+static uint16_t modulate_bf16(float x, float shift, float scale) {
+  const float one_plus = 1.0f + scale; /* IEEE single */
+  const float t = x * one_plus;        /* IEEE single */
+  const float z = t + shift;           /* IEEE single */
+  return oracle_bf16_rne((double)z);   /* exact widening, one rounding to bf16 */
+}
+
+/* 2^n as an fp32 (n in [-126, 127]), built from its bit pattern. */
+static float pow2_f32(int n) {
+  const uint32_t u = (uint32_t)(n + 127) << 23;
+  float f;
+  memcpy(&f, &u, sizeof f);
+  return f;
+}
+
+/* e^x for x <= 0 in fp32 steps.  Cody and Waite's argument reduction: n = rint(x log2 e),
+ * r = x - n ln2 with ln2 split into a 15-bit high part (whose product with n is exact for
+ * |n| <= 150) and a low part, each subtracted by one fused multiply-add; e^r by its Taylor
+ * polynomial to degree 8 in Horner form with fused multiply-adds (|r| <= 0.35, the truncation
+ * below 2^-32); then e^x = 2^n e^r, the power of two applied by one product, or by two where
+ * 2^n is below the normal range (each product one IEEE rounding).  Below x = -104, e^x rounds
+ * to 0 in fp32 and 0 is returned. */
+static float exp_neg_f32(float x) {
+  if (x < -104.0f) return 0.0f;
+  const float n = rintf(x * 0x1.715476p+0f);
+  float r = fmaf(-n, 0x1.62e4p-1f, x);
+  r = fmaf(-n, 0x1.7f7d1cp-20f, r);
+  float p = 0x1.a01a02p-16f;        /* 1/8! */
+  p = fmaf(p, r, 0x1.a01a02p-13f);  /* 1/7! */
+  p = fmaf(p, r, 0x1.6c16c2p-10f);  /* 1/6! */
+  p = fmaf(p, r, 0x1.111112p-7f);   /* 1/5! */
+  p = fmaf(p, r, 0x1.555556p-5f);   /* 1/4! */
+  p = fmaf(p, r, 0x1.555556p-3f);   /* 1/3! */
+  p = fmaf(p, r, 0x1p-1f);          /* 1/2! */
+  p = fmaf(p, r, 1.0f);
+  p = fmaf(p, r, 1.0f);
+  const int ni = (int)n;
+  if (ni >= -126) return p * pow2_f32(ni);
+  return (p * pow2_f32(ni + 64)) * 0x1p-64f;
+}
+
+/* The tanh GELU of one value in fp32 steps (the reading in the section header):
+ * u = fl32(0.7978846 * fl32(h + fl32(0.044715 * fl32(fl32(h * h) * h)))), sigma(2u) as
+ * 1 / (1 + e^{-2u}) for u >= 0 and e^{2u} / (1 + e^{2u}) for u < 0 (exp_neg_f32), and
+ * g = fl32(h * sigma); +-0 gives +-0. */
+float oracle_gelu_tanh_f32(float h) {
+  if (h == 0.0f) return h;
+  const float h3 = (h * h) * h;
+  const float p = h + 0x1.6e4e26p-5f * h3;
+  const float u = 0x1.988454p-1f * p;
+  float sig;
+  if (u >= 0.0f) {
+    sig = 1.0f / (1.0f + exp_neg_f32(-2.0f * u));
+  } else {
+    const float e = exp_neg_f32(2.0f * u);
+    sig = e / (1.0f + e);
+  }
+  return h * sig;
+}
+
+void oracle_modulate_quantize_bf16(const uint16_t* x, int64_t M, int64_t K, int64_t ldx, const float* shift,
+                                   const float* scale, int64_t tokens_per_sample, int64_t G, uint16_t* z,
+                                   int8_t* codes, float* scales) {
+  const int64_t ng = K / G;
+#pragma omp parallel for schedule(static)
+  for (int64_t m = 0; m < M; ++m) {
+    const int64_t b = m / tokens_per_sample;
+    float* zf = (float*)malloc((size_t)K * sizeof(float));
+    for (int64_t k = 0; k < K; ++k) {
+      const uint16_t zb = modulate_bf16(bf16_bits_to_float(x[m * ldx + k]), shift[b * K + k], scale[b * K + k]);
+      z[m * K + k] = zb;
+      zf[k] = bf16_bits_to_float(zb);
+    }
+    for (int64_t g = 0; g < ng; ++g)
+      scales[m * ng + g] = quantize_group(zf + g * G, G, codes + m * K + g * G);
+    free(zf);
+  }
+}
+
+void oracle_gelu_quantize_bf16(const uint16_t* h, int64_t M, int64_t K, int64_t ldh, int64_t G, uint16_t* z,
+                               int8_t* codes, float* scales) {
+  const int64_t ng = K / G;
+#pragma omp parallel for schedule(static)
+  for (int64_t m = 0; m < M; ++m) {
+    float* zf = (float*)malloc((size_t)K * sizeof(float));
+    for (int64_t k = 0; k < K; ++k) {
+      const uint16_t zb = oracle_bf16_rne((double)oracle_gelu_tanh_f32(bf16_bits_to_float(h[m * ldh + k])));
+      z[m * K + k] = zb;
+      zf[k] = bf16_bits_to_float(zb);
+    }
+    for (int64_t g = 0; g < ng; ++g)
+      scales[m * ng + g] = quantize_group(zf + g * G, G, codes + m * K + g * G);
+    free(zf);
+  }
+}

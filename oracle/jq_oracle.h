@@ -37,6 +37,12 @@ void oracle_fake_quant_bf16(const uint16_t* x, int64_t M, int64_t K, int64_t G, 
 void oracle_fake_quant_f32(const float* w, int64_t N, int64_t K, int64_t G, const float* s_in,
                            float* what, uint8_t* mask, float* s_out);
 void oracle_ste_backward_bf16(const uint16_t* grad, const uint8_t* mask, int64_t n, uint16_t* grad_x);
+float oracle_gelu_tanh_f32(float h);
+void oracle_modulate_quantize_bf16(const uint16_t* x, int64_t M, int64_t K, int64_t ldx, const float* shift,
+                                   const float* scale, int64_t tokens_per_sample, int64_t G, uint16_t* z,
+                                   int8_t* codes, float* scales);
+void oracle_gelu_quantize_bf16(const uint16_t* h, int64_t M, int64_t K, int64_t ldh, int64_t G, uint16_t* z,
+                               int8_t* codes, float* scales);
 #ifdef __cplusplus
 }
 #endif

@@ -27,7 +27,7 @@ __all__ = [
     "jq_fused_quant_linear", "jq_w4a4_group_partials", "jq_device_status", "jq_status_string",
     "jq_w4a4_linear_noalloc", "jq_pack_weight_ternary", "jq_w158a4_workspace_size", "jq_w158a4_linear",
     "jq_debug_wait_timeout", "jq_fake_quant_act", "jq_fake_quant_weight",
-    "jq_ste_backward",
+    "jq_ste_backward", "jq_modulate_quantize_act", "jq_gelu_quantize_act",
 ]
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
@@ -70,6 +70,8 @@ def _load() -> ctypes.CDLL:
                 "jq_w4a4_linear_noalloc": [vp, vp, vp, vp, vp, vp, i64, i64, i64, i32, vp],
                 "jq_pack_weight_ternary": [vp, i64, i64, i32, vp, vp, vp],
                 "jq_w158a4_linear": [vp, vp, vp, vp, vp, vp, i64, i64, i64, i32, vp, sz, vp],
+                "jq_modulate_quantize_act": [vp, i64, i64, i64, vp, vp, i64, i32, vp, vp, vp],
+                "jq_gelu_quantize_act": [vp, i64, i64, i64, i32, vp, vp, vp],
             }
             for name, args in sig.items():
                 f = getattr(lib, name)
@@ -211,6 +213,51 @@ def jq_quantize_act(x: torch.Tensor, group: int, q: torch.Tensor | None = None, 
         s_a = torch.empty((M, K // group if group else 0), dtype=torch.float32, device=x.device)
     _check("jq_quantize_act", _load().jq_quantize_act(_ptr(x), M, K, x.stride(0), group, _ptr(q), _ptr(s_a),
                                                       _stream(stream)))
+    return q, s_a
+
+
+def jq_modulate_quantize_act(x: torch.Tensor, shift: torch.Tensor, scale: torch.Tensor, tokens_per_sample: int,
+                             group: int, q: torch.Tensor | None = None, s_a: torch.Tensor | None = None, stream=None):
+    """adaLN modulation fused with the activation quantiser (DiT block linears): the codes and
+    scales of bf16(x * (1 + scale[b]) + shift[b]) for token m of sample b = m // tokens_per_sample.
+
+    x bf16 [M, K] (row stride >= K); shift, scale fp32 [ceil(M / tokens_per_sample), K]
+    -> (packed codes uint8 [M, K/2], scales fp32 [M, K/G])."""
+    fn = "jq_modulate_quantize_act"
+    _expect_x(fn, x)
+    M, K = x.shape
+    if tokens_per_sample <= 0:
+        raise ValueError(f"{fn}: tokens_per_sample must be positive")
+    samples = -(-M // tokens_per_sample)
+    _expect(fn, "shift", shift, torch.float32, (samples, K), x.device)
+    _expect(fn, "scale", scale, torch.float32, (samples, K), x.device)
+    _expect(fn, "q", q, torch.uint8, (M, K // 2), x.device)
+    _expect(fn, "s_a", s_a, torch.float32, (M, _groups(K, group)), x.device)
+    _need_cuda(x, shift, scale, stream=stream)
+    if q is None:
+        q = torch.empty((M, K // 2), dtype=torch.uint8, device=x.device)
+    if s_a is None:
+        s_a = torch.empty((M, K // group if group else 0), dtype=torch.float32, device=x.device)
+    _check(fn, _load().jq_modulate_quantize_act(_ptr(x), M, K, x.stride(0), _ptr(shift), _ptr(scale),
+                                                tokens_per_sample, group, _ptr(q), _ptr(s_a), _stream(stream)))
+    return q, s_a
+
+
+def jq_gelu_quantize_act(h: torch.Tensor, group: int, q: torch.Tensor | None = None,
+                         s_a: torch.Tensor | None = None, stream=None):
+    """tanh GELU fused with the activation quantiser (the input of a DiT MLP's second linear):
+    the codes and scales of bf16(GELU(h)).  h bf16 [M, K] -> (uint8 [M, K/2], fp32 [M, K/G])."""
+    fn = "jq_gelu_quantize_act"
+    _expect_x(fn, h)
+    M, K = h.shape
+    _expect(fn, "q", q, torch.uint8, (M, K // 2), h.device)
+    _expect(fn, "s_a", s_a, torch.float32, (M, _groups(K, group)), h.device)
+    _need_cuda(h, stream=stream)
+    if q is None:
+        q = torch.empty((M, K // 2), dtype=torch.uint8, device=h.device)
+    if s_a is None:
+        s_a = torch.empty((M, K // group if group else 0), dtype=torch.float32, device=h.device)
+    _check(fn, _load().jq_gelu_quantize_act(_ptr(h), M, K, h.stride(0), group, _ptr(q), _ptr(s_a), _stream(stream)))
     return q, s_a
 
 

@@ -119,6 +119,34 @@ jq_status jq_quantize_act(const void* x_bf16, int64_t M, int64_t K, int64_t ldx,
                                            d->sms));
 }
 
+jq_status jq_modulate_quantize_act(const void* x_bf16, int64_t M, int64_t K, int64_t ldx, const float* shift,
+                                   const float* scale, int64_t tokens_per_sample, int32_t group, uint8_t* q, float* s_a,
+                                   void* stream) {
+  if (M < 0 || !group_ok(K, group) || ldx < K || tokens_per_sample <= 0) return JQ_ERR_INVALID_ARG;
+  if (M == 0) return JQ_OK;
+  if (x_bf16 == nullptr || shift == nullptr || scale == nullptr || q == nullptr || s_a == nullptr)
+    return JQ_ERR_INVALID_ARG;
+  if (!aligned16(x_bf16) || !aligned16(shift) || !aligned16(scale) || !aligned16(q) || !aligned16(s_a) ||
+      (ldx * 2) % 16 != 0)
+    return JQ_ERR_MISALIGNED;
+  const DeviceInfo* d = current_device();
+  if (d == nullptr) return JQ_ERR_UNSUPPORTED;
+  return from_cuda(jq::launch_modulate_quantize_act(x_bf16, M, K, ldx, shift, scale, tokens_per_sample, group, q, s_a,
+                                                    static_cast<cudaStream_t>(stream), d->sms));
+}
+
+jq_status jq_gelu_quantize_act(const void* h_bf16, int64_t M, int64_t K, int64_t ldh, int32_t group, uint8_t* q,
+                               float* s_a, void* stream) {
+  if (M < 0 || !group_ok(K, group) || ldh < K) return JQ_ERR_INVALID_ARG;
+  if (M == 0) return JQ_OK;
+  if (h_bf16 == nullptr || q == nullptr || s_a == nullptr) return JQ_ERR_INVALID_ARG;
+  if (!aligned16(h_bf16) || !aligned16(q) || !aligned16(s_a) || (ldh * 2) % 16 != 0) return JQ_ERR_MISALIGNED;
+  const DeviceInfo* d = current_device();
+  if (d == nullptr) return JQ_ERR_UNSUPPORTED;
+  return from_cuda(jq::launch_gelu_quantize_act(h_bf16, M, K, ldh, group, q, s_a, static_cast<cudaStream_t>(stream),
+                                                d->sms));
+}
+
 jq_status jq_pack_weight(const float* w, int64_t N, int64_t K, int32_t group, uint8_t* qw, float* s_w,
                          void* stream) {
   if (N < 0 || !group_ok(K, group)) return JQ_ERR_INVALID_ARG;

@@ -75,6 +75,14 @@ cudaError_t launch_quantize_act(const void* x, int64_t M, int64_t K, int64_t ldx
 // (fused path; the corrections are 8 * the group's code sum in 2^-18 units, operand.cuh).
 cudaError_t launch_quantize_act_operand(const void* x, int64_t M, int64_t K, int64_t ldx, int G, uint8_t* op,
                                         float* s_a, float* corr, cudaStream_t stream, int sms);
+// DiT neighbour operations fused with the activation quantiser (quantize.cu): the adaLN
+// modulation bf16(x (1 + scale[b]) + shift[b]) of token m of sample b = m / tokens_per_sample,
+// shift / scale fp32 [samples, K]; the tanh GELU of h.  Output as launch_quantize_act.
+cudaError_t launch_modulate_quantize_act(const void* x, int64_t M, int64_t K, int64_t ldx, const float* shift,
+                                         const float* scale, int64_t tokens_per_sample, int G, uint8_t* q, float* s_a,
+                                         cudaStream_t stream, int sms);
+cudaError_t launch_gelu_quantize_act(const void* h, int64_t M, int64_t K, int64_t ldh, int G, uint8_t* q, float* s_a,
+                                     cudaStream_t stream, int sms);
 // fp32 weights [N, K] -> packed codes [N, K/2] + scales [K/G, N].
 cudaError_t launch_pack_weight(const float* w, int64_t N, int64_t K, int G, uint8_t* qw, float* s_w,
                                cudaStream_t stream, int sms);

@@ -92,6 +92,93 @@ __device__ __forceinline__ void quantize32(const float (&x)[32], float s, uint32
   }
 }
 
+// ---------------------------------------------------------------- DiT neighbour operations
+// The inputs of a DiT-XL/2 block's linears come from the adaLN modulation (before the attention's
+// QKV projection and the MLP's first linear) and from the MLP's tanh GELU (before its second
+// linear).  Fusing them here makes the quantiser read the operation's input instead of a bf16
+// tensor the operation wrote.  Each yields the bf16 value the linear layer would receive.
+enum NeighbourOp : int { kOpNone = 0, kOpModulate = 1, kOpGelu = 2 };
+
+struct OpArgs {
+  const float* shift = nullptr;  // modulation: [samples, K]
+  const float* scale = nullptr;  // modulation: [samples, K]
+  int64_t tokens_per_sample = 1;
+};
+
+// bf16( fl32( fl32( x * fl32(1 + scale) ) + shift ) ): IEEE single steps, no contraction, one
+// rounding to bf16 (round to nearest even).
+__device__ __forceinline__ float modulate_bf16(float x, float shift, float scale) {
+  const float z = __fadd_rn(__fmul_rn(x, __fadd_rn(1.0f, scale)), shift);
+  return __bfloat162float(__float2bfloat16_rn(z));
+}
+
+// e^x for x <= 0 in fp32 steps: Cody and Waite's reduction n = rint(x log2 e), r = x - n ln2 with
+// ln2 split into a 15-bit high part (n * ln2_hi exact for |n| <= 150) and a low part, e^r by its
+// Taylor polynomial to degree 8 (Horner, fused multiply-adds; |r| <= 0.35, truncation below
+// 2^-32), e^x = 2^n e^r by one exact-exponent product (two below the normal range); 0 below
+// x = -104.  Every step is one IEEE operation, so the CPU oracle reproduces it bit for bit.
+__device__ __forceinline__ float pow2_f32(int n) { return __int_as_float((n + 127) << 23); }
+
+__device__ __forceinline__ float exp_neg_f32(float x) {
+  // branch-free (selects only), so that the caller's independent elements interleave; the values
+  // are those of the stepwise definition: below -104 the result is 0, and below the normal range
+  // the power of two is applied as 2^(n+64) then 2^-64 (the second product is by exactly 1 above)
+  const bool zero = x < -104.0f;
+  x = fmaxf(x, -104.0f);
+  const float n = rintf(__fmul_rn(x, 0x1.715476p+0f));
+  float r = __fmaf_rn(-n, 0x1.62e4p-1f, x);
+  r = __fmaf_rn(-n, 0x1.7f7d1cp-20f, r);
+  float p = 0x1.a01a02p-16f;           // 1/8!
+  p = __fmaf_rn(p, r, 0x1.a01a02p-13f);  // 1/7!
+  p = __fmaf_rn(p, r, 0x1.6c16c2p-10f);  // 1/6!
+  p = __fmaf_rn(p, r, 0x1.111112p-7f);   // 1/5!
+  p = __fmaf_rn(p, r, 0x1.555556p-5f);   // 1/4!
+  p = __fmaf_rn(p, r, 0x1.555556p-3f);   // 1/3!
+  p = __fmaf_rn(p, r, 0x1p-1f);          // 1/2!
+  p = __fmaf_rn(p, r, 1.0f);
+  p = __fmaf_rn(p, r, 1.0f);
+  const int ni = static_cast<int>(n);
+  const bool low = ni < -126;
+  const float v = __fmul_rn(__fmul_rn(p, pow2_f32(low ? ni + 64 : ni)), low ? 0x1p-64f : 1.0f);
+  return zero ? 0.0f : v;
+}
+
+// The tanh GELU of one value evaluated in fp32 by a fixed sequence of IEEE operations (the same
+// as the oracle's): u = 0.7978846 (h + 0.044715 h^3), 1 + tanh(u) = 2 sigma(2u) with the logistic
+// as 1 / (1 + e^{-2u}) (u >= 0) or e^{2u} / (1 + e^{2u}) (u < 0), g = h sigma(2u); then rounded to
+// bf16 as a bf16 model stores it.  +-0 stays +-0.
+__device__ __forceinline__ float gelu_bf16(float h) {
+  // straight-line: the logistic takes one division with a selected numerator, 1 / (1 + e^{-2u})
+  // for u >= 0 and e^{2u} / (1 + e^{2u}) for u < 0 (e = e^{-2|u|} in both); h = +-0 gives +-0
+  const float h3 = __fmul_rn(__fmul_rn(h, h), h);
+  const float p = __fadd_rn(h, __fmul_rn(0x1.6e4e26p-5f, h3));
+  const float u = __fmul_rn(0x1.988454p-1f, p);
+  const float e = exp_neg_f32(__fmul_rn(-2.0f, fabsf(u)));
+  const float sig = __fdiv_rn(u >= 0.0f ? 1.0f : e, __fadd_rn(1.0f, e));
+  return __bfloat162float(__float2bfloat16_rn(__fmul_rn(h, sig)));
+}
+
+// Applies the neighbour operation to 32 consecutive values of row `row` from K index `col`.
+template <int kOp>
+__device__ __forceinline__ void apply_op(float (&v)[32], int64_t row, int64_t col, int64_t K, const OpArgs& op) {
+  if constexpr (kOp == kOpModulate) {
+    const int64_t base = (row / op.tokens_per_sample) * K + col;
+    const float4* sh = reinterpret_cast<const float4*>(op.shift + base);
+    const float4* sc = reinterpret_cast<const float4*>(op.scale + base);
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      const float4 a = __ldg(sh + i), c = __ldg(sc + i);
+      v[4 * i] = modulate_bf16(v[4 * i], a.x, c.x);
+      v[4 * i + 1] = modulate_bf16(v[4 * i + 1], a.y, c.y);
+      v[4 * i + 2] = modulate_bf16(v[4 * i + 2], a.z, c.z);
+      v[4 * i + 3] = modulate_bf16(v[4 * i + 3], a.w, c.w);
+    }
+  } else if constexpr (kOp == kOpGelu) {
+#pragma unroll
+    for (int i = 0; i < 32; ++i) v[i] = gelu_bf16(v[i]);
+  }
+}
+
 // 32 codes of one row starting at K index `col` (a multiple of 32): packed codes go to the
 // row-major [rows, K/2] array; operand bytes go to the A-operand image (operand.cuh).
 template <bool kOperand>
@@ -112,10 +199,11 @@ __device__ __forceinline__ void store32(uint8_t* out, int64_t row, int64_t col, 
 
 // G = 32 * L (L = 2 or 4): each thread quantises 32 consecutive elements; the L threads of a
 // group are adjacent lanes and reduce amax with xor-shuffles.
-template <typename In, int L, bool kOperand, bool kScaleT>
+template <typename In, int L, bool kOperand, bool kScaleT, int kOp = kOpNone>
 __global__ void __launch_bounds__(256) quantize_groups_kernel(const In* __restrict__ x, int64_t M, int64_t K,
                                                               int64_t ldx, uint8_t* __restrict__ out,
-                                                              float* __restrict__ scales, float* __restrict__ corr) {
+                                                              float* __restrict__ scales, float* __restrict__ corr,
+                                                              const OpArgs op) {
   // The activation quantiser lets the next kernel (the linear layer, which starts by streaming
   // its weights) launch at once; the weight packer does not, so nothing reads weights early.
   if (!kScaleT) pdl_launch_dependents();
@@ -131,6 +219,7 @@ __global__ void __launch_bounds__(256) quantize_groups_kernel(const In* __restri
     float v[32];
     if (valid) {
       load32(x + row * ldx + col, v);
+      apply_op<kOp>(v, row, col, K, op);
     } else {
 #pragma unroll
       for (int i = 0; i < 32; ++i) v[i] = 0.0f;
@@ -161,10 +250,11 @@ __global__ void __launch_bounds__(256) quantize_groups_kernel(const In* __restri
 
 // G = K: one block per row; pass 1 reduces the row amax, pass 2 quantises (the second read
 // of the row hits L1/L2).
-template <typename In, bool kOperand, bool kScaleT>
+template <typename In, bool kOperand, bool kScaleT, int kOp = kOpNone>
 __global__ void __launch_bounds__(128) quantize_rows_kernel(const In* __restrict__ x, int64_t M, int64_t K,
                                                             int64_t ldx, uint8_t* __restrict__ out,
-                                                            float* __restrict__ scales, float* __restrict__ corr) {
+                                                            float* __restrict__ scales, float* __restrict__ corr,
+                                                            const OpArgs op) {
   __shared__ float red[4];
   __shared__ int red_cs[4];
   if (!kScaleT) pdl_launch_dependents();  // as in quantize_groups_kernel
@@ -175,6 +265,7 @@ __global__ void __launch_bounds__(128) quantize_rows_kernel(const In* __restrict
     for (int64_t col = threadIdx.x * 32; col < K; col += 32 * blockDim.x) {
       float v[32];
       load32(xr + col, v);
+      apply_op<kOp>(v, row, col, K, op);
       a = fmaxf(a, amax32(v));
     }
 #pragma unroll
@@ -188,6 +279,7 @@ __global__ void __launch_bounds__(128) quantize_rows_kernel(const In* __restrict
     for (int64_t col = threadIdx.x * 32; col < K; col += 32 * blockDim.x) {
       float v[32];
       load32(xr + col, v);
+      apply_op<kOp>(v, row, col, K, op);
       uint32_t pk[4];
       quantize32(v, s, pk);
       store32<kOperand>(out, row, col, K, pk);
@@ -282,21 +374,21 @@ int grid_for(int64_t work_items, int threads, int sms) {
   return static_cast<int>(blocks);
 }
 
-template <typename In, bool kOperand, bool kScaleT>
+template <typename In, bool kOperand, bool kScaleT, int kOp = kOpNone>
 cudaError_t launch_quantize(const In* x, int64_t M, int64_t K, int64_t ldx, int G, uint8_t* out, float* scales,
-                            float* corr, cudaStream_t stream, int sms) {
+                            float* corr, cudaStream_t stream, int sms, const OpArgs& op = OpArgs()) {
   if (M == 0) return cudaSuccess;
   if (G == K) {
     int blocks = static_cast<int>(M < static_cast<int64_t>(sms) * 16 ? M : static_cast<int64_t>(sms) * 16);
-    return launch_pdl(quantize_rows_kernel<In, kOperand, kScaleT>, dim3(blocks), dim3(128), 0, stream, x, M, K, ldx,
-                      out, scales, corr);
+    return launch_pdl(quantize_rows_kernel<In, kOperand, kScaleT, kOp>, dim3(blocks), dim3(128), 0, stream, x, M, K,
+                      ldx, out, scales, corr, op);
   }
   const int grid = grid_for(M * (K / 32), 256, sms);
   if (G == 64)
-    return launch_pdl(quantize_groups_kernel<In, 2, kOperand, kScaleT>, dim3(grid), dim3(256), 0, stream, x, M, K,
-                      ldx, out, scales, corr);
-  return launch_pdl(quantize_groups_kernel<In, 4, kOperand, kScaleT>, dim3(grid), dim3(256), 0, stream, x, M, K, ldx,
-                    out, scales, corr);
+    return launch_pdl(quantize_groups_kernel<In, 2, kOperand, kScaleT, kOp>, dim3(grid), dim3(256), 0, stream, x, M,
+                      K, ldx, out, scales, corr, op);
+  return launch_pdl(quantize_groups_kernel<In, 4, kOperand, kScaleT, kOp>, dim3(grid), dim3(256), 0, stream, x, M, K,
+                    ldx, out, scales, corr, op);
 }
 
 }  // namespace
@@ -329,6 +421,27 @@ cudaError_t launch_expand_operand(const uint8_t* packed, int64_t rows, int64_t K
   const int grid = grid_for(chunks, 256, sms);
   if (G == 64) return launch_pdl(expand_operand_kernel<2>, dim3(grid), dim3(256), 0, stream, packed, rows, K, op, corr);
   return launch_pdl(expand_operand_kernel<4>, dim3(grid), dim3(256), 0, stream, packed, rows, K, op, corr);
+}
+
+}  // namespace jq
+
+namespace jq {
+
+cudaError_t launch_modulate_quantize_act(const void* x, int64_t M, int64_t K, int64_t ldx, const float* shift,
+                                         const float* scale, int64_t tokens_per_sample, int G, uint8_t* q, float* s_a,
+                                         cudaStream_t stream, int sms) {
+  OpArgs op;
+  op.shift = shift;
+  op.scale = scale;
+  op.tokens_per_sample = tokens_per_sample;
+  return launch_quantize<__nv_bfloat16, false, false, kOpModulate>(static_cast<const __nv_bfloat16*>(x), M, K, ldx, G, q,
+                                                                    s_a, nullptr, stream, sms, op);
+}
+
+cudaError_t launch_gelu_quantize_act(const void* h, int64_t M, int64_t K, int64_t ldh, int G, uint8_t* q, float* s_a,
+                                     cudaStream_t stream, int sms) {
+  return launch_quantize<__nv_bfloat16, false, false, kOpGelu>(static_cast<const __nv_bfloat16*>(h), M, K, ldh, G, q,
+                                                                s_a, nullptr, stream, sms);
 }
 
 }  // namespace jq

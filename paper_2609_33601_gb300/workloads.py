@@ -30,6 +30,12 @@ drawn in fp64/fp32 and rounded once to bf16, round-to-nearest-even):
 * ``sweep_a`` / ``sweep_b``: M tokens x (K=4096 -> N=12288) or
               (K=3072 -> N=3072); X ~ N(0,1) with 1% of channels x20;
               W ~ N(0, 0.02); no bias.
+* ``dit``   : DiT-XL/2 block linears (hidden 1152, MLP 4608, 256 tokens per
+              256x256 image: 16 images = 4096 tokens), group128 (Appendix
+              "DiT-XL/2 experimental details").  X ~ N(0,1) (layer-normalised
+              tokens, or the MLP's pre-activation for the GELU); the adaLN
+              modulation's shift and scale per image ~ N(0, 0.5^2)
+              (``dit_modulation``); W ~ N(0, 0.02); bias ~ N(0, 0.01).
 """
 from __future__ import annotations
 
@@ -46,7 +52,9 @@ WORKLOADS = {
     "flux_out": (4608, 15360, 3072, 64, True),
     "sweep_a": (None, 4096, 12288, 128, False),
     "sweep_b": (None, 3072, 3072, 64, False),
+    "dit": (4096, 1152, 3456, 128, True),
 }
+DIT_TOKENS_PER_IMAGE = 256  # 256x256 images, 32x32 latent, patch 2
 SWEEP_M = (1, 16, 64, 256, 1024, 4096, 16384)
 
 
@@ -106,6 +114,8 @@ def _activations(name: str, rng: np.random.Generator, M: int, K: int) -> np.ndar
         x[:, :attn] = rng.standard_normal((M, attn), dtype=np.float32)
         h = rng.standard_normal((M, K - attn))
         x[:, attn:] = _gelu_exact(h).astype(np.float32)
+    elif name == "dit":
+        x = rng.standard_normal((M, K), dtype=np.float32)
     elif name in ("sweep_a", "sweep_b", "custom"):
         x = rng.standard_normal((M, K), dtype=np.float32)
         n_out = max(1, int(round(0.01 * K)))
@@ -147,3 +157,11 @@ def random_codes(rng: np.random.Generator, rows: int, K: int, low: int = -8, hig
     """Uniform random INT4 codes in [low, high], as int8 [rows, K] (for GEMM
     tests that feed the full code range, including -8, straight to the GEMM)."""
     return rng.integers(low, high + 1, size=(rows, K), dtype=np.int8)
+
+
+def dit_modulation(seed: int, samples: int, K: int):
+    """The adaLN modulation's per-image shift and scale, fp32 [samples, K] each, ~ N(0, 0.5^2)."""
+    rng = np.random.default_rng(seed)
+    shift = (rng.standard_normal((samples, K)) * 0.5).astype(np.float32)
+    scale = (rng.standard_normal((samples, K)) * 0.5).astype(np.float32)
+    return shift, scale

@@ -237,3 +237,29 @@ def test_fake_quant_binding_refuses_wrong_tensors():
         jq.jq_ste_backward(x, torch.zeros((4, 255), dtype=torch.uint8))
     with pytest.raises(ValueError, match="CUDA tensors only"):
         jq.jq_ste_backward(x, torch.zeros((4, 256), dtype=torch.uint8))
+
+
+def test_dit_neighbour_entry_points_check_arguments(lib):
+    """jq_modulate_quantize_act / jq_gelu_quantize_act refuse bad arguments before any launch."""
+    vp = ctypes.c_void_p
+    lib.jq_modulate_quantize_act.argtypes = [vp, ctypes.c_int64, ctypes.c_int64, ctypes.c_int64, vp, vp,
+                                             ctypes.c_int64, ctypes.c_int32, vp, vp, vp]
+    lib.jq_gelu_quantize_act.argtypes = [vp, ctypes.c_int64, ctypes.c_int64, ctypes.c_int64, ctypes.c_int32, vp, vp,
+                                         vp]
+    p = vp(4096)
+    odd = vp(4100)
+    mod = lib.jq_modulate_quantize_act
+    assert mod(p, 4, 256, 256, p, p, 1, 64, p, p, None) == 3          # valid: no sm_103 device here
+    assert mod(p, 0, 256, 256, p, p, 1, 64, p, p, None) == 0          # empty batch
+    assert mod(p, 4, 256, 256, p, p, 0, 64, p, p, None) == 1          # tokens_per_sample <= 0
+    assert mod(p, 4, 256, 256, None, p, 1, 64, p, p, None) == 1       # no shift
+    assert mod(p, 4, 256, 256, p, None, 1, 64, p, p, None) == 1       # no scale
+    assert mod(p, 4, 256, 128, p, p, 1, 64, p, p, None) == 1          # ldx < K
+    assert mod(p, 4, 256, 256, p, p, 1, 96, p, p, None) == 1          # unsupported group
+    assert mod(p, 4, 256, 256, odd, p, 1, 64, p, p, None) == 2        # misaligned x
+    assert mod(p, 4, 256, 256, p, odd, 1, 64, p, p, None) == 2        # misaligned shift
+    gelu = lib.jq_gelu_quantize_act
+    assert gelu(p, 4, 256, 256, 128, p, p, None) == 3
+    assert gelu(p, 4, 256, 260, 128, p, p, None) == 2                 # ldh * 2 not a multiple of 16
+    assert gelu(None, 4, 256, 256, 128, p, p, None) == 1
+    assert gelu(p, 4, 200, 256, 128, p, p, None) == 1                 # K not a multiple of 128
