@@ -94,8 +94,8 @@ FP8_PER_BF16 = 2.0  # nominal dense FP8 / BF16 tensor-core ratio on GB300 (4.5 /
 # capture was taken on (kernel_hash); once the code changes the figure no longer applies and the
 # bench reports null until a new capture is recorded here.
 KERNEL_TRAFFIC: dict = {
-    ("flux_qkv", "d0d1b1f0f83343fb"): 54.647296e6 + 143.780096e6,
-    ("dllm", "d0d1b1f0f83343fb"): 31.236864e6 + 0.134656e6,
+    ("flux_qkv", "22124523f93a78bb"): 54.730240e6 + 143.731712e6,
+    ("dllm", "22124523f93a78bb"): 31.241728e6 + 0.144384e6,
 }
 
 

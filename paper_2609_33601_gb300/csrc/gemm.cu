@@ -197,30 +197,183 @@ __device__ __forceinline__ void drain_export(const Args& args, const Pair& pr, u
   }
 }
 
-// Linear path, 256-column tiles (one-group problems).  Warp w (drain index d = w - 8) owns TMEM
-// lanes 32*(w%4).. (32 rows) and columns 128*(d/4).. of each accumulator, read with the 16x256b
-// shape: thread t holds rows t/4 + {0, 8, 16, 24} of those 32 and columns 8j + 2(t%4) + {0, 1},
-// j = 0..15.  So a thread needs only 32 weight scales and 4 activation scales per group; it loads
-// all of them at the start of the group (the tensor core's operand reads starve shared-memory
-// loads issued one chunk ahead of their use, but not loads issued a group ahead).
+__device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
+  const __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
+  return *reinterpret_cast<const uint32_t*>(&v);
+}
+
+// Linear path, 256-column tiles, several groups (sign-magnitude weight codes): warp w (drain index
+// d = w - 8) owns one row per thread -- TMEM
+// lane 32*(w%4) + lane -- and columns 128*(d/4).. of each accumulator, read 16 at a time with the
+// 32x32b shape: two loads in flight, the next 16 columns arriving while the current ones are
+// scaled.  The running sums are float2 pairs, the operand form of the packed fp32 instructions,
+// so y += (acc * s_w) * (s_a * 2^18) costs one FMUL2 and one FFMA2 per two outputs.  The weight
+// scales are the same for every lane (broadcast LDS.128 from the scale ring); the activation
+// scale is one value per thread and group.  (Per group the lanes of a warp fill 16 KB of registers
+// with weight scales this way, four times the 16x256b layout's share, but its 8 wide TMEM loads
+// per group against 32 narrow ones make it the faster of the two when every group is drained.)
 template <class T, bool kOffset>
-__device__ __forceinline__ void drain_linear(const Args& args, const Pair& pr, uint32_t tmem_base, const Bars& b,
-                                             uint8_t* sSc, volatile int* abort_flag) {
-  static_assert(T::kBN == 256, "the 128-column tiles drain in drain_linear128");
+__device__ __forceinline__ void drain_linear_rows(const Args& args, const Pair& pr, uint32_t tmem_base,
+                                                  const Bars& b, uint8_t* sSc, volatile int* abort_flag) {
+  static_assert(T::kBN == 256, "drain layout for 256-column tiles");
+  const uint32_t warp = warp_id(), lane = lane_id();
+  const int M = args.M, N = args.N, groups = args.groups;
+  const uint32_t quarter = warp & 3u, half = (warp - kDrainWarp0) >> 2;
+  const uint32_t trow = quarter * 32u + lane;  // row within the CTA's 128
+  uint32_t chunk_it = 0, sc_it = 0;
+  bool ok = true;
+  bool next_full = false;  // the next accumulator was seen complete during the current group
+  for (int tile = pr.cluster; ok && tile < args.num_tiles; tile += pr.num_clusters) {
+    const int mt2 = tile % args.num_m2, nt = tile / args.num_m2;
+    const int row = mt2 * kPairM + (int)pr.rank * kBM + (int)trow;
+    const int col0 = nt * T::kBN + half * 128;
+    const bool row_ok = row < M;
+    float2 y[64];
+#pragma unroll
+    for (int i = 0; i < 64; ++i) y[i] = make_float2(0.0f, 0.0f);
+    for (int g = 0; g < groups; ++g) {
+      const uint32_t ab = acc_buf<T>(chunk_it);
+      const int gi = g % kScGroups;
+      const uint32_t sslot = sc_it % kScSlots;
+      if (gi == 0) {
+        ok = __all_sync(0xffffffffu, mbar_wait(&b.sc_full[sslot], ring_parity(sc_it, kScSlots), abort_flag, args.status));
+        if (!ok) break;
+      }
+      const uint8_t* slot = sSc + sslot * T::kScSlotBytes;
+      const float4* sw4 = reinterpret_cast<const float4*>(reinterpret_cast<const float*>(slot) + gi * T::kBN + half * 128);
+      float sa;
+      if (args.sa_tma)
+        sa = reinterpret_cast<const float*>(slot + T::kScSwBytes)[trow * kScGroups + gi];
+      else
+        sa = row_ok ? __ldg(args.s_a + (int64_t)row * groups + g) : 0.0f;
+      // one-group offset-code weights: the exact partial is the accumulator less 8 * the code sum
+      const float cr = (kOffset && row_ok) ? -__ldg(args.corr + (int64_t)row * groups + g) : 0.0f;
+      // Warp-collective tcgen05.ld follows: the whole warp proceeds or none of it (a timeout in
+      // one lane must not leave the others in an aligned instruction).
+      if (!__all_sync(0xffffffffu, next_full)) {
+        ok = __all_sync(0xffffffffu, mbar_wait(&b.acc_full[ab], acc_parity<T>(chunk_it), abort_flag, args.status));
+        if (!ok) break;
+      }
+      next_full = false;
+      tc_fence_after();
+      const uint32_t taddr = tmem_base + ((quarter * 32u) << 16) + ab * T::kBN + half * 128;
+      auto release = [&]() {  // every column of this accumulator is in registers: hand it back
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive_remote_cta(leader_bar(&b.acc_empty[ab]));
+      };
+      // Both arithmetic forms are exact-partial * scales in fp32; the second is needed when
+      // s_a * 2^18 would overflow.  The choice is made for the whole warp: both issue
+      // warp-collective tcgen05.ld / __syncwarp, which every lane must reach.
+      if (__all_sync(0xffffffffu, sa * kOperandUnitInv <= FLT_MAX)) {
+        const float2 f = make_float2(sa * kOperandUnitInv, sa * kOperandUnitInv);
+        const float2 c2 = make_float2(cr, cr);
+        auto scale16 = [&](int c, const uint32_t (&r)[16]) {
+#pragma unroll
+          for (int q = 0; q < 4; ++q) {
+            const float4 w = sw4[(c >> 2) + q];
+            float2 d0 = make_float2(__uint_as_float(r[4 * q]), __uint_as_float(r[4 * q + 1]));
+            float2 d1 = make_float2(__uint_as_float(r[4 * q + 2]), __uint_as_float(r[4 * q + 3]));
+            if (kOffset) {  // integers below 2^24: exact
+              d0 = __fadd2_rn(d0, c2);
+              d1 = __fadd2_rn(d1, c2);
+            }
+            float2& y0 = y[(c >> 1) + 2 * q];
+            float2& y1 = y[(c >> 1) + 2 * q + 1];
+            y0 = __ffma2_rn(__fmul2_rn(d0, make_float2(w.x, w.y)), f, y0);
+            y1 = __ffma2_rn(__fmul2_rn(d1, make_float2(w.z, w.w)), f, y1);
+          }
+        };
+        uint32_t ra[16], rb[16];
+        tmem_ld16(taddr, ra);
+        tmem_ld_wait();
+#pragma unroll
+        for (int c = 0; c < 128; c += 32) {
+          tmem_ld16(taddr + c + 16, rb);
+          scale16(c, ra);
+          tmem_ld_wait();
+          if (c == 96) release();
+          if (c < 96) tmem_ld16(taddr + c + 32, ra);
+          if (c == 64)  // the next accumulator: seen complete yet?
+            next_full = mbar_test_wait(&b.acc_full[acc_buf<T>(chunk_it + 1)], acc_parity<T>(chunk_it + 1));
+          scale16(c + 16, rb);
+          if (c < 96) tmem_ld_wait();
+        }
+      } else {  // some |s_a| > 2^110: apply 2^18 to the exact partials first so nothing overflows
+#pragma unroll
+        for (int c = 0; c < 128; c += 16) {
+          uint32_t r[16];
+          tmem_ld16(taddr + c, r);
+          tmem_ld_wait();
+          if (c == 112) release();
+#pragma unroll
+          for (int q = 0; q < 4; ++q) {
+            const float4 w = sw4[(c >> 2) + q];
+            const float wv[4] = {w.x, w.y, w.z, w.w};
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+              float& yv = (e & 1) ? y[(c >> 1) + 2 * q + (e >> 1)].y : y[(c >> 1) + 2 * q + (e >> 1)].x;
+              yv = fmaf(((__uint_as_float(r[4 * q + e]) + cr) * kOperandUnitInv) * sa, wv[e], yv);
+            }
+          }
+        }
+      }
+      if (gi == kScGroups - 1 || g == groups - 1) {  // done with this scale slot
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&b.sc_empty[sslot]);
+        ++sc_it;
+      }
+      ++chunk_it;
+    }
+    if (!ok) break;
+    // + bias, round to bf16, store: each thread writes its row's 128 columns, 8 (16 bytes) at a time
+    if (row_ok) {
+#pragma unroll
+      for (int c = 0; c < 128; c += 8) {
+        const int col = col0 + c;
+        if (col < N) {  // N % 8 == 0: a chunk is wholly inside or outside
+          float4 b0 = make_float4(0.f, 0.f, 0.f, 0.f), b1 = b0;
+          if (args.bias != nullptr) {
+            b0 = __ldg(reinterpret_cast<const float4*>(args.bias + col));
+            b1 = __ldg(reinterpret_cast<const float4*>(args.bias + col + 4));
+          }
+          const float2* yy = y + (c >> 1);
+          uint4 o;
+          o.x = pack_bf16x2(yy[0].x + b0.x, yy[0].y + b0.y);
+          o.y = pack_bf16x2(yy[1].x + b0.z, yy[1].y + b0.w);
+          o.z = pack_bf16x2(yy[2].x + b1.x, yy[2].y + b1.y);
+          o.w = pack_bf16x2(yy[3].x + b1.z, yy[3].y + b1.w);
+          *reinterpret_cast<uint4*>(args.y + (int64_t)row * N + col) = o;
+        }
+      }
+    }
+  }
+}
+// Linear path, 256-column tiles, one group (offset weight codes, drained once per tile): warp w
+// (drain index d = w - 8) owns TMEM lanes 32*(w%4).. (32 rows) and columns 128*(d/4).. of each
+// accumulator, read with the 16x256b shape: thread t holds rows t/4 + {0, 8, 16, 24} of those 32
+// and columns 8j + 2(t%4) + {0, 1}, j = 0..15, so it needs only 32 weight scales and 4 activation
+// scales, loaded at the start of the group, and its bf16 stores are 4-byte pairs of neighbouring
+// lanes (the row layout's 16-byte stores per row measured slower here, where the epilogue runs
+// after every group).
+template <class T, bool kOffset>
+__device__ __forceinline__ void drain_linear_quads(const Args& args, const Pair& pr, uint32_t tmem_base,
+                                                   const Bars& b, uint8_t* sSc, volatile int* abort_flag) {
+  static_assert(T::kBN == 256, "drain layout for 256-column tiles");
   const uint32_t warp = warp_id(), lane = lane_id();
   const int M = args.M, N = args.N, groups = args.groups;
   const uint32_t quarter = warp & 3u, half = (warp - kDrainWarp0) >> 2;
   const uint32_t tq = lane & 3u, t4 = lane >> 2;
   uint32_t chunk_it = 0, sc_it = 0;
   bool ok = true;
+  bool next_full = false;
   for (int tile = pr.cluster; ok && tile < args.num_tiles; tile += pr.num_clusters) {
     const int mt2 = tile % args.num_m2, nt = tile / args.num_m2;
     const int row0 = mt2 * kPairM + (int)pr.rank * kBM + (int)(quarter * 32u + t4);  // + 8 * rr
     const int col0 = nt * T::kBN + half * 128 + 2 * (int)tq;                           // + 8 * j
-    // y layout: y[(rr * 16 + j) * 2 + e], rr = row index 0..3 (offset 8 * rr)
-    float y[128];
+    float2 y[64];  // y[rr * 16 + j]
 #pragma unroll
-    for (int i = 0; i < 128; ++i) y[i] = 0.0f;
+    for (int i = 0; i < 64; ++i) y[i] = make_float2(0.0f, 0.0f);
     for (int g = 0; g < groups; ++g) {
       const uint32_t ab = acc_buf<T>(chunk_it);
       const int gi = g % kScGroups;
@@ -234,83 +387,83 @@ __device__ __forceinline__ void drain_linear(const Args& args, const Pair& pr, u
       float2 w[16];
 #pragma unroll
       for (int j = 0; j < 16; ++j) w[j] = *reinterpret_cast<const float2*>(sws + 8 * j);
-      // per row: s_a, and (offset-code weights, one group) -8 * the activation code sum
-      float f[4], cr[4];
+      float sa[4], cr[4];
 #pragma unroll
       for (int rr = 0; rr < 4; ++rr) {
         const int row = row0 + 8 * rr;
-        float sa;
         if (args.sa_tma)
-          sa = reinterpret_cast<const float*>(slot + T::kScSwBytes)[(quarter * 32u + t4 + 8u * rr) * kScGroups + gi];
+          sa[rr] = reinterpret_cast<const float*>(slot + T::kScSwBytes)[(quarter * 32u + t4 + 8u * rr) * kScGroups + gi];
         else
-          sa = row < M ? __ldg(args.s_a + (int64_t)row * groups + g) : 0.0f;
-        f[rr] = sa;
+          sa[rr] = row < M ? __ldg(args.s_a + (int64_t)row * groups + g) : 0.0f;
         cr[rr] = (kOffset && row < M) ? -__ldg(args.corr + (int64_t)row * groups + g) : 0.0f;
       }
-      // Warp-collective tcgen05.ld follows: the whole warp proceeds or none of it (a timeout in
-      // one lane must not leave the others in an aligned instruction).
-      ok = __all_sync(0xffffffffu, mbar_wait(&b.acc_full[ab], acc_parity<T>(chunk_it), abort_flag, args.status));
-      if (!ok) break;
+      if (!__all_sync(0xffffffffu, next_full)) {
+        ok = __all_sync(0xffffffffu, mbar_wait(&b.acc_full[ab], acc_parity<T>(chunk_it), abort_flag, args.status));
+        if (!ok) break;
+      }
+      next_full = false;
       tc_fence_after();
       const uint32_t taddr = tmem_base + ((quarter * 32u) << 16) + ab * T::kBN + half * 128;
-      // The two arithmetic forms below are both exact-partial * scales in fp32; the slow one is
-      // needed when s_a * 2^18 would overflow.  The choice is made for the whole warp: both
-      // paths issue warp-collective tcgen05.ld / __syncwarp, which every lane must reach.
+      auto release = [&]() {
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive_remote_cta(leader_bar(&b.acc_empty[ab]));
+      };
+      auto load = [&](int j, uint32_t (&r)[8]) {
+        tmem_ld16x256b_x1(taddr + j * 8, *reinterpret_cast<uint32_t(*)[4]>(&r[0]));
+        tmem_ld16x256b_x1(taddr + (16u << 16) + j * 8, *reinterpret_cast<uint32_t(*)[4]>(&r[4]));
+      };
       bool finite = true;
 #pragma unroll
-      for (int rr = 0; rr < 4; ++rr) finite = finite && (f[rr] * kOperandUnitInv <= FLT_MAX);
-      finite = __all_sync(0xffffffffu, finite);
-      if (finite) {
+      for (int rr = 0; rr < 4; ++rr) finite = finite && (sa[rr] * kOperandUnitInv <= FLT_MAX);
+      if (__all_sync(0xffffffffu, finite)) {
+        float2 f[4], c2[4];
 #pragma unroll
-        for (int rr = 0; rr < 4; ++rr) f[rr] *= kOperandUnitInv;  // s_a * 2^18
-#pragma unroll
-        for (int j = 0; j < 16; ++j) {  // 8 columns per step
-          uint32_t r0[4], r1[4];        // lanes 0-15 and 16-31 of the quarter
-          tmem_ld16x256b_x1(taddr + j * 8, r0);
-          tmem_ld16x256b_x1(taddr + (16u << 16) + j * 8, r1);
-          tmem_ld_wait();
-          if (j == 15) {  // every column of this accumulator is in registers: hand it back
-            tc_fence_before();
-            __syncwarp();
-            if (lane == 0) mbar_arrive_remote_cta(leader_bar(&b.acc_empty[ab]));
-          }
-#pragma unroll
-          for (int rr = 0; rr < 4; ++rr) {  // r0: rows +0 / +8; r1: rows +16 / +24
-            const uint32_t* r = rr < 2 ? r0 : r1;
-            const int e = 2 * (rr & 1);
-            float2 d = make_float2(__uint_as_float(r[e]), __uint_as_float(r[e + 1]));
-            if (kOffset)  // the exact partial: the offset-code sum less the correction (integers < 2^24)
-              d = __fadd2_rn(d, make_float2(cr[rr], cr[rr]));
-            const float2 t = __fmul2_rn(d, w[j]);
-            float* yy = y + (rr * 16 + j) * 2;
-            const float2 v = __ffma2_rn(t, make_float2(f[rr], f[rr]), make_float2(yy[0], yy[1]));
-            yy[0] = v.x;
-            yy[1] = v.y;
-          }
+        for (int rr = 0; rr < 4; ++rr) {
+          f[rr] = make_float2(sa[rr] * kOperandUnitInv, sa[rr] * kOperandUnitInv);
+          c2[rr] = make_float2(cr[rr], cr[rr]);
         }
-      } else {  // some |s_a| > 2^110: apply 2^18 to the exact partials first so nothing overflows
-#pragma unroll
-        for (int j = 0; j < 16; ++j) {
-          uint32_t r0[4], r1[4];
-          tmem_ld16x256b_x1(taddr + j * 8, r0);
-          tmem_ld16x256b_x1(taddr + (16u << 16) + j * 8, r1);
-          tmem_ld_wait();
-          if (j == 15) {
-            tc_fence_before();
-            __syncwarp();
-            if (lane == 0) mbar_arrive_remote_cta(leader_bar(&b.acc_empty[ab]));
-          }
+        auto scale = [&](int j, const uint32_t (&r)[8]) {  // r[0..3]: rows +0 / +8; r[4..7]: +16 / +24
 #pragma unroll
           for (int rr = 0; rr < 4; ++rr) {
-            const uint32_t* r = rr < 2 ? r0 : r1;
-            const int e = 2 * (rr & 1);
-            float* yy = y + (rr * 16 + j) * 2;
-            yy[0] = fmaf(((__uint_as_float(r[e]) + cr[rr]) * kOperandUnitInv) * f[rr], w[j].x, yy[0]);
-            yy[1] = fmaf(((__uint_as_float(r[e + 1]) + cr[rr]) * kOperandUnitInv) * f[rr], w[j].y, yy[1]);
+            const int e = 4 * (rr >> 1) + 2 * (rr & 1);
+            float2 d = make_float2(__uint_as_float(r[e]), __uint_as_float(r[e + 1]));
+            if (kOffset) d = __fadd2_rn(d, c2[rr]);
+            y[rr * 16 + j] = __ffma2_rn(__fmul2_rn(d, w[j]), f[rr], y[rr * 16 + j]);
+          }
+        };
+        uint32_t ra[8], rb[8];
+        load(0, ra);
+        tmem_ld_wait();
+#pragma unroll
+        for (int j = 0; j < 16; j += 2) {
+          load(j + 1, rb);
+          scale(j, ra);
+          tmem_ld_wait();
+          if (j == 14) release();
+          if (j < 14) load(j + 2, ra);
+          if (j == 8)
+            next_full = mbar_test_wait(&b.acc_full[acc_buf<T>(chunk_it + 1)], acc_parity<T>(chunk_it + 1));
+          scale(j + 1, rb);
+          if (j < 14) tmem_ld_wait();
+        }
+      } else {
+#pragma unroll
+        for (int j = 0; j < 16; ++j) {
+          uint32_t r[8];
+          load(j, r);
+          tmem_ld_wait();
+          if (j == 15) release();
+#pragma unroll
+          for (int rr = 0; rr < 4; ++rr) {
+            const int e = 4 * (rr >> 1) + 2 * (rr & 1);
+            float2& yy = y[rr * 16 + j];
+            yy.x = fmaf(((__uint_as_float(r[e]) + cr[rr]) * kOperandUnitInv) * sa[rr], w[j].x, yy.x);
+            yy.y = fmaf(((__uint_as_float(r[e + 1]) + cr[rr]) * kOperandUnitInv) * sa[rr], w[j].y, yy.y);
           }
         }
       }
-      if (gi == kScGroups - 1 || g == groups - 1) {  // done with this scale slot
+      if (gi == kScGroups - 1 || g == groups - 1) {
         __syncwarp();
         if (lane == 0) mbar_arrive(&b.sc_empty[sslot]);
         ++sc_it;
@@ -318,7 +471,6 @@ __device__ __forceinline__ void drain_linear(const Args& args, const Pair& pr, u
       ++chunk_it;
     }
     if (!ok) break;
-    // + bias, round to bf16, store: each (row, j) pair of columns is 4 bytes
 #pragma unroll
     for (int j = 0; j < 16; ++j) {
       const int col = col0 + 8 * j;
@@ -328,11 +480,9 @@ __device__ __forceinline__ void drain_linear(const Args& args, const Pair& pr, u
 #pragma unroll
         for (int rr = 0; rr < 4; ++rr) {
           const int row = row0 + 8 * rr;
-          if (row < M) {
-            const float* yy = y + (rr * 16 + j) * 2;
-            __nv_bfloat162 v = __floats2bfloat162_rn(yy[0] + bj.x, yy[1] + bj.y);
-            *reinterpret_cast<__nv_bfloat162*>(args.y + (int64_t)row * N + col) = v;
-          }
+          if (row < M)
+            *reinterpret_cast<__nv_bfloat162*>(args.y + (int64_t)row * N + col) =
+                __floats2bfloat162_rn(y[rr * 16 + j].x + bj.x, y[rr * 16 + j].y + bj.y);
         }
       }
     }
@@ -686,8 +836,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;\n" ::"n"(kRegsDrain) : "memory");
     if (kExport)
       drain_export<T, kOffset>(args, pr, tmem_base, b, abort_flag);
+    else if (kOffset)
+      drain_linear_quads<T, kOffset>(args, pr, tmem_base, b, sSc, abort_flag);
     else
-      drain_linear<T, kOffset>(args, pr, tmem_base, b, sSc, abort_flag);
+      drain_linear_rows<T, kOffset>(args, pr, tmem_base, b, sSc, abort_flag);
   } else if (warp >= kUnpackWarp0) {
     asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;\n" ::"n"(kRegsUnpack) : "memory");
     unpack_role<T, kOffset>(args, pr, sB, b, abort_flag);
