@@ -4,14 +4,17 @@ The paper deploys DiT-XL/2 (a 0.6B DiT; Sec. 1's remark that small matrices and 
 limit the speed-up, and the Appendix table "DiT-XL/2 experimental details" with W4A4 /
 W1.58A4, group128).  In its blocks the linears are fed by the adaLN modulation
 x (1 + scale) + shift and by the MLP's tanh GELU.  The readings (jq_oracle.c): the modulation in
-IEEE single steps without contraction, rounded once to bf16; the GELU's exact value rounded once
-to bf16; then the activation rule.  Pinned here by
+IEEE single steps without contraction, rounded once to bf16; the GELU as a fixed sequence of IEEE
+single operations (the logistic form, an own exponential), rounded to bf16; then the activation
+rule.  Pinned here by
   * an exact-rational evaluation of the modulation with fp32 / bf16 roundings written from the
     formats (not a retyping of the oracle's expression in the same arithmetic), on random,
     extreme and tie-constructed inputs, and its identities (scale 0 and shift 0 give x; scale -1
     gives bf16(shift); scale 2^j - 1 with shift 0 scales x exactly);
-  * a 50-digit mpmath evaluation of 0.5 h (1 + tanh(sqrt(2/pi)(h + 0.044715 h^3))) rounded to
-    bf16, over every bf16 h in [-16, 16] and extreme magnitudes, and the GELU's invariants;
+  * a 50-digit mpmath evaluation of 0.5 h (1 + tanh(sqrt(2/pi)(h + 0.044715 h^3))): the fp32
+    sequence within its error bound of it for every bf16 h in [-9, 16], its bf16 result equal to
+    the exact value rounded once except within that bound of a rounding boundary, extreme
+    magnitudes, and the GELU's invariants;
   * a hand-worked modulated group with its codes and scale;
   * planted mistakes (a fused multiply-add, a double rounding through bf16, the cancelling
     1 + tanh(u) form in fp64) that each fail one of these checks.
