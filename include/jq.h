@@ -291,6 +291,54 @@ JQ_API jq_status jq_ste_backward(const void* grad_bf16, const uint8_t* mask, int
                                  void* stream);
 
 /*
+ * NVFP4 W4A4, the format of the paper's LLaDA-8B rows (Appendix table "ELF-B and LLaDA-8B
+ * experimental details": "NVFP4 W4A4"; the paper defines nothing more, the reading is the
+ * published NVFP4 format): E2M1 elements, one E4M3 scale per 16 consecutive K elements of a row,
+ * one fp32 scale g per tensor.  Per block b: s_b = e4m3(fl32(amax_b / fl32(6 g))), S_b =
+ * fl32(s_b g), q = e2m1(fl32(x / S_b)), both nearest with ties to the even mantissa and
+ * saturating (448, 6); q = 0 where g = 0 or S_b = 0.  Codes: 4-bit E2M1 (bit 3 sign, bits 1-2
+ * exponent, bit 0 mantissa), element 2j in the low nibble of byte j; block scales: E4M3 bytes.
+ *
+ * Activations with the caller's (calibrated) tensor scale g_a >= 0:
+ *   x_bf16 : bf16 [M, ldx] (device);  codes : uint8 [M, K/2] (output);  scales : uint8 [M, K/16]
+ * K a multiple of 64, at most 262016; x, codes 16-byte aligned, ldx*2 a multiple of 16; M = 0
+ * is a no-op.  Errors: JQ_ERR_INVALID_ARG (null, K, M < 0, ldx < K, g_a negative or not finite),
+ * JQ_ERR_MISALIGNED, JQ_ERR_UNSUPPORTED, JQ_ERR_CUDA.
+ */
+JQ_API jq_status jq_nvfp4_quantize_act(const void* x_bf16, int64_t M, int64_t K, int64_t ldx, float g_a,
+                                       uint8_t* codes, uint8_t* scales, void* stream);
+
+/*
+ * Weights, with their tensor scale computed on the device: g_w = fl32(amax |w| / 2688).
+ *   w : fp32 [N, K] (device);  codes : uint8 [N, K/2];  scales : uint8 [N, K/16];
+ *   g_w : one fp32 (device, output; the linear layer reads it there)
+ * K as above; w, codes and g_w 16-byte aligned.  Errors as jq_nvfp4_quantize_act.
+ */
+JQ_API jq_status jq_nvfp4_pack_weight(const float* w, int64_t N, int64_t K, uint8_t* codes, uint8_t* scales,
+                                      float* g_w, void* stream);
+
+/* Workspace bytes jq_nvfp4_linear needs: two bf16 operand images (activations and weights). */
+JQ_API size_t jq_nvfp4_workspace_size(int64_t M, int64_t N, int64_t K);
+
+/*
+ * The NVFP4 linear layer:
+ *   y[m,n] = bf16( sum_b (sum_{k in b} qa qw) sa_b sw_b * g_a * g_w + bias[n] )
+ * Each element's value q * s_b is exact in bf16; the layer multiplies those in the tensor core
+ * (exact products) and sums them in fp32 over all of K, then scales by g_a and g_w and adds the
+ * bias in fp32.  The fp32 sum is the one step that is not exact: |y - y64| is within one bf16 ulp
+ * plus (K + 2) * 2^-24 * (sum_k |term| + |bias|).
+ *   codes_a, scales_a : jq_nvfp4_quantize_act's output for [M, K];  g_a as given there
+ *   codes_w, scales_w, g_w : jq_nvfp4_pack_weight's output for [N, K]
+ *   bias : fp32 [N] or NULL;  y_bf16 : bf16 [M, N] (output)
+ * K as above, N % 8 == 0; codes, y and bias 16-byte aligned; workspace >= jq_nvfp4_workspace_size
+ * bytes, 16-byte aligned; M = 0 or N = 0 is a no-op.  Errors: JQ_ERR_INVALID_ARG,
+ * JQ_ERR_MISALIGNED, JQ_ERR_WORKSPACE, JQ_ERR_UNSUPPORTED, JQ_ERR_CUDA.
+ */
+JQ_API jq_status jq_nvfp4_linear(const uint8_t* codes_a, const uint8_t* scales_a, float g_a, const uint8_t* codes_w,
+                                 const uint8_t* scales_w, const float* g_w, const float* bias, void* y_bf16, int64_t M,
+                                 int64_t N, int64_t K, void* workspace, size_t workspace_bytes, void* stream);
+
+/*
  * Verification export for failure handling (computes nothing; no counterpart in the paper):
  * launches one block in which one
  * thread waits, with the bounded wait every kernel of this library uses, on an mbarrier phase

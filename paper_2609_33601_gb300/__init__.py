@@ -27,7 +27,8 @@ __all__ = [
     "jq_fused_quant_linear", "jq_w4a4_group_partials", "jq_device_status", "jq_status_string",
     "jq_w4a4_linear_noalloc", "jq_pack_weight_ternary", "jq_w158a4_workspace_size", "jq_w158a4_linear",
     "jq_debug_wait_timeout", "jq_fake_quant_act", "jq_fake_quant_weight",
-    "jq_ste_backward", "jq_modulate_quantize_act", "jq_gelu_quantize_act",
+    "jq_ste_backward", "jq_modulate_quantize_act", "jq_gelu_quantize_act", "jq_nvfp4_quantize_act", "jq_nvfp4_pack_weight",
+    "jq_nvfp4_workspace_size", "jq_nvfp4_linear",
 ]
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
@@ -72,6 +73,9 @@ def _load() -> ctypes.CDLL:
                 "jq_w158a4_linear": [vp, vp, vp, vp, vp, vp, i64, i64, i64, i32, vp, sz, vp],
                 "jq_modulate_quantize_act": [vp, i64, i64, i64, vp, vp, i64, i32, vp, vp, vp],
                 "jq_gelu_quantize_act": [vp, i64, i64, i64, i32, vp, vp, vp],
+                "jq_nvfp4_quantize_act": [vp, i64, i64, i64, ctypes.c_float, vp, vp, vp],
+                "jq_nvfp4_pack_weight": [vp, i64, i64, vp, vp, vp, vp],
+                "jq_nvfp4_linear": [vp, vp, ctypes.c_float, vp, vp, vp, vp, vp, i64, i64, i64, vp, sz, vp],
             }
             for name, args in sig.items():
                 f = getattr(lib, name)
@@ -81,6 +85,8 @@ def _load() -> ctypes.CDLL:
             lib.jq_workspace_size.restype = ctypes.c_size_t
             lib.jq_w158a4_workspace_size.argtypes = [i64, i64, i64, i32]
             lib.jq_w158a4_workspace_size.restype = ctypes.c_size_t
+            lib.jq_nvfp4_workspace_size.argtypes = [i64, i64, i64]
+            lib.jq_nvfp4_workspace_size.restype = ctypes.c_size_t
             lib.jq_status_string.argtypes = [ctypes.c_int]
             lib.jq_status_string.restype = ctypes.c_char_p
             _lib = lib
@@ -377,6 +383,70 @@ def jq_w158a4_linear(q, s_a, qw2, s_w, bias, group: int, y=None, workspace=None,
     _check("jq_w158a4_linear",
            _load().jq_w158a4_linear(_ptr(q), _ptr(s_a), _ptr(qw2), _ptr(s_w), _ptr(bias), _ptr(y), M, N, K, group,
                                     _ptr(workspace), ws_bytes, _stream(stream)))
+    return y
+
+
+def jq_nvfp4_quantize_act(x: torch.Tensor, g_a: float, codes=None, scales=None, stream=None):
+    """NVFP4 activations: bf16 [M, K] (K % 64 == 0) with the tensor scale g_a ->
+    (E2M1 codes uint8 [M, K/2], E4M3 block-scale bytes uint8 [M, K/16])."""
+    fn = "jq_nvfp4_quantize_act"
+    _expect_x(fn, x)
+    M, K = x.shape
+    dev = x.device
+    _expect(fn, "codes", codes, torch.uint8, (M, K // 2), dev)
+    _expect(fn, "scales", scales, torch.uint8, (M, K // 16), dev)
+    _need_cuda(x, stream=stream)
+    if codes is None:
+        codes = torch.empty((M, K // 2), dtype=torch.uint8, device=dev)
+    if scales is None:
+        scales = torch.empty((M, K // 16), dtype=torch.uint8, device=dev)
+    _check(fn, _load().jq_nvfp4_quantize_act(_ptr(x), M, K, x.stride(0), float(g_a), _ptr(codes), _ptr(scales),
+                                             _stream(stream)))
+    return codes, scales
+
+
+def jq_nvfp4_pack_weight(w: torch.Tensor, stream=None):
+    """NVFP4 weights: fp32 [N, K] -> (codes uint8 [N, K/2], block-scale bytes uint8 [N, K/16],
+    tensor scale fp32 [1] on the device)."""
+    fn = "jq_nvfp4_pack_weight"
+    if w.dim() != 2:
+        raise ValueError(f"{fn}: w must be 2-D, got shape {list(w.shape)}")
+    N, K = w.shape
+    _expect(fn, "w", w, torch.float32, (N, K), w.device)
+    _need_cuda(w, stream=stream)
+    codes = torch.empty((N, K // 2), dtype=torch.uint8, device=w.device)
+    scales = torch.empty((N, K // 16), dtype=torch.uint8, device=w.device)
+    g_w = torch.empty(4, dtype=torch.float32, device=w.device)  # one used; 16 bytes for the alignment rule
+    _check(fn, _load().jq_nvfp4_pack_weight(_ptr(w), N, K, _ptr(codes), _ptr(scales), _ptr(g_w), _stream(stream)))
+    return codes, scales, g_w[:1]
+
+
+def jq_nvfp4_workspace_size(M: int, N: int, K: int) -> int:
+    return int(_load().jq_nvfp4_workspace_size(M, N, K))
+
+
+def jq_nvfp4_linear(codes_a, scales_a, g_a: float, codes_w, scales_w, g_w, bias, y=None, workspace=None,
+                    stream=None):
+    """NVFP4 W4A4: y = bf16(sum_b (sum qa qw) sa_b sw_b g_a g_w + bias) from the quantiser's and
+    the packer's outputs (g_w: the packer's one-element device tensor)."""
+    fn = "jq_nvfp4_linear"
+    M, K, N = _codes_shapes(fn, codes_a, codes_w, 2)
+    dev = codes_a.device
+    _expect(fn, "scales_a", scales_a, torch.uint8, (M, K // 16), dev)
+    _expect(fn, "scales_w", scales_w, torch.uint8, (N, K // 16), dev)
+    _expect(fn, "g_w", g_w, torch.float32, (1,), dev)
+    _expect(fn, "bias", bias, torch.float32, (N,), dev)
+    _expect(fn, "y", y, torch.bfloat16, (M, N), dev)
+    _expect_workspace(fn, workspace, dev)
+    _need_cuda(codes_a, scales_a, codes_w, scales_w, g_w, bias, stream=stream)
+    if y is None:
+        y = torch.empty((M, N), dtype=torch.bfloat16, device=dev)
+    if workspace is None:
+        workspace = torch.empty(max(jq_nvfp4_workspace_size(M, N, K), 16), dtype=torch.uint8, device=dev)
+    ws_bytes = workspace.numel() * workspace.element_size()
+    _check(fn, _load().jq_nvfp4_linear(_ptr(codes_a), _ptr(scales_a), float(g_a), _ptr(codes_w), _ptr(scales_w),
+                                       _ptr(g_w), _ptr(bias), _ptr(y), M, N, K, _ptr(workspace), ws_bytes,
+                                       _stream(stream)))
     return y
 
 

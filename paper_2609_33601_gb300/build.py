@@ -17,7 +17,8 @@ CSRC = os.path.join(HERE, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 BUILD = os.path.join(HERE, "_build")
 LIB = os.path.join(HERE, "libjq.so")
-SOURCES = ["api.cu", "quantize.cu", "gemm.cu", "skinny.cu", "noalloc.cu", "ternary.cu", "fakequant.cu"]
+SOURCES = ["api.cu", "quantize.cu", "gemm.cu", "skinny.cu", "noalloc.cu", "ternary.cu", "fakequant.cu",
+           "nvfp4.cu"]
 HEADERS = ["kernels.cuh", "operand.cuh", "ptx.cuh"]
 
 NVCC_FLAGS = [

@@ -1,6 +1,7 @@
 // api.cu -- the C ABI declared in include/jq.h: synchronous argument checks, then kernel
 // launches on the caller's stream.  No allocation, no synchronisation (except in
 // jq_device_status), no exceptions.
+#include <cfloat>
 #include <cstdint>
 #include <mutex>
 
@@ -367,6 +368,62 @@ jq_status jq_debug_wait_timeout(void* stream) {
   if (d == nullptr) return JQ_ERR_UNSUPPORTED;
   wait_timeout_probe_kernel<<<1, 32, 0, static_cast<cudaStream_t>(stream)>>>(d->status);
   return from_cuda(cudaGetLastError());
+}
+
+// ---- NVFP4 W4A4 (nvfp4.cu)
+namespace {
+bool nvfp4_k_ok(int64_t K) { return K > 0 && K % 64 == 0 && K <= kMaxK; }
+}  // namespace
+
+jq_status jq_nvfp4_quantize_act(const void* x_bf16, int64_t M, int64_t K, int64_t ldx, float g_a, uint8_t* codes,
+                                uint8_t* scales, void* stream) {
+  if (M < 0 || !nvfp4_k_ok(K) || ldx < K || !(g_a >= 0.0f && g_a <= FLT_MAX)) return JQ_ERR_INVALID_ARG;
+  if (M == 0) return JQ_OK;
+  if (x_bf16 == nullptr || codes == nullptr || scales == nullptr) return JQ_ERR_INVALID_ARG;
+  if (!aligned16(x_bf16) || !aligned16(codes) || (ldx * 2) % 16 != 0) return JQ_ERR_MISALIGNED;
+  const DeviceInfo* d = current_device();
+  if (d == nullptr) return JQ_ERR_UNSUPPORTED;
+  return from_cuda(jq::launch_nvfp4_quantize_act(x_bf16, M, K, ldx, g_a, codes, scales,
+                                                 static_cast<cudaStream_t>(stream), d->sms));
+}
+
+jq_status jq_nvfp4_pack_weight(const float* w, int64_t N, int64_t K, uint8_t* codes, uint8_t* scales, float* g_w,
+                               void* stream) {
+  if (N < 0 || !nvfp4_k_ok(K)) return JQ_ERR_INVALID_ARG;
+  if (N == 0) return JQ_OK;
+  if (w == nullptr || codes == nullptr || scales == nullptr || g_w == nullptr) return JQ_ERR_INVALID_ARG;
+  if (!aligned16(w) || !aligned16(codes) || !aligned16(g_w)) return JQ_ERR_MISALIGNED;
+  const DeviceInfo* d = current_device();
+  if (d == nullptr) return JQ_ERR_UNSUPPORTED;
+  return from_cuda(jq::launch_nvfp4_pack_weight(w, N, K, codes, scales, g_w, static_cast<cudaStream_t>(stream),
+                                                d->sms));
+}
+
+size_t jq_nvfp4_workspace_size(int64_t M, int64_t N, int64_t K) {
+  if (M <= 0 || N <= 0 || !nvfp4_k_ok(K)) return 0;
+  return jq::nvfp4_image_bytes(M, K) + jq::nvfp4_image_bytes(N, K);
+}
+
+jq_status jq_nvfp4_linear(const uint8_t* codes_a, const uint8_t* scales_a, float g_a, const uint8_t* codes_w,
+                          const uint8_t* scales_w, const float* g_w, const float* bias, void* y_bf16, int64_t M,
+                          int64_t N, int64_t K, void* workspace, size_t workspace_bytes, void* stream) {
+  if (M < 0 || N < 0 || N % 8 != 0 || M > INT32_MAX || N > INT32_MAX || !nvfp4_k_ok(K) ||
+      !(g_a >= 0.0f && g_a <= FLT_MAX))
+    return JQ_ERR_INVALID_ARG;
+  if (M == 0 || N == 0) return JQ_OK;
+  if (codes_a == nullptr || scales_a == nullptr || codes_w == nullptr || scales_w == nullptr || g_w == nullptr ||
+      y_bf16 == nullptr)
+    return JQ_ERR_INVALID_ARG;
+  if (!aligned16(codes_a) || !aligned16(codes_w) || !aligned16(y_bf16) || (bias != nullptr && !aligned16(bias)) ||
+      (reinterpret_cast<uintptr_t>(g_w) & 3u) != 0)
+    return JQ_ERR_MISALIGNED;
+  if (workspace == nullptr || !aligned16(workspace) || workspace_bytes < jq_nvfp4_workspace_size(M, N, K))
+    return JQ_ERR_WORKSPACE;
+  const DeviceInfo* d = current_device();
+  if (d == nullptr) return JQ_ERR_UNSUPPORTED;
+  return from_cuda(jq::launch_nvfp4_linear(codes_a, scales_a, g_a, codes_w, scales_w, g_w, bias, y_bf16, M, N, K,
+                                           static_cast<uint8_t*>(workspace), d->status,
+                                           static_cast<cudaStream_t>(stream), d->sms));
 }
 
 jq_status jq_device_status(void* stream, int32_t reset) {

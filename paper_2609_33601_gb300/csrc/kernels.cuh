@@ -106,6 +106,18 @@ cudaError_t launch_ste_backward(const void* grad, const uint8_t* mask, int64_t n
 cudaError_t launch_expand_operand(const uint8_t* packed, int64_t rows, int64_t K, int G, uint8_t* op, float* corr,
                                   cudaStream_t stream, int sms);
 
+// NVFP4 (nvfp4.cu): activations bf16 [M, ldx] -> E2M1 codes [M, K/2] + E4M3 block-scale bytes
+// [M, K/16] with the caller's tensor scale g; weights fp32 [N, K] -> the same, with g computed
+// into the device scalar *g; the linear layer from both (workspace: two bf16 operand images).
+size_t nvfp4_image_bytes(int64_t rows, int64_t K);
+cudaError_t launch_nvfp4_quantize_act(const void* x, int64_t M, int64_t K, int64_t ldx, float g, uint8_t* codes,
+                                      uint8_t* scales, cudaStream_t stream, int sms);
+cudaError_t launch_nvfp4_pack_weight(const float* w, int64_t N, int64_t K, uint8_t* codes, uint8_t* scales, float* g,
+                                     cudaStream_t stream, int sms);
+cudaError_t launch_nvfp4_linear(const uint8_t* qa, const uint8_t* sa, float ga, const uint8_t* qw, const uint8_t* sw,
+                                const float* gw, const float* bias, void* y, int64_t M, int64_t N, int64_t K,
+                                uint8_t* workspace, uint32_t* status, cudaStream_t stream, int sms);
+
 // Workspace of the GEMM path, each part on a 256-byte boundary: the A-operand image (whole
 // 128-row tiles of K operand bytes), the corrections fp32 [M, K/G], and for the fused path the
 // activation scales fp32 [M, K/G].

@@ -1,0 +1,430 @@
+// nvfp4.cu -- the NVFP4 W4A4 linear layer (the format of the paper's LLaDA-8B rows, Appendix
+// table "ELF-B and LLaDA-8B experimental details": "NVFP4 W4A4").
+//
+// The format: FP4 E2M1 elements (magnitudes 0, 0.5, 1, 1.5, 2, 3, 4, 6), one FP8 E4M3 scale per
+// block of 16 consecutive reduction-axis elements of a row, one fp32 scale g per tensor.  Per
+// block b:  s_b = e4m3(fl32(amax_b / fl32(6 g))),  S_b = fl32(s_b g),  q = e2m1(fl32(x / S_b)),
+// both roundings to nearest with ties to the even mantissa and saturating (448, 6); q = 0 where
+// g == 0 or S_b == 0.  Weights: g = fl32(amax |w| / 2688); activations: g given by the caller.
+// The layer: y = sum_b (sum_{k in b} qa qw) sa_b sw_b ga gw + bias.
+//
+// Kernels:
+//   nvfp4_amax_kernel / nvfp4_finish_g_kernel  the weights' tensor amax and g (three launches
+//                      with the quantiser; the packing is offline)
+//   nvfp4_quantize_kernel<In>  one thread per block of 16: E4M3 scale byte and 8 bytes of codes
+//   nvfp4_expand_kernel  codes and block scales -> a bf16 operand image: every element's exact
+//                      value q * s_b (E2M1 x E4M3 needs at most 6 significant bits and lies in
+//                      [2^-10, 2688], so bf16 holds it exactly), in the 128-byte-swizzled K-major
+//                      layout of the GEMM's operand images with a stage of 64 elements (128 B)
+//   nvfp4_gemm_kernel  tcgen05 kind::f16 with bf16 operands from both images by TMA, fp32
+//                      accumulation in TMEM over the whole K (the block scales are inside the
+//                      operands), epilogue y = (acc * ga) * gw + bias -> bf16
+// The products q_a s_a,b * q_w s_w,b are exact in the tensor core; its fp32 sum over K is not,
+// and its error is bounded by the fp32 summation bound over K products.
+//
+// Why bf16 operands and not the FP4 tensor-core kind: kind::mxf4nvf4.block_scale reads the block
+// scales from tensor memory in a layout fixed by the instruction (scale-factor tiles copied by
+// tcgen05.cp, scale-factor IDs in the instruction descriptor) that could not be checked against
+// its documentation here; the bf16 path needs only forms the rest of the library already runs.
+#include <cfloat>
+#include <cstdint>
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+
+#include "kernels.cuh"
+#include "operand.cuh"
+#include "ptx.cuh"
+
+namespace jq {
+
+namespace {
+
+// ---------------------------------------------------------------- roundings (the format)
+__device__ __forceinline__ float pow2f(int n) { return __int_as_float((n + 127) << 23); }  // n in [-126, 127]
+
+// Nearest E4M3 value to a (finite, >= 0): 3 mantissa bits, exponent bias 7, normals down to 2^-6,
+// subnormals in steps of 2^-9, ties to even, saturating at 448.  Scaling by the quantum is exact.
+__device__ __forceinline__ float e4m3_round(float a) {
+  if (a == 0.0f) return 0.0f;
+  const int e = (int)((__float_as_uint(a) >> 23) & 255u) - 127;  // floor(log2 a) for normal a
+  int q = e - 3;                                                   // the quantum's exponent
+  if (q < -9) q = -9;                                              // subnormal quantum
+  const float n = rintf(a * pow2f(-q));                            // ties to even
+  const float r = n * pow2f(q);                                    // exact (inf only past 448)
+  return r > 448.0f ? 448.0f : r;
+}
+// The E4M3 byte of a value e4m3_round returned.
+__device__ __forceinline__ uint32_t e4m3_byte(float r) {
+  if (r == 0.0f) return 0u;
+  if (r < 0x1p-6f) return (uint32_t)(r * 512.0f);                // subnormal: m * 2^-9
+  const int e = (int)((__float_as_uint(r) >> 23) & 255u) - 127;  // in [-6, 8]
+  const uint32_t m = (__float_as_uint(r) >> 20) & 7u;            // 3 mantissa bits
+  return ((uint32_t)(e + 7) << 3) | m;
+}
+__device__ __forceinline__ float e4m3_value(uint32_t b) {
+  const uint32_t e = (b >> 3) & 15u, m = b & 7u;
+  return e == 0u ? (float)m * 0x1p-9f : (float)(8u + m) * pow2f((int)e - 10);
+}
+// Nearest E2M1 magnitude to a (>= 0) as its 3-bit index into (0, 0.5, 1, 1.5, 2, 3, 4, 6), ties
+// to the even mantissa (the even indices), saturating at 6.
+__device__ __forceinline__ uint32_t e2m1_index(float a) {
+  if (a <= 0.25f) return 0u;
+  if (a < 0.75f) return 1u;
+  if (a <= 1.25f) return 2u;
+  if (a < 1.75f) return 3u;
+  if (a <= 2.5f) return 4u;
+  if (a < 3.5f) return 5u;
+  if (a <= 5.0f) return 6u;
+  return 7u;
+}
+
+// ---------------------------------------------------------------- weights' tensor scale
+__global__ void __launch_bounds__(256) nvfp4_amax_kernel(const float* __restrict__ w, int64_t n,
+                                                        unsigned int* __restrict__ amax_bits) {
+  pdl_wait();
+  float m = 0.0f;
+  for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x)
+    m = fmaxf(m, fabsf(__ldg(w + i)));
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) m = fmaxf(m, __shfl_xor_sync(0xFFFFFFFFu, m, o));
+  if ((threadIdx.x & 31) == 0) atomicMax(amax_bits, __float_as_uint(m));  // non-negative: bits order as values
+}
+__global__ void nvfp4_finish_g_kernel(float* g) {
+  pdl_wait();
+  *g = __fdiv_rn(__uint_as_float(*reinterpret_cast<const unsigned int*>(g)), 2688.0f);
+}
+
+// ---------------------------------------------------------------- quantiser
+__device__ __forceinline__ void load16(const __nv_bfloat16* p, float (&x)[16]) {
+  const uint4* v = reinterpret_cast<const uint4*>(p);
+#pragma unroll
+  for (int i = 0; i < 2; ++i) {
+    const uint4 u = __ldg(v + i);
+    const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      x[8 * i + 2 * j] = __uint_as_float(w[j] << 16);
+      x[8 * i + 2 * j + 1] = __uint_as_float(w[j] & 0xFFFF0000u);
+    }
+  }
+}
+__device__ __forceinline__ void load16(const float* p, float (&x)[16]) {
+  const float4* v = reinterpret_cast<const float4*>(p);
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const float4 u = __ldg(v + i);
+    x[4 * i] = u.x;
+    x[4 * i + 1] = u.y;
+    x[4 * i + 2] = u.z;
+    x[4 * i + 3] = u.w;
+  }
+}
+
+// One thread per block of 16 elements: codes [rows, K/2] (element 2j in the low nibble of byte
+// j), scale bytes [rows, K/16].  g from g_dev when given (the weights' computed scale), else g_host.
+template <typename In>
+__global__ void __launch_bounds__(256) nvfp4_quantize_kernel(const In* __restrict__ x, int64_t rows, int64_t K,
+                                                            int64_t ldx, float g_host, const float* g_dev,
+                                                            uint8_t* __restrict__ codes, uint8_t* __restrict__ scales) {
+  if (sizeof(In) == 2) pdl_launch_dependents();
+  pdl_wait();
+  const float g = g_dev != nullptr ? *g_dev : g_host;
+  const int64_t nb = K / 16, total = rows * nb;
+  for (int64_t t = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; t < total; t += (int64_t)gridDim.x * blockDim.x) {
+    const int64_t r = t / nb, b = t % nb;
+    float v[16];
+    load16(x + r * ldx + b * 16, v);
+    float amax = 0.0f;
+#pragma unroll
+    for (int i = 0; i < 16; ++i) amax = fmaxf(amax, fabsf(v[i]));
+    float s = 0.0f, S = 0.0f;
+    if (g != 0.0f) {
+      s = e4m3_round(__fdiv_rn(amax, 6.0f * g));
+      S = s * g;
+    }
+    uint32_t lo = 0u, hi = 0u;
+    if (S != 0.0f) {
+#pragma unroll
+      for (int i = 0; i < 16; ++i) {
+        const float q = __fdiv_rn(v[i], S);
+        const uint32_t idx = e2m1_index(fabsf(q));
+        const uint32_t c = idx | ((q < 0.0f && idx != 0u) ? 8u : 0u);
+        if (i < 8) lo |= c << (4 * i);
+        else hi |= c << (4 * (i - 8));
+      }
+    }
+    *reinterpret_cast<uint2*>(codes + r * (K / 2) + b * 8) = make_uint2(lo, hi);
+    scales[r * nb + b] = (uint8_t)e4m3_byte(s);
+  }
+}
+
+// ---------------------------------------------------------------- bf16 operand images
+constexpr int kStageK = 64;  // bf16 elements per 128-byte operand row of a stage
+
+// One thread per 8 elements (a 16-byte chunk of the image).  rows may be short of a whole
+// 128-row tile: the image's rows past them are never written (their outputs are never kept).
+__global__ void __launch_bounds__(256) nvfp4_expand_kernel(const uint8_t* __restrict__ codes,
+                                                          const uint8_t* __restrict__ scales, int64_t rows, int64_t K,
+                                                          uint8_t* __restrict__ image) {
+  pdl_launch_dependents();
+  pdl_wait();
+  const int64_t per_row = K / 8, total = rows * per_row;
+  const uint32_t k_stages = (uint32_t)(K / kStageK);
+  for (int64_t t = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; t < total; t += (int64_t)gridDim.x * blockDim.x) {
+    const int64_t r = t / per_row, k0 = (t % per_row) * 8;
+    const uint32_t c = __ldg(reinterpret_cast<const uint32_t*>(codes + r * (K / 2) + k0 / 2));
+    const float s = e4m3_value(__ldg(scales + r * (K / 16) + k0 / 16));
+    uint32_t out[4];
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      float v[2];
+#pragma unroll
+      for (int h = 0; h < 2; ++h) {
+        const uint32_t nib = (c >> (8 * i + 4 * h)) & 15u;
+        // E2M1: exponent bits e = idx >> 1, mantissa bit m = idx & 1: m/2 for e = 0 (subnormal),
+        // (1 + m/2) 2^(e-1) otherwise -- 0, 0.5, 1, 1.5, 2, 3, 4, 6
+        const uint32_t idx = nib & 7u, ee = idx >> 1, mm = idx & 1u;
+        const float mag = ee == 0u ? 0.5f * (float)mm : (1.0f + 0.5f * (float)mm) * (float)(1u << (ee - 1u));
+        const float val = mag * s;  // exact
+        v[h] = (nib & 8u) ? -val : val;
+      }
+      const __nv_bfloat162 p = __floats2bfloat162_rn(v[0], v[1]);  // exact
+      out[i] = *reinterpret_cast<const uint32_t*>(&p);
+    }
+    const uint32_t kb = (uint32_t)(k0 / kStageK), c16 = (uint32_t)((k0 % kStageK) / 8);
+    *reinterpret_cast<uint4*>(image + image_chunk_offset(r, kb, c16, k_stages)) = make_uint4(out[0], out[1], out[2], out[3]);
+  }
+}
+
+// ---------------------------------------------------------------- GEMM
+constexpr int kTileM = 128, kTileN = 256, kStages = 4, kThreadsG = 192;
+constexpr uint32_t kABytes = kTileM * 128, kBBytes = kTileN * 128, kStageBytes = kABytes + kBBytes;  // 48 KB
+constexpr uint32_t kOffBars = kStages * kStageBytes;
+constexpr uint32_t kSmemG = kOffBars + (2 * kStages + 1) * 8 + 16;
+constexpr uint32_t kTmemColsG = 256;
+// kind::f16, bf16 A and B (both K-major), fp32 accumulator: D format [4,6) = 1, A format [7,10)
+// = 1 (BF16), B format [10,13) = 1 (BF16), N >> 3 at [17,23), M >> 4 at [24,29).
+constexpr uint32_t kIdescBf16 = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(kTileN >> 3) << 17) |
+                                ((uint32_t)(kTileM >> 4) << 24);
+
+__device__ __forceinline__ void umma_bf16(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc, uint32_t idesc,
+                                          uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
+      "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+
+struct NvArgs {
+  int M, N, k_stages, num_m;
+  float ga;
+  const float* gw;   // device scalar
+  const float* bias;  // [N] or nullptr
+  __nv_bfloat16* y;   // [M, N]
+  uint32_t* status;
+};
+
+// One 128 x 256 output tile per CTA (tiles M-fastest, so that the CTAs resident at once share
+// weight tiles).  Warp 0: TMA producer (A: one 128-row box, B: two, per 64-element stage).
+// Warp 1: TMEM owner and MMA issuer (four 128x256x16 MMAs per stage, one commit per stage to free
+// the slot, one at the end for the drain).  Warps 2-5: drain, one accumulator row per thread.
+__global__ void __launch_bounds__(kThreadsG, 1)
+    nvfp4_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
+                      const NvArgs a) {
+  extern __shared__ __align__(1024) uint8_t smem[];
+  if ((smem_u32(smem) & 1023u) != 0) {
+    if (threadIdx.x == 0 && a.status != nullptr) atomicExch(a.status, (uint32_t)kDevSmemAlign);
+    return;
+  }
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + kOffBars);
+  uint64_t* empty = full + kStages;
+  uint64_t* acc_full = empty + kStages;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(acc_full + 1);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+  const uint32_t warp = warp_id(), lane = lane_id();
+  const int mt = (int)(blockIdx.x % (uint32_t)a.num_m), nt = (int)(blockIdx.x / (uint32_t)a.num_m);
+  const int ks = a.k_stages;
+  if (threadIdx.x == 0) {
+    *abort_flag = 0;
+    for (int i = 0; i < kStages; ++i) {
+      mbar_init(&full[i], 1);
+      mbar_init(&empty[i], 1);
+    }
+    mbar_init(acc_full, 1);
+    fence_mbar_init();
+    tma_prefetch_desc(&tmA);
+    tma_prefetch_desc(&tmB);
+  }
+  if (warp == 1) {
+    tmem_alloc(tmem_slot, kTmemColsG);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_slot;
+  pdl_launch_dependents();
+  pdl_wait();  // the images come from the kernels before this one
+
+  if (warp == 0) {
+    if (lane == 0) {
+      for (int kb = 0; kb < ks; ++kb) {
+        const int s = kb % kStages;
+        if (!mbar_wait(&empty[s], (uint32_t)((kb / kStages) & 1) ^ 1u, abort_flag, a.status)) break;
+        uint8_t* st = smem + (uint32_t)s * kStageBytes;
+        mbar_arrive_expect_tx(&full[s], kStageBytes);
+        tma_load_2d(st, &tmA, &full[s], 0, (mt * ks + kb) * kTileM);
+        tma_load_2d(st + kABytes, &tmB, &full[s], 0, ((2 * nt) * ks + kb) * 128);
+        tma_load_2d(st + kABytes + kBBytes / 2, &tmB, &full[s], 0, ((2 * nt + 1) * ks + kb) * 128);
+      }
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      bool ok = true;
+      for (int kb = 0; ok && kb < ks; ++kb) {
+        const int s = kb % kStages;
+        if (!(ok = mbar_wait(&full[s], (uint32_t)((kb / kStages) & 1), abort_flag, a.status))) break;
+        tc_fence_after();
+        const uint32_t sa = smem_u32(smem + (uint32_t)s * kStageBytes);
+        const uint64_t ad = sdesc_kmajor_sw128(sa), bd = sdesc_kmajor_sw128(sa + kABytes);
+#pragma unroll
+        for (int k4 = 0; k4 < 4; ++k4)  // 16 bf16 (32 bytes) of K per MMA: +2 in the descriptor's 16-byte units
+          umma_bf16(tmem_base, ad + 2u * (uint32_t)k4, bd + 2u * (uint32_t)k4, kIdescBf16, (kb | k4) != 0 ? 1u : 0u);
+        umma_commit(&empty[s]);
+      }
+      if (ok) umma_commit(acc_full);
+    }
+  } else {  // drain: warp w reads TMEM lanes 32 (w % 4) .. (all four quarters over warps 2-5)
+    const uint32_t quarter = warp & 3u;
+    const int row = mt * kTileM + (int)(quarter * 32u + lane);
+    const bool ok = __all_sync(0xffffffffu, mbar_wait(acc_full, 0, abort_flag, a.status));
+    if (ok) {
+      tc_fence_after();
+      const float gw = *a.gw;
+#pragma unroll 1
+      for (int c = 0; c < kTileN; c += 32) {
+        uint32_t r[32];
+        tmem_ld32(tmem_base + ((quarter * 32u) << 16) + (uint32_t)c, r);
+        tmem_ld_wait();
+        const int col0 = nt * kTileN + c;
+        if (row < a.M) {
+#pragma unroll
+          for (int v8 = 0; v8 < 4; ++v8) {
+            const int col = col0 + 8 * v8;
+            if (col < a.N) {  // N % 8 == 0: a chunk of 8 is wholly inside or outside
+              uint32_t o[4];
+#pragma unroll
+              for (int i = 0; i < 4; ++i) {
+                const int cc = 8 * v8 + 2 * i;
+                const float b0 = a.bias != nullptr ? __ldg(a.bias + col + 2 * i) : 0.0f;
+                const float b1 = a.bias != nullptr ? __ldg(a.bias + col + 2 * i + 1) : 0.0f;
+                const float y0 = (__uint_as_float(r[cc]) * a.ga) * gw + b0;
+                const float y1 = (__uint_as_float(r[cc + 1]) * a.ga) * gw + b1;
+                const __nv_bfloat162 p = __floats2bfloat162_rn(y0, y1);
+                o[i] = *reinterpret_cast<const uint32_t*>(&p);
+              }
+              *reinterpret_cast<uint4*>(a.y + (int64_t)row * a.N + col) = make_uint4(o[0], o[1], o[2], o[3]);
+            }
+          }
+        }
+      }
+    }
+  }
+  // Every TMA copy issued has landed (the MMA waited for each; a producer that gave up issued no
+  // more), every MMA has completed (the drain waited for the last commit, or all gave up).
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 0 && lane == 0 && *abort_flag) {  // unwinding: wait (bounded) for copies in flight
+    for (int kb = (ks > kStages ? ks - kStages : 0); kb < ks; ++kb) {
+      int dummy = 0;
+      mbar_wait(&full[kb % kStages], (uint32_t)((kb / kStages) & 1), &dummy, a.status);
+    }
+  }
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem_base, kTmemColsG);
+  }
+}
+
+int grid_cap(int64_t items, int threads, int sms) {
+  int64_t b = (items + threads - 1) / threads;
+  const int64_t cap = (int64_t)sms * 8;
+  return (int)(b < 1 ? 1 : (b > cap ? cap : b));
+}
+
+}  // namespace
+
+size_t nvfp4_image_bytes(int64_t rows, int64_t K) { return (size_t)((rows + 127) / 128 * 128) * (size_t)K * 2; }
+
+cudaError_t launch_nvfp4_quantize_act(const void* x, int64_t M, int64_t K, int64_t ldx, float g, uint8_t* codes,
+                                      uint8_t* scales, cudaStream_t stream, int sms) {
+  if (M == 0) return cudaSuccess;
+  return launch_pdl(nvfp4_quantize_kernel<__nv_bfloat16>, dim3(grid_cap(M * (K / 16), 256, sms)), dim3(256), 0,
+                    stream, static_cast<const __nv_bfloat16*>(x), M, K, ldx, g, (const float*)nullptr, codes, scales);
+}
+
+cudaError_t launch_nvfp4_pack_weight(const float* w, int64_t N, int64_t K, uint8_t* codes, uint8_t* scales, float* g,
+                                     cudaStream_t stream, int sms) {
+  if (N == 0) return cudaSuccess;
+  cudaError_t e = cudaMemsetAsync(g, 0, sizeof(float), stream);
+  if (e != cudaSuccess) return e;
+  if ((e = launch_pdl(nvfp4_amax_kernel, dim3(grid_cap(N * K, 256, sms)), dim3(256), 0, stream, w, N * K,
+                      reinterpret_cast<unsigned int*>(g))) != cudaSuccess)
+    return e;
+  if ((e = launch_pdl(nvfp4_finish_g_kernel, dim3(1), dim3(1), 0, stream, g)) != cudaSuccess) return e;
+  return launch_pdl(nvfp4_quantize_kernel<float>, dim3(grid_cap(N * (K / 16), 256, sms)), dim3(256), 0, stream, w, N,
+                    K, K, 0.0f, (const float*)g, codes, scales);
+}
+
+cudaError_t launch_nvfp4_linear(const uint8_t* qa, const uint8_t* sa, float ga, const uint8_t* qw, const uint8_t* sw,
+                                const float* gw, const float* bias, void* y, int64_t M, int64_t N, int64_t K,
+                                uint8_t* workspace, uint32_t* status, cudaStream_t stream, int sms) {
+  if (M == 0 || N == 0) return cudaSuccess;
+  uint8_t* img_a = workspace;
+  uint8_t* img_b = workspace + nvfp4_image_bytes(M, K);
+  cudaError_t e;
+  if ((e = launch_pdl(nvfp4_expand_kernel, dim3(grid_cap(M * (K / 8), 256, sms)), dim3(256), 0, stream, qa, sa, M, K,
+                      img_a)) != cudaSuccess)
+    return e;
+  if ((e = launch_pdl(nvfp4_expand_kernel, dim3(grid_cap(N * (K / 8), 256, sms)), dim3(256), 0, stream, qw, sw, N, K,
+                      img_b)) != cudaSuccess)
+    return e;
+  // The set-up CUDA keeps per device: the dynamic shared-memory size of the GEMM kernel.
+  static PerDevice<bool> attr;
+  bool done = false;
+  if ((e = attr.get(
+           [](bool& v) {
+             v = true;
+             return cudaFuncSetAttribute(nvfp4_gemm_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemG);
+           },
+           done)) != cudaSuccess)
+    return e;
+  // Both images as rows of 128 bytes; one box = one 128-row block of a stage, copied as it is
+  // (already in the 128-byte swizzle).
+  const int ks = (int)(K / kStageK);
+  const int64_t rows_a = (M + 127) / 128 * 128 * ks, rows_b = (N + 127) / 128 * 128 * ks;
+  CUtensorMap tmA, tmB;
+  if (!encode_2d(&tmA, CU_TENSOR_MAP_DATA_TYPE_UINT8, img_a, 128, (uint64_t)rows_a, 128, 128, 128,
+                 CU_TENSOR_MAP_SWIZZLE_NONE) ||
+      !encode_2d(&tmB, CU_TENSOR_MAP_DATA_TYPE_UINT8, img_b, 128, (uint64_t)rows_b, 128, 128, 128,
+                 CU_TENSOR_MAP_SWIZZLE_NONE))
+    return cudaErrorInvalidValue;
+  NvArgs a;
+  a.M = (int)M;
+  a.N = (int)N;
+  a.k_stages = ks;
+  a.num_m = (int)((M + kTileM - 1) / kTileM);
+  a.ga = ga;
+  a.gw = gw;
+  a.bias = bias;
+  a.y = static_cast<__nv_bfloat16*>(y);
+  a.status = status;
+  const int tiles = a.num_m * (int)((N + kTileN - 1) / kTileN);
+  return launch_pdl(nvfp4_gemm_kernel, dim3(tiles), dim3(kThreadsG), kSmemG, stream, tmA, tmB, a);
+}
+
+}  // namespace jq

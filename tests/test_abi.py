@@ -263,3 +263,38 @@ def test_dit_neighbour_entry_points_check_arguments(lib):
     assert gelu(p, 4, 256, 260, 128, p, p, None) == 2                 # ldh * 2 not a multiple of 16
     assert gelu(None, 4, 256, 256, 128, p, p, None) == 1
     assert gelu(p, 4, 200, 256, 128, p, p, None) == 1                 # K not a multiple of 128
+
+
+def test_nvfp4_entry_points_check_arguments(lib):
+    """jq_nvfp4_quantize_act / _pack_weight / _linear refuse bad arguments before any launch."""
+    vp, i64, f32, sz = ctypes.c_void_p, ctypes.c_int64, ctypes.c_float, ctypes.c_size_t
+    lib.jq_nvfp4_quantize_act.argtypes = [vp, i64, i64, i64, f32, vp, vp, vp]
+    lib.jq_nvfp4_pack_weight.argtypes = [vp, i64, i64, vp, vp, vp, vp]
+    lib.jq_nvfp4_linear.argtypes = [vp, vp, f32, vp, vp, vp, vp, vp, i64, i64, i64, vp, sz, vp]
+    lib.jq_nvfp4_workspace_size.argtypes = [i64, i64, i64]
+    lib.jq_nvfp4_workspace_size.restype = sz
+    p, odd = vp(4096), vp(4100)
+    qa = lib.jq_nvfp4_quantize_act
+    assert qa(p, 4, 192, 192, 0.01, p, p, None) == 3               # valid (K % 64 == 0): no sm_103 device here
+    assert qa(p, 0, 192, 192, 0.01, p, p, None) == 0               # empty batch
+    assert qa(p, 4, 200, 200, 0.01, p, p, None) == 1               # K not a multiple of 64
+    assert qa(p, 4, 192, 128, 0.01, p, p, None) == 1               # ldx < K
+    assert qa(p, 4, 192, 192, -1.0, p, p, None) == 1               # negative tensor scale
+    assert qa(p, 4, 192, 192, float("inf"), p, p, None) == 1       # infinite tensor scale
+    assert qa(p, 4, 192, 192, float("nan"), p, p, None) == 1       # NaN tensor scale
+    assert qa(odd, 4, 192, 192, 0.01, p, p, None) == 2             # misaligned x
+    assert qa(p, 4, 192, 196, 0.01, p, p, None) == 2               # ldx * 2 not a multiple of 16
+    pw = lib.jq_nvfp4_pack_weight
+    assert pw(p, 8, 128, p, p, p, None) == 3
+    assert pw(p, 8, 128, p, p, None, None) == 1                    # no output for g_w
+    assert pw(p, 8, 128, p, p, odd, None) == 2
+    need = lib.jq_nvfp4_workspace_size(64, 256, 128)
+    assert need == 128 * 128 * 2 + 256 * 128 * 2                  # two bf16 operand images, whole 128-row tiles
+    assert lib.jq_nvfp4_workspace_size(64, 256, 100) == 0
+    ln = lib.jq_nvfp4_linear
+    assert ln(p, p, 1.0, p, p, p, None, p, 64, 256, 128, p, need, None) == 3
+    assert ln(p, p, 1.0, p, p, p, None, p, 64, 252, 128, p, need, None) == 1   # N % 8 != 0
+    assert ln(p, p, 1.0, p, p, None, None, p, 64, 256, 128, p, need, None) == 1  # no g_w
+    assert ln(p, p, 1.0, p, p, p, None, p, 64, 256, 128, p, need - 1, None) == 6  # short workspace
+    assert ln(p, p, 1.0, p, p, p, None, odd, 64, 256, 128, p, need, None) == 2   # misaligned y
+    assert ln(p, p, 1.0, p, p, p, None, p, 0, 256, 128, None, 0, None) == 0      # empty
