@@ -137,16 +137,18 @@ def whole_job_tops(world: int, ops_per_step: float, steps: int, seconds: float) 
 
 
 def metric_name(args) -> str:
-    return "W1.58A4 linear TOPS" if args.weights == "ternary" else "W4A4 linear TOPS"
+    return {"ternary": "W1.58A4 linear TOPS", "nvfp4": "NVFP4 W4A4 linear TOPS"}.get(args.weights, "W4A4 linear TOPS")
 
 
-def launches_per_step(M: int, few: bool, fused: bool, ternary: bool) -> int:
+def launches_per_step(M: int, few: bool, fused: bool, ternary: bool, nvfp4: bool = False) -> int:
     """Kernels of this library per timed step: the activation quantiser (or, fused, the
     quantise-to-operand kernel), the operand expansion when the linear kernel reads the operand
     image (more than 16 tokens), the ternary -> INT4 rewrite (ternary weights, GEMM), and the
     linear kernel itself."""
     if fused:
         return 2
+    if nvfp4:  # quantiser, the two operand images, GEMM
+        return 4
     return 1 + (1 if M > 16 else 0) + (1 if ternary and not few else 0) + 1
 
 
@@ -218,16 +220,23 @@ class OracleSample:
     sampled activation rows and evaluate the linear layer for them (the weights are packed
     once, outside the timing, as on the GPU)."""
 
-    def __init__(self, name: str, seed: int = 7, ternary: bool = False):
+    def __init__(self, name: str, seed: int = 7, ternary: bool = False, fmt: str | None = None):
         import oracle
         from paper_2609_33601_gb300 import workloads as wl
         self.oracle = oracle
+        self.wl = wl
         self.name = name
+        self.fmt = fmt or ("ternary" if ternary else "int4")
         self.desc, self.M, self.K, self.N, self.G, gen = WORKLOADS[name]
         w = wl.make(gen, seed=seed, M=self.M, K=self.K, N=self.N, G=self.G)
         self.x_bits, self.bias = w.x_bits, w.bias
-        quant = oracle.quantize_ternary_f32 if ternary else oracle.quantize_f32
-        self.qw, self.sw = quant(w.w, self.G)
+        if self.fmt == "nvfp4":  # weights with their own tensor scale; activations with a calibrated one
+            self.gw = oracle.nvfp4_tensor_scale(w.w)
+            self.qw, self.sw = oracle.quantize_nvfp4(w.w, self.gw)
+            self.ga = oracle.nvfp4_tensor_scale(wl.bf16_bits_to_f32(self.x_bits))
+        else:
+            quant = oracle.quantize_ternary_f32 if self.fmt == "ternary" else oracle.quantize_f32
+            self.qw, self.sw = quant(w.w, self.G)
         self.rows = 8
         self.run_s = 0.0
         self.tokens_per_sample = wl.DIT_TOKENS_PER_IMAGE
@@ -235,6 +244,10 @@ class OracleSample:
 
     def run(self, rows: int) -> float:
         t0 = time.perf_counter()
+        if self.fmt == "nvfp4":
+            qa2, sa = self.oracle.quantize_nvfp4(self.wl.bf16_bits_to_f32(self.x_bits[:rows]), self.ga)
+            self.oracle.linear_nvfp4(qa2, sa, self.ga, self.qw, self.sw, self.gw, self.bias)
+            return time.perf_counter() - t0
         prologue = DIT_PROLOGUE.get(self.name)
         if prologue == "modulate":
             _, qa, sa = self.oracle.modulate_quantize_bf16(self.x_bits[:rows], self.mod[0], self.mod[1],
@@ -288,7 +301,7 @@ def run_reference(args):
     rank, world, _ = dist_env()
     if rank != 0:
         return 0
-    o = OracleSample(args.workload, ternary=args.weights == "ternary")
+    o = OracleSample(args.workload, fmt=args.weights)
     per_step = min(args.ref_seconds, 120.0 / (args.steps + args.warmup))
     o.calibrate(per_step)
     for _ in range(args.warmup):
@@ -658,7 +671,8 @@ def run_ours(args):
     from paper_2609_33601_gb300 import workloads as wl
 
     desc, M, K, N, G, gen = WORKLOADS[args.workload]
-    few = M <= FEW_TOKENS
+    nv = args.weights == "nvfp4"
+    few = M <= FEW_TOKENS and not nv  # NVFP4 has no few-token kernel: every M takes its GEMM
     dev = torch.device("cuda", local)
     sets = []
     # rotating weight sets: together several times larger than the 126 MB L2
@@ -666,8 +680,14 @@ def run_ours(args):
     for i in range(n_sets):
         w = wl.make(gen, seed=100 + 17 * rank + i, M=M, K=K, N=N, G=G)
         x = torch.from_numpy(w.x_bits.view(np.int16)).to(dev).view(torch.bfloat16)
-        pack = jq.jq_pack_weight_ternary if args.weights == "ternary" else jq.jq_pack_weight
-        qw, sw = pack(torch.from_numpy(w.w).to(dev), G)
+        if nv:  # codes, (block-scale bytes, device tensor scale)
+            codes_w, scales_w, g_w = jq.jq_nvfp4_pack_weight(torch.from_numpy(w.w).to(dev))
+            qw, sw = codes_w, (scales_w, g_w)
+            if i == 0:  # the activations' tensor scale, calibrated once on the first input set
+                ga = float(np.float32(np.abs(wl.bf16_bits_to_f32(w.x_bits)).max()) / np.float32(2688.0))
+        else:
+            pack = jq.jq_pack_weight_ternary if args.weights == "ternary" else jq.jq_pack_weight
+            qw, sw = pack(torch.from_numpy(w.w).to(dev), G)
         b = None if w.bias is None else torch.from_numpy(w.bias).to(dev)
         sets.append((x, qw, sw, b))
         del w
@@ -677,9 +697,17 @@ def run_ours(args):
     y = torch.empty((M, N), dtype=torch.bfloat16, device=dev)
     fused = args.fused
     ternary = args.weights == "ternary"
-    need = jq.jq_w158a4_workspace_size(M, N, K, G) if ternary else jq.jq_workspace_size(M, N, K, G, fused)
+    need = (jq.jq_nvfp4_workspace_size(M, N, K) if nv else
+            jq.jq_w158a4_workspace_size(M, N, K, G) if ternary else jq.jq_workspace_size(M, N, K, G, fused))
     ws = torch.empty(max(need, 16), dtype=torch.uint8, device=dev)
     linear_call = jq.jq_w158a4_linear if ternary else jq.jq_w4a4_linear
+    if nv:
+        codes_a = torch.empty((M, K // 2), dtype=torch.uint8, device=dev)
+        scales_a = torch.empty((M, K // 16), dtype=torch.uint8, device=dev)
+
+        def linear_call(q_, s_, qw_, sw_, b_, g_, y=None, workspace=None, stream=None):
+            return jq.jq_nvfp4_linear(codes_a, scales_a, ga, qw_, sw_[0], sw_[1], b_, y=y, workspace=workspace,
+                                      stream=stream)
     stream = torch.cuda.current_stream()
 
     prologue = DIT_PROLOGUE.get(args.workload)
@@ -690,7 +718,9 @@ def run_ours(args):
 
     def quantize(i, st):
         x = sets[i % n_sets][0]
-        if prologue == "modulate":
+        if nv:
+            jq.jq_nvfp4_quantize_act(x, ga, codes_a, scales_a, stream=st)
+        elif prologue == "modulate":
             sh, sc = mods[i % n_sets]
             jq.jq_modulate_quantize_act(x, sh, sc, T, G, q, s_a, stream=st)
         elif prologue == "gelu":
@@ -776,7 +806,9 @@ def run_ours(args):
     y_free = [None] * nb  # the copy out of y_dev[k] is done
 
     def quantize_x(x, i, st):
-        if prologue == "modulate":
+        if nv:
+            jq.jq_nvfp4_quantize_act(x, ga, codes_a, scales_a, stream=st)
+        elif prologue == "modulate":
             sh, sc = mods[i % n_sets]
             jq.jq_modulate_quantize_act(x, sh, sc, T, G, q, s_a, stream=st)
         elif prologue == "gelu":
@@ -838,16 +870,22 @@ def run_ours(args):
     bf16_peak, hbm_peak, peak_src = measured_peaks()
     fp8_peak = bf16_peak * FP8_PER_BF16
     kernel_file = "skinny.cu" if few else "gemm.cu"
-    traffic = None if (fused or ternary) else recorded_traffic(args.workload, kernel_file)
+    traffic = None if (fused or ternary or nv) else recorded_traffic(args.workload, kernel_file)
     # algorithmic bytes of one linear call: packed weights and their scales, packed activation
     # codes and scales (the fused call reads bf16 activations instead), bias, bf16 output
     groups = K // G
     act_bytes = M * K * 2 if fused else M * K // 2 + M * groups * 4
     wbytes = N * K // 4 if ternary else N * K // 2  # 2-bit ternary or 4-bit INT4 weight codes
     alg_bytes = wbytes + groups * N * 4 + act_bytes + (0 if sets[0][3] is None else N * 4) + M * N * 2
+    tensor_peak, tensor_src = fp8_peak, f"{peak_src} bf16 {bf16_peak} TFLOP/s x nominal FP8/BF16 ratio {FP8_PER_BF16}"
+    if nv:  # E2M1 codes and E4M3 block-scale bytes of both operands; the layer's MMA is bf16
+        alg_bytes = (M + N) * (K // 2 + K // 16) + (0 if sets[0][3] is None else N * 4) + M * N * 2
+        tensor_peak, tensor_src = bf16_peak, f"{peak_src} bf16 {bf16_peak} TFLOP/s (the layer's MMA is bf16)"
     # the bound is whichever of the tensor time and the HBM time is larger
-    t_tensor, t_hbm = ops_step / (fp8_peak * 1e12), alg_bytes / (hbm_peak * 1e9)
-    what = ("jq_w158a4_linear (few-token kernel, 2-bit weights)" if ternary and few else
+    t_tensor, t_hbm = ops_step / (tensor_peak * 1e12), alg_bytes / (hbm_peak * 1e9)
+    what = ("jq_nvfp4_linear (bf16 operand images of the exact block-scaled values + tcgen05 kind::f16 GEMM)"
+            if nv else
+            "jq_w158a4_linear (few-token kernel, 2-bit weights)" if ternary and few else
             "jq_w158a4_linear (ternary -> INT4 rewrite + operand expansion + tcgen05 GEMM)" if ternary else
             "jq_fused_quant_linear (quantise-to-operand + tcgen05 GEMM)" if fused else
             "jq_w4a4_linear (few-token weight-streaming kernel)" if few else
@@ -860,11 +898,11 @@ def run_ours(args):
                     "peak_source": f"{peak_src} HBM copy bandwidth {hbm_peak} GB/s"}
     else:
         achieved = ops_step / (gemm_ms * 1e-3) / 1e12
-        roofline = {"bound": "tensor", "achieved": achieved, "peak": fp8_peak, "unit": "TFLOP/s",
-                    "frac": achieved / fp8_peak, "frac_of_bf16_peak": achieved / bf16_peak,
+        roofline = {"bound": "tensor", "achieved": achieved, "peak": tensor_peak, "unit": "TFLOP/s",
+                    "frac": achieved / tensor_peak, "frac_of_bf16_peak": achieved / bf16_peak,
                     "traffic": traffic, "algorithmic_bytes": alg_bytes,
                     "kernel": what + ", CUDA events around a graph of K launches",
-                    "peak_source": f"{peak_src} bf16 {bf16_peak} TFLOP/s x nominal FP8/BF16 ratio {FP8_PER_BF16}"}
+                    "peak_source": tensor_src}
     context = None
     if not args.no_context:
         context = {"cublas_bf16": cublas_context(torch, dev, sets, M, N, K, args, world)}
@@ -879,20 +917,22 @@ def run_ours(args):
         return 0
     cpu = None
     if world == 1 and not args.no_cpu_baseline:
-        o = OracleSample(args.workload, ternary=ternary)
+        o = OracleSample(args.workload, fmt=args.weights)
         o.calibrate(args.ref_seconds)
         cpu = o.describe(o.run(o.rows), single_s=args.ref_single_seconds)
     line = {
         "metric": metric_name(args), "value": value, "unit": "TOPS", "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": total_ms / args.steps, "higher_is_better": True, "scaling": "weak",
-        "vs_baseline": None, "dtype": "int4", "data": "synthetic",
+        "vs_baseline": None, "dtype": "nvfp4" if nv else "int4", "data": "synthetic",
         "config": {"workload": desc, "M": M, "K": K, "N": N, "group": G,
-                   "step": ("jq_fused_quant_linear" if fused else
+                   "step": ("jq_nvfp4_quantize_act + jq_nvfp4_linear" if nv else
+                            "jq_fused_quant_linear" if fused else
                             "jq_quantize_act + jq_w158a4_linear" if ternary else
                             "jq_modulate_quantize_act + jq_w4a4_linear" if prologue == "modulate" else
                             "jq_gelu_quantize_act + jq_w4a4_linear" if prologue == "gelu" else
                             "jq_quantize_act + jq_w4a4_linear"),
-                   "weights": "ternary (2-bit)" if ternary else "INT4",
+                   "weights": ("NVFP4 (E2M1, E4M3 scale per 16, fp32 tensor scale)" if nv else
+                               "ternary (2-bit)" if ternary else "INT4"),
                    "launch": "CUDA graph of the K steps",
                    "parallelism": f"replicas x{world}",
                    "l2": f"{n_sets} rotating input/weight sets larger than L2"},
@@ -902,7 +942,7 @@ def run_ours(args):
         "e2e": {"value": e2e_value, "unit": "TOPS", "h2d_bytes_per_step": M * K * 2, "d2h_bytes_per_step": M * N * 2,
                 "copies": ("pinned host buffers, on two copy streams overlapping the neighbouring steps' kernels"
                            if pipelined else "pinned host buffers, on the compute stream around the kernels")},
-        "gpu_launches": launches_per_step(M, few, fused, ternary) * args.steps,
+        "gpu_launches": launches_per_step(M, few, fused, ternary, nv) * args.steps,
         "clocks": clocks.summary(),
     }
     print(json.dumps(line), flush=True)
@@ -925,14 +965,17 @@ def main():
                     help="CPU seconds for the oracle's single-thread sample (0: skip it)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--fused", action="store_true", help="time jq_fused_quant_linear (bf16 activations in)")
-    ap.add_argument("--weights", choices=["int4", "ternary"], default="int4",
-                    help="ternary: the W1.58A4 layer (jq_pack_weight_ternary + jq_w158a4_linear)")
+    ap.add_argument("--weights", choices=["int4", "ternary", "nvfp4"], default="int4",
+                    help="ternary: the W1.58A4 layer (jq_pack_weight_ternary + jq_w158a4_linear); nvfp4: the "
+                         "NVFP4 W4A4 layer (jq_nvfp4_pack_weight + jq_nvfp4_quantize_act + jq_nvfp4_linear)")
     ap.add_argument("--no-context", action="store_true", help="skip the cuBLAS bf16 GEMM of the same shape")
     args = ap.parse_args()
     if args.warmup < 3:
         ap.error("--warmup must be at least 3")
-    if args.fused and args.weights == "ternary":
+    if args.fused and args.weights != "int4":
         ap.error("--fused is an INT4-weight call")
+    if args.weights == "nvfp4" and (args.workload in DIT_PROLOGUE or args.workload in STREAM_WORKLOADS):
+        ap.error("--weights nvfp4 runs the plain linear layer workloads")
     if args.workload in STREAM_WORKLOADS:
         if args.impl == "reference":
             return run_stream_reference(args)
