@@ -16,9 +16,9 @@
 //                      value q * s_b (E2M1 x E4M3 needs at most 6 significant bits and lies in
 //                      [2^-10, 2688], so bf16 holds it exactly), in the 128-byte-swizzled K-major
 //                      layout of the GEMM's operand images with a stage of 64 elements (128 B)
-//   nvfp4_gemm_kernel  tcgen05 kind::f16 with bf16 operands from both images by TMA, fp32
-//                      accumulation in TMEM over the whole K (the block scales are inside the
-//                      operands), epilogue y = (acc * ga) * gw + bias -> bf16
+//   nvfp4_gemm_kernel  persistent tcgen05 kind::f16 GEMM with bf16 operands from both images by
+//                      TMA, fp32 accumulation in TMEM over the whole K (the block scales are
+//                      inside the operands), two accumulators, epilogue y = (acc * ga) * gw + bias
 // The products q_a s_a,b * q_w s_w,b are exact in the tensor core; its fp32 sum over K is not,
 // and its error is bounded by the fp32 summation bound over K products.
 //
@@ -198,11 +198,12 @@ __global__ void __launch_bounds__(256) nvfp4_expand_kernel(const uint8_t* __rest
 }
 
 // ---------------------------------------------------------------- GEMM
-constexpr int kTileM = 128, kTileN = 256, kStages = 4, kThreadsG = 192;
+constexpr int kTileM = 128, kTileN = 256, kStages = 4, kThreadsG = 192, kAccBufs = 2;
 constexpr uint32_t kABytes = kTileM * 128, kBBytes = kTileN * 128, kStageBytes = kABytes + kBBytes;  // 48 KB
 constexpr uint32_t kOffBars = kStages * kStageBytes;
-constexpr uint32_t kSmemG = kOffBars + (2 * kStages + 1) * 8 + 16;
-constexpr uint32_t kTmemColsG = 256;
+constexpr uint32_t kNumBarsG = 2 * kStages + 2 * kAccBufs;
+constexpr uint32_t kSmemG = kOffBars + kNumBarsG * 8 + 16;
+constexpr uint32_t kTmemColsG = kAccBufs * kTileN;  // 512: two accumulators
 // kind::f16, bf16 A and B (both K-major), fp32 accumulator: D format [4,6) = 1, A format [7,10)
 // = 1 (BF16), B format [10,13) = 1 (BF16), N >> 3 at [17,23), M >> 4 at [24,29).
 constexpr uint32_t kIdescBf16 = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(kTileN >> 3) << 17) |
@@ -219,7 +220,7 @@ __device__ __forceinline__ void umma_bf16(uint32_t d_tmem, uint64_t a_desc, uint
 }
 
 struct NvArgs {
-  int M, N, k_stages, num_m;
+  int M, N, k_stages, num_m, num_tiles;
   float ga;
   const float* gw;   // device scalar
   const float* bias;  // [N] or nullptr
@@ -227,10 +228,13 @@ struct NvArgs {
   uint32_t* status;
 };
 
-// One 128 x 256 output tile per CTA (tiles M-fastest, so that the CTAs resident at once share
-// weight tiles).  Warp 0: TMA producer (A: one 128-row box, B: two, per 64-element stage).
-// Warp 1: TMEM owner and MMA issuer (four 128x256x16 MMAs per stage, one commit per stage to free
-// the slot, one at the end for the drain).  Warps 2-5: drain, one accumulator row per thread.
+// Persistent: CTA c computes 128 x 256 output tiles c, c + grid, ... (tiles M-fastest, so that the
+// tiles in flight at once share weight tiles), with two TMEM accumulators so that a tile's
+// epilogue runs under the next tile's MMAs.  Warp 0: TMA producer (A: one 128-row box, B: two,
+// per 64-element stage, into a 4-stage ring that runs on across tiles).  Warp 1: TMEM owner and
+// MMA issuer (four 128x256x16 MMAs per stage, one commit per stage to free the slot, one per tile
+// for the drain).  Warps 2-5: drain, one accumulator row per thread, handing the accumulator back
+// once its last columns are in registers.
 __global__ void __launch_bounds__(kThreadsG, 1)
     nvfp4_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                       const NvArgs a) {
@@ -242,10 +246,10 @@ __global__ void __launch_bounds__(kThreadsG, 1)
   uint64_t* full = reinterpret_cast<uint64_t*>(smem + kOffBars);
   uint64_t* empty = full + kStages;
   uint64_t* acc_full = empty + kStages;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(acc_full + 1);
+  uint64_t* acc_empty = acc_full + kAccBufs;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(acc_empty + kAccBufs);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
   const uint32_t warp = warp_id(), lane = lane_id();
-  const int mt = (int)(blockIdx.x % (uint32_t)a.num_m), nt = (int)(blockIdx.x / (uint32_t)a.num_m);
   const int ks = a.k_stages;
   if (threadIdx.x == 0) {
     *abort_flag = 0;
@@ -253,7 +257,10 @@ __global__ void __launch_bounds__(kThreadsG, 1)
       mbar_init(&full[i], 1);
       mbar_init(&empty[i], 1);
     }
-    mbar_init(acc_full, 1);
+    for (int i = 0; i < kAccBufs; ++i) {
+      mbar_init(&acc_full[i], 1);
+      mbar_init(&acc_empty[i], 4);  // the four drain warps
+    }
     fence_mbar_init();
     tma_prefetch_desc(&tmA);
     tma_prefetch_desc(&tmB);
@@ -269,46 +276,69 @@ __global__ void __launch_bounds__(kThreadsG, 1)
   pdl_launch_dependents();
   pdl_wait();  // the images come from the kernels before this one
 
+  uint32_t issued = 0;  // producer: stages issued (ring position)
   if (warp == 0) {
     if (lane == 0) {
-      for (int kb = 0; kb < ks; ++kb) {
-        const int s = kb % kStages;
-        if (!mbar_wait(&empty[s], (uint32_t)((kb / kStages) & 1) ^ 1u, abort_flag, a.status)) break;
-        uint8_t* st = smem + (uint32_t)s * kStageBytes;
-        mbar_arrive_expect_tx(&full[s], kStageBytes);
-        tma_load_2d(st, &tmA, &full[s], 0, (mt * ks + kb) * kTileM);
-        tma_load_2d(st + kABytes, &tmB, &full[s], 0, ((2 * nt) * ks + kb) * 128);
-        tma_load_2d(st + kABytes + kBBytes / 2, &tmB, &full[s], 0, ((2 * nt + 1) * ks + kb) * 128);
+      bool ok = true;
+      for (int t = (int)blockIdx.x; ok && t < a.num_tiles; t += (int)gridDim.x) {
+        const int mt = t % a.num_m, nt = t / a.num_m;
+        for (int kb = 0; kb < ks; ++kb, ++issued) {
+          const uint32_t s = issued % kStages;
+          if (!(ok = mbar_wait(&empty[s], ((issued / kStages) & 1u) ^ 1u, abort_flag, a.status))) break;
+          uint8_t* st = smem + s * kStageBytes;
+          mbar_arrive_expect_tx(&full[s], kStageBytes);
+          tma_load_2d(st, &tmA, &full[s], 0, (mt * ks + kb) * kTileM);
+          tma_load_2d(st + kABytes, &tmB, &full[s], 0, ((2 * nt) * ks + kb) * 128);
+          tma_load_2d(st + kABytes + kBBytes / 2, &tmB, &full[s], 0, ((2 * nt + 1) * ks + kb) * 128);
+        }
       }
     }
   } else if (warp == 1) {
     if (lane == 0) {
       bool ok = true;
-      for (int kb = 0; ok && kb < ks; ++kb) {
-        const int s = kb % kStages;
-        if (!(ok = mbar_wait(&full[s], (uint32_t)((kb / kStages) & 1), abort_flag, a.status))) break;
+      uint32_t it = 0, tile_it = 0;
+      for (int t = (int)blockIdx.x; ok && t < a.num_tiles; t += (int)gridDim.x, ++tile_it) {
+        const uint32_t ab = tile_it % kAccBufs;
+        // the drain has emptied this accumulator (tile_it - 2's)
+        if (!(ok = mbar_wait(&acc_empty[ab], ((tile_it / kAccBufs) & 1u) ^ 1u, abort_flag, a.status))) break;
         tc_fence_after();
-        const uint32_t sa = smem_u32(smem + (uint32_t)s * kStageBytes);
-        const uint64_t ad = sdesc_kmajor_sw128(sa), bd = sdesc_kmajor_sw128(sa + kABytes);
+        const uint32_t d = tmem_base + ab * (uint32_t)kTileN;
+        for (int kb = 0; kb < ks; ++kb, ++it) {
+          const uint32_t s = it % kStages;
+          if (!(ok = mbar_wait(&full[s], (it / kStages) & 1u, abort_flag, a.status))) break;
+          tc_fence_after();
+          const uint32_t sa = smem_u32(smem + s * kStageBytes);
+          const uint64_t ad = sdesc_kmajor_sw128(sa), bd = sdesc_kmajor_sw128(sa + kABytes);
 #pragma unroll
-        for (int k4 = 0; k4 < 4; ++k4)  // 16 bf16 (32 bytes) of K per MMA: +2 in the descriptor's 16-byte units
-          umma_bf16(tmem_base, ad + 2u * (uint32_t)k4, bd + 2u * (uint32_t)k4, kIdescBf16, (kb | k4) != 0 ? 1u : 0u);
-        umma_commit(&empty[s]);
+          for (int k4 = 0; k4 < 4; ++k4)  // 16 bf16 (32 bytes) of K per MMA: +2 in the descriptor's 16-byte units
+            umma_bf16(d, ad + 2u * (uint32_t)k4, bd + 2u * (uint32_t)k4, kIdescBf16, (kb | k4) != 0 ? 1u : 0u);
+          umma_commit(&empty[s]);
+        }
+        if (ok) umma_commit(&acc_full[ab]);
       }
-      if (ok) umma_commit(acc_full);
     }
   } else {  // drain: warp w reads TMEM lanes 32 (w % 4) .. (all four quarters over warps 2-5)
     const uint32_t quarter = warp & 3u;
-    const int row = mt * kTileM + (int)(quarter * 32u + lane);
-    const bool ok = __all_sync(0xffffffffu, mbar_wait(acc_full, 0, abort_flag, a.status));
-    if (ok) {
+    const float gw = *a.gw;
+    uint32_t tile_it = 0;
+    for (int t = (int)blockIdx.x; t < a.num_tiles; t += (int)gridDim.x, ++tile_it) {
+      const int mt = t % a.num_m, nt = t / a.num_m;
+      const uint32_t ab = tile_it % kAccBufs;
+      const bool ok = __all_sync(0xffffffffu, mbar_wait(&acc_full[ab], (tile_it / kAccBufs) & 1u, abort_flag, a.status));
+      if (!ok) break;
       tc_fence_after();
-      const float gw = *a.gw;
+      const int row = mt * kTileM + (int)(quarter * 32u + lane);
+      const uint32_t taddr = tmem_base + ((quarter * 32u) << 16) + ab * (uint32_t)kTileN;
 #pragma unroll 1
       for (int c = 0; c < kTileN; c += 32) {
         uint32_t r[32];
-        tmem_ld32(tmem_base + ((quarter * 32u) << 16) + (uint32_t)c, r);
+        tmem_ld32(taddr + (uint32_t)c, r);
         tmem_ld_wait();
+        if (c + 32 == kTileN) {  // every column of this accumulator is in registers: hand it back
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(&acc_empty[ab]);
+        }
         const int col0 = nt * kTileN + c;
         if (row < a.M) {
 #pragma unroll
@@ -333,14 +363,14 @@ __global__ void __launch_bounds__(kThreadsG, 1)
       }
     }
   }
-  // Every TMA copy issued has landed (the MMA waited for each; a producer that gave up issued no
-  // more), every MMA has completed (the drain waited for the last commit, or all gave up).
+  // Every TMA copy issued has landed (the MMA waited for each, or the abort path below waits),
+  // every MMA has completed (the drain waited for each tile's last commit, or all gave up).
   tc_fence_before();
   __syncthreads();
   if (warp == 0 && lane == 0 && *abort_flag) {  // unwinding: wait (bounded) for copies in flight
-    for (int kb = (ks > kStages ? ks - kStages : 0); kb < ks; ++kb) {
+    for (uint32_t i = (issued > (uint32_t)kStages ? issued - kStages : 0u); i < issued; ++i) {
       int dummy = 0;
-      mbar_wait(&full[kb % kStages], (uint32_t)((kb / kStages) & 1), &dummy, a.status);
+      mbar_wait(&full[i % kStages], (i / kStages) & 1u, &dummy, a.status);
     }
   }
   __syncthreads();
@@ -418,13 +448,14 @@ cudaError_t launch_nvfp4_linear(const uint8_t* qa, const uint8_t* sa, float ga, 
   a.N = (int)N;
   a.k_stages = ks;
   a.num_m = (int)((M + kTileM - 1) / kTileM);
+  a.num_tiles = a.num_m * (int)((N + kTileN - 1) / kTileN);
   a.ga = ga;
   a.gw = gw;
   a.bias = bias;
   a.y = static_cast<__nv_bfloat16*>(y);
   a.status = status;
-  const int tiles = a.num_m * (int)((N + kTileN - 1) / kTileN);
-  return launch_pdl(nvfp4_gemm_kernel, dim3(tiles), dim3(kThreadsG), kSmemG, stream, tmA, tmB, a);
+  const int grid = a.num_tiles < sms ? a.num_tiles : sms;  // persistent: one CTA per SM
+  return launch_pdl(nvfp4_gemm_kernel, dim3(grid), dim3(kThreadsG), kSmemG, stream, tmA, tmB, a);
 }
 
 }  // namespace jq
