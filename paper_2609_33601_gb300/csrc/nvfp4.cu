@@ -130,9 +130,10 @@ __global__ void __launch_bounds__(256) nvfp4_quantize_kernel(const In* __restric
   if (sizeof(In) == 2) pdl_launch_dependents();
   pdl_wait();
   const float g = g_dev != nullptr ? *g_dev : g_host;
-  const int64_t nb = K / 16, total = rows * nb;
-  for (int64_t t = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; t < total; t += (int64_t)gridDim.x * blockDim.x) {
-    const int64_t r = t / nb, b = t % nb;
+  const int64_t nb = K / 16;
+  const int64_t b = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;  // the block of 16 within the row
+  if (b >= nb) return;
+  for (int64_t r = blockIdx.y; r < rows; r += gridDim.y) {
     float v[16];
     load16(x + r * ldx + b * 16, v);
     float amax = 0.0f;
@@ -162,38 +163,49 @@ __global__ void __launch_bounds__(256) nvfp4_quantize_kernel(const In* __restric
 // ---------------------------------------------------------------- bf16 operand images
 constexpr int kStageK = 64;  // bf16 elements per 128-byte operand row of a stage
 
-// One thread per 8 elements (a 16-byte chunk of the image).  rows may be short of a whole
-// 128-row tile: the image's rows past them are never written (their outputs are never kept).
-__global__ void __launch_bounds__(256) nvfp4_expand_kernel(const uint8_t* __restrict__ codes,
+// One thread per 32 elements of a row (four 16-byte chunks of the image, all in one stage); grid
+// x over the row's 32-element units, y over rows.  rows may be short of a whole 128-row tile:
+// the image's rows past them are never written (their outputs are never kept).
+__device__ __forceinline__ uint32_t e2m1_bf16_pair(uint32_t byte, float s) {
+  float v[2];
+#pragma unroll
+  for (int h = 0; h < 2; ++h) {
+    const uint32_t nib = (byte >> (4 * h)) & 15u;
+    // E2M1: exponent bits e = idx >> 1, mantissa bit m = idx & 1: m/2 for e = 0 (subnormal),
+    // (1 + m/2) 2^(e-1) otherwise -- 0, 0.5, 1, 1.5, 2, 3, 4, 6
+    const uint32_t idx = nib & 7u, ee = idx >> 1, mm = idx & 1u;
+    const float mag = ee == 0u ? 0.5f * (float)mm : (1.0f + 0.5f * (float)mm) * (float)(1u << (ee - 1u));
+    const float val = mag * s;  // exact
+    v[h] = (nib & 8u) ? -val : val;
+  }
+  const __nv_bfloat162 p = __floats2bfloat162_rn(v[0], v[1]);  // exact
+  return *reinterpret_cast<const uint32_t*>(&p);
+}
+
+__global__ void __launch_bounds__(128) nvfp4_expand_kernel(const uint8_t* __restrict__ codes,
                                                           const uint8_t* __restrict__ scales, int64_t rows, int64_t K,
                                                           uint8_t* __restrict__ image) {
   pdl_launch_dependents();
   pdl_wait();
-  const int64_t per_row = K / 8, total = rows * per_row;
+  const int64_t u = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;  // 32-element unit of the row
+  if (u >= K / 32) return;
   const uint32_t k_stages = (uint32_t)(K / kStageK);
-  for (int64_t t = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; t < total; t += (int64_t)gridDim.x * blockDim.x) {
-    const int64_t r = t / per_row, k0 = (t % per_row) * 8;
-    const uint32_t c = __ldg(reinterpret_cast<const uint32_t*>(codes + r * (K / 2) + k0 / 2));
-    const float s = e4m3_value(__ldg(scales + r * (K / 16) + k0 / 16));
-    uint32_t out[4];
+  const int64_t k0 = u * 32;
+  const uint32_t kb = (uint32_t)(k0 / kStageK), c16 = (uint32_t)((k0 % kStageK) / 8);
+  for (int64_t r = blockIdx.y; r < rows; r += gridDim.y) {
+    const uint4 c = __ldg(reinterpret_cast<const uint4*>(codes + r * (K / 2) + k0 / 2));
+    const uint8_t* sr = scales + r * (K / 16) + k0 / 16;  // byte loads: the scales carry no alignment rule
+    const float s0 = e4m3_value(__ldg(sr)), s1 = e4m3_value(__ldg(sr + 1));  // elements 0-15, 16-31
+    const uint32_t w[4] = {c.x, c.y, c.z, c.w};
 #pragma unroll
-    for (int i = 0; i < 4; ++i) {
-      float v[2];
+    for (int q = 0; q < 4; ++q) {  // chunk q: elements 8q .. 8q + 7 (4 code bytes)
+      const float sq = q < 2 ? s0 : s1;
+      uint32_t out[4];
 #pragma unroll
-      for (int h = 0; h < 2; ++h) {
-        const uint32_t nib = (c >> (8 * i + 4 * h)) & 15u;
-        // E2M1: exponent bits e = idx >> 1, mantissa bit m = idx & 1: m/2 for e = 0 (subnormal),
-        // (1 + m/2) 2^(e-1) otherwise -- 0, 0.5, 1, 1.5, 2, 3, 4, 6
-        const uint32_t idx = nib & 7u, ee = idx >> 1, mm = idx & 1u;
-        const float mag = ee == 0u ? 0.5f * (float)mm : (1.0f + 0.5f * (float)mm) * (float)(1u << (ee - 1u));
-        const float val = mag * s;  // exact
-        v[h] = (nib & 8u) ? -val : val;
-      }
-      const __nv_bfloat162 p = __floats2bfloat162_rn(v[0], v[1]);  // exact
-      out[i] = *reinterpret_cast<const uint32_t*>(&p);
+      for (int i = 0; i < 4; ++i) out[i] = e2m1_bf16_pair((w[q] >> (8 * i)) & 0xFFu, sq);
+      *reinterpret_cast<uint4*>(image + image_chunk_offset(r, kb, c16 + (uint32_t)q, k_stages)) =
+          make_uint4(out[0], out[1], out[2], out[3]);
     }
-    const uint32_t kb = (uint32_t)(k0 / kStageK), c16 = (uint32_t)((k0 % kStageK) / 8);
-    *reinterpret_cast<uint4*>(image + image_chunk_offset(r, kb, c16, k_stages)) = make_uint4(out[0], out[1], out[2], out[3]);
   }
 }
 
@@ -380,6 +392,13 @@ __global__ void __launch_bounds__(kThreadsG, 1)
   }
 }
 
+// Grid of (units of a row / threads) x rows, the rows capped at the grid's y limit (the kernels
+// stride over the rest).
+dim3 grid_rows(int64_t units, int threads, int64_t rows) {
+  const int64_t gx = (units + threads - 1) / threads;
+  return dim3((unsigned)gx, (unsigned)(rows < 65535 ? rows : 65535), 1);
+}
+
 int grid_cap(int64_t items, int threads, int sms) {
   int64_t b = (items + threads - 1) / threads;
   const int64_t cap = (int64_t)sms * 8;
@@ -393,8 +412,8 @@ size_t nvfp4_image_bytes(int64_t rows, int64_t K) { return (size_t)((rows + 127)
 cudaError_t launch_nvfp4_quantize_act(const void* x, int64_t M, int64_t K, int64_t ldx, float g, uint8_t* codes,
                                       uint8_t* scales, cudaStream_t stream, int sms) {
   if (M == 0) return cudaSuccess;
-  return launch_pdl(nvfp4_quantize_kernel<__nv_bfloat16>, dim3(grid_cap(M * (K / 16), 256, sms)), dim3(256), 0,
-                    stream, static_cast<const __nv_bfloat16*>(x), M, K, ldx, g, (const float*)nullptr, codes, scales);
+  return launch_pdl(nvfp4_quantize_kernel<__nv_bfloat16>, grid_rows(K / 16, 128, M), dim3(128), 0, stream,
+                    static_cast<const __nv_bfloat16*>(x), M, K, ldx, g, (const float*)nullptr, codes, scales);
 }
 
 cudaError_t launch_nvfp4_pack_weight(const float* w, int64_t N, int64_t K, uint8_t* codes, uint8_t* scales, float* g,
@@ -406,8 +425,8 @@ cudaError_t launch_nvfp4_pack_weight(const float* w, int64_t N, int64_t K, uint8
                       reinterpret_cast<unsigned int*>(g))) != cudaSuccess)
     return e;
   if ((e = launch_pdl(nvfp4_finish_g_kernel, dim3(1), dim3(1), 0, stream, g)) != cudaSuccess) return e;
-  return launch_pdl(nvfp4_quantize_kernel<float>, dim3(grid_cap(N * (K / 16), 256, sms)), dim3(256), 0, stream, w, N,
-                    K, K, 0.0f, (const float*)g, codes, scales);
+  return launch_pdl(nvfp4_quantize_kernel<float>, grid_rows(K / 16, 128, N), dim3(128), 0, stream, w, N, K, K, 0.0f,
+                    (const float*)g, codes, scales);
 }
 
 cudaError_t launch_nvfp4_linear(const uint8_t* qa, const uint8_t* sa, float ga, const uint8_t* qw, const uint8_t* sw,
@@ -417,11 +436,11 @@ cudaError_t launch_nvfp4_linear(const uint8_t* qa, const uint8_t* sa, float ga, 
   uint8_t* img_a = workspace;
   uint8_t* img_b = workspace + nvfp4_image_bytes(M, K);
   cudaError_t e;
-  if ((e = launch_pdl(nvfp4_expand_kernel, dim3(grid_cap(M * (K / 8), 256, sms)), dim3(256), 0, stream, qa, sa, M, K,
-                      img_a)) != cudaSuccess)
+  if ((e = launch_pdl(nvfp4_expand_kernel, grid_rows(K / 32, 128, M), dim3(128), 0, stream, qa, sa, M, K, img_a)) !=
+      cudaSuccess)
     return e;
-  if ((e = launch_pdl(nvfp4_expand_kernel, dim3(grid_cap(N * (K / 8), 256, sms)), dim3(256), 0, stream, qw, sw, N, K,
-                      img_b)) != cudaSuccess)
+  if ((e = launch_pdl(nvfp4_expand_kernel, grid_rows(K / 32, 128, N), dim3(128), 0, stream, qw, sw, N, K, img_b)) !=
+      cudaSuccess)
     return e;
   // The set-up CUDA keeps per device: the dynamic shared-memory size of the GEMM kernel.
   static PerDevice<bool> attr;
