@@ -215,6 +215,33 @@ def test_weight_quantiser_equals_activation_rule_on_bf16_exact_values():
     assert np.array_equal(ca, cw) and np.array_equal(sa, sw)
 
 
+@pytest.mark.parametrize("seed", [0, 1])
+def test_weight_quantiser_matches_exact_rational_rule_on_fp32_values(seed):
+    """The fp32 weight path on values that are not bf16-exact (24 significant bits), against the
+    exact-rational rule directly: random magnitudes over many binades, fp32 subnormals, groups
+    whose quotients fall on exact ties (x = (k + 1/2) s with s = amax/7 representable), and
+    values one fp32 ulp either side of such ties."""
+    rng = np.random.default_rng(100 + seed)
+    G = 16
+    w = (rng.standard_normal((48, G)) * np.exp(rng.uniform(-30, 30, (48, 1)))).astype(np.float32)
+    w[0] = 0.0
+    w[1, :] = np.float32(3e-42)                       # fp32 subnormal group
+    w[1, 5] = np.float32(7e-42)
+    s = np.float32(0.25)                              # amax 1.75 gives s = fl32(1.75 / 7) = 0.25
+    w[2] = np.float32(0.0)
+    w[2, :8] = np.array([1.75, 0.625, -0.625, 0.875, -1.125, 0.375, 0.125, -0.125], np.float32)
+    w[3] = w[2]
+    w[3, 1:8] = np.nextafter(w[2, 1:8], np.float32(np.inf))     # just above the ties
+    w[4] = w[2]
+    w[4, 1:8] = np.nextafter(w[2, 1:8], np.float32(-np.inf))    # just below
+    assert np.float32(np.float32(1.75) / np.float32(7)) == s
+    codes, scales = oracle.quantize_f32(w, group=G)
+    for r in range(w.shape[0]):
+        q_ref, s_ref = quant_ref(w[r])
+        assert scales[r, 0] == np.float32(s_ref), r
+        assert codes[r].tolist() == q_ref, r
+
+
 # ---------------------------------------------------------------- packing ----
 
 def test_pack_all_byte_values_round_trip():
