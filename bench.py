@@ -94,8 +94,9 @@ FP8_PER_BF16 = 2.0  # nominal dense FP8 / BF16 tensor-core ratio on GB300 (4.5 /
 # capture was taken on (kernel_hash); once the code changes the figure no longer applies and the
 # bench reports null until a new capture is recorded here.
 KERNEL_TRAFFIC: dict = {
-    ("flux_qkv", "22124523f93a78bb"): 54.730240e6 + 143.731712e6,
-    ("dllm", "22124523f93a78bb"): 31.241728e6 + 0.144384e6,
+    ("flux_qkv", "f01c650c0bc1bb2c"): 54.967552e6 + 143.880448e6,
+    ("dllm", "f01c650c0bc1bb2c"): 31.267584e6 + 0.160256e6,
+    ("dllm/ternary", "f01c650c0bc1bb2c"): 18.689792e6 + 0.122368e6,
 }
 
 
@@ -140,16 +141,16 @@ def metric_name(args) -> str:
     return {"ternary": "W1.58A4 linear TOPS", "nvfp4": "NVFP4 W4A4 linear TOPS"}.get(args.weights, "W4A4 linear TOPS")
 
 
-def launches_per_step(M: int, few: bool, fused: bool, ternary: bool, nvfp4: bool = False) -> int:
+def launches_per_step(M: int, fused: bool, nvfp4: bool = False) -> int:
     """Kernels of this library per timed step: the activation quantiser (or, fused, the
     quantise-to-operand kernel), the operand expansion when the linear kernel reads the operand
-    image (more than 16 tokens), the ternary -> INT4 rewrite (ternary weights, GEMM), and the
-    linear kernel itself."""
+    image (more than 16 tokens), and the linear kernel itself (ternary weights are read as
+    2-bit codes by both linear kernels)."""
     if fused:
         return 2
     if nvfp4:  # quantiser, the two operand images, GEMM
         return 4
-    return 1 + (1 if M > 16 else 0) + (1 if ternary and not few else 0) + 1
+    return 1 + (1 if M > 16 else 0) + 1
 
 
 def dist_env():
@@ -870,7 +871,8 @@ def run_ours(args):
     bf16_peak, hbm_peak, peak_src = measured_peaks()
     fp8_peak = bf16_peak * FP8_PER_BF16
     kernel_file = "skinny.cu" if few else "gemm.cu"
-    traffic = None if (fused or ternary or nv) else recorded_traffic(args.workload, kernel_file)
+    traffic = None if (fused or nv) else recorded_traffic(args.workload + ("/ternary" if ternary else ""),
+                                                          kernel_file)
     # algorithmic bytes of one linear call: packed weights and their scales, packed activation
     # codes and scales (the fused call reads bf16 activations instead), bias, bf16 output
     groups = K // G
@@ -886,7 +888,7 @@ def run_ours(args):
     what = ("jq_nvfp4_linear (bf16 operand images of the exact block-scaled values + tcgen05 kind::f16 GEMM)"
             if nv else
             "jq_w158a4_linear (few-token kernel, 2-bit weights)" if ternary and few else
-            "jq_w158a4_linear (ternary -> INT4 rewrite + operand expansion + tcgen05 GEMM)" if ternary else
+            "jq_w158a4_linear (operand expansion + tcgen05 GEMM reading the 2-bit codes)" if ternary else
             "jq_fused_quant_linear (quantise-to-operand + tcgen05 GEMM)" if fused else
             "jq_w4a4_linear (few-token weight-streaming kernel)" if few else
             "jq_w4a4_linear (operand expansion + tcgen05 GEMM)")
@@ -942,7 +944,7 @@ def run_ours(args):
         "e2e": {"value": e2e_value, "unit": "TOPS", "h2d_bytes_per_step": M * K * 2, "d2h_bytes_per_step": M * N * 2,
                 "copies": ("pinned host buffers, on two copy streams overlapping the neighbouring steps' kernels"
                            if pipelined else "pinned host buffers, on the compute stream around the kernels")},
-        "gpu_launches": launches_per_step(M, few, fused, ternary, nv) * args.steps,
+        "gpu_launches": launches_per_step(M, fused, nv) * args.steps,
         "clocks": clocks.summary(),
     }
     print(json.dumps(line), flush=True)

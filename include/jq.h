@@ -236,10 +236,12 @@ JQ_API size_t jq_w158a4_workspace_size(int64_t M, int64_t N, int64_t K, int32_t 
  *   y = bf16( sum_g acc[m,n,g] * s_a[m,g] * s_w[g,n] + bias[n] ),  acc over qa * qw, qw in {-1,0,1}.
  *   q, s_a    : packed INT4 activation codes and scales (jq_quantize_act)
  *   qw2, s_w  : packed ternary weights and scales (jq_pack_weight_ternary, or any ternary codes
- *               and finite scales in these layouts)
- *   workspace : >= jq_w158a4_workspace_size(M, N, K, group) bytes, 16-byte aligned
- * Up to 64 tokens the few-token kernel streams the 2-bit codes (half the bytes of INT4 weights);
- * for more tokens the codes are rewritten as INT4 into the workspace and the INT4 GEMM runs.
+ *               and finite scales in these layouts; a 2-bit field of 3 is not a code and gives an
+ *               unspecified result)
+ *   workspace : >= jq_w158a4_workspace_size(M, N, K, group) bytes, 16-byte aligned (the same
+ *               size as jq_workspace_size(M, N, K, group, 0))
+ * Both kernels read the 2-bit codes directly (half the weight bytes of INT4): up to 64 tokens the
+ * few-token kernel, for more tokens the INT4 GEMM, whose weight-unpack warps convert them.
  * Other arguments, shapes and errors as jq_w4a4_linear.
  */
 JQ_API jq_status jq_w158a4_linear(const uint8_t* q, const float* s_a, const uint8_t* qw2, const float* s_w,

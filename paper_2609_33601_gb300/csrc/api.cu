@@ -262,11 +262,8 @@ jq_status jq_pack_weight_ternary(const float* w, int64_t N, int64_t K, int32_t g
 }
 
 size_t jq_w158a4_workspace_size(int64_t M, int64_t N, int64_t K, int32_t group) {
-  if (M <= 0 || N < 0 || K <= 0 || group <= 0 || K % group != 0) return 0;
-  // as jq_w4a4_linear, + the weights rewritten as packed INT4 for the GEMM (M > 64)
-  size_t bytes = jq_workspace_size(M, N, K, group, 0);
-  if (!jq::skinny_supports(M, K, group)) bytes += round_up(static_cast<size_t>(N) * static_cast<size_t>(K / 2), 256);
-  return bytes;
+  // as jq_w4a4_linear: both kernels read the 2-bit codes directly
+  return jq_workspace_size(M, N, K, group, 0);
 }
 
 jq_status jq_w158a4_linear(const uint8_t* q, const float* s_a, const uint8_t* qw2, const float* s_w, const float* bias,
@@ -294,12 +291,11 @@ jq_status jq_w158a4_linear(const uint8_t* q, const float* s_a, const uint8_t* qw
     }
     return from_cuda(jq::launch_w4a4_skinny(p, s, d->sms));
   }
-  // many tokens: the compute-bound GEMM, fed the same codes as INT4
-  uint8_t* qw4 = a_op + jq_workspace_size(M, N, K, group, 0);
-  if (jq::launch_ternary_to_int4(qw2, N, K, qw4, s, d->sms) != cudaSuccess) return JQ_ERR_CUDA;
+  // many tokens: the compute-bound GEMM, its weight-unpack warps reading the 2-bit codes
   if (jq::launch_expand_operand(q, M, K, group, a_op, corr, s, d->sms) != cudaSuccess) return JQ_ERR_CUDA;
-  jq::GemmProblem p{static_cast<int>(M), static_cast<int>(N), static_cast<int>(K), group, a_op, s_a, corr, qw4, s_w,
+  jq::GemmProblem p{static_cast<int>(M), static_cast<int>(N), static_cast<int>(K), group, a_op, s_a, corr, qw2, s_w,
                     bias, y_bf16, nullptr, d->status};
+  p.ternary = 1;
   return from_cuda(jq::launch_w4a4_gemm(p, s, d->sms));
 }
 

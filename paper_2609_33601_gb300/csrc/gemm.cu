@@ -37,6 +37,7 @@
 // of a pair meet at a final cluster barrier before the pair's TMEM is released.
 #include <cfloat>
 #include <cstdint>
+#include <type_traits>
 #include <cuda.h>
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
@@ -110,6 +111,7 @@ struct Args {
   int num_m2, num_tiles, k_stages, slots_per_tile;
   int groups, sc_boxes;  // K / G, and scale-ring slots per tile (ceil(groups / kScGroups))
   int sa_tma;            // activation scales come through the scale ring (groups % 4 == 0)
+  int ternary;           // qw holds 2-bit ternary codes [N, K/4] (ternary.cu), not INT4 [N, K/2]
   const uint8_t* qw;
   const float* s_a;
   const float* corr;     // [M, K/G]: 8 * the group's activation code sum in 2^-18 units (offset codes)
@@ -664,18 +666,30 @@ struct UnpackCursor {
   int tile, j;
 };
 
-template <class T>
+// One stage's packed chunks of one thread: 16 bytes of INT4 codes, or the same 32 codes as 8 bytes
+// of ternary codes (W1.58A4, qw [N, K/4]).
+template <bool kTernary>
+using PackedChunk = typename std::conditional<kTernary, uint2, uint4>::type;
+
+template <class T, bool kTernary>
 __device__ __forceinline__ void unpack_load(const Args& args, const Pair& pr, const UnpackCursor& c, uint32_t ug,
-                                            uint32_t u, uint4 (&buf)[T::kChunksPerThread]) {
-  const int K2 = args.K / 2;
+                                            uint32_t u, PackedChunk<kTernary> (&buf)[T::kChunksPerThread]) {
   const int kb = c.j * kStagesPerSlot + (int)ug;
   if (c.tile < args.num_tiles && kb < args.k_stages) {
     const int n0 = (c.tile / args.num_m2) * T::kBN + (int)pr.rank * T::kBNHalf;
-    const uint8_t* src = args.qw + kb * (kBK / 2) + (u & 3u) * 16;
+    constexpr int kRowDiv = kTernary ? 4 : 2;  // K elements per packed byte
+    constexpr int kChunk = (int)sizeof(PackedChunk<kTernary>);
+    const int row_bytes = args.K / kRowDiv;
+    const uint8_t* src = args.qw + kb * (kBK / kRowDiv) + (u & 3u) * kChunk;
 #pragma unroll
     for (int i = 0; i < T::kChunksPerThread; ++i) {
       const int n = n0 + (int)(u >> 2) + 16 * i;
-      buf[i] = n < args.N ? __ldg(reinterpret_cast<const uint4*>(src + (int64_t)n * K2)) : make_uint4(0u, 0u, 0u, 0u);
+      if constexpr (kTernary)  // rows past N: zero codes
+        buf[i] = n < args.N ? __ldg(reinterpret_cast<const uint2*>(src + (int64_t)n * row_bytes))
+                            : make_uint2(kTernaryZeroWord, kTernaryZeroWord);
+      else
+        buf[i] = n < args.N ? __ldg(reinterpret_cast<const uint4*>(src + (int64_t)n * row_bytes))
+                            : make_uint4(0u, 0u, 0u, 0u);
     }
   }
 }
@@ -689,9 +703,10 @@ __device__ __forceinline__ void unpack_advance(const Args& args, const Pair& pr,
 
 // Converts this group's stage of ring slot (q % kSlots) into the slot's B half for that stage
 // (or, for the missing second stage of an odd K-stage count, only signals the slot).
-template <class T, bool kOffset>
+template <class T, bool kOffset, bool kTernary>
 __device__ __forceinline__ bool unpack_store(const Args& args, uint8_t* sB, const Bars& b, uint32_t ug, uint32_t u,
-                                             uint32_t q, bool has_stage, const uint4 (&buf)[T::kChunksPerThread],
+                                             uint32_t q, bool has_stage,
+                                             const PackedChunk<kTernary> (&buf)[T::kChunksPerThread],
                                              volatile int* abort_flag) {
   const uint32_t o = q % T::kSlots;
   if (!__all_sync(0xffffffffu, mbar_wait(&b.empty[o], ring_parity(q, T::kSlots) ^ 1u, abort_flag, args.status)))
@@ -703,10 +718,15 @@ __device__ __forceinline__ bool unpack_store(const Args& args, uint8_t* sB, cons
     for (int i = 0; i < T::kChunksPerThread; ++i) {
       const uint32_t r = (u >> 2) + 16u * i, r7 = r & 7u;
       uint4 lo, hi;
-      if (kOffset)
+      if constexpr (kTernary) {  // operand.cuh: each 16-code word is one operand chunk
+        static_assert(!kOffset, "ternary weights enter the MMA in sign-magnitude form only");
+        lo = tern16_to_operand(buf[i].x);
+        hi = tern16_to_operand(buf[i].y);
+      } else if constexpr (kOffset) {
         nib32_to_operand_offset(buf[i], lo, hi);  // offset weight codes (operand.cuh)
-      else
+      } else {
         nib32_to_operand(buf[i], lo, hi);
+      }
       const uint32_t row_base = dst + (r >> 3) * 1024u + r7 * 128u;
       st_shared_v4(row_base + (((2u * jc) ^ r7) << 4), lo.x, lo.y, lo.z, lo.w);
       st_shared_v4(row_base + (((2u * jc + 1u) ^ r7) << 4), hi.x, hi.y, hi.z, hi.w);
@@ -723,7 +743,7 @@ __device__ __forceinline__ bool unpack_store(const Args& args, uint8_t* sB, cons
   return true;
 }
 
-template <class T, bool kOffset>
+template <class T, bool kOffset, bool kTernary>
 __device__ __forceinline__ void unpack_role(const Args& args, const Pair& pr, uint8_t* sB, const Bars& b,
                                             volatile int* abort_flag) {
   const uint32_t ut = threadIdx.x - kUnpackWarp0 * 32;
@@ -733,22 +753,22 @@ __device__ __forceinline__ void unpack_role(const Args& args, const Pair& pr, ui
   const uint32_t total = static_cast<uint32_t>(my_tiles) * static_cast<uint32_t>(args.slots_per_tile);
   UnpackCursor sc{pr.cluster, 0};  // the slot being stored
   UnpackCursor lc = sc;            // the slot being loaded (two ahead)
-  uint4 b0[T::kChunksPerThread], b1[T::kChunksPerThread];
-  unpack_load<T>(args, pr, lc, ug, u, b0);
+  PackedChunk<kTernary> b0[T::kChunksPerThread], b1[T::kChunksPerThread];
+  unpack_load<T, kTernary>(args, pr, lc, ug, u, b0);
   unpack_advance(args, pr, lc);
-  unpack_load<T>(args, pr, lc, ug, u, b1);
+  unpack_load<T, kTernary>(args, pr, lc, ug, u, b1);
   unpack_advance(args, pr, lc);
   for (uint32_t q = 0; q < total; q += 2) {
     bool has = sc.j * kStagesPerSlot + (int)ug < args.k_stages;
-    if (!unpack_store<T, kOffset>(args, sB, b, ug, u, q, has, b0, abort_flag)) return;
+    if (!unpack_store<T, kOffset, kTernary>(args, sB, b, ug, u, q, has, b0, abort_flag)) return;
     unpack_advance(args, pr, sc);
-    unpack_load<T>(args, pr, lc, ug, u, b0);
+    unpack_load<T, kTernary>(args, pr, lc, ug, u, b0);
     unpack_advance(args, pr, lc);
     if (q + 1 < total) {
       has = sc.j * kStagesPerSlot + (int)ug < args.k_stages;
-      if (!unpack_store<T, kOffset>(args, sB, b, ug, u, q + 1, has, b1, abort_flag)) return;
+      if (!unpack_store<T, kOffset, kTernary>(args, sB, b, ug, u, q + 1, has, b1, abort_flag)) return;
       unpack_advance(args, pr, sc);
-      unpack_load<T>(args, pr, lc, ug, u, b1);
+      unpack_load<T, kTernary>(args, pr, lc, ug, u, b1);
       unpack_advance(args, pr, lc);
     }
   }
@@ -842,7 +862,14 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
       drain_linear_rows<T, kOffset>(args, pr, tmem_base, b, sSc, abort_flag);
   } else if (warp >= kUnpackWarp0) {
     asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;\n" ::"n"(kRegsUnpack) : "memory");
-    unpack_role<T, kOffset>(args, pr, sB, b, abort_flag);
+    bool done = false;
+    if constexpr (!kExport && !kOffset) {  // W1.58A4 weights (the host never pairs them with offset codes)
+      if (args.ternary) {
+        unpack_role<T, kOffset, true>(args, pr, sB, b, abort_flag);
+        done = true;
+      }
+    }
+    if (!done) unpack_role<T, kOffset, false>(args, pr, sB, b, abort_flag);
   } else {
     asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;\n" ::"n"(kRegsCtl) : "memory");
     if (warp == kWarpProdA) {
@@ -933,6 +960,7 @@ cudaError_t launch_impl(const GemmProblem& p, cudaStream_t stream, int sms) {
   a.groups = groups;
   a.sc_boxes = (groups + kScGroups - 1) / kScGroups;
   a.sa_tma = sa_tma ? 1 : 0;
+  a.ternary = p.ternary ? 1 : 0;
   a.qw = p.qw;
   a.s_a = p.s_a;
   a.corr = p.corr;
@@ -981,7 +1009,9 @@ cudaError_t launch_w4a4_gemm(const GemmProblem& p, cudaStream_t stream, int sms)
   // One group: offset-code weights (see w4a4_gemm_kernel), exact while the whole K run fits the
   // offset form's fp32 range (operand.cuh); longer one-group runs keep the sign-magnitude form,
   // whose sums stay below 2^24 for every K the library accepts.  Group scales: 128-column tiles.
-  const bool offset = p.G == p.K && p.K <= kOffsetMaxRun;
+  // Ternary weights keep the sign-magnitude form in every mode (one form keeps the unpack role's
+  // registers within the kernel's budget).
+  const bool offset = p.G == p.K && p.K <= kOffsetMaxRun && !p.ternary;
   if (p.partials != nullptr)
     return offset ? launch_impl<true, true, 256>(p, stream, sms) : launch_impl<true, false, 256>(p, stream, sms);
   return offset ? launch_impl<false, true, 256>(p, stream, sms) : launch_impl<false, false, 256>(p, stream, sms);

@@ -89,9 +89,6 @@ cudaError_t launch_pack_weight(const float* w, int64_t N, int64_t K, int G, uint
 // fp32 weights [N, K] -> packed ternary codes [N, K/4] + scales [K/G, N] (ternary.cu).
 cudaError_t launch_pack_weight_ternary(const float* w, int64_t N, int64_t K, int G, uint8_t* qw, float* s_w,
                                        cudaStream_t stream, int sms);
-// packed ternary codes [N, K/4] -> packed INT4 codes [N, K/2] (ternary.cu).
-cudaError_t launch_ternary_to_int4(const uint8_t* qw2, int64_t N, int64_t K, uint8_t* qw4, cudaStream_t stream,
-                                   int sms);
 // bf16 activations [M, K] (dense rows) -> fake-quantised bf16 [M, K] + pass-through mask u8 [M, K]
 // + scales fp32 [M, K/G]; s_in (nullable) gives the scales instead of the amax rule (fakequant.cu).
 cudaError_t launch_fake_quant_act(const void* x, int64_t M, int64_t K, int G, const float* s_in, void* xhat,
@@ -133,12 +130,13 @@ struct GemmProblem {
   const uint8_t* a_operand;  // [M, K] operand bytes (workspace)
   const float* s_a;          // [M, K/G]
   const float* corr;         // [M, K/G]: 8 * sum of the group's activation codes, in 2^-18 units
-  const uint8_t* qw;         // [N, K/2] packed
+  const uint8_t* qw;         // [N, K/2] packed INT4 (or [N, K/4] ternary, below)
   const float* s_w;          // [K/G, N]
   const float* bias;         // [N] or nullptr
   void* y;                   // bf16 [M, N] (or nullptr when exporting partials)
   int32_t* partials;         // int32 [M, N, K/G] or nullptr
   uint32_t* status;          // device status word
+  int ternary = 0;           // qw holds packed ternary codes [N, K/4] (ternary.cu) instead of INT4
 };
 
 // Device address of the library's status word on the current device, or nullptr.

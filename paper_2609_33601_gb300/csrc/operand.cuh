@@ -76,6 +76,24 @@ __device__ __forceinline__ int nib32_sum(uint4 p) {
 }
 constexpr int kOffsetMaxRun = 139808;
 
+// Packed ternary codes (the W1.58A4 weights, 16 codes per 32-bit word, ternary.cu) -> operand
+// bytes.  Bits 0-1 of byte j of (word >> 2i) hold c = q + 1 in {0, 1, 2} for elements
+// {2j, 2j+1, 8+2j, 9+2j}[i], so the four shifts give the operand chunk of the word's 16 elements
+// in operand order with no byte movement.  Sign-magnitude bytes: c = 2 -> 0x01, c = 1 -> 0x00,
+// c = 0 -> 0x81; the magnitude bit is the complement of bit 0 of c and the sign is set where
+// neither bit of c is.
+__device__ __forceinline__ uint32_t tern4_to_operand(uint32_t p) {
+  const uint32_t mag = ~p & 0x01010101u;
+  const uint32_t neg = ~(p | (p >> 1)) & 0x01010101u;
+  return mag | (neg << 7);
+}
+__device__ __forceinline__ uint4 tern16_to_operand(uint32_t w) {
+  return make_uint4(tern4_to_operand(w), tern4_to_operand(w >> 2), tern4_to_operand(w >> 4),
+                    tern4_to_operand(w >> 6));
+}
+// The packed ternary word of 16 zero codes.
+constexpr uint32_t kTernaryZeroWord = 0x55555555u;
+
 // A-operand image (the GEMM's activation operand in global memory): for every 128-row tile
 // mt and every 128-element K stage kb, one contiguous 16 KB block that is byte for byte the
 // shared-memory image the tensor core reads -- 128 rows of 128 operand bytes in the 128-byte

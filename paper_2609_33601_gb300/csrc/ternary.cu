@@ -12,10 +12,7 @@
 // and 9+2j in bits 0-1, 2-3, 4-5 and 6-7.  So (word >> 2i) & 0x03030303, i = 0..3, are directly
 // the MMA operand bytes of elements {0,2,4,6}, {1,3,5,7}, {8,10,12,14}, {9,11,13,15}: the byte
 // order the INT4 operand uses (operand.cuh), in offset form q + 1, which E4M3 reads exactly.
-//
-// Expansion.  For the large-M GEMM the packed ternary codes are rewritten as packed INT4 codes
-// (4-bit two's complement, element 2j in the low nibble of byte j), which the GEMM consumes as
-// any INT4 weights.
+// Both the few-token kernel and the GEMM read this format directly (operand.cuh).
 #include <cstdint>
 #include <cuda_runtime.h>
 
@@ -70,26 +67,6 @@ __global__ void __launch_bounds__(128) pack_ternary_kernel(const float* __restri
   }
 }
 
-// One 32-bit word of 16 ternary codes -> 8 bytes of packed INT4 codes.
-__global__ void __launch_bounds__(256) ternary_to_int4_kernel(const uint32_t* __restrict__ in, int64_t words,
-                                                              uint2* __restrict__ out) {
-  pdl_launch_dependents();
-  pdl_wait();
-  for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < words; i += (int64_t)gridDim.x * blockDim.x) {
-    const uint32_t w = __ldg(in + i);
-    uint32_t lo = 0, hi = 0;
-#pragma unroll
-    for (int e = 0; e < 16; ++e) {
-      const uint32_t nib = (((w >> tern_bit(e)) & 3u) + 15u) & 15u;  // q + 1 -> q, 4-bit two's complement
-      if (e < 8)
-        lo |= nib << (4 * e);
-      else
-        hi |= nib << (4 * (e - 8));
-    }
-    out[i] = make_uint2(lo, hi);
-  }
-}
-
 int grid_cap(int64_t items, int threads, int sms) {
   int64_t blocks = (items + threads - 1) / threads;
   const int64_t cap = static_cast<int64_t>(sms) * 8;
@@ -103,14 +80,6 @@ cudaError_t launch_pack_weight_ternary(const float* w, int64_t N, int64_t K, int
   if (N == 0) return cudaSuccess;
   return launch_pdl(pack_ternary_kernel, dim3(grid_cap(N * (K / G), 128, sms)), dim3(128), 0, stream, w, N, K, G, qw,
                     s_w);
-}
-
-cudaError_t launch_ternary_to_int4(const uint8_t* qw2, int64_t N, int64_t K, uint8_t* qw4, cudaStream_t stream,
-                                   int sms) {
-  const int64_t words = N * K / 16;
-  if (words == 0) return cudaSuccess;
-  return launch_pdl(ternary_to_int4_kernel, dim3(grid_cap(words, 256, sms)), dim3(256), 0, stream,
-                    reinterpret_cast<const uint32_t*>(qw2), words, reinterpret_cast<uint2*>(qw4));
 }
 
 }  // namespace jq

@@ -127,9 +127,10 @@ def test_w158a4_entry_points(lib):
     lib.jq_workspace_size.argtypes = [i64, i64, i64, i32, i32]
     lib.jq_workspace_size.restype = sz
     ws, ws4 = lib.jq_w158a4_workspace_size, lib.jq_workspace_size
-    # few tokens: as the INT4 linear; many tokens: + the weights rewritten as packed INT4
+    # as the INT4 linear at every size: both kernels read the 2-bit codes in place
     assert ws(64, 12288, 4096, 128) == ws4(64, 12288, 4096, 128, 0)
-    assert ws(1024, 12288, 4096, 128) == ws4(1024, 12288, 4096, 128, 0) + 12288 * 4096 // 2
+    assert ws(1024, 12288, 4096, 128) == ws4(1024, 12288, 4096, 128, 0)
+    assert ws(4608, 3072, 15360, 15360) == ws4(4608, 3072, 15360, 15360, 0)
     assert ws(0, 8, 256, 64) == 0
     A, odd = _fake(0x10000), _fake(0x10008)
     P = lib.jq_pack_weight_ternary

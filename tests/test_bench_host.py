@@ -36,18 +36,17 @@ def test_recorded_traffic_applies_only_to_the_code_it_was_captured_on(monkeypatc
     assert bench.recorded_traffic("flux_out", "gemm.cu") is None
 
 
-@pytest.mark.parametrize("M,few,fused,ternary,expect", [
-    (1, True, False, False, 2),      # quantiser + few-token kernel
-    (16, True, False, False, 2),
-    (64, True, False, False, 3),     # + operand expansion (pre-expanded tokens)
-    (1024, False, False, False, 3),  # quantiser + operand expansion + GEMM
-    (1024, False, False, True, 4),   # + ternary -> INT4 rewrite
-    (64, True, False, True, 3),
-    (4608, False, True, False, 2),   # quantise-to-operand + GEMM
-    (1, True, True, False, 2),
+@pytest.mark.parametrize("M,fused,nvfp4,expect", [
+    (1, False, False, 2),      # quantiser + few-token kernel
+    (16, False, False, 2),
+    (64, False, False, 3),     # + operand expansion (pre-expanded tokens)
+    (1024, False, False, 3),   # quantiser + operand expansion + GEMM (INT4 or ternary weights)
+    (4608, True, False, 2),    # quantise-to-operand + GEMM
+    (1, True, False, 2),
+    (1024, False, True, 4),    # NVFP4: quantiser + two operand images + GEMM
 ])
-def test_launches_per_step(M, few, fused, ternary, expect):
-    assert bench.launches_per_step(M, few, fused, ternary) == expect
+def test_launches_per_step(M, fused, nvfp4, expect):
+    assert bench.launches_per_step(M, fused, nvfp4) == expect
 
 
 def test_metric_names():

@@ -61,7 +61,7 @@ def test_pack_weight_ternary_bit_exact(N, K, G):
     assert np.array_equal(qw2.cpu().numpy(), oracle.pack_ternary(codes)), "packed codes differ from the oracle"
 
 
-@pytest.mark.parametrize("M", [1, 9, 16, 40, 64, 200])
+@pytest.mark.parametrize("M", [1, 9, 16, 40, 64, 200, 300])
 @pytest.mark.parametrize("N,K,G,bias", [(264, 512, 64, True), (136, 1024, 128, False), (264, 2048, 2048, True)])
 def test_w158a4_linear_matches_oracle(M, N, K, G, bias):
     rng = np.random.default_rng(7 * M + K + G)
