@@ -13,7 +13,9 @@
 // Those rare elements (and groups whose scale is subnormal, where 1/s may overflow) take the
 // IEEE division __fdiv_rn.  rint(y) itself comes from one fp32 add of 1.5*2^23 + 8: the sum is
 // an integer 0x4B400008 + rint(y) whose low nibble is the offset code q + 8.
+#include <climits>
 #include <cstdint>
+#include <type_traits>
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
 
@@ -197,6 +199,38 @@ __device__ __forceinline__ void store32(uint8_t* out, int64_t row, int64_t col, 
   }
 }
 
+// The rest of one thread's 32 elements once they are in registers (as the bf16 value the linear
+// layer receives): the group amax over the group's L adjacent lanes, the scale, the codes and their
+// store, and the group's scale (and, for the operand image, its code-sum correction) from the
+// group's first lane.  Every lane of the warp takes part (the shuffles); `valid` lanes hold data.
+template <int L, bool kOperand, bool kScaleT>
+__device__ __forceinline__ void finish_chunk(const float (&v)[32], bool valid, int64_t row, int64_t col, int64_t M,
+                                             int64_t K, uint8_t* __restrict__ out, float* __restrict__ scales,
+                                             float* __restrict__ corr) {
+  float a = amax32(v);
+#pragma unroll
+  for (int o = 1; o < L; o <<= 1) a = fmaxf(a, __shfl_xor_sync(0xFFFFFFFFu, a, o));
+  const float s = __fdiv_rn(a, 7.0f);
+  uint32_t pk[4] = {0x88888888u, 0x88888888u, 0x88888888u, 0x88888888u};  // sums to 0 past the end
+  if (valid) {
+    quantize32(v, s, pk);
+    store32<kOperand>(out, row, col, K, pk);
+  }
+  int cs = 0;
+  if constexpr (kOperand) {  // the group's code sum, over its L lanes
+    cs = valid ? nib32_sum(make_uint4(pk[0], pk[1], pk[2], pk[3])) : 0;
+#pragma unroll
+    for (int o = 1; o < L; o <<= 1) cs += __shfl_xor_sync(0xFFFFFFFFu, cs, o);
+  }
+  if (valid && (threadIdx.x & (L - 1)) == 0) {
+    const int64_t ng = K / (32 * L);
+    const int64_t g = col / (32 * L);
+    if constexpr (kScaleT) scales[g * M + row] = s;
+    else scales[row * ng + g] = s;
+    if constexpr (kOperand) corr[row * ng + g] = (float)(8 * cs) * kOperandUnit;
+  }
+}
+
 // G = 32 * L (L = 2 or 4): each thread quantises 32 consecutive elements; the L threads of a
 // group are adjacent lanes and reduce amax with xor-shuffles.
 template <typename In, int L, bool kOperand, bool kScaleT, int kOp = kOpNone>
@@ -210,7 +244,6 @@ __global__ void __launch_bounds__(256) quantize_groups_kernel(const In* __restri
   pdl_wait();
   const int64_t chunks_per_row = K / 32;
   const int64_t total = M * chunks_per_row;
-  const int64_t ng = K / (32 * L);
   for (int64_t c = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; c - (threadIdx.x & 31) < total;
        c += (int64_t)gridDim.x * blockDim.x) {
     const bool valid = c < total;
@@ -224,15 +257,152 @@ __global__ void __launch_bounds__(256) quantize_groups_kernel(const In* __restri
 #pragma unroll
       for (int i = 0; i < 32; ++i) v[i] = 0.0f;
     }
-    float a = amax32(v);
+    finish_chunk<L, kOperand, kScaleT>(v, valid, row, col, M, K, out, scales, corr);
+  }
+}
+
+// The same quantiser for bf16 activations with many rows, the input staged through shared memory
+// by TMA: tiles of 64 rows x 256 elements (32 KB) in a 3-slot ring per CTA, two CTAs per SM, so
+// that the bytes in flight are set by the rings (up to 192 KB per SM), not by registers.  Warp 16
+// (one thread) issues the tile loads; warps 0-15 take a tile's 512 chunks of 32 elements, one per
+// thread (chunk j: row j / 8 of the tile, elements 32 (j % 8) ..), and release the slot.  A chunk
+// is read from shared memory twice (the group amax, then the codes) so that few values live in
+// registers.  The codes follow the same reciprocal rule as quantize32 with the fp32 steps in
+// packed pairs; the elements near a tie are then redone with the IEEE quotient one by one.  Rows past M and columns past
+// K arrive as zeros and are skipped.  Tiles are ordered column-fastest.
+constexpr int kQtRows = 64, kQtCols = 256, kQtSlots = 3, kQtConsumerWarps = 16;
+constexpr int kQtThreads = 32 * (kQtConsumerWarps + 1);
+constexpr uint32_t kQtSlotBytes = kQtRows * kQtCols * 2;
+constexpr uint32_t kQtSmemBytes = kQtSlots * kQtSlotBytes + 2 * kQtSlots * 8 + 16;
+static_assert(32 * kQtConsumerWarps * 32 == kQtRows * kQtCols, "one chunk of 32 elements per consumer thread");
+
+// 8 bf16 values (one 16-byte unit) -> their offset codes q + 8 as the 8 nibbles of one word in
+// packed order (element 2j in the low nibble of byte j), with r = RN(1/s).  `ties` gets bit
+// 8j + 7 for even element 2j and bit 8j + 6 for odd element 2j + 1 when that element's y may lie
+// within 2^-19 of a half-integer (its nibble then needs the IEEE quotient).  The test is
+// d^2 - c >= 0 with d = y - rint(y) and c just below (1/2 - 2^-19)^2, in one fused operation:
+// every element the reciprocal rule may get wrong is flagged, and a few more.
+constexpr float kTieSq = 0x1.ffffp-3f;  // 2^-2 - 2^-19: (1/2 - 2^-19)^2 = 2^-2 - 2^-19 + 2^-38, rounded down
+
+__device__ __forceinline__ uint32_t codes8_offset(uint4 u, float r, uint32_t& ties) {
+  const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+  const float2 r2 = make_float2(r, r), m2 = make_float2(kRintMagic, kRintMagic);
+  const float2 nm2 = make_float2(-kRintMagic, -kRintMagic), neg1 = make_float2(-1.0f, -1.0f);
+  const float2 nc2 = make_float2(-kTieSq, -kTieSq);
+  uint32_t t[8], v[8];
+#pragma unroll
+  for (int e = 0; e < 4; ++e) {
+    const float2 x = make_float2(__uint_as_float(w[e] << 16), __uint_as_float(w[e] & 0xFFFF0000u));
+    const float2 y = __fmul2_rn(x, r2);
+    const float2 tt = __fadd2_rn(y, m2);         // 1.5 * 2^23 + 8 + rint(y): low byte q + 8
+    const float2 rt = __fadd2_rn(tt, nm2);       // rint(y), exact
+    const float2 d = __ffma2_rn(rt, neg1, y);    // y - rint(y), exact
+    const float2 g = __ffma2_rn(d, d, nc2);      // d^2 - c: sign clear for a (possible) near-tie
+    t[2 * e] = __float_as_uint(tt.x);
+    t[2 * e + 1] = __float_as_uint(tt.y);
+    v[2 * e] = __float_as_uint(g.x);
+    v[2 * e + 1] = __float_as_uint(g.y);
+  }
+  // low bytes of the even elements to bytes 0-3, of the odd elements likewise, then nibbles
+  const uint32_t ev = __byte_perm(__byte_perm(t[0], t[2], 0x0040), __byte_perm(t[4], t[6], 0x0040), 0x5410);
+  const uint32_t od = __byte_perm(__byte_perm(t[1], t[3], 0x0040), __byte_perm(t[5], t[7], 0x0040), 0x5410);
+  // top bytes (signs) of the tie tests likewise
+  const uint32_t tv = __byte_perm(__byte_perm(v[0], v[2], 0x0073), __byte_perm(v[4], v[6], 0x0073), 0x5410);
+  const uint32_t to = __byte_perm(__byte_perm(v[1], v[3], 0x0073), __byte_perm(v[5], v[7], 0x0073), 0x5410);
+  ties = (~tv & 0x80808080u) | ((~to & 0x80808080u) >> 1);
+  return ev | (od << 4);
+}
+
+template <int L, bool kOperand>
+__global__ void __launch_bounds__(kQtThreads, 2) quantize_tiles_kernel(const __grid_constant__ CUtensorMap tmX,
+                                                                       int64_t M, int64_t K,
+                                                                       uint8_t* __restrict__ out,
+                                                                       float* __restrict__ scales,
+                                                                       float* __restrict__ corr, uint32_t* status) {
+  extern __shared__ __align__(1024) uint8_t smem[];
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + kQtSlots * kQtSlotBytes);
+  uint64_t* empty = full + kQtSlots;
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(empty + kQtSlots);
+  const uint32_t warp = warp_id(), lane = lane_id();
+  if (threadIdx.x == 0) {
+    for (int i = 0; i < kQtSlots; ++i) {
+      mbar_init(&full[i], 1);
+      mbar_init(&empty[i], kQtConsumerWarps);
+    }
+    *abort_flag = 0;
+    fence_mbar_init();
+  }
+  __syncthreads();
+  pdl_launch_dependents();  // as in quantize_groups_kernel
+  pdl_wait();
+  const int64_t col_tiles = (K + kQtCols - 1) / kQtCols;
+  const int64_t tiles = (M + kQtRows - 1) / kQtRows * col_tiles;
+  if (warp == kQtConsumerWarps) {  // TMA producer
+    if (lane == 0) {
+      tma_prefetch_desc(&tmX);
+      uint32_t it = 0;
+      for (int64_t t = blockIdx.x; t < tiles; t += gridDim.x, ++it) {
+        const uint32_t slot = it % kQtSlots;
+        if (!mbar_wait(&empty[slot], ((it / kQtSlots) & 1u) ^ 1u, abort_flag, status)) break;
+        mbar_arrive_expect_tx(&full[slot], kQtSlotBytes);
+        tma_load_2d(smem + slot * kQtSlotBytes, &tmX, &full[slot], (int)((t % col_tiles) * kQtCols),
+                    (int)((t / col_tiles) * kQtRows));
+      }
+      // After an abort, let the loads already issued land before the CTA's shared memory goes.
+      if (*abort_flag) {
+        int dummy = 0;
+        const uint32_t issued = it;
+        for (uint32_t k = issued > (uint32_t)kQtSlots ? issued - kQtSlots : 0; k < issued; ++k)
+          (void)mbar_wait(&full[k % kQtSlots], (k / kQtSlots) & 1u, &dummy, nullptr);
+      }
+    }
+    return;
+  }
+  const int j = (int)threadIdx.x;  // this thread's chunk of every tile
+  uint32_t it = 0;
+  for (int64_t t = blockIdx.x; t < tiles; t += gridDim.x, ++it) {
+    const uint32_t slot = it % kQtSlots;
+    if (!__all_sync(0xFFFFFFFFu, mbar_wait(&full[slot], (it / kQtSlots) & 1u, abort_flag, status))) break;
+    const int64_t row = (t / col_tiles) * kQtRows + (j >> 3), col = (t % col_tiles) * kQtCols + 32 * (j & 7);
+    const bool valid = row < M && col < K;
+    const uint4* src = reinterpret_cast<const uint4*>(smem + slot * kQtSlotBytes + (j >> 3) * (kQtCols * 2) +
+                                                      (j & 7) * 64);
+    // amax over bf16 pairs (|x| by clearing the signs; finite inputs), then as fp32
+    __nv_bfloat162 m2 = __floats2bfloat162_rn(0.0f, 0.0f);  // zeros past the ends
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      const uint4 u = src[q];
+      const uint32_t w[4] = {u.x & 0x7FFF7FFFu, u.y & 0x7FFF7FFFu, u.z & 0x7FFF7FFFu, u.w & 0x7FFF7FFFu};
+#pragma unroll
+      for (int e = 0; e < 4; ++e) m2 = __hmax2(m2, *reinterpret_cast<const __nv_bfloat162*>(&w[e]));
+    }
+    float a = fmaxf(__low2float(m2), __high2float(m2));
 #pragma unroll
     for (int o = 1; o < L; o <<= 1) a = fmaxf(a, __shfl_xor_sync(0xFFFFFFFFu, a, o));
     const float s = __fdiv_rn(a, 7.0f);
-    uint32_t pk[4] = {0x88888888u, 0x88888888u, 0x88888888u, 0x88888888u};  // sums to 0 past the end
-    if (valid) {
-      quantize32(v, s, pk);
-      store32<kOperand>(out, row, col, K, pk);
+    uint32_t pk[4] = {0u, 0u, 0u, 0u};  // an all-zero group (s = 0) has zero codes
+    if (valid && s != 0.0f) {
+      const bool normal = s >= 0x1p-126f;  // 1/s representable: the reciprocal rule applies
+      const float r = __frcp_rn(s);
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        uint32_t ties = 0xC0C0C0C0u, word = 0;  // a subnormal scale: every element by division
+        if (normal) word = codes8_offset(src[q], r, ties);
+        // the elements near a tie (all of them for a subnormal scale) take the IEEE quotient
+        while (ties != 0) {
+          const int bit = __ffs(ties) - 1;  // 8j + 7: element 2j, 8j + 6: element 2j + 1
+          ties &= ties - 1;
+          const int e = 2 * (bit >> 3) + ((bit & 7) == 6 ? 1 : 0);
+          const uint16_t b = reinterpret_cast<const uint16_t*>(src + q)[e];
+          const uint32_t c = code_offset(__uint_as_float((uint32_t)b << 16), s, r, true);
+          word = (word & ~(0xFu << (4 * e))) | (c << (4 * e));
+        }
+        pk[q] = word ^ 0x88888888u;
+      }
     }
+    __syncwarp();
+    if (lane == 0) mbar_arrive(&empty[slot]);  // the slot's bytes are no longer read
+    if (valid) store32<kOperand>(out, row, col, K, pk);
     int cs = 0;
     if constexpr (kOperand) {  // the group's code sum, over its L lanes
       cs = valid ? nib32_sum(make_uint4(pk[0], pk[1], pk[2], pk[3])) : 0;
@@ -240,9 +410,8 @@ __global__ void __launch_bounds__(256) quantize_groups_kernel(const In* __restri
       for (int o = 1; o < L; o <<= 1) cs += __shfl_xor_sync(0xFFFFFFFFu, cs, o);
     }
     if (valid && (threadIdx.x & (L - 1)) == 0) {
-      const int64_t g = col / (32 * L);
-      if constexpr (kScaleT) scales[g * M + row] = s;
-      else scales[row * ng + g] = s;
+      const int64_t ng = K / (32 * L), g = col / (32 * L);
+      scales[row * ng + g] = s;
       if constexpr (kOperand) corr[row * ng + g] = (float)(8 * cs) * kOperandUnit;
     }
   }
@@ -374,6 +543,38 @@ int grid_for(int64_t work_items, int threads, int sms) {
   return static_cast<int>(blocks);
 }
 
+// bf16 activations (with no neighbour operation) take the TMA-staged kernel when every CTA gets
+// at least two tiles (each CTA's first tile waits for its whole copy; smaller inputs are better
+// served by the register kernel's many small loads).
+constexpr int64_t kQtMinRows = 64;
+constexpr int kQtMinTilesPerSm = 4;
+
+template <int L, bool kOperand>
+cudaError_t launch_quantize_tiles(const __nv_bfloat16* x, int64_t M, int64_t K, int64_t ldx, uint8_t* out,
+                                  float* scales, float* corr, cudaStream_t stream, int sms) {
+  // The input as a 2-D tensor [M, K] of row pitch ldx (the callers check that the base and the
+  // pitch are 16-byte aligned, as the tensor map needs); boxes of 256 x 64, zeros past the ends.
+  CUtensorMap tm;
+  if (!encode_2d(&tm, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, x, (uint64_t)K, (uint64_t)M, (uint64_t)ldx * 2, kQtCols,
+                 kQtRows, CU_TENSOR_MAP_SWIZZLE_NONE))
+    return cudaErrorInvalidValue;
+  static PerDevice<bool> smem_attr;  // once per device and instantiation
+  bool attr_ok = false;
+  cudaError_t ae = smem_attr.get(
+      [](bool& v) {
+        v = true;
+        return cudaFuncSetAttribute(quantize_tiles_kernel<L, kOperand>,
+                                    cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kQtSmemBytes);
+      },
+      attr_ok);
+  if (ae != cudaSuccess) return ae;
+  const int64_t tiles = (M + kQtRows - 1) / kQtRows * ((K + kQtCols - 1) / kQtCols);
+  const int64_t cap = 2 * static_cast<int64_t>(sms);  // two CTAs per SM
+  const int grid = static_cast<int>(tiles < cap ? tiles : cap);
+  return launch_pdl(quantize_tiles_kernel<L, kOperand>, dim3(grid), dim3(kQtThreads), kQtSmemBytes, stream, tm, M, K,
+                    out, scales, corr, device_status_word());
+}
+
 template <typename In, bool kOperand, bool kScaleT, int kOp = kOpNone>
 cudaError_t launch_quantize(const In* x, int64_t M, int64_t K, int64_t ldx, int G, uint8_t* out, float* scales,
                             float* corr, cudaStream_t stream, int sms, const OpArgs& op = OpArgs()) {
@@ -382,6 +583,12 @@ cudaError_t launch_quantize(const In* x, int64_t M, int64_t K, int64_t ldx, int 
     int blocks = static_cast<int>(M < static_cast<int64_t>(sms) * 16 ? M : static_cast<int64_t>(sms) * 16);
     return launch_pdl(quantize_rows_kernel<In, kOperand, kScaleT, kOp>, dim3(blocks), dim3(128), 0, stream, x, M, K,
                       ldx, out, scales, corr, op);
+  }
+  if constexpr (std::is_same<In, __nv_bfloat16>::value && !kScaleT && kOp == kOpNone) {
+    const int64_t tiles = (M + kQtRows - 1) / kQtRows * ((K + kQtCols - 1) / kQtCols);
+    if (M >= kQtMinRows && M <= INT32_MAX && tiles >= kQtMinTilesPerSm * static_cast<int64_t>(sms))
+      return G == 64 ? launch_quantize_tiles<2, kOperand>(x, M, K, ldx, out, scales, corr, stream, sms)
+                     : launch_quantize_tiles<4, kOperand>(x, M, K, ldx, out, scales, corr, stream, sms);
   }
   const int grid = grid_for(M * (K / 32), 256, sms);
   if (G == 64)

@@ -49,3 +49,21 @@ def test_reciprocal_shortcut_matches_the_exact_quotient_for_every_bf16_pair():
     assert pairs > 1_000_000_000
     assert mismatches == {k: 0 for k in mismatches}, mismatches
     assert fallbacks < pairs // 1000  # the exact division stays rare
+
+
+def test_tiled_kernel_tie_test_covers_the_band():
+    """The TMA-staged quantiser flags a near-tie by fma(d, d, -c) >= 0 with d = y - rint(y), whose
+    sign is that of the exact d^2 - c.  Every element of the band above (|d| > 1/2 - 2^-19) must
+    be flagged, so c must lie below (1/2 - 2^-19)^2; and c close to 1/4 keeps the extra
+    fallbacks rare.  The constant is read from the kernel source."""
+    import os
+    import re
+    from fractions import Fraction
+    src = open(os.path.join(os.path.dirname(os.path.dirname(os.path.abspath(__file__))),
+                            "paper_2609_33601_gb300", "csrc", "quantize.cu")).read()
+    lit = re.search(r"constexpr float kTieSq = (0x[0-9a-fA-F.]+p-?\d+)f;", src).group(1)
+    c = Fraction(float.fromhex(lit))
+    assert float(np.float32(float(c))) == float(c), "the constant is an fp32 value"
+    band = Fraction(1, 2) - Fraction(1, 2 ** 19)
+    assert c < band * band
+    assert c > Fraction(1, 4) - Fraction(1, 2 ** 18)

@@ -74,7 +74,12 @@ def act_bits(M, K, seed, special=True, extreme=True):
 
 @pytest.mark.parametrize("M,K,G,pad", [(300, 512, 64, 0), (300, 512, 128, 0), (300, 512, 512, 0),
                                        (9, 15360, 64, 0), (7, 4096, 4096, 0), (1, 128, 128, 0),
-                                       (37, 256, 64, 72)])
+                                       (37, 256, 64, 72), (63, 384, 64, 0),
+                                       (64, 15360, 64, 0), (130, 1152, 64, 0), (130, 384, 128, 40),
+                                       (65, 4096, 128, 8), (200, 128, 64, 0),
+                                       # at least 4 tiles of 64 x 256 per SM: the TMA-staged kernel,
+                                       # with a ragged last row tile and a half-empty last column tile
+                                       (4100, 2432, 64, 40), (4100, 2432, 128, 0)])
 def test_quantize_act_bit_exact(M, K, G, pad):
     x = act_bits(M, K, seed=M + K + G)
     ref_codes, ref_s = oracle.quantize_bf16(x, G)
