@@ -94,9 +94,9 @@ FP8_PER_BF16 = 2.0  # nominal dense FP8 / BF16 tensor-core ratio on GB300 (4.5 /
 # capture was taken on (kernel_hash); once the code changes the figure no longer applies and the
 # bench reports null until a new capture is recorded here.
 KERNEL_TRAFFIC: dict = {
-    ("flux_qkv", "f01c650c0bc1bb2c"): 54.967552e6 + 143.880448e6,
-    ("dllm", "f01c650c0bc1bb2c"): 31.267584e6 + 0.160256e6,
-    ("dllm/ternary", "f01c650c0bc1bb2c"): 18.689792e6 + 0.122368e6,
+    ("flux_qkv", "17f2efcfd35bda35"): 55.028224e6 + 144.056576e6,
+    ("dllm", "17f2efcfd35bda35"): 31.280896e6 + 0.182784e6,
+    ("dllm/ternary", "17f2efcfd35bda35"): 18.673152e6 + 0.105216e6,
 }
 
 

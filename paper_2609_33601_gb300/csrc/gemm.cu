@@ -10,14 +10,13 @@
 // so the fp32 TMEM accumulator holds acc[m,n,g] * 2^-18 exactly.
 //
 // Persistent kernel on CTA pairs (clusters of two SMs, tcgen05 cta_group::2).  A pair owns a
-// 256 x kBN output tile at a time (kBN = 256): CTA r of the pair holds A rows 128r..128r+127 and B
-// rows (output columns) r*kBN/2.. of the tile, and the even CTA issues 256 x kBN x 32 MMAs that
-// read both CTAs' shared memory and write 128 rows x kBN columns into each CTA's TMEM (two
-// accumulators fill its 512 columns).  Per SM this halves the B bytes the tensor core reads and
-// the B nibbles each SM unpacks, against a one-SM tile.  The tile width is a parameter of the
-// layout (Tile): a 128-column tile with four accumulators was built and measured for the group
-// modes, and ran at half this tile's rate -- the per-group rescale costs about the same time per
-// group at either width, so the wider tile does twice the work per rescale.  K stages of 128;
+// 256 x kBN output tile at a time: CTA r of the pair holds A rows 128r..128r+127 and B rows
+// (output columns) r*kBN/2.. of the tile, and the even CTA issues 256 x kBN x 32 MMAs that read
+// both CTAs' shared memory and write 128 rows x kBN columns into each CTA's TMEM (two
+// accumulators of 256 columns fill its 512).  Per SM this halves the B bytes the tensor core
+// reads and the B nibbles each SM unpacks, against a one-SM tile.  The tile width is a parameter
+// of the layout (Tile): 256 normally; with several groups, 224 or 128 when their tile count
+// leaves the pairs' last round of tiles fuller (grouped_tile_width).  K stages of 128;
 // 16 warps per CTA:
 //   warp 0      A producer: one 2-D TMA per two K stages (256 rows x 128 bytes of the
 //               pre-swizzled A-operand image, 32 KB) -> A ring, completing on the even CTA's
@@ -81,7 +80,7 @@ struct Tile {
   static constexpr int kBNHalf = kBN / 2;                    // B rows per CTA
   static constexpr int kAccBufs = kTmemCols / kBN;           // TMEM accumulators (2 or 4)
   static constexpr int kDrainCols = kBN / 2;                 // accumulator columns per drain warp
-  static constexpr int kSlots = kBN == 256 ? 3 : 4;          // operand ring slots (what fits in shared memory)
+  static constexpr int kSlots = kBN > 128 ? 3 : 4;           // operand ring slots (what fits in shared memory)
   static constexpr uint32_t kOpBBytes = kBNHalf * kBK;       // B bytes per K stage per CTA
   static constexpr uint32_t kSlotBBytes = kStagesPerSlot * kOpBBytes;
   static constexpr int kChunksPerThread = kBNHalf * (kBK / 2) / 16 / kUnpackGroupThreads;  // packed 16-byte chunks
@@ -94,7 +93,8 @@ struct Tile {
   static constexpr uint32_t kNumBars = 2 * kSlots + 2 * kAccBufs + 1 + 2 * kScSlots;
   static constexpr uint32_t kOffMisc = kOffBar + kNumBars * 8;
   static constexpr uint32_t kSmemBytes = kOffMisc + 16;
-  static_assert(kBN == 128 || kBN == 256, "tile widths");
+  static_assert(kBN % 32 == 0 && kBN >= 128 && kBN <= 256, "tile widths (the MMA's N, a multiple of 16 per CTA)");
+  static_assert(kDrainCols % 16 == 0, "the drain reads 16 columns at a time");
   static_assert(kChunksPerThread * kUnpackGroupThreads * 16 == kBNHalf * (kBK / 2), "unpack covers the B half");
   static_assert(kOffBar % 8 == 0 && kOffMisc % 8 == 0, "mbarriers need 8-byte alignment");
   static_assert(kOffSc % 128 == 0 && kScSlotBytes % 128 == 0 && kScSwBytes % 128 == 0,
@@ -204,11 +204,10 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
   return *reinterpret_cast<const uint32_t*>(&v);
 }
 
-// Linear path, 256-column tiles, several groups (sign-magnitude weight codes): warp w (drain index
-// d = w - 8) owns one row per thread -- TMEM
-// lane 32*(w%4) + lane -- and columns 128*(d/4).. of each accumulator, read 16 at a time with the
-// 32x32b shape: two loads in flight, the next 16 columns arriving while the current ones are
-// scaled.  The running sums are float2 pairs, the operand form of the packed fp32 instructions,
+// Linear path, several groups (sign-magnitude weight codes): warp w (drain index d = w - 8) owns
+// one row per thread -- TMEM lane 32*(w%4) + lane -- and columns D*(d/4).. of each accumulator
+// (D = kBN/2: 128 for the 256-column tile), read 16 at a time with the 32x32b shape: two loads in
+// flight, the next 16 columns arriving while the current ones are scaled.  The running sums are float2 pairs, the operand form of the packed fp32 instructions,
 // so y += (acc * s_w) * (s_a * 2^18) costs one FMUL2 and one FFMA2 per two outputs.  The weight
 // scales are the same for every lane (broadcast LDS.128 from the scale ring); the activation
 // scale is one value per thread and group.  (Per group the lanes of a warp fill 16 KB of registers
@@ -217,7 +216,8 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
 template <class T, bool kOffset>
 __device__ __forceinline__ void drain_linear_rows(const Args& args, const Pair& pr, uint32_t tmem_base,
                                                   const Bars& b, uint8_t* sSc, volatile int* abort_flag) {
-  static_assert(T::kBN == 256, "drain layout for 256-column tiles");
+  constexpr int D = T::kDrainCols, kBatches = D / 16;
+  static_assert(kBatches >= 2, "the load pipeline needs two batches");
   const uint32_t warp = warp_id(), lane = lane_id();
   const int M = args.M, N = args.N, groups = args.groups;
   const uint32_t quarter = warp & 3u, half = (warp - kDrainWarp0) >> 2;
@@ -228,11 +228,11 @@ __device__ __forceinline__ void drain_linear_rows(const Args& args, const Pair& 
   for (int tile = pr.cluster; ok && tile < args.num_tiles; tile += pr.num_clusters) {
     const int mt2 = tile % args.num_m2, nt = tile / args.num_m2;
     const int row = mt2 * kPairM + (int)pr.rank * kBM + (int)trow;
-    const int col0 = nt * T::kBN + half * 128;
+    const int col0 = nt * T::kBN + half * D;
     const bool row_ok = row < M;
-    float2 y[64];
+    float2 y[D / 2];
 #pragma unroll
-    for (int i = 0; i < 64; ++i) y[i] = make_float2(0.0f, 0.0f);
+    for (int i = 0; i < D / 2; ++i) y[i] = make_float2(0.0f, 0.0f);
     for (int g = 0; g < groups; ++g) {
       const uint32_t ab = acc_buf<T>(chunk_it);
       const int gi = g % kScGroups;
@@ -242,7 +242,7 @@ __device__ __forceinline__ void drain_linear_rows(const Args& args, const Pair& 
         if (!ok) break;
       }
       const uint8_t* slot = sSc + sslot * T::kScSlotBytes;
-      const float4* sw4 = reinterpret_cast<const float4*>(reinterpret_cast<const float*>(slot) + gi * T::kBN + half * 128);
+      const float4* sw4 = reinterpret_cast<const float4*>(reinterpret_cast<const float*>(slot) + gi * T::kBN + half * D);
       float sa;
       if (args.sa_tma)
         sa = reinterpret_cast<const float*>(slot + T::kScSwBytes)[trow * kScGroups + gi];
@@ -258,7 +258,7 @@ __device__ __forceinline__ void drain_linear_rows(const Args& args, const Pair& 
       }
       next_full = false;
       tc_fence_after();
-      const uint32_t taddr = tmem_base + ((quarter * 32u) << 16) + ab * T::kBN + half * 128;
+      const uint32_t taddr = tmem_base + ((quarter * 32u) << 16) + ab * T::kBN + half * D;
       auto release = [&]() {  // every column of this accumulator is in registers: hand it back
         tc_fence_before();
         __syncwarp();
@@ -290,24 +290,23 @@ __device__ __forceinline__ void drain_linear_rows(const Args& args, const Pair& 
         tmem_ld16(taddr, ra);
         tmem_ld_wait();
 #pragma unroll
-        for (int c = 0; c < 128; c += 32) {
-          tmem_ld16(taddr + c + 16, rb);
-          scale16(c, ra);
-          tmem_ld_wait();
-          if (c == 96) release();
-          if (c < 96) tmem_ld16(taddr + c + 32, ra);
-          if (c == 64)  // the next accumulator: seen complete yet?
+        for (int bi = 0; bi < kBatches; ++bi) {  // batch bi is in ra (even) or rb (odd)
+          uint32_t(&cur)[16] = (bi & 1) ? rb : ra;
+          uint32_t(&nxt)[16] = (bi & 1) ? ra : rb;
+          if (bi + 1 < kBatches) tmem_ld16(taddr + 16 * (bi + 1), nxt);
+          if (bi == kBatches / 2 + 1)  // the next accumulator: seen complete yet?
             next_full = mbar_test_wait(&b.acc_full[acc_buf<T>(chunk_it + 1)], acc_parity<T>(chunk_it + 1));
-          scale16(c + 16, rb);
-          if (c < 96) tmem_ld_wait();
+          scale16(16 * bi, cur);
+          if (bi + 1 < kBatches) tmem_ld_wait();
+          if (bi + 2 == kBatches) release();  // the last batch is in registers
         }
       } else {  // some |s_a| > 2^110: apply 2^18 to the exact partials first so nothing overflows
 #pragma unroll
-        for (int c = 0; c < 128; c += 16) {
+        for (int c = 0; c < D; c += 16) {
           uint32_t r[16];
           tmem_ld16(taddr + c, r);
           tmem_ld_wait();
-          if (c == 112) release();
+          if (c == D - 16) release();
 #pragma unroll
           for (int q = 0; q < 4; ++q) {
             const float4 w = sw4[(c >> 2) + q];
@@ -328,10 +327,10 @@ __device__ __forceinline__ void drain_linear_rows(const Args& args, const Pair& 
       ++chunk_it;
     }
     if (!ok) break;
-    // + bias, round to bf16, store: each thread writes its row's 128 columns, 8 (16 bytes) at a time
+    // + bias, round to bf16, store: each thread writes its row's D columns, 8 (16 bytes) at a time
     if (row_ok) {
 #pragma unroll
-      for (int c = 0; c < 128; c += 8) {
+      for (int c = 0; c < D; c += 8) {
         const int col = col0 + c;
         if (col < N) {  // N % 8 == 0: a chunk is wholly inside or outside
           float4 b0 = make_float4(0.f, 0.f, 0.f, 0.f), b1 = b0;
@@ -854,9 +853,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
   // MMA (warps 0-3) 32, unpack (warps 4-7) 96, drain (warps 8-15, the running sums) 192.
   if (warp >= kDrainWarp0) {
     asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;\n" ::"n"(kRegsDrain) : "memory");
-    if (kExport)
+    if constexpr (kExport)
       drain_export<T, kOffset>(args, pr, tmem_base, b, abort_flag);
-    else if (kOffset)
+    else if constexpr (kOffset)
       drain_linear_quads<T, kOffset>(args, pr, tmem_base, b, sSc, abort_flag);
     else
       drain_linear_rows<T, kOffset>(args, pr, tmem_base, b, sSc, abort_flag);
@@ -1004,6 +1003,31 @@ bool encode_2d(CUtensorMap* map, CUtensorMapDataType dtype, const void* base, ui
             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// Tile width of the grouped (sign-magnitude, several groups) linear path.  Every pair of CTAs
+// takes ceil(tiles / pairs) tiles at most, each costing time in proportion to its width, so the
+// width with the smallest ceil(tiles / pairs) * width finishes first; a narrower tile is taken
+// only when it wins by 3 % (it re-reads the A operand more often).  E.g. 1024 x 4096 -> 12288:
+// 192 tiles of 256 on 76 pairs (3 rounds, the last half full) against 220 of 224 (3 rounds, nearly
+// full); 4096 x 4608 -> 1152: 80 tiles of 256 (2 rounds, the second with 4 tiles) against 144
+// of 128 (2 full rounds).
+int grouped_tile_width(const GemmProblem& p, int sms) {
+  const int64_t num_m2 = (p.M + kPairM - 1) / kPairM, pairs = sms / 2 > 0 ? sms / 2 : 1;
+  auto cost = [&](int64_t bn) {
+    const int64_t tiles = num_m2 * ((p.N + bn - 1) / bn);
+    return ((tiles + pairs - 1) / pairs) * bn;
+  };
+  int best = 256;
+  int64_t c_best = cost(256);
+  for (int bn : {224, 128}) {
+    const int64_t c = cost(bn);
+    if (c * 100 < c_best * 97) {
+      best = bn;
+      c_best = c;
+    }
+  }
+  return best;
+}
+
 cudaError_t launch_w4a4_gemm(const GemmProblem& p, cudaStream_t stream, int sms) {
   if (p.M == 0 || p.N == 0) return cudaSuccess;
   // One group: offset-code weights (see w4a4_gemm_kernel), exact while the whole K run fits the
@@ -1014,7 +1038,17 @@ cudaError_t launch_w4a4_gemm(const GemmProblem& p, cudaStream_t stream, int sms)
   const bool offset = p.G == p.K && p.K <= kOffsetMaxRun && !p.ternary;
   if (p.partials != nullptr)
     return offset ? launch_impl<true, true, 256>(p, stream, sms) : launch_impl<true, false, 256>(p, stream, sms);
-  return offset ? launch_impl<false, true, 256>(p, stream, sms) : launch_impl<false, false, 256>(p, stream, sms);
+  // One group: 256-column tiles always (their 16x256b drain; the row drain on narrower tiles
+  // measured slower there: 1024 x 4096 -> 12288 with G = K, 1615 -> 1557 TFLOP/s at width 224).
+  if (offset) return launch_impl<false, true, 256>(p, stream, sms);
+  switch (grouped_tile_width(p, sms)) {
+    case 224:
+      return launch_impl<false, false, 224>(p, stream, sms);
+    case 128:
+      return launch_impl<false, false, 128>(p, stream, sms);
+    default:
+      return launch_impl<false, false, 256>(p, stream, sms);
+  }
 }
 
 }  // namespace jq

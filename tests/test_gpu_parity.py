@@ -200,7 +200,12 @@ def run_linear(ref: Reference, x_bits, fused: bool):
                                           # holds one stage): DiT-XL/2's hidden size 1152 = 9 x 128
                                           (300, 264, 384, 64, True), (300, 264, 384, 128, False),
                                           (300, 264, 384, 384, True), (257, 520, 1152, 128, True),
-                                          (257, 136, 1152, 1152, False), (40, 264, 1152, 128, True)])
+                                          (257, 136, 1152, 1152, False), (40, 264, 1152, 128, True),
+                                          # the GEMM's tile width follows the tile count (128 for
+                                          # the small shapes above); 224 here, ragged in M and N
+                                          (1000, 12200, 256, 64, False), (1000, 12200, 1152, 128, True),
+                                          # and 256 (several rounds of tiles, ragged in M and N)
+                                          (4500, 3000, 512, 64, True)])
 def test_linear_matches_oracle(M, N, K, G, bias):
     w = wl.make("custom", seed=11 + M, M=M, K=K, N=N, G=G, bias=bias)
     x = act_bits(M, K, seed=3 + M, extreme=False) if M >= 8 else w.x_bits
