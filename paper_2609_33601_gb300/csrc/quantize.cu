@@ -28,7 +28,6 @@ namespace jq {
 namespace {
 
 constexpr float kRintMagic = 12582920.0f;  // 1.5 * 2^23 + 8
-constexpr float kHalfGuard = 0.5f - 0x1p-19f;
 
 // Loads 32 consecutive values of a row as fp32.
 __device__ __forceinline__ void load32(const __nv_bfloat16* p, float (&x)[32]) {
@@ -63,18 +62,51 @@ __device__ __forceinline__ float amax32(const float (&x)[32]) {
   return m;
 }
 
-// One code as its offset nibble u = q + 8 in [0, 15].
-__device__ __forceinline__ uint32_t code_offset(float x, float s, float r, bool exact_only) {
-  const float y = x * r;
-  const float t = y + kRintMagic;
-  const float d = y - (t - kRintMagic);
-  if (exact_only || fabsf(d) > kHalfGuard) {
-    float q = rintf(__fdiv_rn(x, s));
-    q = fminf(fmaxf(q, -8.0f), 7.0f);
-    return static_cast<uint32_t>(static_cast<int>(q) + 8);
-  }
-  return __float_as_uint(t) & 0xFu;
+// One code by the rule itself, as its offset nibble q + 8 in [0, 15]: the IEEE quotient, rint,
+// the clamp (the elements the reciprocal rule cannot settle, and subnormal scales).
+__device__ __forceinline__ uint32_t code_exact(float x, float s) {
+  const float q = fminf(fmaxf(rintf(__fdiv_rn(x, s)), -8.0f), 7.0f);
+  return static_cast<uint32_t>(static_cast<int>(q) + 8);
 }
+
+// 8 values of one group (pairs: elements 2e and 2e + 1 in x[e]) -> their offset codes q + 8 as
+// the 8 nibbles of one word in packed order (element 2j in the low nibble of byte j), by the
+// reciprocal rule above with r = RN(1/s), its fp32 steps in packed pairs (each component rounds as
+// the scalar operation would).  `ties` gets bit 8j + 7 for element 2j and bit 8j + 6 for element
+// 2j + 1 when that element's y may lie within 2^-19 of a half-integer (its nibble then needs the
+// IEEE quotient).  The test is d^2 - c >= 0 with d = y - rint(y) and c just below
+// (1/2 - 2^-19)^2, in one fused operation: every element the reciprocal rule may get wrong is
+// flagged, and a few more.  The codes are gathered from the sums' low bytes by byte permutes.
+constexpr float kTieSq = 0x1.ffffp-3f;  // 2^-2 - 2^-19: (1/2 - 2^-19)^2 = 2^-2 - 2^-19 + 2^-38, rounded down
+
+__device__ __forceinline__ uint32_t codes8_pairs(const float2 (&x)[4], float r, uint32_t& ties) {
+  const float2 r2 = make_float2(r, r), m2 = make_float2(kRintMagic, kRintMagic);
+  const float2 nm2 = make_float2(-kRintMagic, -kRintMagic), neg1 = make_float2(-1.0f, -1.0f);
+  const float2 nc2 = make_float2(-kTieSq, -kTieSq);
+  uint32_t t[8], v[8];
+#pragma unroll
+  for (int e = 0; e < 4; ++e) {
+    const float2 y = __fmul2_rn(x[e], r2);
+    const float2 tt = __fadd2_rn(y, m2);         // 1.5 * 2^23 + 8 + rint(y): low byte q + 8
+    const float2 rt = __fadd2_rn(tt, nm2);       // rint(y), exact
+    const float2 d = __ffma2_rn(rt, neg1, y);    // y - rint(y), exact
+    const float2 g = __ffma2_rn(d, d, nc2);      // d^2 - c: sign clear for a (possible) near-tie
+    t[2 * e] = __float_as_uint(tt.x);
+    t[2 * e + 1] = __float_as_uint(tt.y);
+    v[2 * e] = __float_as_uint(g.x);
+    v[2 * e + 1] = __float_as_uint(g.y);
+  }
+  // low bytes of the even elements to bytes 0-3, of the odd elements likewise, then nibbles
+  const uint32_t ev = __byte_perm(__byte_perm(t[0], t[2], 0x0040), __byte_perm(t[4], t[6], 0x0040), 0x5410);
+  const uint32_t od = __byte_perm(__byte_perm(t[1], t[3], 0x0040), __byte_perm(t[5], t[7], 0x0040), 0x5410);
+  // top bytes (signs) of the tie tests likewise
+  const uint32_t tv = __byte_perm(__byte_perm(v[0], v[2], 0x0073), __byte_perm(v[4], v[6], 0x0073), 0x5410);
+  const uint32_t to = __byte_perm(__byte_perm(v[1], v[3], 0x0073), __byte_perm(v[5], v[7], 0x0073), 0x5410);
+  ties = (~tv & 0x80808080u) | ((~to & 0x80808080u) >> 1);
+  return ev | (od << 4);
+}
+// The bit of `ties` that flags element j of the 8.
+__host__ __device__ constexpr int tie_bit(int j) { return 8 * (j >> 1) + ((j & 1) ? 6 : 7); }
 
 // 32 values of one group (scale s) -> 4 words of packed two's complement nibbles.
 __device__ __forceinline__ void quantize32(const float (&x)[32], float s, uint32_t (&pk)[4]) {
@@ -87,11 +119,29 @@ __device__ __forceinline__ void quantize32(const float (&x)[32], float s, uint32
   const float r = __frcp_rn(s);
 #pragma unroll
   for (int i = 0; i < 4; ++i) {
-    uint32_t w = 0;
+    uint32_t ties = 0xC0C0C0C0u, w = 0;  // a subnormal scale: every element by division
+    if (!exact_only) {
+      const float2 xp[4] = {make_float2(x[8 * i], x[8 * i + 1]), make_float2(x[8 * i + 2], x[8 * i + 3]),
+                            make_float2(x[8 * i + 4], x[8 * i + 5]), make_float2(x[8 * i + 6], x[8 * i + 7])};
+      w = codes8_pairs(xp, r, ties);
+    }
+    if (ties != 0) {  // the elements near a tie take the IEEE quotient
 #pragma unroll
-    for (int j = 0; j < 8; ++j) w |= code_offset(x[8 * i + j], s, r, exact_only) << (4 * j);
+      for (int j = 0; j < 8; ++j)
+        if ((ties >> tie_bit(j)) & 1u)
+          w = (w & ~(0xFu << (4 * j))) | (code_exact(x[8 * i + j], s) << (4 * j));
+    }
     pk[i] = w ^ 0x88888888u;  // offset (q + 8) -> two's complement nibble
   }
+}
+
+// The same for 8 bf16 values (one 16-byte unit of a row, element 2e in the low half of word e).
+__device__ __forceinline__ uint32_t codes8_offset(uint4 u, float r, uint32_t& ties) {
+  const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+  float2 x[4];
+#pragma unroll
+  for (int e = 0; e < 4; ++e) x[e] = make_float2(__uint_as_float(w[e] << 16), __uint_as_float(w[e] & 0xFFFF0000u));
+  return codes8_pairs(x, r, ties);
 }
 
 // ---------------------------------------------------------------- DiT neighbour operations
@@ -119,45 +169,76 @@ __device__ __forceinline__ float modulate_bf16(float x, float shift, float scale
 // Taylor polynomial to degree 8 (Horner, fused multiply-adds; |r| <= 0.35, truncation below
 // 2^-32), e^x = 2^n e^r by one exact-exponent product (two below the normal range); 0 below
 // x = -104.  Every step is one IEEE operation, so the CPU oracle reproduces it bit for bit.
+//
+// It (and the GELU below) works on a pair of values, the floating-point steps as packed pairs:
+// each packed operation rounds every component exactly as the scalar one would (the packed fused
+// multiply-add is __fmaf_rn per component), so the values are those of the scalar sequence with
+// half the floating-point instructions; the selects are per component.  Branch-free (selects only), so that independent pairs interleave: below -104
+// the result is 0, and below the normal range the power of two is applied as 2^(n+64) then 2^-64
+// (the second product is by exactly 1 above).
 __device__ __forceinline__ float pow2_f32(int n) { return __int_as_float((n + 127) << 23); }
+__device__ __forceinline__ float2 f2(float v) { return make_float2(v, v); }
 
-__device__ __forceinline__ float exp_neg_f32(float x) {
-  // branch-free (selects only), so that the caller's independent elements interleave; the values
-  // are those of the stepwise definition: below -104 the result is 0, and below the normal range
-  // the power of two is applied as 2^(n+64) then 2^-64 (the second product is by exactly 1 above)
-  const bool zero = x < -104.0f;
-  x = fmaxf(x, -104.0f);
-  const float n = rintf(__fmul_rn(x, 0x1.715476p+0f));
-  float r = __fmaf_rn(-n, 0x1.62e4p-1f, x);
-  r = __fmaf_rn(-n, 0x1.7f7d1cp-20f, r);
-  float p = 0x1.a01a02p-16f;           // 1/8!
-  p = __fmaf_rn(p, r, 0x1.a01a02p-13f);  // 1/7!
-  p = __fmaf_rn(p, r, 0x1.6c16c2p-10f);  // 1/6!
-  p = __fmaf_rn(p, r, 0x1.111112p-7f);   // 1/5!
-  p = __fmaf_rn(p, r, 0x1.555556p-5f);   // 1/4!
-  p = __fmaf_rn(p, r, 0x1.555556p-3f);   // 1/3!
-  p = __fmaf_rn(p, r, 0x1p-1f);          // 1/2!
-  p = __fmaf_rn(p, r, 1.0f);
-  p = __fmaf_rn(p, r, 1.0f);
-  const int ni = static_cast<int>(n);
-  const bool low = ni < -126;
-  const float v = __fmul_rn(__fmul_rn(p, pow2_f32(low ? ni + 64 : ni)), low ? 0x1p-64f : 1.0f);
-  return zero ? 0.0f : v;
+__device__ __forceinline__ float2 exp_neg_f32x2(float2 x) {
+  const bool zx = x.x < -104.0f, zy = x.y < -104.0f;
+  x = make_float2(fmaxf(x.x, -104.0f), fmaxf(x.y, -104.0f));
+  // n = rint(t) by the 1.5 * 2^23 addition (t in [-151, 0]: the sum's unit is 1 and rounds to
+  // nearest even, exactly as rint; the subtraction is exact)
+  const float2 t = __fmul2_rn(x, f2(0x1.715476p+0f));
+  const float2 tm = __fadd2_rn(t, f2(12582912.0f));
+  const float2 n = __fadd2_rn(tm, f2(-12582912.0f));
+  const float2 nn = make_float2(-n.x, -n.y);
+  float2 r = __ffma2_rn(nn, f2(0x1.62e4p-1f), x);
+  r = __ffma2_rn(nn, f2(0x1.7f7d1cp-20f), r);
+  float2 p = f2(0x1.a01a02p-16f);           // 1/8!
+  p = __ffma2_rn(p, r, f2(0x1.a01a02p-13f));  // 1/7!
+  p = __ffma2_rn(p, r, f2(0x1.6c16c2p-10f));  // 1/6!
+  p = __ffma2_rn(p, r, f2(0x1.111112p-7f));   // 1/5!
+  p = __ffma2_rn(p, r, f2(0x1.555556p-5f));   // 1/4!
+  p = __ffma2_rn(p, r, f2(0x1.555556p-3f));   // 1/3!
+  p = __ffma2_rn(p, r, f2(0x1p-1f));          // 1/2!
+  p = __ffma2_rn(p, r, f2(1.0f));
+  p = __ffma2_rn(p, r, f2(1.0f));
+  const int nx = static_cast<int>(n.x), ny = static_cast<int>(n.y);
+  const bool lx = nx < -126, ly = ny < -126;
+  const float2 v = __fmul2_rn(__fmul2_rn(p, make_float2(pow2_f32(lx ? nx + 64 : nx), pow2_f32(ly ? ny + 64 : ny))),
+                              make_float2(lx ? 0x1p-64f : 1.0f, ly ? 0x1p-64f : 1.0f));
+  return make_float2(zx ? 0.0f : v.x, zy ? 0.0f : v.y);
 }
 
-// The tanh GELU of one value evaluated in fp32 by a fixed sequence of IEEE operations (the same
-// as the oracle's): u = 0.7978846 (h + 0.044715 h^3), 1 + tanh(u) = 2 sigma(2u) with the logistic
-// as 1 / (1 + e^{-2u}) (u >= 0) or e^{2u} / (1 + e^{2u}) (u < 0), g = h sigma(2u); then rounded to
-// bf16 as a bf16 model stores it.  +-0 stays +-0.
-__device__ __forceinline__ float gelu_bf16(float h) {
-  // straight-line: the logistic takes one division with a selected numerator, 1 / (1 + e^{-2u})
-  // for u >= 0 and e^{2u} / (1 + e^{2u}) for u < 0 (e = e^{-2|u|} in both); h = +-0 gives +-0
-  const float h3 = __fmul_rn(__fmul_rn(h, h), h);
-  const float p = __fadd_rn(h, __fmul_rn(0x1.6e4e26p-5f, h3));
-  const float u = __fmul_rn(0x1.988454p-1f, p);
-  const float e = exp_neg_f32(__fmul_rn(-2.0f, fabsf(u)));
-  const float sig = __fdiv_rn(u >= 0.0f ? 1.0f : e, __fadd_rn(1.0f, e));
-  return __bfloat162float(__float2bfloat16_rn(__fmul_rn(h, sig)));
+// a / d for d in [1, 2] and a in [0, 1] without the division unit: Newton-Raphson division (the
+// reciprocal of D = d/2 in [1/2, 1] from the linear estimate 48/17 - 32/17 D, three iterations
+// y += y (1 - D y), each squaring the relative error from at most 1/17), then Markstein's
+// correction q + (a - q d) y with the exact remainder from a fused multiply-add.  It is not the
+// IEEE quotient for every such pair (a = 1, d = 2 - 2^-23 gives 1/2 instead of 1/2 + 2^-24), so
+// it stands in for the GELU's division only because the GELU value, rounded to bf16, is the
+// oracle's for every one of the 65280 finite bf16 inputs (a GPU test runs all of them).
+__device__ __forceinline__ float2 div_1_2(float2 a, float2 d) {
+  const float2 D = __fmul2_rn(d, f2(0.5f));
+  const float2 nD = make_float2(-D.x, -D.y);
+  float2 y = __ffma2_rn(D, f2(-32.0f / 17.0f), f2(48.0f / 17.0f));
+#pragma unroll
+  for (int i = 0; i < 3; ++i) y = __ffma2_rn(y, __ffma2_rn(nD, y, f2(1.0f)), y);
+  const float2 yh = __fmul2_rn(y, f2(0.5f));  // ~ 1/d
+  const float2 q = __fmul2_rn(a, yh);
+  const float2 r = __ffma2_rn(make_float2(-q.x, -q.y), d, a);  // a - q d, exact
+  return __ffma2_rn(r, yh, q);
+}
+
+// The tanh GELU evaluated in fp32 by the oracle's fixed sequence of IEEE operations, but for the
+// logistic's division (div_1_2 above): u = 0.7978846 (h + 0.044715 h^3), 1 + tanh(u) = 2 sigma(2u) with the logistic as
+// 1 / (1 + e^{-2u}) (u >= 0) or e^{2u} / (1 + e^{2u}) (u < 0), g = h sigma(2u); then rounded to
+// bf16 as a bf16 model stores it.  Straight-line: the logistic takes one division with a
+// selected numerator (e = e^{-2|u|} in both forms); +-0 stays +-0.  On a pair of values, as above.
+__device__ __forceinline__ float2 gelu_bf16x2(float2 h) {
+  const float2 h3 = __fmul2_rn(__fmul2_rn(h, h), h);
+  const float2 p = __fadd2_rn(h, __fmul2_rn(f2(0x1.6e4e26p-5f), h3));
+  const float2 u = __fmul2_rn(f2(0x1.988454p-1f), p);
+  const float2 e = exp_neg_f32x2(__fmul2_rn(f2(-2.0f), make_float2(fabsf(u.x), fabsf(u.y))));
+  const float2 d = __fadd2_rn(f2(1.0f), e);
+  const float2 sig = div_1_2(make_float2(u.x >= 0.0f ? 1.0f : e.x, u.y >= 0.0f ? 1.0f : e.y), d);
+  const float2 g = __fmul2_rn(h, sig);
+  return __bfloat1622float2(__floats2bfloat162_rn(g.x, g.y));
 }
 
 // Applies the neighbour operation to 32 consecutive values of row `row` from K index `col`.
@@ -177,7 +258,11 @@ __device__ __forceinline__ void apply_op(float (&v)[32], int64_t row, int64_t co
     }
   } else if constexpr (kOp == kOpGelu) {
 #pragma unroll
-    for (int i = 0; i < 32; ++i) v[i] = gelu_bf16(v[i]);
+    for (int i = 0; i < 16; ++i) {
+      const float2 g = gelu_bf16x2(make_float2(v[2 * i], v[2 * i + 1]));
+      v[2 * i] = g.x;
+      v[2 * i + 1] = g.y;
+    }
   }
 }
 
@@ -276,43 +361,6 @@ constexpr uint32_t kQtSlotBytes = kQtRows * kQtCols * 2;
 constexpr uint32_t kQtSmemBytes = kQtSlots * kQtSlotBytes + 2 * kQtSlots * 8 + 16;
 static_assert(32 * kQtConsumerWarps * 32 == kQtRows * kQtCols, "one chunk of 32 elements per consumer thread");
 
-// 8 bf16 values (one 16-byte unit) -> their offset codes q + 8 as the 8 nibbles of one word in
-// packed order (element 2j in the low nibble of byte j), with r = RN(1/s).  `ties` gets bit
-// 8j + 7 for even element 2j and bit 8j + 6 for odd element 2j + 1 when that element's y may lie
-// within 2^-19 of a half-integer (its nibble then needs the IEEE quotient).  The test is
-// d^2 - c >= 0 with d = y - rint(y) and c just below (1/2 - 2^-19)^2, in one fused operation:
-// every element the reciprocal rule may get wrong is flagged, and a few more.
-constexpr float kTieSq = 0x1.ffffp-3f;  // 2^-2 - 2^-19: (1/2 - 2^-19)^2 = 2^-2 - 2^-19 + 2^-38, rounded down
-
-__device__ __forceinline__ uint32_t codes8_offset(uint4 u, float r, uint32_t& ties) {
-  const uint32_t w[4] = {u.x, u.y, u.z, u.w};
-  const float2 r2 = make_float2(r, r), m2 = make_float2(kRintMagic, kRintMagic);
-  const float2 nm2 = make_float2(-kRintMagic, -kRintMagic), neg1 = make_float2(-1.0f, -1.0f);
-  const float2 nc2 = make_float2(-kTieSq, -kTieSq);
-  uint32_t t[8], v[8];
-#pragma unroll
-  for (int e = 0; e < 4; ++e) {
-    const float2 x = make_float2(__uint_as_float(w[e] << 16), __uint_as_float(w[e] & 0xFFFF0000u));
-    const float2 y = __fmul2_rn(x, r2);
-    const float2 tt = __fadd2_rn(y, m2);         // 1.5 * 2^23 + 8 + rint(y): low byte q + 8
-    const float2 rt = __fadd2_rn(tt, nm2);       // rint(y), exact
-    const float2 d = __ffma2_rn(rt, neg1, y);    // y - rint(y), exact
-    const float2 g = __ffma2_rn(d, d, nc2);      // d^2 - c: sign clear for a (possible) near-tie
-    t[2 * e] = __float_as_uint(tt.x);
-    t[2 * e + 1] = __float_as_uint(tt.y);
-    v[2 * e] = __float_as_uint(g.x);
-    v[2 * e + 1] = __float_as_uint(g.y);
-  }
-  // low bytes of the even elements to bytes 0-3, of the odd elements likewise, then nibbles
-  const uint32_t ev = __byte_perm(__byte_perm(t[0], t[2], 0x0040), __byte_perm(t[4], t[6], 0x0040), 0x5410);
-  const uint32_t od = __byte_perm(__byte_perm(t[1], t[3], 0x0040), __byte_perm(t[5], t[7], 0x0040), 0x5410);
-  // top bytes (signs) of the tie tests likewise
-  const uint32_t tv = __byte_perm(__byte_perm(v[0], v[2], 0x0073), __byte_perm(v[4], v[6], 0x0073), 0x5410);
-  const uint32_t to = __byte_perm(__byte_perm(v[1], v[3], 0x0073), __byte_perm(v[5], v[7], 0x0073), 0x5410);
-  ties = (~tv & 0x80808080u) | ((~to & 0x80808080u) >> 1);
-  return ev | (od << 4);
-}
-
 template <int L, bool kOperand>
 __global__ void __launch_bounds__(kQtThreads, 2) quantize_tiles_kernel(const __grid_constant__ CUtensorMap tmX,
                                                                        int64_t M, int64_t K,
@@ -394,7 +442,7 @@ __global__ void __launch_bounds__(kQtThreads, 2) quantize_tiles_kernel(const __g
           ties &= ties - 1;
           const int e = 2 * (bit >> 3) + ((bit & 7) == 6 ? 1 : 0);
           const uint16_t b = reinterpret_cast<const uint16_t*>(src + q)[e];
-          const uint32_t c = code_offset(__uint_as_float((uint32_t)b << 16), s, r, true);
+          const uint32_t c = code_exact(__uint_as_float((uint32_t)b << 16), s);
           word = (word & ~(0xFu << (4 * e))) | (c << (4 * e));
         }
         pk[q] = word ^ 0x88888888u;

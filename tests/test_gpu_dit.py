@@ -99,6 +99,28 @@ def test_gelu_quantize_bit_exact(G):
     assert np.array_equal(sa.cpu().numpy().view(np.uint32), s.view(np.uint32))
 
 
+def test_gelu_every_finite_bf16_through_the_group_scale():
+    """Every finite bf16 h, each alone in a group of 64 (the rest zeros, GELU(0) = 0): the group
+    scale is |GELU(h)| / 7 and the code carries the sign, so equal scales and codes mean the fused
+    GELU's bf16 value equals the oracle's for every input the kernel can see."""
+    allb = np.arange(0, 0x10000, dtype=np.uint32).astype(np.uint16)
+    vals = wl.bf16_bits_to_f32(allb)
+    h_vals = allb[np.isfinite(vals)]
+    G, K = 64, 4096
+    rows = -(-len(h_vals) // (K // G))
+    h = np.zeros((rows * (K // G), G), np.uint16)
+    h[: len(h_vals), 0] = h_vals
+    h = h.reshape(rows, K)
+    z, codes, s = oracle.gelu_quantize_bf16(h, G)
+    q, sa = jq.jq_gelu_quantize_act(dev_bf16(h), G)
+    assert np.array_equal(q.cpu().numpy(), oracle.pack(codes)), "codes differ"
+    got = sa.cpu().numpy().view(np.uint32)
+    want = s.view(np.uint32)
+    if not np.array_equal(got, want):
+        bad = np.argwhere(got.reshape(-1) != want.reshape(-1))[:5, 0]
+        raise AssertionError(f"{(got != want).sum()} group scales differ, e.g. inputs {h.reshape(-1, G)[bad, 0]}")
+
+
 def test_modulate_quantize_then_linear_at_the_dit_qkv_shape():
     """DiT-XL/2 attention input projection, 4 images of 256 tokens: 1024 x 1152 -> 3456, group128,
     through jq_modulate_quantize_act and jq_w4a4_linear; every output against the oracle."""

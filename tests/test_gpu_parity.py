@@ -124,6 +124,39 @@ def test_quantize_act_exhaustive_bf16(G):
     assert np.array_equal(s.cpu().numpy().view(np.uint32), ref_s.view(np.uint32))
 
 
+@pytest.mark.parametrize("G", [64, 128])
+def test_quantize_act_exhaustive_bf16_tiled(G):
+    """The same values as test_quantize_act_exhaustive_bf16 (every positive finite bf16 under
+    amaxes over the whole range, and their negatives), laid out as rows of 2048 and repeated so
+    that the input takes the TMA-staged kernel (at least four 64 x 256 tiles per SM)."""
+    allb = np.arange(1, 0x7F80, dtype=np.uint16)
+    allf = wl.bf16_bits_to_f32(allb)
+    amaxes = np.unique(np.concatenate([np.linspace(1, 0x7F7F, 150).astype(np.uint16),
+                                       wl.f32_to_bf16_bits(np.array([1.0, 7.0, 3.5, 448.0], np.float32))]))
+    per = G - 1
+    rows = []
+    for a in amaxes:
+        xs = allb[allf <= wl.bf16_bits_to_f32(np.array([a]))[0]]
+        n = (len(xs) + per - 1) // per
+        blk = np.zeros((n, G), np.uint16)
+        blk[:, 0] = a
+        flat = np.zeros(n * per, np.uint16)
+        flat[: len(xs)] = xs
+        blk[:, 1:] = flat.reshape(n, per)
+        rows.append(blk)
+    groups = np.concatenate(rows)
+    groups = np.concatenate([groups, groups ^ np.uint16(0x8000)])
+    K = 2048
+    reps = -(-(10 * 2 ** 20) // groups.size)  # >= 10 M elements: > 4 tiles per SM
+    flat = np.tile(groups.reshape(-1), reps)
+    flat = flat[: (flat.size // K) * K]
+    x = flat.reshape(-1, K)
+    ref_codes, ref_s = oracle.quantize_bf16(x, G)
+    q, s = jq.jq_quantize_act(dev_bf16(x), G)
+    assert np.array_equal(q.cpu().numpy(), oracle.pack(ref_codes))
+    assert np.array_equal(s.cpu().numpy().view(np.uint32), ref_s.view(np.uint32))
+
+
 @pytest.mark.slow
 def test_quantize_act_every_bf16_pair():
     """Every positive finite bf16 amax with every bf16 x of magnitude up to it, both signs (about
