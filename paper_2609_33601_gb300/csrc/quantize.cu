@@ -241,6 +241,21 @@ __device__ __forceinline__ float2 gelu_bf16x2(float2 h) {
   return __bfloat1622float2(__floats2bfloat162_rn(g.x, g.y));
 }
 
+// The GELU's input is a bf16 value, so the whole function is a table of 65536 bf16 results: the
+// fused quantiser looks each value up instead of evaluating the sequence (about 35 operations an
+// element, which made that kernel compute-bound).  The table is filled on the device by
+// gelu_bf16x2 itself -- the same values by construction -- once per device before the first
+// fused GELU call (launch_gelu_quantize_act).
+__device__ uint16_t g_gelu_bf16[65536];
+
+__global__ void __launch_bounds__(256) gelu_table_kernel() {
+  const uint32_t i = blockIdx.x * 256u + threadIdx.x;  // entries 2i, 2i + 1
+  if (i >= 32768u) return;
+  const float2 g = gelu_bf16x2(make_float2(__uint_as_float((2u * i) << 16), __uint_as_float((2u * i + 1u) << 16)));
+  g_gelu_bf16[2u * i] = static_cast<uint16_t>(__float_as_uint(g.x) >> 16);
+  g_gelu_bf16[2u * i + 1u] = static_cast<uint16_t>(__float_as_uint(g.y) >> 16);
+}
+
 // Applies the neighbour operation to 32 consecutive values of row `row` from K index `col`.
 template <int kOp>
 __device__ __forceinline__ void apply_op(float (&v)[32], int64_t row, int64_t col, int64_t K, const OpArgs& op) {
@@ -256,13 +271,10 @@ __device__ __forceinline__ void apply_op(float (&v)[32], int64_t row, int64_t co
       v[4 * i + 2] = modulate_bf16(v[4 * i + 2], a.z, c.z);
       v[4 * i + 3] = modulate_bf16(v[4 * i + 3], a.w, c.w);
     }
-  } else if constexpr (kOp == kOpGelu) {
+  } else if constexpr (kOp == kOpGelu) {  // v[i] holds a bf16 value: its bits index the table
 #pragma unroll
-    for (int i = 0; i < 16; ++i) {
-      const float2 g = gelu_bf16x2(make_float2(v[2 * i], v[2 * i + 1]));
-      v[2 * i] = g.x;
-      v[2 * i + 1] = g.y;
-    }
+    for (int i = 0; i < 32; ++i)
+      v[i] = __uint_as_float(static_cast<uint32_t>(__ldg(g_gelu_bf16 + (__float_as_uint(v[i]) >> 16))) << 16);
   }
 }
 
@@ -695,6 +707,31 @@ cudaError_t launch_modulate_quantize_act(const void* x, int64_t M, int64_t K, in
 
 cudaError_t launch_gelu_quantize_act(const void* h, int64_t M, int64_t K, int64_t ldh, int G, uint8_t* q, float* s_a,
                                      cudaStream_t stream, int sms) {
+  // The GELU table: filled once per device and waited for before it counts as ready, so a call
+  // on any stream of the device may read it.  A first call made while `stream` is being captured
+  // into a graph cannot wait: it puts the filling kernel into the graph ahead of the quantiser
+  // (every replay rewrites the same values) and leaves the once-per-device filling to a later
+  // call made outside a capture.
+  static PerDevice<bool> table;
+  cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
+  if (cudaStreamIsCapturing(stream, &cs) != cudaSuccess) return cudaGetLastError();
+  if (cs == cudaStreamCaptureStatusNone) {
+    bool ready = false;
+    cudaError_t e = table.get(
+        [stream](bool& v) {
+          gelu_table_kernel<<<128, 256, 0, stream>>>();
+          cudaError_t le = cudaGetLastError();
+          if (le == cudaSuccess) le = cudaStreamSynchronize(stream);
+          v = le == cudaSuccess;
+          return le;
+        },
+        ready);
+    if (e != cudaSuccess) return e;
+  } else {
+    gelu_table_kernel<<<128, 256, 0, stream>>>();
+    cudaError_t le = cudaGetLastError();
+    if (le != cudaSuccess) return le;
+  }
   return launch_quantize<__nv_bfloat16, false, false, kOpGelu>(static_cast<const __nv_bfloat16*>(h), M, K, ldh, G, q,
                                                                 s_a, nullptr, stream, sms);
 }
