@@ -377,6 +377,41 @@ def cublas_context(torch, dev, sets, M, N, K, args, world):
             "what": "torch.matmul bf16 x[M,K] @ W[N,K]^T, same M, N, K"}
 
 
+def copy_context(torch, dev, nbytes, args, world):
+    """What a device-to-device copy of as many bytes as the linear layer moves takes, for the
+    HBM-bound lines (the measured HBM peak is a copy rate): rotating source and destination
+    buffers (together larger than L2), K copies captured in a CUDA graph and timed with CUDA
+    events like the linear layer; GB/s counts the bytes read and written.  At a few MB a
+    launch's fixed costs, not HBM, set the copy's rate too."""
+    n = max(4096, (nbytes // 16) * 16)
+    n_b = max(2, -(-300_000_000 // (2 * n)))
+    src = [torch.ones(n, dtype=torch.uint8, device=dev) for _ in range(n_b)]
+    dst = [torch.empty(n, dtype=torch.uint8, device=dev) for _ in range(n_b)]
+    cap = torch.cuda.Stream()
+    cap.wait_stream(torch.cuda.current_stream())
+    with torch.cuda.stream(cap):
+        for i in range(args.warmup):
+            dst[i % n_b].copy_(src[i % n_b])
+    cap.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=cap):
+        for i in range(args.steps):
+            dst[i % n_b].copy_(src[i % n_b])
+    g.replay()
+    torch.cuda.synchronize()
+    t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    t0.record()
+    g.replay()
+    t1.record()
+    torch.cuda.synchronize()
+    ms = t0.elapsed_time(t1) / args.steps
+    del src, dst, g
+    torch.cuda.empty_cache()
+    return {"value": world * 2 * n / (ms * 1e-3) / 1e9, "unit": "GB/s", "ms_per_call": ms, "bytes": n,
+            "what": "device-to-device copy of the linear's algorithmic bytes (rotating buffers > L2), K copies "
+                    "in a CUDA graph; GB/s counts bytes read + written, like the measured HBM peak"}
+
+
 def prologue_context(torch, jq, sets, mods, prologue, G, T, q, s_a, args):
     """The DiT neighbour operation fused into the quantiser against the same operation done
     separately (PyTorch bf16 ops writing the activation, then jq_quantize_act reading it back),
@@ -908,6 +943,8 @@ def run_ours(args):
     context = None
     if not args.no_context:
         context = {"cublas_bf16": cublas_context(torch, dev, sets, M, N, K, args, world)}
+        if few:
+            context["copy_same_bytes"] = copy_context(torch, dev, alg_bytes, args, world)
         if prologue is not None:
             context["prologue"] = prologue_context(torch, jq, sets, mods if prologue == "modulate" else None, prologue,
                                                    G, T, q, s_a, args)
