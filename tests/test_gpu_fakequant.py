@@ -47,8 +47,10 @@ def _gen(seed, M, K):
     return wl.f32_to_bf16_bits(x)
 
 
+# Four rows per block from 2432 rows on (152 SMs), else one: a ragged last block at 2433 rows.
 @pytest.mark.parametrize("M,K,G", [(64, 256, 64), (64, 256, 128), (64, 256, 256), (37, 384, 384),
-                                   (37, 384, 128), (5, 6144, 64), (3, 6144, 6144), (1500, 128, 128)])
+                                   (37, 384, 128), (5, 6144, 64), (3, 6144, 6144), (1500, 128, 128),
+                                   (2433, 256, 64), (2436, 384, 384), (2437, 1024, 128)])
 def test_amax_rule_matches_the_oracle(M, K, G):
     xb = _gen(M * 7 + K + G, M, K)
     xb[min(2, M - 1), :G] = 0  # an all-zero group
@@ -56,7 +58,7 @@ def test_amax_rule_matches_the_oracle(M, K, G):
     assert om.all()
 
 
-@pytest.mark.parametrize("M,K,G", [(33, 256, 64), (9, 2304, 128), (4, 384, 384)])
+@pytest.mark.parametrize("M,K,G", [(33, 256, 64), (9, 2304, 128), (4, 384, 384), (2435, 256, 64)])
 def test_given_scales_clamp_like_the_oracle(M, K, G):
     xb = _gen(100 + M, M, K)
     rng = np.random.default_rng(M)
@@ -104,7 +106,8 @@ def test_forward_mask_feeds_the_backward():
 
 
 @pytest.mark.parametrize("N,K,G,given", [(256, 256, 64, False), (96, 384, 384, False), (300, 4096, 128, False),
-                                         (1300, 128, 128, False), (40, 2304, 128, True)])
+                                         (1300, 128, 128, False), (40, 2304, 128, True), (2434, 3072, 64, False),
+                                         (2441, 512, 128, True)])
 def test_weight_fake_quant_matches_the_oracle(N, K, G, given):
     rng = np.random.default_rng(N + K)
     w = (rng.standard_normal((N, K)) * 0.02).astype(np.float32)
