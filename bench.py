@@ -94,9 +94,9 @@ FP8_PER_BF16 = 2.0  # nominal dense FP8 / BF16 tensor-core ratio on GB300 (4.5 /
 # capture was taken on (kernel_hash); once the code changes the figure no longer applies and the
 # bench reports null until a new capture is recorded here.
 KERNEL_TRAFFIC: dict = {
-    ("flux_qkv", "17f2efcfd35bda35"): 55.028224e6 + 144.056576e6,
-    ("dllm", "17f2efcfd35bda35"): 31.280896e6 + 0.182784e6,
-    ("dllm/ternary", "17f2efcfd35bda35"): 18.673152e6 + 0.105216e6,
+    ("flux_qkv", "b083073b8736b564"): 54.676992e6 + 143.107328e6,
+    ("dllm", "b083073b8736b564"): 31.281152e6 + 0.165376e6,
+    ("dllm/ternary", "b083073b8736b564"): 18.681088e6 + 0.109568e6,
 }
 
 

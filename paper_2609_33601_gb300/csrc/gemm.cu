@@ -112,6 +112,7 @@ struct Args {
   int groups, sc_boxes;  // K / G, and scale-ring slots per tile (ceil(groups / kScGroups))
   int sa_tma;            // activation scales come through the scale ring (groups % 4 == 0)
   int ternary;           // qw holds 2-bit ternary codes [N, K/4] (ternary.cu), not INT4 [N, K/2]
+  int prefetch_slots;    // L2 prefetch distance of the packed weights, in ring slots (producer_a)
   const uint8_t* qw;
   const float* s_a;
   const float* corr;     // [M, K/G]: 8 * the group's activation code sum in 2^-18 units (offset codes)
@@ -521,11 +522,32 @@ __device__ __forceinline__ void scale_producer(const Args& args, const Pair& pr,
 // ------------------------------------------------------------------ A producer
 // Both CTAs load their own 128 rows of a slot's two K stages; the transfers complete on the even
 // CTA's full barrier, which the even CTA arms with the bytes of both.
+// The same thread prefetches into L2 this CTA's packed weight rows of the slot args.prefetch_slots
+// ahead of the one it loads A for: the unpack warps fetch weights with plain loads only two slots
+// ahead, which left slots waiting for DRAM when a weight tile serves few M tiles.  Measured over
+// one-group problems 4096 -> 12288 (linear alone, weight sets larger than L2), with 0 / 2 / 4
+// slots: M = 1024 1568 / 1720 / 1703 TFLOP/s, M = 4096 1988 / 2076 / 2077, but M = 16384 2377 /
+// 2327 / 2274 (there the weights stay in L2 for the 64 M tiles that share them) and M = 256
+// 942 / 922 / 877; so two slots, for 2 to 16 pair tiles along M (launch_impl).
+constexpr int kPrefetchSlots = 2;
+
 template <class T>
-__device__ __forceinline__ void producer_a(const Args& args, const Pair& pr, const CUtensorMap* tmA, uint8_t* sA,
-                                           const Bars& b, volatile int* abort_flag) {
+__device__ __forceinline__ void producer_a(const Args& args, const Pair& pr, const CUtensorMap* tmA,
+                                           const CUtensorMap* tmW, uint8_t* sA, const Bars& b,
+                                           volatile int* abort_flag) {
   uint32_t it = 0;
   bool ok = true;
+  const int wslot_bytes = kStagesPerSlot * kBK / (args.ternary ? 4 : 2);  // packed weight bytes of a slot
+  int ptile = pr.cluster, pj = 0;  // the slot whose weights are prefetched next
+  auto prefetch_next = [&]() {
+    if (ptile >= args.num_tiles) return;
+    tma_prefetch_l2_2d(tmW, pj * wslot_bytes, (ptile / args.num_m2) * T::kBN + (int)pr.rank * T::kBNHalf);
+    if (++pj == args.slots_per_tile) {
+      pj = 0;
+      ptile += pr.num_clusters;
+    }
+  };
+  for (int i = 0; i < args.prefetch_slots; ++i) prefetch_next();
   for (int tile = pr.cluster; ok && tile < args.num_tiles; tile += pr.num_clusters) {
     const int mt = (tile % args.num_m2) * 2 + (int)pr.rank;  // 128-row block of the operand image
     for (int j = 0; j < args.slots_per_tile; ++j) {
@@ -534,6 +556,7 @@ __device__ __forceinline__ void producer_a(const Args& args, const Pair& pr, con
       if (pr.rank == 0) mbar_arrive_expect_tx(&b.full[s], 2 * kSlotABytes);
       const int image_row = (mt * args.k_stages + j * kStagesPerSlot) * kBM;
       tma_load_2d_pair(sA + s * kSlotABytes, tmA, leader_bar(&b.full[s]), 0, image_row);
+      if (args.prefetch_slots > 0) prefetch_next();
       ++it;
     }
   }
@@ -780,7 +803,8 @@ __device__ __forceinline__ void unpack_role(const Args& args, const Pair& pr, ui
 template <bool kExport, bool kOffset, int kBN>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     w4a4_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmSW,
-                     const __grid_constant__ CUtensorMap tmSA, const Args args) {
+                     const __grid_constant__ CUtensorMap tmSA, const __grid_constant__ CUtensorMap tmW,
+                     const Args args) {
   using T = Tile<kBN>;
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   if ((smem_u32(smem_raw) & 1023u) != 0) {  // uniform across the grid: nothing has been touched yet
@@ -827,6 +851,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     }
     fence_mbar_init();
     tma_prefetch_desc(&tmA);
+    tma_prefetch_desc(&tmW);
     if (!kExport) {
       tma_prefetch_desc(&tmSW);
       if (args.sa_tma) tma_prefetch_desc(&tmSA);
@@ -872,7 +897,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
   } else {
     asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;\n" ::"n"(kRegsCtl) : "memory");
     if (warp == kWarpProdA) {
-      if (lane == 0) producer_a<T>(args, pr, &tmA, sA, b, abort_flag);
+      if (lane == 0) producer_a<T>(args, pr, &tmA, &tmW, sA, b, abort_flag);
     } else if (warp == kWarpScale) {
       if (!kExport && lane == 0) scale_producer<T>(args, pr, &tmSW, &tmSA, sSc, b, abort_flag);
     } else if (warp == kWarpMma && lane == 0) {
@@ -910,6 +935,16 @@ cudaError_t launch_impl(const GemmProblem& p, cudaStream_t stream, int sms) {
   if (!encode_2d(&tmA, CU_TENSOR_MAP_DATA_TYPE_UINT8, p.a_operand, kBK, image_rows, kBK, kBK,
                  kStagesPerSlot * kBM, CU_TENSOR_MAP_SWIZZLE_NONE))
     return cudaErrorInvalidValue;
+  // The packed weights as rows of bytes, for the L2 prefetch of a slot's rows (producer_a): one
+  // box is one slot's bytes (two K stages) of this CTA's half of the tile's columns.
+  CUtensorMap tmW;
+  {
+    const uint64_t wrow = p.ternary ? (uint64_t)p.K / 4 : (uint64_t)p.K / 2;
+    if (!encode_2d(&tmW, CU_TENSOR_MAP_DATA_TYPE_UINT8, p.qw, wrow, (uint64_t)p.N, wrow,
+                   (uint32_t)(kStagesPerSlot * kBK / (p.ternary ? 4 : 2)), (uint32_t)T::kBNHalf,
+                   CU_TENSOR_MAP_SWIZZLE_NONE))
+      return cudaErrorInvalidValue;
+  }
   // Scale maps (the export path reads no scales: it passes the A map in their place, unused).
   const int groups = p.K / p.G;
   const bool sa_tma = !kExport && groups % kScGroups == 0;
@@ -960,6 +995,7 @@ cudaError_t launch_impl(const GemmProblem& p, cudaStream_t stream, int sms) {
   a.sc_boxes = (groups + kScGroups - 1) / kScGroups;
   a.sa_tma = sa_tma ? 1 : 0;
   a.ternary = p.ternary ? 1 : 0;
+  a.prefetch_slots = (a.num_m2 >= 2 && a.num_m2 <= 16) ? kPrefetchSlots : 0;
   a.qw = p.qw;
   a.s_a = p.s_a;
   a.corr = p.corr;
@@ -970,7 +1006,7 @@ cudaError_t launch_impl(const GemmProblem& p, cudaStream_t stream, int sms) {
   a.status = p.status;
   const int pairs = a.num_tiles < max_pairs ? a.num_tiles : max_pairs;
   return launch_pdl(w4a4_gemm_kernel<kExport, kOffset, kBN>, dim3(2 * pairs), dim3(kThreads), T::kSmemBytes, stream,
-                    tmA, tmSW, tmSA, a);
+                    tmA, tmSW, tmSA, tmW, a);
 }
 
 }  // namespace
