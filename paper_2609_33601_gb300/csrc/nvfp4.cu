@@ -166,19 +166,32 @@ constexpr int kStageK = 64;  // bf16 elements per 128-byte operand row of a stag
 // One thread per 32 elements of a row (four 16-byte chunks of the image, all in one stage); grid
 // x over the row's 32-element units, y over rows.  rows may be short of a whole 128-row tile:
 // the image's rows past them are never written (their outputs are never kept).
-__device__ __forceinline__ uint32_t e2m1_bf16_pair(uint32_t byte, float s) {
-  float v[2];
+// 8 E2M1 codes (one 32-bit word, element i in bits 4i..4i+3) -> their values as 4 bf16 pairs
+// (elements 2k, 2k+1 in word k), without conversions: byte permutes look up the low and high
+// bytes of each magnitude's bf16 bits in 8-entry tables (0, 0.5, 1, 1.5, 2, 3, 4, 6 are 0000,
+// 3F00, 3F80, 3FC0, 4000, 4040, 4080, 40C0), a third permute turns each sign bit into 0x00 or
+// 0x80 for the high byte, and two more interleave low and high bytes into pairs.
+__device__ __forceinline__ uint4 e2m1x8_bf16(uint32_t w) {
+  constexpr uint32_t kLoA = 0xC0800000u, kLoB = 0xC0804000u;  // low bytes of idx 0-3, 4-7
+  constexpr uint32_t kHiA = 0x3F3F3F00u, kHiB = 0x40404040u;  // high bytes of idx 0-3, 4-7
+  const uint32_t mag = w & 0x77777777u;                        // magnitude index per nibble
+  const uint32_t sgn = (w >> 3) & 0x11111111u;                 // sign per nibble: byte 0 or 1
+  uint32_t out[4];
 #pragma unroll
-  for (int h = 0; h < 2; ++h) {
-    const uint32_t nib = (byte >> (4 * h)) & 15u;
-    // E2M1: exponent bits e = idx >> 1, mantissa bit m = idx & 1: m/2 for e = 0 (subnormal),
-    // (1 + m/2) 2^(e-1) otherwise -- 0, 0.5, 1, 1.5, 2, 3, 4, 6
-    const uint32_t idx = nib & 7u, ee = idx >> 1, mm = idx & 1u;
-    const float mag = ee == 0u ? 0.5f * (float)mm : (1.0f + 0.5f * (float)mm) * (float)(1u << (ee - 1u));
-    const float val = mag * s;  // exact
-    v[h] = (nib & 8u) ? -val : val;
+  for (int h = 0; h < 2; ++h) {  // elements 4h .. 4h + 3
+    const uint32_t sel = (mag >> (16 * h)) & 0xFFFFu, ssel = (sgn >> (16 * h)) & 0xFFFFu;
+    const uint32_t lo = __byte_perm(kLoA, kLoB, sel);
+    const uint32_t hi = __byte_perm(kHiA, kHiB, sel) | __byte_perm(0x8000u, 0u, ssel);
+    out[2 * h] = __byte_perm(lo, hi, 0x5140);
+    out[2 * h + 1] = __byte_perm(lo, hi, 0x7362);
   }
-  const __nv_bfloat162 p = __floats2bfloat162_rn(v[0], v[1]);  // exact
+  return make_uint4(out[0], out[1], out[2], out[3]);
+}
+
+// A bf16 pair times the block scale (an E4M3 value, exact in bf16): every product has at most 6
+// significant bits and lies in [2^-10, 2688], so the bf16 multiply is exact.
+__device__ __forceinline__ uint32_t bf16x2_scale(uint32_t v, __nv_bfloat162 s2) {
+  const __nv_bfloat162 p = __hmul2(*reinterpret_cast<const __nv_bfloat162*>(&v), s2);
   return *reinterpret_cast<const uint32_t*>(&p);
 }
 
@@ -195,16 +208,15 @@ __global__ void __launch_bounds__(128) nvfp4_expand_kernel(const uint8_t* __rest
   for (int64_t r = blockIdx.y; r < rows; r += gridDim.y) {
     const uint4 c = __ldg(reinterpret_cast<const uint4*>(codes + r * (K / 2) + k0 / 2));
     const uint8_t* sr = scales + r * (K / 16) + k0 / 16;  // byte loads: the scales carry no alignment rule
-    const float s0 = e4m3_value(__ldg(sr)), s1 = e4m3_value(__ldg(sr + 1));  // elements 0-15, 16-31
+    const __nv_bfloat162 s0 = __float2bfloat162_rn(e4m3_value(__ldg(sr)));      // elements 0-15
+    const __nv_bfloat162 s1 = __float2bfloat162_rn(e4m3_value(__ldg(sr + 1)));  // elements 16-31
     const uint32_t w[4] = {c.x, c.y, c.z, c.w};
 #pragma unroll
     for (int q = 0; q < 4; ++q) {  // chunk q: elements 8q .. 8q + 7 (4 code bytes)
-      const float sq = q < 2 ? s0 : s1;
-      uint32_t out[4];
-#pragma unroll
-      for (int i = 0; i < 4; ++i) out[i] = e2m1_bf16_pair((w[q] >> (8 * i)) & 0xFFu, sq);
+      const __nv_bfloat162 sq = q < 2 ? s0 : s1;
+      const uint4 m = e2m1x8_bf16(w[q]);
       *reinterpret_cast<uint4*>(image + image_chunk_offset(r, kb, c16 + (uint32_t)q, k_stages)) =
-          make_uint4(out[0], out[1], out[2], out[3]);
+          make_uint4(bf16x2_scale(m.x, sq), bf16x2_scale(m.y, sq), bf16x2_scale(m.z, sq), bf16x2_scale(m.w, sq));
     }
   }
 }
