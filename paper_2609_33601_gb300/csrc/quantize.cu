@@ -331,7 +331,7 @@ __device__ __forceinline__ void finish_chunk(const float (&v)[32], bool valid, i
 // G = 32 * L (L = 2 or 4): each thread quantises 32 consecutive elements; the L threads of a
 // group are adjacent lanes and reduce amax with xor-shuffles.
 template <typename In, int L, bool kOperand, bool kScaleT, int kOp = kOpNone>
-__global__ void __launch_bounds__(256) quantize_groups_kernel(const In* __restrict__ x, int64_t M, int64_t K,
+__global__ void __launch_bounds__(256, kOp == kOpModulate ? 4 : 1) quantize_groups_kernel(const In* __restrict__ x, int64_t M, int64_t K,
                                                               int64_t ldx, uint8_t* __restrict__ out,
                                                               float* __restrict__ scales, float* __restrict__ corr,
                                                               const OpArgs op) {
