@@ -26,8 +26,9 @@
  *     Weight scales s_w:     fp32 [K/group, N] (group-major: one row of N channel scales per
  *     K-group).  bias: fp32 [N] or NULL.  Outputs y: bf16 [M, N].
  *   - All data pointers are DEVICE pointers owned by the caller.  The library allocates
- *     nothing, never synchronises, and enqueues its kernels on `stream` (a cudaStream_t passed
- *     as void*; NULL = legacy default stream).
+ *     nothing, never synchronises (one exception: jq_gelu_quantize_act, below, once per
+ *     device), and enqueues its kernels on `stream` (a cudaStream_t passed as void*; NULL =
+ *     legacy default stream).
  *   - Supported shapes: group in {64, 128, K}; K % 128 == 0; K <= 262016 (so every exact
  *     per-group sum, |acc| <= 64*K, stays below 2^24); N % 8 == 0; M >= 0 (M == 0 is a no-op).
  *   - Pointers must be 16-byte aligned and ldx*2 a multiple of 16 bytes.
@@ -123,6 +124,13 @@ JQ_API jq_status jq_pack_weight(const float* w, int64_t N, int64_t K, int32_t gr
  *   q, s_a          : outputs as jq_quantize_act
  * Errors as jq_quantize_act (JQ_ERR_INVALID_ARG also for tokens_per_sample <= 0 or a NULL
  * shift / scale).
+ * The GELU is read from a table of its value at every bf16 input (65536 entries, in the
+ * library's device memory), computed on the device by the first call on each device: outside
+ * a stream capture that call runs the filling kernel on `stream` and synchronises `stream` once
+ * (later calls on any stream then read the finished table); a first call made while `stream`
+ * is being captured puts the filling kernel into the graph ahead of the quantiser instead
+ * (each replay rewrites the same values) and leaves the once-per-device filling to the first
+ * call made outside a capture.
  */
 JQ_API jq_status jq_modulate_quantize_act(const void* x_bf16, int64_t M, int64_t K, int64_t ldx, const float* shift,
                                           const float* scale, int64_t tokens_per_sample, int32_t group, uint8_t* q,
