@@ -160,32 +160,120 @@ def dist_env():
     return rank, world, local
 
 
+class NvmlClocks:
+    """SM clock, its maximum, the clock-event (throttle) reason bits and the power draw of one
+    GPU, read through NVML (libnvidia-ml, installed with the driver) by ctypes: read-only
+    queries, a few microseconds each, so the timed region gets sampled many times."""
+
+    CLOCK_SM = 1  # NVML_CLOCK_SM
+
+    def __init__(self, index: int, uuid: str | None = None):
+        import ctypes
+        c = ctypes
+        lib = c.CDLL("libnvidia-ml.so.1")
+        lib.nvmlDeviceGetHandleByIndex_v2.argtypes = [c.c_uint, c.POINTER(c.c_void_p)]
+        lib.nvmlDeviceGetUUID.argtypes = [c.c_void_p, c.c_char_p, c.c_uint]
+        lib.nvmlDeviceGetClockInfo.argtypes = [c.c_void_p, c.c_int, c.POINTER(c.c_uint)]
+        lib.nvmlDeviceGetMaxClockInfo.argtypes = [c.c_void_p, c.c_int, c.POINTER(c.c_uint)]
+        lib.nvmlDeviceGetPowerUsage.argtypes = [c.c_void_p, c.POINTER(c.c_uint)]
+        reasons = getattr(lib, "nvmlDeviceGetCurrentClocksEventReasons", None)
+        if reasons is None:
+            reasons = lib.nvmlDeviceGetCurrentClocksThrottleReasons
+        reasons.argtypes = [c.c_void_p, c.POINTER(c.c_ulonglong)]
+        if lib.nvmlInit_v2() != 0:
+            raise OSError("nvmlInit_v2 failed")
+        self._c, self._lib, self._reasons = c, lib, reasons
+        self.handle = self._find(index, uuid)
+
+    def _find(self, index, uuid):
+        """The device whose UUID is the CUDA device's (CUDA and NVML may number GPUs differently),
+        else NVML index `index`."""
+        c, lib = self._c, self._lib
+        count = c.c_uint(0)
+        if uuid and lib.nvmlDeviceGetCount_v2(c.byref(count)) == 0:
+            buf = c.create_string_buffer(96)
+            for i in range(count.value):
+                h = c.c_void_p()
+                if (lib.nvmlDeviceGetHandleByIndex_v2(i, c.byref(h)) == 0
+                        and lib.nvmlDeviceGetUUID(h, buf, 96) == 0
+                        and buf.value.decode().lower().endswith(uuid.lower())):
+                    return h
+        h = c.c_void_p()
+        if lib.nvmlDeviceGetHandleByIndex_v2(index, c.byref(h)) != 0:
+            raise OSError(f"no NVML device {index}")
+        return h
+
+    def sample(self):
+        c, lib, h = self._c, self._lib, self.handle
+        sm, mx, pw, r = c.c_uint(), c.c_uint(), c.c_uint(), c.c_ulonglong()
+        if (lib.nvmlDeviceGetClockInfo(h, self.CLOCK_SM, c.byref(sm)) != 0
+                or lib.nvmlDeviceGetMaxClockInfo(h, self.CLOCK_SM, c.byref(mx)) != 0
+                or self._reasons(h, c.byref(r)) != 0):
+            return None
+        power = pw.value / 1000.0 if lib.nvmlDeviceGetPowerUsage(h, c.byref(pw)) == 0 else None
+        return sm.value, mx.value, r.value, power
+
+    def close(self):
+        self._lib.nvmlShutdown()
+
+
+# NVML clock-event reason bits (nvmlClocksEventReason*) and the names nvidia-smi gives them.
+CLOCK_REASON_BITS = {0x4: "sw_power_cap", 0x8: "hw_slowdown", 0x20: "sw_thermal_slowdown",
+                     0x40: "hw_thermal_slowdown", 0x80: "hw_power_brake_slowdown"}
+
+
 class ClockSampler:
-    """Samples SM clocks and throttle reasons with nvidia-smi while the timed region runs."""
+    """Samples SM clocks and throttle reasons while the timed region runs: through NVML every
+    5 ms, or, where NVML cannot be loaded, with nvidia-smi (one sample per call, ~0.2 s apart)."""
 
     QUERY = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+    NAMES = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
 
-    def __init__(self, gpu_index: int):
+    def __init__(self, gpu_index: int, uuid: str | None = None, nvml=None):
         self.gpu = gpu_index
-        self.samples = []
+        self.uuid = uuid
+        self.samples = []  # (sm MHz, max MHz, reason names, power W)
+        self.source = None
+        self._nvml = nvml
         self._stop = threading.Event()
         self._thread = None
 
-    def _run(self):
+    def _run_nvml(self):
+        while not self._stop.is_set():
+            s = self._nvml.sample()
+            if s is not None:
+                sm, mx, bits, power = s
+                self.samples.append((float(sm), float(mx),
+                                     [n for b, n in CLOCK_REASON_BITS.items() if bits & b], power))
+            self._stop.wait(0.005)
+
+    def _run_smi(self):
+        gpu = f"GPU-{self.uuid}" if self.uuid and not self.uuid.startswith("GPU-") else (self.uuid or self.gpu)
         while not self._stop.is_set():
             try:
-                out = subprocess.run(["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.QUERY}",
+                out = subprocess.run(["nvidia-smi", f"--id={gpu}", f"--query-gpu={self.QUERY}",
                                       "--format=csv,noheader,nounits"], capture_output=True, text=True, timeout=5)
                 if out.returncode == 0 and out.stdout.strip():
-                    self.samples.append([v.strip() for v in out.stdout.strip().split(",")])
+                    v = [x.strip() for x in out.stdout.strip().split(",")]
+                    num = lambda t: float(t) if t.replace(".", "").isdigit() else None  # noqa: E731
+                    self.samples.append((num(v[1]), num(v[2]),
+                                         [n for n, a in zip(self.NAMES, v[5:9]) if a.lower() == "active"],
+                                         num(v[3])))
             except Exception:
                 return
             self._stop.wait(0.2)
 
     def __enter__(self):
-        self._thread = threading.Thread(target=self._run, daemon=True)
+        if self._nvml is None:
+            try:
+                self._nvml = NvmlClocks(self.gpu, self.uuid)
+            except Exception:
+                self._nvml = None
+        self.source = "nvml" if self._nvml is not None else "nvidia-smi"
+        self._thread = threading.Thread(target=self._run_nvml if self._nvml is not None else self._run_smi,
+                                        daemon=True)
         self._thread.start()
         return self
 
@@ -193,16 +281,26 @@ class ClockSampler:
         self._stop.set()
         if self._thread:
             self._thread.join(timeout=10)
+        if isinstance(self._nvml, NvmlClocks):
+            self._nvml.close()
 
     def summary(self):
         if not self.samples:
-            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unsampled"]}
-        sm = [float(s[1]) for s in self.samples if s[1].replace(".", "").isdigit()]
-        mx = [float(s[2]) for s in self.samples if s[2].replace(".", "").isdigit()]
-        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
-        reasons = sorted({n for s in self.samples for n, v in zip(names, s[5:9]) if v.lower() == "active"})
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unsampled"], "source": self.source}
+        sm = [s[0] for s in self.samples if s[0] is not None]
+        mx = [s[1] for s in self.samples if s[1] is not None]
+        pw = [s[3] for s in self.samples if s[3] is not None]
         return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(mx) if mx else None,
-                "reasons": reasons, "samples": len(self.samples)}
+                "reasons": sorted({n for s in self.samples for n in s[2]}), "samples": len(self.samples),
+                "power_w": round(statistics.median(pw), 1) if pw else None, "source": self.source}
+
+
+def device_uuid(torch, dev) -> str | None:
+    """The CUDA device's UUID (to find the same GPU in NVML), where this PyTorch reports it."""
+    try:
+        return str(torch.cuda.get_device_properties(dev).uuid)
+    except Exception:
+        return None
 
 
 def measured_peaks():
@@ -616,7 +714,7 @@ def run_stream(args):
         import torch.distributed as dist
         dist.barrier()
     torch.cuda.synchronize()
-    with ClockSampler(local) as clocks:
+    with ClockSampler(local, device_uuid(torch, dev)) as clocks:
         t0.record(stream)
         g.replay()
         t1.record(stream)
@@ -810,7 +908,7 @@ def run_ours(args):
     l_start, l_end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     barrier()
     torch.cuda.synchronize()
-    with ClockSampler(local) as clocks:
+    with ClockSampler(local, device_uuid(torch, dev)) as clocks:
         t_start.record(stream)
         g_steps.replay()
         t_end.record(stream)

@@ -89,3 +89,38 @@ def test_cpu_baseline_reports_an_all_cores_and_a_single_thread_sample(monkeypatc
     assert st["cores"] == 1 and st["value"] > 0
     assert oracle.max_threads() == threads  # restored
     assert "single_thread" not in o.describe(o.run(o.rows))
+
+
+class _FakeNvml:
+    """Stands in for NvmlClocks: a fixed SM clock, its maximum, reason bits and power."""
+
+    def __init__(self, bits):
+        self.bits = bits
+        self.calls = 0
+
+    def sample(self):
+        self.calls += 1
+        return 1965, 2070, self.bits, 1180.5
+
+
+def test_clock_sampler_decodes_nvml_reason_bits():
+    import time
+    with bench.ClockSampler(0, nvml=_FakeNvml(0x4 | 0x8 | 0x1)) as c:  # power cap, hw slowdown, idle
+        time.sleep(0.05)
+    s = c.summary()
+    assert s["source"] == "nvml" and s["samples"] >= 2
+    assert s["sm_mhz"] == 1965 and s["sm_max_mhz"] == 2070 and s["power_w"] == 1180.5
+    # the idle bit is not a throttle reason; the two others keep nvidia-smi's names
+    assert s["reasons"] == ["hw_slowdown", "sw_power_cap"]
+    with bench.ClockSampler(0, nvml=_FakeNvml(0)) as c:
+        time.sleep(0.02)
+    assert c.summary()["reasons"] == []
+
+
+def test_clock_sampler_reports_an_unsampled_region():
+    class Dead:
+        def sample(self):
+            return None
+    with bench.ClockSampler(0, nvml=Dead()) as c:
+        pass
+    assert c.summary()["reasons"] == ["unsampled"]
