@@ -205,6 +205,81 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
   return *reinterpret_cast<const uint32_t*>(&v);
 }
 
+// The epilogue of the row-layout drain.  Lane l holds output row row0 + l; written as it is held,
+// each 16-byte store instruction would touch 32 rows (32 memory lines).  Instead the lanes of each
+// aligned group of W exchange 16-byte chunks (a W x W transpose by xor-shuffle butterflies: at
+// distance d a lane swaps chunk k | d or k, by bit d of its lane index, with its partner's other
+// one), after which lane g + j holds chunk j of rows g .. g + W - 1, and each store instruction
+// writes W consecutive chunks (16 W contiguous bytes) of each of 32 / W rows.
+template <int W>
+__device__ __forceinline__ void transpose_chunks(uint4 (&o)[W], uint32_t lane) {
+#pragma unroll
+  for (int d = 1; d < W; d <<= 1) {
+    const bool up = (lane & (uint32_t)d) != 0;
+#pragma unroll
+    for (int k = 0; k < W; ++k) {
+      if (k & d) continue;
+      const uint4 send = up ? o[k] : o[k | d];
+      uint4 recv;
+      recv.x = __shfl_xor_sync(0xffffffffu, send.x, d);
+      recv.y = __shfl_xor_sync(0xffffffffu, send.y, d);
+      recv.z = __shfl_xor_sync(0xffffffffu, send.z, d);
+      recv.w = __shfl_xor_sync(0xffffffffu, send.w, d);
+      if (up)
+        o[k] = recv;
+      else
+        o[k | d] = recv;
+    }
+  }
+}
+
+// Columns c0 .. c0 + 8W - 1 of the warp's D (relative to col0): + bias, bf16, transposed, stored.
+// Rows at or past M and chunks at or past N (N % 8 == 0: a chunk is wholly inside or outside)
+// are not written.
+template <int W, int D, int C0>
+__device__ __forceinline__ void store_block(const Args& args, const float2 (&y)[D / 2], int row0, int col0,
+                                            uint32_t lane) {
+  uint4 o[W];
+#pragma unroll
+  for (int k = 0; k < W; ++k) {
+    const int c = C0 + 8 * k, col = col0 + c;
+    float4 b0 = make_float4(0.f, 0.f, 0.f, 0.f), b1 = b0;
+    if (args.bias != nullptr && col < args.N) {
+      b0 = __ldg(reinterpret_cast<const float4*>(args.bias + col));
+      b1 = __ldg(reinterpret_cast<const float4*>(args.bias + col + 4));
+    }
+    const float2* yy = y + (c >> 1);
+    o[k].x = pack_bf16x2(yy[0].x + b0.x, yy[0].y + b0.y);
+    o[k].y = pack_bf16x2(yy[1].x + b0.z, yy[1].y + b0.w);
+    o[k].z = pack_bf16x2(yy[2].x + b1.x, yy[2].y + b1.y);
+    o[k].w = pack_bf16x2(yy[3].x + b1.z, yy[3].y + b1.w);
+  }
+  transpose_chunks<W>(o, lane);
+  const uint32_t j = lane & (uint32_t)(W - 1);
+  const int col = col0 + C0 + 8 * (int)j;
+  const int rg = row0 + (int)(lane - j);
+#pragma unroll
+  for (int t = 0; t < W; ++t) {
+    const int r = rg + t;
+    if (r < args.M && col < args.N) *reinterpret_cast<uint4*>(args.y + (int64_t)r * args.N + col) = o[t];
+  }
+}
+
+// Columns C0 .. D - 1: blocks of 8W columns while they fit, the rest (D % 16 == 0) in narrower
+// blocks.
+template <int W, int D, int C0>
+__device__ __forceinline__ void store_rows(const Args& args, const float2 (&y)[D / 2], int row0, int col0,
+                                           uint32_t lane) {
+  static_assert(D % 16 == 0 && W >= 2, "16-column blocks at the least");
+  if constexpr (C0 + 8 * W <= D) {
+    store_block<W, D, C0>(args, y, row0, col0, lane);
+    store_rows<W, D, C0 + 8 * W>(args, y, row0, col0, lane);
+  } else if constexpr (C0 < D) {
+    store_rows<W / 2, D, C0>(args, y, row0, col0, lane);
+  }
+}
+constexpr int kStoreLanes = 4;
+
 // Linear path, several groups (sign-magnitude weight codes): warp w (drain index d = w - 8) owns
 // one row per thread -- TMEM lane 32*(w%4) + lane -- and columns D*(d/4).. of each accumulator
 // (D = kBN/2: 128 for the 256-column tile), read 16 at a time with the 32x32b shape: two loads in
@@ -220,7 +295,7 @@ __device__ __forceinline__ void drain_linear_rows(const Args& args, const Pair& 
   constexpr int D = T::kDrainCols, kBatches = D / 16;
   static_assert(kBatches >= 2, "the load pipeline needs two batches");
   const uint32_t warp = warp_id(), lane = lane_id();
-  const int M = args.M, N = args.N, groups = args.groups;
+  const int M = args.M, groups = args.groups;
   const uint32_t quarter = warp & 3u, half = (warp - kDrainWarp0) >> 2;
   const uint32_t trow = quarter * 32u + lane;  // row within the CTA's 128
   uint32_t chunk_it = 0, sc_it = 0;
@@ -328,27 +403,8 @@ __device__ __forceinline__ void drain_linear_rows(const Args& args, const Pair& 
       ++chunk_it;
     }
     if (!ok) break;
-    // + bias, round to bf16, store: each thread writes its row's D columns, 8 (16 bytes) at a time
-    if (row_ok) {
-#pragma unroll
-      for (int c = 0; c < D; c += 8) {
-        const int col = col0 + c;
-        if (col < N) {  // N % 8 == 0: a chunk is wholly inside or outside
-          float4 b0 = make_float4(0.f, 0.f, 0.f, 0.f), b1 = b0;
-          if (args.bias != nullptr) {
-            b0 = __ldg(reinterpret_cast<const float4*>(args.bias + col));
-            b1 = __ldg(reinterpret_cast<const float4*>(args.bias + col + 4));
-          }
-          const float2* yy = y + (c >> 1);
-          uint4 o;
-          o.x = pack_bf16x2(yy[0].x + b0.x, yy[0].y + b0.y);
-          o.y = pack_bf16x2(yy[1].x + b0.z, yy[1].y + b0.w);
-          o.z = pack_bf16x2(yy[2].x + b1.x, yy[2].y + b1.y);
-          o.w = pack_bf16x2(yy[3].x + b1.z, yy[3].y + b1.w);
-          *reinterpret_cast<uint4*>(args.y + (int64_t)row * N + col) = o;
-        }
-      }
-    }
+    // + bias, round to bf16, store (whole-warp shuffles: every lane takes part)
+    store_rows<kStoreLanes, D, 0>(args, y, row - (int)lane, col0, lane);
   }
 }
 // Linear path, 256-column tiles, one group (offset weight codes, drained once per tile): warp w
