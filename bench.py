@@ -93,11 +93,7 @@ FP8_PER_BF16 = 2.0  # nominal dense FP8 / BF16 tensor-core ratio on GB300 (4.5 /
 # from an ncu capture of that kernel, keyed by workload and by the hash of the kernel code the
 # capture was taken on (kernel_hash); once the code changes the figure no longer applies and the
 # bench reports null until a new capture is recorded here.
-KERNEL_TRAFFIC: dict = {
-    ("flux_qkv", "b083073b8736b564"): 54.676992e6 + 143.107328e6,
-    ("dllm", "b083073b8736b564"): 31.281152e6 + 0.165376e6,
-    ("dllm/ternary", "b083073b8736b564"): 18.681088e6 + 0.109568e6,
-}
+KERNEL_TRAFFIC: dict = {}
 
 
 def recorded_traffic(workload: str, kernel_file: str):
