@@ -179,7 +179,11 @@ class NvmlClocks:
         if lib.nvmlInit_v2() != 0:
             raise OSError("nvmlInit_v2 failed")
         self._c, self._lib, self._reasons = c, lib, reasons
-        self.handle = self._find(index, uuid)
+        try:
+            self.handle = self._find(index, uuid)
+        except Exception:
+            lib.nvmlShutdown()
+            raise
 
     def _find(self, index, uuid):
         """The device whose UUID is the CUDA device's (CUDA and NVML may number GPUs differently),
