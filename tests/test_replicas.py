@@ -57,3 +57,22 @@ def test_reference_arm_runs_on_rank_zero_only(monkeypatch, capsys):
                                       "--warmup", "3"])
     assert bench.main() == 0
     assert capsys.readouterr().out == ""  # rank 1 exits without work or output
+
+
+@pytest.mark.parametrize("workload,unit", [("dllm", "TOPS"), ("quant_dllm", "GB/s")])
+def test_reference_arm_line_on_rank_zero(monkeypatch, capsys, workload, unit):
+    # the reference arm times the oracle on the host cores and prints the contract's JSON line
+    import json
+    import bench
+    monkeypatch.delenv("RANK", raising=False)
+    monkeypatch.delenv("WORLD_SIZE", raising=False)
+    monkeypatch.setattr(sys, "argv", ["bench.py", "--impl", "reference", "--workload", workload, "--steps", "1",
+                                      "--warmup", "3", "--ref-seconds", "0.2", "--ref-single-seconds", "0.2"])
+    assert bench.main() == 0
+    line = json.loads(capsys.readouterr().out.strip().splitlines()[-1])
+    assert line["impl"] == "reference" and line["unit"] == unit and line["n_gpus"] == 1
+    assert line["steps"] == 1 and line["warmup"] == 3 and line["higher_is_better"] is True
+    assert line["value"] > 0 and line["config"]["workload"]
+    cb = line["cpu_baseline"]
+    assert cb["kind"] == "oracle" and cb["cores"] >= 1 and cb["sample"] and cb["value"] == line["value"]
+    assert line["e2e"] == {"value": line["value"], "unit": unit, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}
